@@ -1,0 +1,259 @@
+/*
+ * oracle.c -- plain CPU oracle (TEST INFRASTRUCTURE ONLY; see oracle.h).
+ *
+ * Written for a reader checking it against the paper: tokens are kept as
+ * their byte strings, the scanner as the raw [Q][256] table, the bracket
+ * stack as an array of symbols.  Loops are the definitions, nothing more.
+ * OpenMP (when compiled in) only splits independent rows across threads.
+ */
+#include "oracle.h"
+
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+#define ORACLE_MAX_DEPTH 32
+
+struct oracle_problem {
+    int32_t n_tokens, eos_id, n_states, max_depth;
+    uint8_t* bytes;      /* all token bytes */
+    int64_t* offsets;    /* [n_tokens + 1] */
+    int32_t* delta;      /* [n_states][256] */
+    uint8_t* live;       /* [n_states] */
+    uint8_t* accepting;  /* [n_states] */
+    oracle_rule* rules;  /* [n_rules] */
+    int32_t* rule_at;    /* [n_states][256]: index into rules or -1 */
+};
+
+static void* dup_bytes(const void* src, size_t n) {
+    void* d = malloc(n ? n : 1);
+    if (d && n) memcpy(d, src, n);
+    return d;
+}
+
+oracle_problem* oracle_new(const uint8_t* bytes, const int64_t* offsets, int32_t n_tokens, int32_t eos_id,
+                           const int32_t* delta, int32_t n_states, const uint8_t* live,
+                           const uint8_t* accepting, const oracle_rule* rules, int32_t n_rules,
+                           int32_t max_depth) {
+    if (n_tokens < 0 || n_states < 1 || max_depth < 0 || max_depth > ORACLE_MAX_DEPTH) return NULL;
+    if (eos_id >= n_tokens) return NULL;
+    for (int64_t i = 0; i < (int64_t)n_states * 256; i++)
+        if (delta[i] < 0 || delta[i] >= n_states) return NULL;
+    oracle_problem* p = (oracle_problem*)calloc(1, sizeof(*p));
+    p->n_tokens = n_tokens;
+    p->eos_id = eos_id;
+    p->n_states = n_states;
+    p->max_depth = max_depth;
+    p->offsets = (int64_t*)dup_bytes(offsets, sizeof(int64_t) * (size_t)(n_tokens + 1));
+    p->bytes = (uint8_t*)dup_bytes(bytes, (size_t)offsets[n_tokens]);
+    p->delta = (int32_t*)dup_bytes(delta, sizeof(int32_t) * (size_t)n_states * 256);
+    p->live = (uint8_t*)dup_bytes(live, (size_t)n_states);
+    p->accepting = (uint8_t*)calloc((size_t)n_states, 1);
+    if (accepting) memcpy(p->accepting, accepting, (size_t)n_states);
+    p->rules = (oracle_rule*)dup_bytes(rules, sizeof(oracle_rule) * (size_t)(n_rules > 0 ? n_rules : 0));
+    p->rule_at = (int32_t*)malloc(sizeof(int32_t) * (size_t)n_states * 256);
+    for (int64_t i = 0; i < (int64_t)n_states * 256; i++) p->rule_at[i] = -1;
+    for (int32_t r = 0; r < n_rules; r++) {
+        const oracle_rule* R = &rules[r];
+        int bad = R->state < 0 || R->state >= n_states || (R->kind != ORACLE_PUSH && R->kind != ORACLE_POP) ||
+                  R->sym > 1;
+        if (!bad && R->kind == ORACLE_POP)
+            bad = R->next_if_empty < 0 || R->next_if_empty >= n_states || R->next_if_top0 < 0 ||
+                  R->next_if_top0 >= n_states || R->next_if_top1 < 0 || R->next_if_top1 >= n_states;
+        int32_t* slot = bad ? NULL : &p->rule_at[(int64_t)R->state * 256 + R->byte];
+        if (bad || *slot != -1) {   /* malformed, or two rules on one (state, byte) */
+            oracle_free(p);
+            return NULL;
+        }
+        *slot = r;
+    }
+    return p;
+}
+
+void oracle_free(oracle_problem* p) {
+    if (!p) return;
+    free(p->bytes); free(p->offsets); free(p->delta); free(p->live); free(p->accepting);
+    free(p->rules); free(p->rule_at);
+    free(p);
+}
+
+/* The bracket stack as the parser sees it: sym[0] is the bottom. */
+typedef struct {
+    int depth;
+    uint8_t sym[ORACLE_MAX_DEPTH];
+} stack_t_;
+
+/* Boundary word -> stack.  Returns 0 when the word is not a valid stack. */
+static int decode_stack(uint64_t w, int max_depth, stack_t_* st) {
+    uint64_t depth = (w >> 32) & 0xFF;
+    uint64_t bits = w & 0xFFFFFFFFull;
+    if ((w >> 40) != 0 || depth > (uint64_t)max_depth) return 0;
+    if (depth < 32 && (bits >> depth) != 0) return 0;   /* symbols above the depth must be zero */
+    st->depth = (int)depth;
+    for (int i = 0; i < st->depth; i++)                  /* top symbol at bit 0 */
+        st->sym[i] = (uint8_t)((bits >> (st->depth - 1 - i)) & 1);
+    return 1;
+}
+
+static uint64_t encode_stack(const stack_t_* st) {
+    uint64_t bits = 0;
+    for (int i = 0; i < st->depth; i++) bits = (bits << 1) | st->sym[i];
+    return ((uint64_t)st->depth << 32) | bits;
+}
+
+static int config_valid(const oracle_problem* p, int32_t state, uint64_t stack, stack_t_* st) {
+    if (state < 0 || state >= p->n_states) return 0;
+    return decode_stack(stack, p->max_depth, st);
+}
+
+/* Walk one token from (s, st); st is updated in place.  Returns 1 when the
+ * token is allowed (Sec. 3.5 at k = infinity), with *end the state reached. */
+static int walk_token(const oracle_problem* p, int32_t s, stack_t_* st, int32_t t, int32_t* end) {
+    int64_t lo = p->offsets[t], hi = p->offsets[t + 1];
+    if (t == p->eos_id) {                         /* forced EOS: accepting and nothing left open */
+        *end = s;
+        return p->accepting[s] && st->depth == 0;
+    }
+    if (hi == lo) return 0;                       /* other empty tokens never advance the output */
+    for (int64_t i = lo; i < hi; i++) {
+        uint8_t c = p->bytes[i];
+        int32_t r = p->rule_at[(int64_t)s * 256 + c];
+        if (r < 0) {
+            s = p->delta[(int64_t)s * 256 + c];
+        } else if (p->rules[r].kind == ORACLE_PUSH) {
+            if (st->depth == p->max_depth) return 0;          /* bounded stack is full */
+            st->sym[st->depth++] = p->rules[r].sym;
+            s = p->delta[(int64_t)s * 256 + c];
+        } else {                                              /* POP */
+            if (st->depth == 0 || st->sym[st->depth - 1] != p->rules[r].sym) return 0;
+            st->depth--;
+            if (st->depth == 0) s = p->rules[r].next_if_empty;
+            else if (st->sym[st->depth - 1] == 0) s = p->rules[r].next_if_top0;
+            else s = p->rules[r].next_if_top1;
+        }
+        if (!p->live[s]) return 0;                /* no continuation can reach acceptance */
+    }
+    *end = s;
+    return 1;
+}
+
+int oracle_check_token(const oracle_problem* p, int32_t state, uint64_t stack, int32_t token,
+                       int32_t* next_state, uint64_t* next_stack) {
+    stack_t_ st;
+    if (!config_valid(p, state, stack, &st) || token < 0 || token >= p->n_tokens) return -1;
+    int32_t end = 0;
+    if (!walk_token(p, state, &st, token, &end)) return 0;
+    if (next_state) *next_state = end;
+    if (next_stack) *next_stack = encode_stack(&st);
+    return 1;
+}
+
+int64_t oracle_step_mask(const oracle_problem* p, const int32_t* states, const uint64_t* stacks,
+                         int32_t batch, uint32_t* mask, int32_t* next, int32_t n_threads) {
+    const int32_t V = p->n_tokens;
+    const int64_t W = ((int64_t)V + 31) / 32;
+    int64_t invalid = 0;
+#ifdef _OPENMP
+    if (n_threads < 1) n_threads = 1;
+#pragma omp parallel for schedule(dynamic, 1) num_threads(n_threads) reduction(+ : invalid)
+#endif
+    for (int32_t b = 0; b < batch; b++) {
+        uint32_t* mrow = mask + (int64_t)b * W;
+        int32_t* nrow = next ? next + (int64_t)b * V : NULL;
+        memset(mrow, 0, sizeof(uint32_t) * (size_t)W);
+        if (nrow) memset(nrow, 0, sizeof(int32_t) * (size_t)V);
+        stack_t_ st0;
+        if (!config_valid(p, states[b], stacks ? stacks[b] : 0, &st0)) {
+            invalid++;
+            continue;
+        }
+        for (int32_t t = 0; t < V; t++) {
+            stack_t_ st = st0;
+            int32_t end = 0;
+            if (walk_token(p, states[b], &st, t, &end)) {
+                mrow[t / 32] |= 1u << (t % 32);
+                if (nrow) nrow[t] = end;
+            }
+        }
+    }
+    return invalid;
+}
+
+static double logit_value(const void* logits, int32_t dtype, int64_t i) {
+    if (dtype == ORACLE_BF16) {
+        uint32_t u = (uint32_t)((const uint16_t*)logits)[i] << 16;   /* bf16 -> f32 is exact */
+        float f;
+        memcpy(&f, &u, sizeof f);
+        return (double)f;
+    }
+    return (double)((const float*)logits)[i];
+}
+
+void oracle_mask_logits(const void* logits, int32_t dtype, int32_t batch, int32_t n_tokens,
+                        int64_t row_stride, const uint32_t* mask, int32_t* argmax, double* lse,
+                        double* logprobs, int32_t n_threads) {
+    const int64_t W = ((int64_t)n_tokens + 31) / 32;
+#ifdef _OPENMP
+    if (n_threads < 1) n_threads = 1;
+#pragma omp parallel for schedule(dynamic, 1) num_threads(n_threads)
+#endif
+    for (int32_t b = 0; b < batch; b++) {
+        const uint32_t* mrow = mask + (int64_t)b * W;
+        const int64_t base = (int64_t)b * row_stride;
+        /* v' = m (.) v with -inf on masked tokens; decode = argmax (lowest index on ties) */
+        double m = -INFINITY;
+        int32_t best = -1;
+        for (int32_t t = 0; t < n_tokens; t++) {
+            if (!((mrow[t / 32] >> (t % 32)) & 1)) continue;
+            double x = logit_value(logits, dtype, base + t);
+            if (x > m) { m = x; best = t; }
+        }
+        argmax[b] = best;
+        double l = -INFINITY;
+        if (best >= 0) {
+            double sum = 0.0;
+            for (int32_t t = 0; t < n_tokens; t++)
+                if ((mrow[t / 32] >> (t % 32)) & 1) sum += exp(logit_value(logits, dtype, base + t) - m);
+            l = m + log(sum);
+        }
+        if (lse) lse[b] = l;
+        if (logprobs) {
+            double* lp = logprobs + (int64_t)b * n_tokens;
+            for (int32_t t = 0; t < n_tokens; t++)
+                lp[t] = ((mrow[t / 32] >> (t % 32)) & 1) ? logit_value(logits, dtype, base + t) - l : -INFINITY;
+        }
+    }
+}
+
+int64_t oracle_advance(const oracle_problem* p, const int32_t* states, const uint64_t* stacks,
+                       const int32_t* tokens, int32_t batch, int32_t start_state, int32_t* states_out,
+                       uint64_t* stacks_out) {
+    int64_t invalid = 0;
+    for (int32_t b = 0; b < batch; b++) {
+        int32_t t = tokens[b];
+        int32_t s = states[b];
+        uint64_t w = stacks ? stacks[b] : 0;
+        int32_t s_out = 0;
+        uint64_t w_out = 0;
+        if (t < 0 || t == p->eos_id) {            /* sequence ended: next one starts at init */
+            s_out = start_state;
+        } else {
+            stack_t_ st;
+            if (t >= p->n_tokens || !config_valid(p, s, w, &st)) {
+                invalid++;
+            } else {
+                int32_t end = 0;
+                if (walk_token(p, s, &st, t, &end)) {
+                    s_out = end;
+                    w_out = encode_stack(&st);
+                }
+            }
+        }
+        states_out[b] = s_out;
+        if (stacks_out) stacks_out[b] = w_out;
+    }
+    return invalid;
+}

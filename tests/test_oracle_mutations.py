@@ -1,0 +1,50 @@
+"""The oracle's pins must catch plausible mistakes.
+
+Each case copies oracle.c, plants one mistake (a dropped term, a wrong index,
+a swapped operand), builds the copy on the CPU and runs the pin suite against
+it in a subprocess: the suite must fail.  The committed oracle is untouched.
+"""
+import os
+import shutil
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+SRC = os.path.join(ROOT, "oracle", "oracle.c")
+
+MUTANTS = {
+    "no_live_check": ("if (!p->live[s]) return 0;", "if (0) return 0;"),
+    "eos_ignores_stack": ("return p->accepting[s] && st->depth == 0;", "return p->accepting[s];"),
+    "pop_ignores_top": ("st->sym[st->depth - 1] != p->rules[r].sym) return 0;", "0) return 0;"),
+    "push_ignores_bound": ("if (st->depth == p->max_depth) return 0;", "if (0) return 0;"),
+    "revealed_swapped": ("else if (st->sym[st->depth - 1] == 0) s = p->rules[r].next_if_top0;",
+                         "else if (st->sym[st->depth - 1] == 1) s = p->rules[r].next_if_top0;"),
+    "ties_highest_index": ("if (x > m) { m = x; best = t; }", "if (x >= m) { m = x; best = t; }"),
+    "lse_drops_max": ("l = m + log(sum);", "l = log(sum);"),
+    "mask_bit_shifted": ("mrow[t / 32] |= 1u << (t % 32);", "mrow[t / 32] |= 1u << ((t + 1) % 32);"),
+    "empty_token_allowed": ("if (hi == lo) return 0;", "if (0) return 0;"),
+    "bf16_wrong_shift": ("((const uint16_t*)logits)[i] << 16;", "((const uint16_t*)logits)[i] << 15;"),
+    "stack_top_at_wrong_end": ("(uint8_t)((bits >> (st->depth - 1 - i)) & 1);", "(uint8_t)((bits >> i) & 1);"),
+    "advance_eos_keeps_state": ("s_out = start_state;", "s_out = s;"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_pins_catch_mutant(tmp_path, name):
+    old, new = MUTANTS[name]
+    src = open(SRC).read()
+    assert src.count(old) == 1, name
+    d = tmp_path / "oracle"
+    d.mkdir()
+    shutil.copy(os.path.join(ROOT, "oracle", "oracle.h"), d / "oracle.h")
+    (d / "oracle.c").write_text(src.replace(old, new))
+    so = d / "liboracle_mutant.so"
+    subprocess.run(["gcc", "-O1", "-std=c11", "-fopenmp", "-fPIC", "-shared", "-o", str(so), str(d / "oracle.c"),
+                    "-lm"], check=True)
+    env = dict(os.environ, DOMINO_ORACLE_SO=str(so))
+    r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",
+                        os.path.join(ROOT, "tests", "test_oracle_pins.py")],
+                       cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
+    assert r.returncode != 0, f"mutant {name} survived the pins:\n{r.stdout[-2000:]}"
