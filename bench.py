@@ -1,0 +1,467 @@
+#!/usr/bin/env python
+"""Masked decode-step throughput of the DOMINO hot path on GB300.
+
+One step = C.mask() (step_mask) -> v' = m (.) v + greedy decode (mask_logits)
+-> C.update() (advance) over one batch (Alg. 1).  Default workload: random
+sparse DFA (Q = 5000, 32 byte classes), V = 128256, batch 256, bf16 logits
+N(0, 3), rotating over enough logits buffers to exceed twice the L2.
+
+Prints ONE JSON line (rank 0).  Metric = token-checks/s (batch x vocabulary
+per second of whole decode steps); masked decode steps/s and per-kernel
+rooflines are extra keys.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 3]
+  python bench.py --impl reference ...   # the CPU oracle on host cores
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "token-checks/s and masked decode steps/s at 1 GB300; mask+logits HBM GB/s vs peak"
+UNIT = "token-checks/s"
+L2_BYTES = 129 * 1024 * 1024
+WORKLOAD_HELP = {1: "kv16_v1024_b1", 2: "kv200_v32000_b32", 3: "sparse5000_v128256_b256",
+                 5: "json300_pda_v152064_b128"}
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=2000)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["domino", "reference"], default="domino")
+    p.add_argument("--workload", type=int, default=3, choices=sorted(WORKLOAD_HELP))
+    p.add_argument("--e2e-steps", type=int, default=100)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-graph", action="store_true", help="launch eagerly (used for ncu launch lists)")
+    p.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle baseline")
+    return p.parse_args()
+
+
+# ----------------------------------------------------------------------------
+# distributed plumbing (replicas only: no data-path collective)
+# ----------------------------------------------------------------------------
+class Dist:
+    def __init__(self):
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.local = int(os.environ.get("LOCAL_RANK", "0"))
+        self.pg = None
+        if self.world > 1:
+            import torch.distributed as dist
+            backend = "nccl" if _cuda_ok() else "gloo"
+            dist.init_process_group(backend)
+            self.pg = dist
+
+    def barrier(self):
+        if self.pg:
+            self.pg.barrier()
+
+    def max(self, x: float) -> float:
+        if not self.pg:
+            return x
+        import torch
+        dev = f"cuda:{self.local}" if _cuda_ok() and self.pg.get_backend() == "nccl" else "cpu"
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX)
+        return float(t.item())
+
+    def close(self):
+        if self.pg:
+            self.pg.destroy_process_group()
+
+
+def _cuda_ok():
+    import torch
+    return torch.cuda.is_available()
+
+
+# ----------------------------------------------------------------------------
+# SM clock / throttle sampling during the timed region (NVML, read only)
+# ----------------------------------------------------------------------------
+REASONS = {0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap", 0x8: "hw_slowdown",
+           0x10: "sync_boost", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown",
+           0x80: "hw_power_brake_slowdown", 0x100: "display_clock_setting"}
+
+
+class ClockSampler:
+    def __init__(self, torch_dev: int, period_s: float = 0.002):
+        self.period = period_s
+        self.samples = []
+        self.reasons = 0
+        self.max_mhz = None
+        self.ok = False
+        self._stop = threading.Event()
+        try:
+            nv = ctypes.CDLL("libnvidia-ml.so.1")
+            if nv.nvmlInit_v2() != 0:
+                return
+            h = ctypes.c_void_p()
+            import torch
+            uuid = None
+            try:
+                uuid = "GPU-" + str(torch.cuda.get_device_properties(torch_dev).uuid)
+            except Exception:
+                pass
+            rc = nv.nvmlDeviceGetHandleByUUID(uuid.encode(), ctypes.byref(h)) if uuid else 1
+            if rc != 0:
+                vis = os.environ.get("CUDA_VISIBLE_DEVICES", "")
+                idx = int(vis.split(",")[torch_dev]) if vis and vis.split(",")[0].isdigit() else torch_dev
+                if nv.nvmlDeviceGetHandleByIndex_v2(idx, ctypes.byref(h)) != 0:
+                    return
+            self.nv, self.h = nv, h
+            c = ctypes.c_uint()
+            if nv.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(c)) == 0:
+                self.max_mhz = c.value
+            self._reason_fn = getattr(nv, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+                getattr(nv, "nvmlDeviceGetCurrentClocksThrottleReasons")
+            self.ok = True
+        except Exception:
+            self.ok = False
+
+    def _run(self):
+        c = ctypes.c_uint()
+        r = ctypes.c_ulonglong()
+        while not self._stop.is_set():
+            if self.nv.nvmlDeviceGetClockInfo(self.h, 1, ctypes.byref(c)) == 0:
+                self.samples.append(c.value)
+            if self._reason_fn(self.h, ctypes.byref(r)) == 0:
+                self.reasons |= r.value & ~0x1
+            time.sleep(self.period)
+
+    def start(self):
+        if self.ok:
+            self._t = threading.Thread(target=self._run, daemon=True)
+            self._t.start()
+
+    def stop(self):
+        if self.ok:
+            self._stop.set()
+            self._t.join()
+
+    def summary(self):
+        if not self.ok or not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": self.max_mhz, "reasons": ["unavailable"]}
+        names = [n for bit, n in REASONS.items() if self.reasons & bit]
+        return {"sm_mhz": statistics.median(self.samples), "sm_max_mhz": self.max_mhz, "reasons": names,
+                "samples": len(self.samples)}
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}, "fallback"
+
+
+# ----------------------------------------------------------------------------
+# CPU oracle baseline (bounded sample of the same workload)
+# ----------------------------------------------------------------------------
+def cpu_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def oracle_step_sample(w, P, states, stacks, rows, step, cores):
+    """One oracle decode step (mask -> masked argmax/lse -> advance) on `rows` rows."""
+    import oracle
+    lg = w.logits(step, batch=rows)           # same values as the first `rows` rows
+    st = states[:rows]
+    sk = stacks[:rows] if w.automaton.rules is not None else None
+    m, _, _ = P.step_mask(st, sk, n_threads=cores)
+    arg, _, _ = oracle.mask_logits(lg, m, want_logprobs=w.want_logprobs, n_threads=cores)
+    P.advance(st, sk, arg, w.automaton.start)
+
+
+def cpu_baseline(w, target_s: float):
+    import oracle
+    cores = cpu_cores()
+    P = oracle.Problem.from_workload(w)
+    states, stacks = w.initial_configs()
+    V = w.vocab.n_tokens
+    rows = min(w.batch, max(1, cores))
+    t0 = time.perf_counter()
+    oracle_step_sample(w, P, states, stacks, rows, 0, cores)
+    t1 = time.perf_counter() - t0
+    reps = max(1, int(target_s / max(t1, 1e-3)))
+    # logits generation is not part of the oracle's work: pre-generate
+    lgs = [w.logits(i, batch=rows) for i in range(min(reps, 4))]
+    t0 = time.perf_counter()
+    for r in range(reps):
+        lg = lgs[r % len(lgs)]
+        st = states[:rows]
+        sk = stacks[:rows] if w.automaton.rules is not None else None
+        m, _, _ = P.step_mask(st, sk, n_threads=cores)
+        arg, _, _ = oracle.mask_logits(lg, m, want_logprobs=w.want_logprobs, n_threads=cores)
+        P.advance(st, sk, arg, w.automaton.start)
+    dt = time.perf_counter() - t0
+    return {"value": rows * V * reps / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{reps} decode steps of {rows} of the {w.batch} rows (full vocabulary V={V}); "
+                      f"step_mask + mask_logits + advance, OpenMP over rows",
+            "steps_per_s_equiv": reps * rows / w.batch / dt}
+
+
+# ----------------------------------------------------------------------------
+# reference arm: the oracle timed on the host cores
+# ----------------------------------------------------------------------------
+def run_reference(args, dist: Dist):
+    from paper_2403_06988_gb300 import synth
+    if dist.rank != 0:
+        return
+    import oracle
+    w = synth.workload(args.workload)
+    cores = cpu_cores()
+    P = oracle.Problem.from_workload(w)
+    states, stacks = w.initial_configs()
+    V = w.vocab.n_tokens
+    rows = min(w.batch, max(1, cores))
+    # size each step's sample so that K + W steps stay within about two minutes
+    t0 = time.perf_counter()
+    oracle_step_sample(w, P, states, stacks, rows, 0, cores)
+    per = time.perf_counter() - t0
+    budget = 120.0 / max(1, args.steps + args.warmup)
+    rows = max(1, min(rows, int(rows * budget / max(per, 1e-4))))
+    for i in range(args.warmup):
+        oracle_step_sample(w, P, states, stacks, rows, i, cores)
+    lgs = [w.logits(i, batch=rows) for i in range(4)]
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        st = states[:rows]
+        sk = stacks[:rows] if w.automaton.rules is not None else None
+        m, _, _ = P.step_mask(st, sk, n_threads=cores)
+        arg, _, _ = oracle.mask_logits(lgs[i % 4], m, want_logprobs=w.want_logprobs, n_threads=cores)
+        P.advance(st, sk, arg, w.automaton.start)
+    dt = time.perf_counter() - t0
+    value = rows * V * args.steps / dt
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3 / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": w.name, "batch": w.batch, "vocab": V,
+                                            "states": w.automaton.n_states, "sample_rows_per_step": rows},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": f"{rows} of {w.batch} rows per step, full vocabulary"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------
+# the GPU arm
+# ----------------------------------------------------------------------------
+def run_domino(args, dist: Dist):
+    import torch
+
+    from paper_2403_06988_gb300 import Domino, synth
+    from paper_2403_06988_gb300 import _binding as B
+
+    dev_id = dist.local
+    torch.cuda.set_device(dev_id)
+    dev = f"cuda:{dev_id}"
+    w = synth.workload(args.workload)
+    a, v = w.automaton, w.vocab
+    d = Domino.from_parts(a, v, device=dev_id)
+    info = d.info()
+    Bsz, V, Wd = w.batch, v.n_tokens, info["n_words"]
+    stack = a.rules is not None
+    states0, stacks0 = w.initial_configs(part=2 + 17 * dist.rank)   # each replica its own batch
+    states = torch.from_numpy(states0).to(dev)
+    stacks = torch.from_numpy(stacks0.view(np.int64)).to(dev) if stack else None
+    esz = 2 if w.logits_dtype == "bf16" else 4
+    logit_bytes = Bsz * V * esz
+    nbuf = max(4, math.ceil(2.2 * L2_BYTES / logit_bytes))
+    host_logits = [w.logits(100 + i) for i in range(nbuf)]
+
+    def to_dev(x):
+        t = torch.from_numpy(x.view(np.int16) if x.dtype == np.uint16 else x).to(dev)
+        return t.view(torch.bfloat16) if x.dtype == np.uint16 else t
+    logits = [to_dev(x) for x in host_logits]
+    mask = torch.empty((Bsz, Wd), dtype=torch.int32, device=dev)
+    argmax = torch.empty(Bsz, dtype=torch.int32, device=dev)
+    lse = torch.empty(Bsz, dtype=torch.float32, device=dev)
+    logprobs = torch.empty((Bsz, V), dtype=torch.float32, device=dev) if w.want_logprobs else None
+    dtype_code = B.DTYPE_BF16 if w.logits_dtype == "bf16" else B.DTYPE_F32
+    L = B.lib()
+    h = d.h
+    # raw pointers once: per-step host work is three C calls
+    p_states, p_stacks = states.data_ptr(), (stacks.data_ptr() if stack else None)
+    p_mask, p_arg, p_lse = mask.data_ptr(), argmax.data_ptr(), lse.data_ptr()
+    p_lp = logprobs.data_ptr() if logprobs is not None else None
+    p_logits = [t.data_ptr() for t in logits]
+    launches_per_step = 3 + (1 if w.want_logprobs else 0)
+
+    def step(i, stream_ptr, ev=None):
+        if ev is not None:
+            ev[0].record()
+        rc = L.domino_step_mask(h, p_states, p_stacks, Bsz, p_mask, None, stream_ptr)
+        if ev is not None:
+            ev[1].record()
+        rc |= L.domino_mask_logits(h, p_logits[i % nbuf], dtype_code, Bsz, V, p_mask, p_arg, p_lse, p_lp,
+                                   stream_ptr)
+        if ev is not None:
+            ev[2].record()
+        rc |= L.domino_advance(h, p_states, p_stacks, p_arg, Bsz, p_states, p_stacks, stream_ptr)
+        if ev is not None:
+            ev[3].record()
+        if rc:
+            raise RuntimeError(f"domino call failed ({rc})")
+
+    K, Wm = args.steps, args.warmup
+    s = torch.cuda.Stream(device=dev)
+    with torch.cuda.stream(s):
+        sp = s.cuda_stream
+        for i in range(Wm):
+            step(i, sp)
+    torch.cuda.synchronize()
+
+    try:
+        events = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(4)] for _ in range(K)]
+        have_ext = True
+    except TypeError:
+        events, have_ext = None, False
+    graph = None
+    if not args.no_graph:
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=s, capture_error_mode="relaxed"):
+            sp = torch.cuda.current_stream().cuda_stream
+            for i in range(K):
+                step(i, sp, events[i] if have_ext else None)
+        graph.replay()                      # upload + one untimed pass
+        torch.cuda.synchronize()
+
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(dev_id)
+    dist.barrier()
+    torch.cuda.synchronize()
+    sampler.start()
+    with torch.cuda.stream(s):
+        t_start.record()
+        if graph is not None:
+            graph.replay()
+        else:
+            sp = s.cuda_stream
+            for i in range(K):
+                step(i, sp, events[i] if events else None)
+        t_end.record()
+    torch.cuda.synchronize()
+    sampler.stop()
+    dist.barrier()
+    ms = t_start.elapsed_time(t_end)
+    ms_max = dist.max(ms)
+    err = d.device_error()
+    if err:
+        raise RuntimeError(f"device error word {err}")
+
+    per_kernel = None
+    if events is not None and (graph is None or have_ext):
+        tk = [0.0, 0.0, 0.0]
+        for ev in events:
+            for j in range(3):
+                tk[j] += ev[j].elapsed_time(ev[j + 1])
+        per_kernel = {"step_mask": tk[0] / K, "mask_logits": tk[1] / K, "advance": tk[2] / K}
+
+    # ---- end to end through the host-buffer C entry point -------------------
+    Ke = max(3, min(args.e2e_steps, K))
+    pin = [torch.from_numpy(x.view(np.int16) if x.dtype == np.uint16 else x).pin_memory() for x in host_logits[:2]]
+    st_h = torch.from_numpy(states0.copy()).pin_memory()
+    sk_h = torch.from_numpy(stacks0.view(np.int64).copy()).pin_memory() if stack else None
+    tok_h = torch.empty(Bsz, dtype=torch.int32).pin_memory()
+    lse_h = torch.empty(Bsz, dtype=torch.float32).pin_memory()
+    e_start = torch.cuda.Event(enable_timing=True)
+    e_end = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(s):
+        sp = s.cuda_stream
+
+        def e2e_step(i):
+            rc = L.domino_decode_step_host(h, pin[i % 2].data_ptr(), dtype_code, Bsz, st_h.data_ptr(),
+                                           sk_h.data_ptr() if stack else None, tok_h.data_ptr(), lse_h.data_ptr(),
+                                           sp)
+            if rc:
+                raise RuntimeError(f"decode_step_host failed ({rc})")
+        for i in range(3):
+            e2e_step(i)
+        dist.barrier()
+        torch.cuda.synchronize()
+        e_start.record()
+        for i in range(Ke):
+            e2e_step(i)
+        e_end.record()
+    torch.cuda.synchronize()
+    e2e_ms = dist.max(e_start.elapsed_time(e_end))
+    h2d = logit_bytes + Bsz * 4 + (Bsz * 8 if stack else 0)
+    d2h = Bsz * 4 * 3 + (Bsz * 8 if stack else 0)
+
+    # ---- report ---------------------------------------------------------------
+    n = dist.world
+    value = n * Bsz * V * K / (ms_max / 1e3)
+    peaks, peak_kind = measured_peaks()
+    hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
+    kernels = {}
+    if per_kernel:
+        lg_bytes = Bsz * V * esz + Bsz * Wd * 4 + Bsz * 8 + (Bsz * V * 4 if w.want_logprobs else 0)
+        t_ml = per_kernel["mask_logits"] * 1e-3
+        kernels["mask_logits"] = {"us": per_kernel["mask_logits"] * 1e3, "bytes": lg_bytes,
+                                  "gbs": lg_bytes / t_ml / 1e9, "frac_hbm": lg_bytes / t_ml / 1e9 / hbm_peak}
+        t_sm = per_kernel["step_mask"] * 1e-3
+        kernels["step_mask"] = {"us": per_kernel["step_mask"] * 1e3, "checks_per_s": Bsz * V / t_sm,
+                                "mask_bytes": Bsz * Wd * 4}
+        kernels["advance"] = {"us": per_kernel["advance"] * 1e3}
+    roofline = None
+    if per_kernel:
+        km = kernels["mask_logits"]
+        roofline = {"kernel": "mask_logits", "bound": "hbm", "achieved": km["gbs"], "peak": hbm_peak,
+                    "unit": "GB/s", "frac": km["frac_hbm"], "traffic": None, "peak_source": peak_kind,
+                    "note": "dominant HBM-bound kernel; step_mask is reported in `kernels`"}
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": n, "steps": K, "warmup": Wm,
+        "ms_per_step": ms_max / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": w.logits_dtype, "data": "synthetic",
+        "config": {"workload": w.name, "batch": Bsz, "vocab": V, "states": a.n_states,
+                   "byte_classes": info["n_classes"], "table_in_smem": info["table_in_smem"],
+                   "logprobs": w.want_logprobs,
+                   "l2": f"logits rotate over {nbuf} buffers ({nbuf * logit_bytes / 2**20:.0f} MiB > 2x L2)",
+                   "parallelism": f"replicas x{n}", "graph": graph is not None},
+        "masked_decode_steps_per_s": n * K / (ms_max / 1e3),
+        "kernels": kernels, "roofline": roofline,
+        "e2e": {"value": n * Bsz * V * Ke / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "steps": Ke, "api": "domino_decode_step_host (pinned host buffers)"},
+        "gpu_launches": K * launches_per_step,
+        "clocks": sampler.summary(),
+    }
+    if dist.rank == 0 and n == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds)
+    if dist.rank == 0:
+        print(json.dumps(line), flush=True)
+    d.close()
+
+
+def main():
+    args = parse()
+    dist = Dist()
+    try:
+        if args.impl == "reference":
+            run_reference(args, dist)
+        else:
+            run_domino(args, dist)
+    finally:
+        dist.close()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,205 @@
+/*
+ * domino.h -- C ABI of libdomino.so: the per-decode-step hot path of DOMINO
+ * ("Guiding LLMs The Right Way: Fast, Non-Invasive Constrained Generation")
+ * on one GB300 GPU (sm_103a).
+ *
+ * The problem statement the calls follow (Alg. 1, Sec. 2): a checker C with
+ * init / update / mask over a subword vocabulary V; C is a byte-level scanner
+ * (Sec. 3.2) plus, for the context-free case, a bounded bracket-stack parser
+ * (Sec. 3.4); the scanner x vocabulary table is precomputed offline
+ * (Sec. 3.5), and the mask is applied to the logits before decoding
+ * (Alg. 1, v' = m (.) v; decode = argmax).
+ *
+ * Conventions shared by every call
+ *  - Return value: DOMINO_OK (0) or a negative DOMINO_E_* code.  Host-side
+ *    argument checks are synchronous; nothing is launched when they fail.
+ *  - "*_dev" pointers are device memory owned by the caller (e.g. torch
+ *    tensors); kernels run asynchronously on `stream` (a cudaStream_t passed
+ *    as void*, NULL = legacy default stream).  No call synchronises except the
+ *    load calls, domino_get_device_error and domino_decode_step_host.
+ *  - Mask layout: row b has W = ceil(V/32) uint32 words; token t is bit
+ *    (t & 31) of word (t >> 5), least significant bit first; pad bits >= V
+ *    are 0.
+ *  - Stack word (uint64): bits 0..31 hold the bracket symbols with the top of
+ *    the stack at bit 0 (a push shifts left and inserts at bit 0); bits 32..39
+ *    hold the depth (0..max_depth); all other bits and the symbol bits at or
+ *    above the depth are 0.  NULL stacks = every stack empty.
+ *  - Invalid device inputs (state id outside [0, Q), a malformed stack word,
+ *    a token id >= V in domino_advance) are treated as the dead configuration
+ *    (all tokens rejected, next state 0) and set a bit of the sticky device
+ *    error word read by domino_get_device_error.  No kernel traps.
+ *  - A handle is not thread-safe; calls on one handle must be serialised by
+ *    the caller (the kernels of different calls may overlap on the GPU only
+ *    if the caller puts them on different streams).
+ */
+#ifndef DOMINO_H
+#define DOMINO_H
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define DOMINO_OK 0
+#define DOMINO_E_INVALID_ARG (-1)  /* bad pointer, size, id or automaton/vocabulary */
+#define DOMINO_E_NOT_LOADED (-2)   /* vocabulary or automaton missing */
+#define DOMINO_E_UNSUPPORTED (-3)  /* valid request this build does not implement */
+#define DOMINO_E_OOM (-4)          /* device or host allocation failed */
+#define DOMINO_E_CUDA (-5)         /* a CUDA runtime call failed */
+#define DOMINO_E_NO_DEVICE (-6)    /* compute call on a host-only handle */
+
+/* bits of the device error word */
+#define DOMINO_DEVERR_BAD_STATE 1u
+#define DOMINO_DEVERR_BAD_STACK 2u
+#define DOMINO_DEVERR_BAD_TOKEN 4u
+
+#define DOMINO_RULE_PUSH 1
+#define DOMINO_RULE_POP 2
+#define DOMINO_DTYPE_F32 0
+#define DOMINO_DTYPE_BF16 1
+#define DOMINO_MAX_DEPTH 32
+#define DOMINO_MAX_STATES 65535
+
+typedef struct domino_ctx* domino_t;
+
+/* One bracket-stack rule (Sec. 3.4, the parser consulted on each terminal),
+ * 20 bytes.  It fires on byte `byte` read in scanner state `state`, before
+ * the scanner step:
+ *   PUSH sym: rejected if depth == max_depth; else push sym and take the
+ *             scanner transition delta[state][byte].
+ *   POP sym:  rejected if depth == 0 or the top != sym; else pop, and the
+ *             next state is next_if_empty / next_if_top0 / next_if_top1 by the
+ *             symbol the pop reveals (delta[state][byte] is ignored). */
+typedef struct {
+    int32_t state;
+    uint8_t byte;
+    uint8_t kind; /* DOMINO_RULE_PUSH or DOMINO_RULE_POP */
+    uint8_t sym;  /* 0 or 1 */
+    uint8_t pad;  /* must be 0 */
+    int32_t next_if_empty;
+    int32_t next_if_top0;
+    int32_t next_if_top1;
+} domino_stack_rule;
+
+/* What a handle holds (filled by domino_get_info). */
+typedef struct {
+    int32_t n_tokens;      /* V */
+    int32_t n_words;       /* W = ceil(V/32) */
+    int32_t eos_id;        /* -1: none */
+    int32_t max_token_len; /* bytes */
+    int32_t n_states;      /* Q */
+    int32_t n_classes;     /* K, byte classes after compression */
+    int32_t start_state;
+    int32_t max_depth;
+    int32_t n_rules;
+    int32_t has_stack;     /* 1 when stack rules were loaded */
+    int32_t table_in_smem; /* 1 when the transition table is staged in shared memory */
+    int32_t device;        /* CUDA ordinal, -1 for a host-only handle */
+    int64_t device_bytes;  /* device memory the handle owns */
+} domino_info;
+
+/* Creates a handle on CUDA device `cuda_device` (it becomes the current device
+ * of the calling thread).  cuda_device = -1 creates a host-only handle that
+ * validates and preprocesses loads but refuses every compute call with
+ * DOMINO_E_NO_DEVICE.  *out is NULL on failure. */
+int domino_create(domino_t* out, int32_t cuda_device);
+
+/* Frees the handle and all device memory it owns (synchronises the device
+ * first).  NULL is accepted. */
+int domino_destroy(domino_t h);
+
+/* Vocabulary V (Sec. 2, subword tokens; Fig. 3 c).  Token t is the byte
+ * string bytes[offsets[t] .. offsets[t+1]) (host arrays, copied; offsets has
+ * n_tokens + 1 entries, offsets[0] == 0, non-decreasing, each token <= 65535
+ * bytes).  eos_id (-1: none) names the end-of-sequence token; its bytes are
+ * ignored.  Replaces any earlier vocabulary; returns after the device copy is
+ * complete.  1 <= n_tokens <= 2^24. */
+int domino_load_vocab(domino_t h, const uint8_t* bytes, const int64_t* offsets, int32_t n_tokens,
+                      int32_t eos_id);
+
+/* Character scanner (Sec. 3.2, a DFA over bytes) and optional bracket rules
+ * (Sec. 3.4).  delta is [n_states][256] int32 (host), live[q] != 0 marks states
+ * from which acceptance is still reachable, accepting may be NULL (none).
+ * Rejected (DOMINO_E_INVALID_ARG) unless: 1 <= n_states <= 65535; every id is
+ * in [0, n_states); state 0 is non-live, absorbing and carries no rule; every
+ * successor of a non-live state (including POP targets) is non-live;
+ * accepting implies live; start_state is in range; rules name valid states,
+ * kinds and symbols, pad == 0, at most one rule per (state, byte);
+ * 0 <= max_depth <= 32.  Transitions into non-live states are redirected to
+ * state 0 (exact early exit) and bytes that every state treats alike share a
+ * byte class.  Returns after the device copy is complete. */
+int domino_load_automaton(domino_t h, const int32_t* delta, int32_t n_states, const uint8_t* live,
+                          const uint8_t* accepting, int32_t start_state, const domino_stack_rule* rules,
+                          int32_t n_rules, int32_t max_depth);
+
+int domino_get_info(domino_t h, domino_info* out);
+
+/* Byte -> class id map of the loaded automaton (256 bytes, host). */
+int domino_get_byte_classes(domino_t h, uint8_t* classes_out);
+
+/* Offline precompute (Alg. 2's "for every state q, for every token l,
+ * traverse"; Sec. 3.5 "computed before inference starts"): for every state
+ * q < Q, the mask row of q (mask_dev [Q][W]) and the next state of every token
+ * (next_dev [Q][V] int32, 0 for rejected tokens; EOS keeps q).  Row q equals
+ * domino_step_mask with states = {q} and empty stacks.  Either output may be
+ * NULL, not both.  Pushdown automata: DOMINO_E_UNSUPPORTED (a row would
+ * depend on the whole stack). */
+int domino_precompute_table(domino_t h, int32_t* next_dev, uint32_t* mask_dev, void* stream);
+
+/* C.mask() of Alg. 1 at lookahead k = infinity (Sec. 3.5; Definition
+ * "minimally invasive", Sec. 2): for every sequence b < batch and token t,
+ * t is allowed iff its bytes walked from (states_dev[b], stacks_dev[b])
+ * through the scanner and bracket rules never reach a non-live state.  EOS is
+ * allowed iff the state is accepting and the stack is empty (forced EOS,
+ * Sec. 2; Fig. 3 e); other zero-length tokens are rejected.
+ *   states_dev int32 [batch]; stacks_dev uint64 [batch] or NULL;
+ *   mask_dev uint32 [batch][W] (written in full);
+ *   next_dev int32 [batch][V] or NULL: end state of allowed tokens, 0 else.
+ * batch = 0 is a no-op. */
+int domino_step_mask(domino_t h, const int32_t* states_dev, const uint64_t* stacks_dev, int32_t batch,
+                     uint32_t* mask_dev, int32_t* next_dev, void* stream);
+
+/* Alg. 1 "v' = m (.) v; t = decode(v')" with greedy decode, fused: per row b,
+ * over the allowed tokens only, m = max logit, argmax = the lowest token id
+ * with logit m, lse = m + log(sum exp(logit - m)) (fp32 accumulation), and
+ * logprob[t] = logit[t] - lse for allowed t, -inf for masked t.  A row with
+ * no allowed token gives argmax -1, lse -inf and all log-probs -inf.
+ *   logits_dev [batch] rows of V values (dtype DOMINO_DTYPE_F32 or
+ *   DOMINO_DTYPE_BF16), row_stride_elems >= V apart; mask_dev [batch][W];
+ *   argmax_dev int32 [batch] (required); lse_dev float [batch] or NULL;
+ *   logprobs_dev float [batch][V] or NULL.
+ * Logits must be finite.  Uses scratch memory owned by the handle. */
+int domino_mask_logits(domino_t h, const void* logits_dev, int32_t dtype, int32_t batch,
+                       int64_t row_stride_elems, const uint32_t* mask_dev, int32_t* argmax_dev, float* lse_dev,
+                       float* logprobs_dev, void* stream);
+
+/* C.update(o) of Alg. 1 for the token just decoded: walks tokens_dev[b] from
+ * (states_dev[b], stacks_dev[b]).  tokens_dev[b] < 0 (no token) or == eos_id
+ * ends the sequence and the next one starts from init: (start_state, empty).
+ * A rejected token gives (0, empty).  Outputs may alias the inputs.
+ * stacks_out may be NULL only when stacks_dev is NULL. */
+int domino_advance(domino_t h, const int32_t* states_dev, const uint64_t* stacks_dev, const int32_t* tokens_dev,
+                   int32_t batch, int32_t* states_out, uint64_t* stacks_out, void* stream);
+
+/* One whole decode step from HOST memory (end-to-end use): copies logits
+ * (batch rows of V values, dense) and the configurations to the device,
+ * runs step_mask -> mask_logits -> advance, copies tokens_host[b] (the
+ * argmax), lse_host (may be NULL) and the new configurations back into
+ * states_host / stacks_host (stacks_host may be NULL for a DFA), and
+ * synchronises `stream`.  Pinned host memory makes the copies asynchronous.
+ * Device staging buffers are owned by the handle and grown on demand. */
+int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, int32_t batch,
+                            int32_t* states_host, uint64_t* stacks_host, int32_t* tokens_host, float* lse_host,
+                            void* stream);
+
+/* Synchronises `stream`, returns the sticky device error word (DOMINO_DEVERR_*
+ * bits, 0 = none) in *code and clears it. */
+int domino_get_device_error(domino_t h, int32_t* code, void* stream);
+
+/* Static text for a status code. */
+const char* domino_status_string(int status);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

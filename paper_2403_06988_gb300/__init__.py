@@ -1,0 +1,106 @@
+"""DOMINO constrained decoding hot path on GB300 (sm_103a).
+
+The compute lives in libdomino.so (C ABI in include/domino.h, kernels in
+csrc/).  `_binding` exposes every entry point under its C name; `Domino`
+below is a thin holder of one handle that allocates output tensors with torch
+and forwards to those entry points.  There is no CPU fallback: without a
+built libdomino.so the binding raises ImportError, and compute calls on a
+handle created without a GPU raise DominoError(E_NO_DEVICE).
+"""
+from __future__ import annotations
+
+from typing import Optional, Tuple
+
+from . import _binding as B
+from ._binding import DominoError, DTYPE_BF16, DTYPE_F32  # noqa: F401
+
+
+class Domino:
+    """One library handle: a vocabulary plus a scanner (+ bracket rules)."""
+
+    def __init__(self, device: int = 0):
+        self.device = device
+        self.h = B.domino_create(device)
+
+    def close(self):
+        if self.h:
+            B.domino_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    # -- loads ---------------------------------------------------------------
+    def load_vocab(self, vocab) -> None:
+        B.domino_load_vocab(self.h, vocab.data, vocab.offsets, vocab.n_tokens, vocab.eos_id)
+
+    def load_automaton(self, a) -> None:
+        B.domino_load_automaton(self.h, a.delta, a.n_states, a.live, a.accepting, a.start, a.rules, None,
+                                a.max_depth)
+
+    @staticmethod
+    def from_parts(automaton, vocab, device: int = 0) -> "Domino":
+        d = Domino(device)
+        d.load_vocab(vocab)
+        d.load_automaton(automaton)
+        return d
+
+    def info(self) -> dict:
+        return B.domino_get_info(self.h)
+
+    # -- compute (torch tensors on this handle's device) -----------------------
+    def step_mask(self, states, stacks=None, want_next: bool = False, out_mask=None, out_next=None,
+                  stream=None):
+        import torch
+        info = self.info()
+        b = states.shape[0]
+        mask = out_mask if out_mask is not None else torch.empty((b, info["n_words"]), dtype=torch.int32,
+                                                                 device=states.device)
+        nxt = out_next
+        if want_next and nxt is None:
+            nxt = torch.empty((b, info["n_tokens"]), dtype=torch.int32, device=states.device)
+        B.domino_step_mask(self.h, states, stacks, b, mask, nxt, stream)
+        return mask, nxt
+
+    def precompute_table(self, want_next: bool = True, want_mask: bool = True, stream=None):
+        import torch
+        info = self.info()
+        dev = f"cuda:{self.device}"
+        nxt = torch.empty((info["n_states"], info["n_tokens"]), dtype=torch.int32, device=dev) if want_next else None
+        mask = torch.empty((info["n_states"], info["n_words"]), dtype=torch.int32, device=dev) if want_mask else None
+        B.domino_precompute_table(self.h, nxt, mask, stream)
+        return nxt, mask
+
+    def mask_logits(self, logits, mask, want_lse: bool = True, want_logprobs: bool = False, n_tokens: Optional[int]
+                    = None, out=None, stream=None) -> Tuple:
+        import torch
+        b = logits.shape[0]
+        V = n_tokens if n_tokens is not None else self.info()["n_tokens"]
+        dtype = DTYPE_BF16 if logits.dtype == torch.bfloat16 else DTYPE_F32
+        if dtype == DTYPE_F32 and logits.dtype != torch.float32:
+            raise TypeError("logits must be float32 or bfloat16")
+        if logits.stride(1) != 1:
+            raise ValueError("logits rows must be contiguous")
+        argmax, lse, lp = out if out is not None else (None, None, None)
+        if argmax is None:
+            argmax = torch.empty(b, dtype=torch.int32, device=logits.device)
+        if want_lse and lse is None:
+            lse = torch.empty(b, dtype=torch.float32, device=logits.device)
+        if want_logprobs and lp is None:
+            lp = torch.empty((b, V), dtype=torch.float32, device=logits.device)
+        B.domino_mask_logits(self.h, logits.data_ptr(), dtype, b, logits.stride(0), mask, argmax,
+                             lse if want_lse else None, lp if want_logprobs else None, stream)
+        return argmax, (lse if want_lse else None), (lp if want_logprobs else None)
+
+    def advance(self, states, stacks, tokens, states_out=None, stacks_out=None, stream=None):
+        b = states.shape[0]
+        so = states if states_out is None else states_out
+        wo = stacks if stacks_out is None else stacks_out
+        B.domino_advance(self.h, states, stacks, tokens, b, so, wo, stream)
+        return so, wo
+
+    def device_error(self, stream=None) -> int:
+        return B.domino_get_device_error(self.h, stream)

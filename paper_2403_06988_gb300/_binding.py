@@ -1,0 +1,216 @@
+"""ctypes binding of libdomino.so (include/domino.h).
+
+Argument marshalling only: every function here has the name of the C entry
+point it calls, turns torch tensors / numpy arrays into pointers and the
+current CUDA stream into a cudaStream_t, and raises DominoError on a non-zero
+status.  All computation happens in the library's kernels.  Importing this
+module fails loudly when libdomino.so has not been built.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+from typing import Optional
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libdomino.so")
+HEADER = os.path.join(os.path.dirname(_PKG), "include", "domino.h")
+
+DOMINO_OK = 0
+DTYPE_F32 = 0
+DTYPE_BF16 = 1
+DEVERR_BAD_STATE = 1
+DEVERR_BAD_STACK = 2
+DEVERR_BAD_TOKEN = 4
+STATUS = {0: "OK", -1: "E_INVALID_ARG", -2: "E_NOT_LOADED", -3: "E_UNSUPPORTED", -4: "E_OOM", -5: "E_CUDA",
+          -6: "E_NO_DEVICE"}
+
+
+class DominoError(RuntimeError):
+    def __init__(self, fn: str, status: int, text: str):
+        super().__init__(f"{fn} failed: {STATUS.get(status, status)} ({text})")
+        self.status = status
+
+
+class StackRule(ctypes.Structure):
+    _fields_ = [("state", ctypes.c_int32), ("byte", ctypes.c_uint8), ("kind", ctypes.c_uint8),
+                ("sym", ctypes.c_uint8), ("pad", ctypes.c_uint8), ("next_if_empty", ctypes.c_int32),
+                ("next_if_top0", ctypes.c_int32), ("next_if_top1", ctypes.c_int32)]
+
+
+class Info(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in (
+        "n_tokens", "n_words", "eos_id", "max_token_len", "n_states", "n_classes", "start_state", "max_depth",
+        "n_rules", "has_stack", "table_in_smem", "device")] + [("device_bytes", ctypes.c_int64)]
+
+
+_lib = None
+P = ctypes.c_void_p
+I32 = ctypes.c_int32
+I64 = ctypes.c_int64
+
+_SIGS = {
+    "domino_create": [P, I32],
+    "domino_destroy": [P],
+    "domino_load_vocab": [P, P, P, I32, I32],
+    "domino_load_automaton": [P, P, I32, P, P, I32, P, I32, I32],
+    "domino_get_info": [P, P],
+    "domino_get_byte_classes": [P, P],
+    "domino_precompute_table": [P, P, P, P],
+    "domino_step_mask": [P, P, P, I32, P, P, P],
+    "domino_mask_logits": [P, P, I32, I32, I64, P, P, P, P, P],
+    "domino_advance": [P, P, P, P, I32, P, P, P],
+    "domino_decode_step_host": [P, P, I32, I32, P, P, P, P, P],
+    "domino_get_device_error": [P, P, P],
+}
+
+
+def lib() -> ctypes.CDLL:
+    """Loads libdomino.so; raises when it has not been built (no fallback)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise ImportError(f"libdomino.so is not built ({LIB_PATH}); run __graft_entry__.build() "
+                              "or python -m paper_2403_06988_gb300.build")
+        L = ctypes.CDLL(LIB_PATH)
+        for name, args in _SIGS.items():
+            f = getattr(L, name)
+            f.argtypes = args
+            f.restype = ctypes.c_int
+        L.domino_status_string.argtypes = [ctypes.c_int]
+        L.domino_status_string.restype = ctypes.c_char_p
+        _lib = L
+    return _lib
+
+
+def header_symbols():
+    """Entry points declared in include/domino.h."""
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"^\s*(?:int|const char\*)\s+(domino_\w+)\s*\(", text, flags=re.M)))
+
+
+def _check(fn: str, status: int):
+    if status != DOMINO_OK:
+        raise DominoError(fn, status, lib().domino_status_string(status).decode())
+
+
+def _ptr(x) -> Optional[int]:
+    """Device or host address of a torch tensor / numpy array (None passes NULL)."""
+    if x is None:
+        return None
+    if isinstance(x, np.ndarray):
+        assert x.flags["C_CONTIGUOUS"]
+        return x.ctypes.data
+    if hasattr(x, "data_ptr"):
+        assert x.is_contiguous()
+        return x.data_ptr()
+    if isinstance(x, int):
+        return x
+    raise TypeError(type(x))
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is not None:
+        return stream if isinstance(stream, int) else stream.cuda_stream
+    import torch
+    return torch.cuda.current_stream().cuda_stream
+
+
+def status_string(status: int) -> str:
+    return lib().domino_status_string(int(status)).decode()
+
+
+# ----------------------------------------------------------------------------
+# one function per entry point
+# ----------------------------------------------------------------------------
+def domino_create(cuda_device: int) -> int:
+    h = ctypes.c_void_p()
+    _check("domino_create", lib().domino_create(ctypes.byref(h), int(cuda_device)))
+    return h.value
+
+
+def domino_destroy(h: int) -> None:
+    _check("domino_destroy", lib().domino_destroy(h))
+
+
+def domino_load_vocab(h: int, data: np.ndarray, offsets: np.ndarray, n_tokens: int, eos_id: int) -> None:
+    data = np.ascontiguousarray(data, dtype=np.uint8)
+    offsets = np.ascontiguousarray(offsets, dtype=np.int64)
+    _check("domino_load_vocab", lib().domino_load_vocab(h, _ptr(data), _ptr(offsets), int(n_tokens), int(eos_id)))
+
+
+def rules_to_ctypes(rules):
+    if rules is None or len(rules) == 0:
+        return None, 0
+    arr = (StackRule * len(rules))()
+    for i, r in enumerate(rules):
+        arr[i] = StackRule(int(r["state"]), int(r["byte"]), int(r["kind"]), int(r["sym"]), int(r["pad"]),
+                           int(r["next_if_empty"]), int(r["next_if_top0"]), int(r["next_if_top1"]))
+    return arr, len(rules)
+
+
+def domino_load_automaton(h: int, delta: np.ndarray, n_states: int, live: np.ndarray, accepting, start_state: int,
+                          rules, n_rules: Optional[int], max_depth: int) -> None:
+    delta = np.ascontiguousarray(delta, dtype=np.int32)
+    live = np.ascontiguousarray(live, dtype=np.uint8)
+    acc = None if accepting is None else np.ascontiguousarray(accepting, dtype=np.uint8)
+    if isinstance(rules, ctypes.Array):
+        arr, n = rules, len(rules)
+    else:
+        arr, n = rules_to_ctypes(rules)
+    if n_rules is not None:
+        n = int(n_rules)
+    _check("domino_load_automaton", lib().domino_load_automaton(
+        h, _ptr(delta), int(n_states), _ptr(live), _ptr(acc), int(start_state),
+        ctypes.cast(arr, ctypes.c_void_p) if arr is not None else None, n, int(max_depth)))
+
+
+def domino_get_info(h: int) -> dict:
+    info = Info()
+    _check("domino_get_info", lib().domino_get_info(h, ctypes.byref(info)))
+    return {name: getattr(info, name) for name, _ in Info._fields_}
+
+
+def domino_get_byte_classes(h: int) -> np.ndarray:
+    out = np.zeros(256, dtype=np.uint8)
+    _check("domino_get_byte_classes", lib().domino_get_byte_classes(h, _ptr(out)))
+    return out
+
+
+def domino_precompute_table(h: int, next_dev, mask_dev, stream=None) -> None:
+    _check("domino_precompute_table", lib().domino_precompute_table(h, _ptr(next_dev), _ptr(mask_dev),
+                                                                     _stream(stream)))
+
+
+def domino_step_mask(h: int, states_dev, stacks_dev, batch: int, mask_dev, next_dev=None, stream=None) -> None:
+    _check("domino_step_mask", lib().domino_step_mask(h, _ptr(states_dev), _ptr(stacks_dev), int(batch),
+                                                       _ptr(mask_dev), _ptr(next_dev), _stream(stream)))
+
+
+def domino_mask_logits(h: int, logits_dev, dtype: int, batch: int, row_stride_elems: int, mask_dev, argmax_dev,
+                       lse_dev=None, logprobs_dev=None, stream=None) -> None:
+    _check("domino_mask_logits", lib().domino_mask_logits(
+        h, _ptr(logits_dev), int(dtype), int(batch), int(row_stride_elems), _ptr(mask_dev), _ptr(argmax_dev),
+        _ptr(lse_dev), _ptr(logprobs_dev), _stream(stream)))
+
+
+def domino_advance(h: int, states_dev, stacks_dev, tokens_dev, batch: int, states_out, stacks_out=None,
+                   stream=None) -> None:
+    _check("domino_advance", lib().domino_advance(h, _ptr(states_dev), _ptr(stacks_dev), _ptr(tokens_dev),
+                                                   int(batch), _ptr(states_out), _ptr(stacks_out), _stream(stream)))
+
+
+def domino_decode_step_host(h: int, logits_host, dtype: int, batch: int, states_host, stacks_host, tokens_host,
+                            lse_host=None, stream=None) -> None:
+    _check("domino_decode_step_host", lib().domino_decode_step_host(
+        h, _ptr(logits_host), int(dtype), int(batch), _ptr(states_host), _ptr(stacks_host), _ptr(tokens_host),
+        _ptr(lse_host), _stream(stream)))
+
+
+def domino_get_device_error(h: int, stream=None) -> int:
+    code = ctypes.c_int32(0)
+    _check("domino_get_device_error", lib().domino_get_device_error(h, ctypes.byref(code), _stream(stream)))
+    return code.value

@@ -1,0 +1,601 @@
+// host.cpp -- the C ABI of libdomino.so: handle lifetime, loaders (validation,
+// dead-state canonicalisation, byte-class compression, vocabulary arena) and
+// argument checks in front of the kernels in kernels.cu.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdint>
+#include <cstring>
+#include <new>
+#include <numeric>
+#include <unordered_map>
+#include <vector>
+
+#include "domino.h"
+#include "domino_internal.h"
+
+using namespace domino;
+
+namespace {
+
+struct DevBuf {
+    void* p = nullptr;
+    size_t n = 0;
+};
+
+}  // namespace
+
+struct domino_ctx {
+    int device = -1;
+    LaunchEnv env{0, 0};
+
+    // ---- vocabulary (host copy, kept so the arena can be rebuilt per automaton)
+    bool vocab_loaded = false;
+    int32_t V = 0, W = 0, eos_id = -1, max_len = 0;
+    std::vector<uint8_t> tok_bytes;
+    std::vector<int64_t> tok_off;
+
+    // ---- automaton (preprocessed)
+    bool auto_loaded = false;
+    int32_t Q = 0, K = 0, start = 0, max_depth = 0, n_rules = 0;
+    bool stack = false;
+    uint8_t byte_class[256] = {0};
+    std::vector<uint16_t> t16;
+    std::vector<uint32_t> t32;
+    std::vector<uint16_t> ret;
+    std::vector<uint32_t> accept_bits;
+
+    // ---- device copies
+    DevBuf d_head, d_orig, d_len, d_tail_off, d_tail, d_pos_of;
+    DevBuf d_t16, d_t32, d_ret, d_accept;
+    DevBuf d_err, d_partials, d_counters, d_lse_tmp;
+    bool arena_ready = false;
+    int32_t n_windows = 0;
+    // staging for domino_decode_step_host
+    DevBuf s_logits, s_states, s_stacks, s_mask, s_tokens, s_lse;
+};
+
+namespace {
+
+struct DeviceGuard {
+    int prev = -1;
+    bool changed = false;
+    explicit DeviceGuard(int dev) {
+        if (dev < 0) return;
+        if (cudaGetDevice(&prev) == cudaSuccess && prev != dev) {
+            changed = cudaSetDevice(dev) == cudaSuccess;
+        }
+    }
+    ~DeviceGuard() {
+        if (changed) cudaSetDevice(prev);
+    }
+};
+
+void dev_free(DevBuf& b) {
+    if (b.p) cudaFree(b.p);
+    b.p = nullptr;
+    b.n = 0;
+}
+
+int64_t dev_bytes(const domino_ctx* h) {
+    const DevBuf* all[] = {&h->d_head, &h->d_orig, &h->d_len, &h->d_tail_off, &h->d_tail, &h->d_pos_of,
+                           &h->d_t16, &h->d_t32, &h->d_ret, &h->d_accept, &h->d_err, &h->d_partials,
+                           &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_states, &h->s_stacks,
+                           &h->s_mask, &h->s_tokens, &h->s_lse};
+    int64_t n = 0;
+    for (auto* b : all) n += (int64_t)b->n;
+    return n;
+}
+
+// (Re)allocates b to hold n bytes and uploads src (when non-null).
+int dev_upload(DevBuf& b, const void* src, size_t n) {
+    size_t want = ((n ? n : 16) + 15) / 16 * 16;   // vector staging reads whole 16-byte words
+    if (b.n < want) {
+        dev_free(b);
+        if (cudaMalloc(&b.p, want) != cudaSuccess) {
+            cudaGetLastError();
+            b.p = nullptr;
+            return DOMINO_E_OOM;
+        }
+        b.n = want;
+    }
+    if (src && n && cudaMemcpy(b.p, src, n, cudaMemcpyHostToDevice) != cudaSuccess) {
+        cudaGetLastError();
+        return DOMINO_E_CUDA;
+    }
+    return DOMINO_OK;
+}
+
+int dev_reserve(DevBuf& b, size_t n) { return dev_upload(b, nullptr, n); }
+
+bool is_host_only(const domino_ctx* h) { return h->device < 0; }
+
+// Byte-class strings of every token, the window sort and the slot arrays.
+int build_arena(domino_ctx* h) {
+    h->arena_ready = false;
+    if (!h->vocab_loaded || !h->auto_loaded) return DOMINO_OK;
+    const int32_t V = h->V;
+    const int32_t nw = (V + kWin - 1) / kWin;
+    const int64_t n_slots = (int64_t)nw * kWin;
+    std::vector<uint8_t> cls(h->tok_bytes.size());
+    for (size_t i = 0; i < cls.size(); i++) cls[i] = h->byte_class[h->tok_bytes[i]];
+    auto tlen = [&](int32_t t) -> int32_t {
+        return t == h->eos_id ? 0 : (int32_t)(h->tok_off[t + 1] - h->tok_off[t]);
+    };
+    auto less = [&](int32_t a, int32_t b) {
+        int32_t la = tlen(a), lb = tlen(b);
+        int c = std::memcmp(cls.data() + h->tok_off[a], cls.data() + h->tok_off[b], (size_t)std::min(la, lb));
+        if (c != 0) return c < 0;
+        if (la != lb) return la < lb;
+        return a < b;
+    };
+    std::vector<uint8_t> head((size_t)n_slots * kHeadBytes, 0);
+    std::vector<int32_t> orig((size_t)n_slots, -1), tail_off((size_t)n_slots, 0), pos_of((size_t)V, 0);
+    std::vector<uint16_t> len((size_t)n_slots, 0);
+    std::vector<uint8_t> tail;
+    std::vector<int32_t> ids;
+    for (int32_t w = 0; w < nw; w++) {
+        int32_t lo = w * kWin, hi = std::min(V, lo + kWin);
+        ids.resize((size_t)(hi - lo));
+        std::iota(ids.begin(), ids.end(), lo);
+        std::sort(ids.begin(), ids.end(), less);
+        for (int32_t j = 0; j < hi - lo; j++) {
+            int32_t t = ids[(size_t)j];
+            int64_t p = (int64_t)lo + j;
+            int32_t L = tlen(t);
+            orig[(size_t)p] = t;
+            len[(size_t)p] = (uint16_t)L;
+            pos_of[(size_t)t] = (int32_t)p;
+            const uint8_t* c = cls.data() + h->tok_off[t];
+            std::memcpy(head.data() + p * kHeadBytes, c, (size_t)std::min(L, kHeadBytes));
+            if (L > kHeadBytes) {
+                tail_off[(size_t)p] = (int32_t)tail.size();
+                tail.insert(tail.end(), c + kHeadBytes, c + L);
+            }
+        }
+    }
+    if (tail.size() > (size_t)INT32_MAX) return DOMINO_E_UNSUPPORTED;
+    int rc;
+    if ((rc = dev_upload(h->d_head, head.data(), head.size()))) return rc;
+    if ((rc = dev_upload(h->d_orig, orig.data(), orig.size() * 4))) return rc;
+    if ((rc = dev_upload(h->d_len, len.data(), len.size() * 2))) return rc;
+    if ((rc = dev_upload(h->d_tail_off, tail_off.data(), tail_off.size() * 4))) return rc;
+    if ((rc = dev_upload(h->d_tail, tail.data(), tail.size()))) return rc;
+    if ((rc = dev_upload(h->d_pos_of, pos_of.data(), pos_of.size() * 4))) return rc;
+    h->n_windows = nw;
+    h->arena_ready = true;
+    return DOMINO_OK;
+}
+
+StepView make_view(domino_ctx* h) {
+    StepView v{};
+    v.head = (const uint4*)h->d_head.p;
+    v.orig = (const int32_t*)h->d_orig.p;
+    v.len = (const uint16_t*)h->d_len.p;
+    v.tail_off = (const int32_t*)h->d_tail_off.p;
+    v.tail = (const uint8_t*)h->d_tail.p;
+    v.pos_of = (const int32_t*)h->d_pos_of.p;
+    v.V = h->V;
+    v.W = h->W;
+    v.n_windows = h->n_windows;
+    v.eos_id = h->eos_id;
+    v.t16 = (const uint16_t*)h->d_t16.p;
+    v.t32 = (const uint32_t*)h->d_t32.p;
+    v.ret = (const uint16_t*)h->d_ret.p;
+    v.accept_bits = (const uint32_t*)h->d_accept.p;
+    v.Q = h->Q;
+    v.K = h->K;
+    v.start = h->start;
+    v.max_depth = h->max_depth;
+    v.n_ret = (int32_t)(h->ret.size() / 4);
+    size_t tb = h->stack ? h->t32.size() * 4 : h->t16.size() * 2;
+    tb = (tb + 15) / 16 * 16;
+    tb += (h->ret.size() * 2 + 15) / 16 * 16;
+    v.table_bytes = (int32_t)tb;
+    v.err = (uint32_t*)h->d_err.p;
+    return v;
+}
+
+bool table_fits_smem(const domino_ctx* h, const StepView& v, bool next) {
+    if (h->env.max_smem_optin <= 0) return false;
+    return (int64_t)v.table_bytes + step_tile_smem_bytes(next) + 1024 <= (int64_t)h->env.max_smem_optin;
+}
+
+int ready_for_compute(domino_ctx* h) {
+    if (!h) return DOMINO_E_INVALID_ARG;
+    if (is_host_only(h)) return DOMINO_E_NO_DEVICE;
+    if (!h->vocab_loaded || !h->auto_loaded || !h->arena_ready) return DOMINO_E_NOT_LOADED;
+    return DOMINO_OK;
+}
+
+int cuda_status(cudaError_t e) {
+    if (e == cudaSuccess) return DOMINO_OK;
+    cudaGetLastError();
+    return DOMINO_E_CUDA;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* domino_status_string(int s) {
+    switch (s) {
+        case DOMINO_OK: return "ok";
+        case DOMINO_E_INVALID_ARG: return "invalid argument";
+        case DOMINO_E_NOT_LOADED: return "vocabulary or automaton not loaded";
+        case DOMINO_E_UNSUPPORTED: return "unsupported request";
+        case DOMINO_E_OOM: return "out of memory";
+        case DOMINO_E_CUDA: return "CUDA runtime error";
+        case DOMINO_E_NO_DEVICE: return "host-only handle has no device";
+        default: return "unknown status";
+    }
+}
+
+int domino_create(domino_t* out, int32_t cuda_device) {
+    if (!out) return DOMINO_E_INVALID_ARG;
+    *out = nullptr;
+    domino_ctx* h = new (std::nothrow) domino_ctx();
+    if (!h) return DOMINO_E_OOM;
+    h->device = cuda_device < 0 ? -1 : cuda_device;
+    if (h->device >= 0) {
+        int n = 0;
+        if (cudaGetDeviceCount(&n) != cudaSuccess || cuda_device >= n) {
+            cudaGetLastError();
+            delete h;
+            return cuda_device >= n && n > 0 ? DOMINO_E_INVALID_ARG : DOMINO_E_CUDA;
+        }
+        if (cudaSetDevice(h->device) != cudaSuccess) {
+            cudaGetLastError();
+            delete h;
+            return DOMINO_E_CUDA;
+        }
+        cudaDeviceGetAttribute(&h->env.num_sms, cudaDevAttrMultiProcessorCount, h->device);
+        cudaDeviceGetAttribute(&h->env.max_smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device);
+        int rc = dev_reserve(h->d_err, 16);
+        if (!rc) rc = dev_reserve(h->d_partials, sizeof(float4) * (size_t)kMaxLogitRows * kMaxChunks);
+        if (!rc) rc = dev_reserve(h->d_counters, sizeof(uint32_t) * (size_t)kMaxLogitRows);
+        if (!rc) rc = dev_reserve(h->d_lse_tmp, sizeof(float) * (size_t)kMaxLogitRows);
+        if (!rc && (cudaMemset(h->d_err.p, 0, 16) != cudaSuccess ||
+                    cudaMemset(h->d_counters.p, 0, sizeof(uint32_t) * (size_t)kMaxLogitRows) != cudaSuccess)) {
+            cudaGetLastError();
+            rc = DOMINO_E_CUDA;
+        }
+        if (rc) {
+            domino_destroy(h);
+            return rc;
+        }
+    }
+    *out = h;
+    return DOMINO_OK;
+}
+
+int domino_destroy(domino_t h) {
+    if (!h) return DOMINO_OK;
+    if (h->device >= 0) {
+        DeviceGuard g(h->device);
+        cudaDeviceSynchronize();
+        DevBuf* all[] = {&h->d_head, &h->d_orig, &h->d_len, &h->d_tail_off, &h->d_tail, &h->d_pos_of,
+                         &h->d_t16, &h->d_t32, &h->d_ret, &h->d_accept, &h->d_err, &h->d_partials,
+                         &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_states, &h->s_stacks,
+                         &h->s_mask, &h->s_tokens, &h->s_lse};
+        for (auto* b : all) dev_free(*b);
+        cudaGetLastError();
+    }
+    delete h;
+    return DOMINO_OK;
+}
+
+int domino_load_vocab(domino_t h, const uint8_t* bytes, const int64_t* offsets, int32_t n_tokens,
+                      int32_t eos_id) {
+    if (!h || !offsets || n_tokens < 1 || n_tokens > (1 << 24)) return DOMINO_E_INVALID_ARG;
+    if (eos_id < -1 || eos_id >= n_tokens || offsets[0] != 0) return DOMINO_E_INVALID_ARG;
+    int32_t max_len = 0;
+    for (int32_t t = 0; t < n_tokens; t++) {
+        int64_t L = offsets[t + 1] - offsets[t];
+        if (L < 0 || L > 65535) return DOMINO_E_INVALID_ARG;
+        if (t != eos_id) max_len = std::max<int32_t>(max_len, (int32_t)L);
+    }
+    if (offsets[n_tokens] > 0 && !bytes) return DOMINO_E_INVALID_ARG;
+    DeviceGuard g(h->device);
+    h->vocab_loaded = false;
+    h->arena_ready = false;
+    h->tok_off.assign(offsets, offsets + n_tokens + 1);
+    if (bytes && offsets[n_tokens] > 0)
+        h->tok_bytes.assign(bytes, bytes + offsets[n_tokens]);
+    else
+        h->tok_bytes.clear();
+    h->V = n_tokens;
+    h->W = (n_tokens + 31) / 32;
+    h->eos_id = eos_id;
+    h->max_len = max_len;
+    h->vocab_loaded = true;
+    if (is_host_only(h)) return DOMINO_OK;
+    return build_arena(h);
+}
+
+int domino_load_automaton(domino_t h, const int32_t* delta, int32_t n_states, const uint8_t* live,
+                          const uint8_t* accepting, int32_t start_state, const domino_stack_rule* rules,
+                          int32_t n_rules, int32_t max_depth) {
+    if (!h || !delta || !live || n_states < 1 || n_states > DOMINO_MAX_STATES) return DOMINO_E_INVALID_ARG;
+    if (start_state < 0 || start_state >= n_states || max_depth < 0 || max_depth > DOMINO_MAX_DEPTH)
+        return DOMINO_E_INVALID_ARG;
+    if (n_rules < 0 || (n_rules > 0 && !rules)) return DOMINO_E_INVALID_ARG;
+    const int64_t Q = n_states;
+    for (int64_t i = 0; i < Q * 256; i++)
+        if (delta[i] < 0 || delta[i] >= n_states) return DOMINO_E_INVALID_ARG;
+    if (live[0]) return DOMINO_E_INVALID_ARG;
+    for (int c = 0; c < 256; c++)
+        if (delta[c] != 0) return DOMINO_E_INVALID_ARG;          // state 0 absorbing
+    for (int64_t q = 0; q < Q; q++)
+        if (accepting && accepting[q] && !live[q]) return DOMINO_E_INVALID_ARG;
+    // rules: one per (state, byte); index -1 = none
+    std::vector<int32_t> rule_at((size_t)(Q * 256), -1);
+    for (int32_t r = 0; r < n_rules; r++) {
+        const domino_stack_rule& R = rules[r];
+        if (R.state <= 0 || R.state >= n_states || R.pad != 0 || R.sym > 1 ||
+            (R.kind != DOMINO_RULE_PUSH && R.kind != DOMINO_RULE_POP))
+            return DOMINO_E_INVALID_ARG;
+        if (R.kind == DOMINO_RULE_POP) {
+            for (int32_t t : {R.next_if_empty, R.next_if_top0, R.next_if_top1})
+                if (t < 0 || t >= n_states) return DOMINO_E_INVALID_ARG;
+        }
+        int32_t& slot = rule_at[(size_t)R.state * 256 + R.byte];
+        if (slot != -1) return DOMINO_E_INVALID_ARG;
+        slot = r;
+    }
+    // closure: a non-live state only reaches non-live states (makes early exit exact)
+    for (int64_t q = 0; q < Q; q++) {
+        if (live[q]) continue;
+        for (int c = 0; c < 256; c++) {
+            int32_t r = rule_at[(size_t)q * 256 + c];
+            if (r >= 0 && rules[r].kind == DOMINO_RULE_POP) {
+                if (live[rules[r].next_if_empty] || live[rules[r].next_if_top0] || live[rules[r].next_if_top1])
+                    return DOMINO_E_INVALID_ARG;
+            } else if (live[delta[q * 256 + c]]) {
+                return DOMINO_E_INVALID_ARG;
+            }
+        }
+    }
+    auto canon = [&](int32_t t) -> uint32_t { return live[t] ? (uint32_t)t : 0u; };
+    // full entry for every (q, byte): dead-canonicalised, pop targets as deduplicated triples
+    const bool stack = n_rules > 0;
+    std::vector<uint32_t> col((size_t)(256 * Q));   // column-major: [byte][q]
+    std::vector<uint16_t> ret;
+    std::unordered_map<uint64_t, uint32_t> triple_id;
+    for (int64_t q = 0; q < Q; q++) {
+        for (int c = 0; c < 256; c++) {
+            int32_t r = rule_at[(size_t)q * 256 + c];
+            uint32_t e;
+            if (r < 0) {
+                e = canon(delta[q * 256 + c]);
+            } else if (rules[r].kind == DOMINO_RULE_PUSH) {
+                e = canon(delta[q * 256 + c]) | (1u << kKindShift) | ((uint32_t)rules[r].sym << kSymShift);
+            } else {
+                uint64_t key = ((uint64_t)canon(rules[r].next_if_empty) << 32) |
+                               ((uint64_t)canon(rules[r].next_if_top0) << 16) | canon(rules[r].next_if_top1);
+                auto it = triple_id.find(key);
+                uint32_t id;
+                if (it == triple_id.end()) {
+                    id = (uint32_t)(ret.size() / 4);
+                    if (id >= kMaxRetTriples) return DOMINO_E_UNSUPPORTED;
+                    triple_id.emplace(key, id);
+                    ret.push_back((uint16_t)canon(rules[r].next_if_empty));
+                    ret.push_back((uint16_t)canon(rules[r].next_if_top0));
+                    ret.push_back((uint16_t)canon(rules[r].next_if_top1));
+                    ret.push_back(0);
+                } else {
+                    id = it->second;
+                }
+                e = (2u << kKindShift) | ((uint32_t)rules[r].sym << kSymShift) | (id << kRetShift);
+            }
+            col[(size_t)c * Q + q] = e;
+        }
+    }
+    // byte classes: bytes whose columns are identical for every state
+    uint8_t cls[256];
+    int rep[256];
+    int K = 0;
+    std::unordered_map<uint64_t, std::vector<int>> by_hash;
+    for (int c = 0; c < 256; c++) {
+        const uint32_t* cc = col.data() + (size_t)c * Q;
+        uint64_t hsh = 1469598103934665603ull;
+        for (int64_t q = 0; q < Q; q++) hsh = (hsh ^ cc[q]) * 1099511628211ull;
+        int found = -1;
+        for (int k : by_hash[hsh]) {
+            if (std::memcmp(cc, col.data() + (size_t)rep[k] * Q, sizeof(uint32_t) * (size_t)Q) == 0) {
+                found = k;
+                break;
+            }
+        }
+        if (found < 0) {
+            found = K++;
+            rep[found] = c;
+            by_hash[hsh].push_back(found);
+        }
+        cls[c] = (uint8_t)found;
+    }
+    DeviceGuard g(h->device);
+    h->auto_loaded = false;
+    h->arena_ready = false;
+    h->Q = n_states;
+    h->K = K;
+    h->start = start_state;
+    h->max_depth = max_depth;
+    h->n_rules = n_rules;
+    h->stack = stack;
+    std::memcpy(h->byte_class, cls, 256);
+    h->t16.clear();
+    h->t32.clear();
+    if (stack) {
+        h->t32.resize((size_t)(Q * K));
+        for (int64_t q = 0; q < Q; q++)
+            for (int k = 0; k < K; k++) h->t32[(size_t)(q * K + k)] = col[(size_t)rep[k] * Q + q];
+    } else {
+        h->t16.resize((size_t)(Q * K));
+        for (int64_t q = 0; q < Q; q++)
+            for (int k = 0; k < K; k++) h->t16[(size_t)(q * K + k)] = (uint16_t)col[(size_t)rep[k] * Q + q];
+    }
+    h->ret = ret;
+    h->accept_bits.assign((size_t)((Q + 31) / 32), 0u);
+    if (accepting)
+        for (int64_t q = 0; q < Q; q++)
+            if (accepting[q]) h->accept_bits[(size_t)(q / 32)] |= 1u << (q % 32);
+    h->auto_loaded = true;
+    if (is_host_only(h)) return DOMINO_OK;
+    int rc;
+    if (stack) {
+        if ((rc = dev_upload(h->d_t32, h->t32.data(), h->t32.size() * 4))) return rc;
+    } else {
+        if ((rc = dev_upload(h->d_t16, h->t16.data(), h->t16.size() * 2))) return rc;
+    }
+    if ((rc = dev_upload(h->d_ret, h->ret.data(), h->ret.size() * 2))) return rc;
+    if ((rc = dev_upload(h->d_accept, h->accept_bits.data(), h->accept_bits.size() * 4))) return rc;
+    return build_arena(h);
+}
+
+int domino_get_info(domino_t h, domino_info* out) {
+    if (!h || !out) return DOMINO_E_INVALID_ARG;
+    std::memset(out, 0, sizeof(*out));
+    out->n_tokens = h->V;
+    out->n_words = h->W;
+    out->eos_id = h->eos_id;
+    out->max_token_len = h->max_len;
+    out->n_states = h->Q;
+    out->n_classes = h->K;
+    out->start_state = h->start;
+    out->max_depth = h->max_depth;
+    out->n_rules = h->n_rules;
+    out->has_stack = h->stack ? 1 : 0;
+    out->device = h->device;
+    if (h->auto_loaded && h->device >= 0) {
+        StepView v = make_view(h);
+        out->table_in_smem = table_fits_smem(h, v, false) ? 1 : 0;
+    }
+    out->device_bytes = dev_bytes(h);
+    return DOMINO_OK;
+}
+
+int domino_get_byte_classes(domino_t h, uint8_t* classes_out) {
+    if (!h || !classes_out) return DOMINO_E_INVALID_ARG;
+    if (!h->auto_loaded) return DOMINO_E_NOT_LOADED;
+    std::memcpy(classes_out, h->byte_class, 256);
+    return DOMINO_OK;
+}
+
+int domino_step_mask(domino_t h, const int32_t* states_dev, const uint64_t* stacks_dev, int32_t batch,
+                     uint32_t* mask_dev, int32_t* next_dev, void* stream) {
+    int rc = ready_for_compute(h);
+    if (rc) return rc;
+    if (batch < 0 || (batch > 0 && (!states_dev || !mask_dev))) return DOMINO_E_INVALID_ARG;
+    if (batch == 0) return DOMINO_OK;
+    DeviceGuard g(h->device);
+    StepView v = make_view(h);
+    bool smem = table_fits_smem(h, v, next_dev != nullptr);
+    return cuda_status(launch_step_mask(v, h->env, h->stack, smem, states_dev, stacks_dev, batch, false, mask_dev,
+                                        next_dev, (cudaStream_t)stream));
+}
+
+int domino_precompute_table(domino_t h, int32_t* next_dev, uint32_t* mask_dev, void* stream) {
+    int rc = ready_for_compute(h);
+    if (rc) return rc;
+    if (!next_dev && !mask_dev) return DOMINO_E_INVALID_ARG;
+    if (h->stack) return DOMINO_E_UNSUPPORTED;
+    DeviceGuard g(h->device);
+    StepView v = make_view(h);
+    bool smem = table_fits_smem(h, v, next_dev != nullptr);
+    return cuda_status(launch_step_mask(v, h->env, false, smem, nullptr, nullptr, h->Q, true, mask_dev, next_dev,
+                                        (cudaStream_t)stream));
+}
+
+int domino_mask_logits(domino_t h, const void* logits_dev, int32_t dtype, int32_t batch,
+                       int64_t row_stride_elems, const uint32_t* mask_dev, int32_t* argmax_dev, float* lse_dev,
+                       float* logprobs_dev, void* stream) {
+    if (!h) return DOMINO_E_INVALID_ARG;
+    if (is_host_only(h)) return DOMINO_E_NO_DEVICE;
+    if (!h->vocab_loaded) return DOMINO_E_NOT_LOADED;
+    if (dtype != DOMINO_DTYPE_F32 && dtype != DOMINO_DTYPE_BF16) return DOMINO_E_INVALID_ARG;
+    if (batch < 0 || row_stride_elems < h->V) return DOMINO_E_INVALID_ARG;
+    if (batch == 0) return DOMINO_OK;
+    if (!logits_dev || !mask_dev || !argmax_dev) return DOMINO_E_INVALID_ARG;
+    DeviceGuard g(h->device);
+    return cuda_status(launch_mask_logits(h->env, logits_dev, dtype, batch, row_stride_elems, h->V, mask_dev,
+                                          argmax_dev, lse_dev, logprobs_dev, (float4*)h->d_partials.p,
+                                          (uint32_t*)h->d_counters.p, (float*)h->d_lse_tmp.p,
+                                          (cudaStream_t)stream));
+}
+
+int domino_advance(domino_t h, const int32_t* states_dev, const uint64_t* stacks_dev, const int32_t* tokens_dev,
+                   int32_t batch, int32_t* states_out, uint64_t* stacks_out, void* stream) {
+    int rc = ready_for_compute(h);
+    if (rc) return rc;
+    if (batch < 0) return DOMINO_E_INVALID_ARG;
+    if (batch == 0) return DOMINO_OK;
+    if (!states_dev || !tokens_dev || !states_out || (stacks_dev && !stacks_out)) return DOMINO_E_INVALID_ARG;
+    DeviceGuard g(h->device);
+    StepView v = make_view(h);
+    return cuda_status(launch_advance(v, h->stack, states_dev, stacks_dev, tokens_dev, batch, states_out,
+                                      stacks_out, (cudaStream_t)stream));
+}
+
+int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, int32_t batch,
+                            int32_t* states_host, uint64_t* stacks_host, int32_t* tokens_host, float* lse_host,
+                            void* stream) {
+    int rc = ready_for_compute(h);
+    if (rc) return rc;
+    if (dtype != DOMINO_DTYPE_F32 && dtype != DOMINO_DTYPE_BF16) return DOMINO_E_INVALID_ARG;
+    if (batch < 0) return DOMINO_E_INVALID_ARG;
+    if (batch == 0) return DOMINO_OK;
+    if (!logits_host || !states_host || !tokens_host) return DOMINO_E_INVALID_ARG;
+    DeviceGuard g(h->device);
+    cudaStream_t st = (cudaStream_t)stream;
+    const size_t esz = dtype == DOMINO_DTYPE_BF16 ? 2 : 4;
+    const size_t logit_bytes = (size_t)batch * (size_t)h->V * esz;
+    if (h->s_logits.n < logit_bytes || h->s_states.n < (size_t)batch * 4) {
+        if (cudaStreamSynchronize(st) != cudaSuccess) return cuda_status(cudaGetLastError());
+    }
+    if ((rc = dev_reserve(h->s_logits, logit_bytes))) return rc;
+    if ((rc = dev_reserve(h->s_states, (size_t)batch * 4))) return rc;
+    if ((rc = dev_reserve(h->s_stacks, (size_t)batch * 8))) return rc;
+    if ((rc = dev_reserve(h->s_mask, (size_t)batch * (size_t)h->W * 4))) return rc;
+    if ((rc = dev_reserve(h->s_tokens, (size_t)batch * 4))) return rc;
+    if ((rc = dev_reserve(h->s_lse, (size_t)batch * 4))) return rc;
+    int32_t* d_states = (int32_t*)h->s_states.p;
+    uint64_t* d_stacks = stacks_host ? (uint64_t*)h->s_stacks.p : nullptr;
+    cudaError_t e = cudaMemcpyAsync(h->s_logits.p, logits_host, logit_bytes, cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(d_states, states_host, (size_t)batch * 4, cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess && d_stacks)
+        e = cudaMemcpyAsync(d_stacks, stacks_host, (size_t)batch * 8, cudaMemcpyHostToDevice, st);
+    if (e != cudaSuccess) return cuda_status(e);
+    if ((rc = domino_step_mask(h, d_states, d_stacks, batch, (uint32_t*)h->s_mask.p, nullptr, stream))) return rc;
+    if ((rc = domino_mask_logits(h, h->s_logits.p, dtype, batch, h->V, (uint32_t*)h->s_mask.p,
+                                 (int32_t*)h->s_tokens.p, (float*)h->s_lse.p, nullptr, stream)))
+        return rc;
+    if ((rc = domino_advance(h, d_states, d_stacks, (int32_t*)h->s_tokens.p, batch, d_states, d_stacks, stream)))
+        return rc;
+    e = cudaMemcpyAsync(tokens_host, h->s_tokens.p, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess && lse_host)
+        e = cudaMemcpyAsync(lse_host, h->s_lse.p, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(states_host, d_states, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess && d_stacks)
+        e = cudaMemcpyAsync(stacks_host, d_stacks, (size_t)batch * 8, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    return cuda_status(e);
+}
+
+int domino_get_device_error(domino_t h, int32_t* code, void* stream) {
+    if (!h || !code) return DOMINO_E_INVALID_ARG;
+    *code = 0;
+    if (is_host_only(h)) return DOMINO_E_NO_DEVICE;
+    DeviceGuard g(h->device);
+    cudaStream_t st = (cudaStream_t)stream;
+    uint32_t word = 0;
+    cudaError_t e = cudaMemcpyAsync(&word, h->d_err.p, 4, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(h->d_err.p, 0, 4, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_status(e);
+    *code = (int32_t)word;
+    return DOMINO_OK;
+}
+
+}  // extern "C"
