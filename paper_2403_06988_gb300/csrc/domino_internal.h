@@ -11,18 +11,27 @@
 namespace domino {
 
 // Vocabulary windows: original ids [w*kWin, (w+1)*kWin) form window w.  Inside
-// a window the tokens are stored sorted by their byte-class strings, so that a
-// warp walks tokens with common prefixes (same first transitions, same early
-// exit) and the mask bits are scattered back to original ids in shared memory.
+// a window the tokens are stored sorted by their byte-class strings, so tokens
+// with the same first class form one contiguous group and neighbouring tokens
+// share prefixes (same transitions, same early exit for a warp).  The allowed
+// bits are scattered back to original ids in shared memory.
 constexpr int kWin = 1024;
-constexpr int kStepThreads = 256;              // step kernel CTA size
-constexpr int kSlotsPerThread = kWin / kStepThreads;
-constexpr int kRowGroup = 8;                   // rows walked between two write-outs
-constexpr int kHeadBytes = 16;                 // class ids stored inline per token
+constexpr int kStepThreads = 1024;             // step kernel CTA size (one CTA per SM)
+constexpr int kRowsPerTile = 16;               // fewest rows per tile (mask only)
+constexpr int kMaxRowsPerTile = 32;            // most rows per tile (one warp ballot)
+constexpr int kRowsPerTileNext = 8;            // rows per tile when next states are written
+constexpr int kUnitSlots = 32;                 // slots per work unit (one per lane)
+constexpr int kWalkChains = 4;                 // rows walked together by one lane (independent chains)
+constexpr int kHeadBytes = 16;                 // class ids per 16-byte head block
+constexpr int kInlineBytes = 32;               // class ids stored inline per token (two head blocks)
 constexpr int kLogitThreads = 256;
 constexpr int kMaxLogitRows = 4096;            // rows per mask_logits pass (scratch size)
-constexpr int kMaxChunks = 64;                 // CTAs per row in mask_logits
+constexpr int kMaxSegments = 64;               // CTAs sharing one row in mask_logits
 constexpr int kAdvanceThreads = 128;
+
+// slot info word: bits 0..9 original id within the window, bit 10 valid,
+// bits 16..31 byte length (0 for EOS and empty tokens)
+constexpr uint32_t kInfoValid = 1u << 10;
 
 // Table entry of a pushdown automaton (uint32): bits 0..15 next state, bits
 // 16..17 kind (0 none, 1 push, 2 pop), bit 18 symbol, bits 19..31 index of the
@@ -30,22 +39,36 @@ constexpr int kAdvanceThreads = 128;
 constexpr uint32_t kKindShift = 16, kSymShift = 18, kRetShift = 19;
 constexpr uint32_t kMaxRetTriples = 1u << 13;
 
+// Where the step kernel reads transitions from.
+enum TableMode : int {
+    kDenseSmem = 0,    // [Q][K] entries staged in shared memory
+    kSparse32Smem = 1, // per state {live-class mask, base} + packed live entries (K <= 32)
+    kSparse64Smem = 2, // the same with a 64-bit class mask (K <= 64)
+    kDenseGlobal = 3,  // [Q][K] entries read through L1/L2
+};
+
 struct StepView {
     // vocabulary arena (slot order)
-    const uint4* head;        // [n_slots] first 16 class ids
-    const int32_t* orig;      // [n_slots] original id, -1 for padding slots
-    const uint16_t* len;      // [n_slots] byte length (0 for EOS)
-    const int32_t* tail_off;  // [n_slots] offset of bytes 16.. in `tail`
-    const uint8_t* tail;      // class ids of bytes 16.. of long tokens
+    const uint4* head;        // [n_slots][2] class ids of bytes 0..15 and 16..31
+    const uint32_t* info;     // [n_slots] original id in window | valid | length
+    const int32_t* tail_off;  // [n_slots] offset of bytes 32.. in `tail`
+    const uint8_t* tail;      // class ids of bytes 32.. of tokens longer than 32 bytes
     const int32_t* pos_of;    // [V] slot of original id
+    // work units: a unit is <= 32 consecutive slots of one first-class group,
+    // packed as class (bits 0..7) | first slot (bits 8..18) | count-1 (bits 19..23)
+    const uint32_t* units;    // all windows' units, window w at [unit_off[w], unit_off[w+1])
+    const int32_t* unit_off;  // [n_windows + 1]
+    const int16_t* eos_slot;  // [n_windows] window-local slot of EOS, -1 if not in the window
+    int32_t max_units;        // max units of one window
     int32_t V, W, n_windows, eos_id;
     // automaton
     const uint16_t* t16;      // [Q][K] (DFA)
     const uint32_t* t32;      // [Q][K] (pushdown)
+    const uint32_t* sp_info;  // sparse rows: [Q][2] or [Q][4] uint32 words
+    const void* sp_tgt;       // sparse live entries (uint16 or uint32)
     const uint16_t* ret;      // [n_ret][4]
     const uint32_t* accept_bits;
-    int32_t Q, K, start, max_depth, n_ret;
-    int32_t table_bytes;      // bytes of t16/t32 (+ ret) as staged in shared memory
+    int32_t Q, K, start, max_depth, n_ret, sp_nnz;
     uint32_t* err;            // sticky device error word
 };
 
@@ -54,19 +77,23 @@ struct LaunchEnv {
     int max_smem_optin;
 };
 
-cudaError_t launch_step_mask(const StepView& v, const LaunchEnv& env, bool stack, bool smem_table,
-                             const int32_t* states, const uint64_t* stacks, int32_t batch, bool row_is_state,
-                             uint32_t* mask, int32_t* next, cudaStream_t st);
+// Bytes the table of `mode` occupies in shared memory (0 for kDenseGlobal).
+int64_t table_smem_bytes(const StepView& v, bool stack, int mode);
 
-// Shared-memory bytes the step kernel needs for its tiles (without the table).
-int step_tile_smem_bytes(bool next);
+// Shared-memory bytes of the step kernel other than the table.
+int step_fixed_smem_bytes(const StepView& v, bool next);
+
+cudaError_t launch_step_mask(const StepView& v, const LaunchEnv& env, bool stack, int mode, const int32_t* states,
+                             const uint64_t* stacks, int32_t batch, bool row_is_state, uint32_t* mask,
+                             int32_t* next, cudaStream_t st);
 
 cudaError_t launch_mask_logits(const LaunchEnv& env, const void* logits, int dtype, int32_t batch,
                                int64_t row_stride, int32_t V, const uint32_t* mask, int32_t* argmax, float* lse,
                                float* logprobs, float4* partials, uint32_t* counters, float* lse_tmp,
                                cudaStream_t st);
 
-cudaError_t launch_advance(const StepView& v, bool stack, const int32_t* states, const uint64_t* stacks,
+// `mode` names the table image the step kernel reads (it is L2-resident after a step).
+cudaError_t launch_advance(const StepView& v, bool stack, int mode, const int32_t* states, const uint64_t* stacks,
                            const int32_t* tokens, int32_t batch, int32_t* states_out, uint64_t* stacks_out,
                            cudaStream_t st);
 

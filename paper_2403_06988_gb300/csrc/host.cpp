@@ -44,10 +44,14 @@ struct domino_ctx {
     std::vector<uint32_t> t32;
     std::vector<uint16_t> ret;
     std::vector<uint32_t> accept_bits;
+    int32_t sp_nnz = 0;       // live entries of the sparse table (0: no sparse image)
+    int32_t sp_words = 0;     // uint32 words per state in the sparse row info (2 or 4)
+    int64_t dense_ret_off = 0, sp_tgt_off = 0, sp_ret_off = 0;
 
     // ---- device copies
-    DevBuf d_head, d_orig, d_len, d_tail_off, d_tail, d_pos_of;
-    DevBuf d_t16, d_t32, d_ret, d_accept;
+    DevBuf d_head, d_info, d_tail_off, d_tail, d_pos_of, d_units, d_unit_off, d_eos_slot;
+    int32_t max_units = 0;
+    DevBuf d_dense, d_sparse, d_accept;
     DevBuf d_err, d_partials, d_counters, d_lse_tmp;
     bool arena_ready = false;
     int32_t n_windows = 0;
@@ -78,8 +82,8 @@ void dev_free(DevBuf& b) {
 }
 
 int64_t dev_bytes(const domino_ctx* h) {
-    const DevBuf* all[] = {&h->d_head, &h->d_orig, &h->d_len, &h->d_tail_off, &h->d_tail, &h->d_pos_of,
-                           &h->d_t16, &h->d_t32, &h->d_ret, &h->d_accept, &h->d_err, &h->d_partials,
+    const DevBuf* all[] = {&h->d_head, &h->d_info, &h->d_tail_off, &h->d_tail, &h->d_pos_of, &h->d_units,
+                           &h->d_unit_off, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_err, &h->d_partials,
                            &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_states, &h->s_stacks,
                            &h->s_mask, &h->s_tokens, &h->s_lse};
     int64_t n = 0;
@@ -122,16 +126,30 @@ int build_arena(domino_ctx* h) {
     auto tlen = [&](int32_t t) -> int32_t {
         return t == h->eos_id ? 0 : (int32_t)(h->tok_off[t + 1] - h->tok_off[t]);
     };
+    // window order: empty tokens first, then by first class; inside a first-class
+    // group longer tokens first (a warp's lanes then walk similar lengths), then
+    // by class string (shared prefixes take the same transitions)
     auto less = [&](int32_t a, int32_t b) {
         int32_t la = tlen(a), lb = tlen(b);
-        int c = std::memcmp(cls.data() + h->tok_off[a], cls.data() + h->tok_off[b], (size_t)std::min(la, lb));
+        if ((la == 0) != (lb == 0)) return la == 0;
+        if (la == 0) return a < b;
+        const uint8_t* ca = cls.data() + h->tok_off[a];
+        const uint8_t* cb = cls.data() + h->tok_off[b];
+        if (ca[0] != cb[0]) return ca[0] < cb[0];
+        if (la != lb) return la > lb;
+        int c = std::memcmp(ca, cb, (size_t)la);
         if (c != 0) return c < 0;
-        if (la != lb) return la < lb;
         return a < b;
     };
-    std::vector<uint8_t> head((size_t)n_slots * kHeadBytes, 0);
-    std::vector<int32_t> orig((size_t)n_slots, -1), tail_off((size_t)n_slots, 0), pos_of((size_t)V, 0);
-    std::vector<uint16_t> len((size_t)n_slots, 0);
+    const int K = h->K;
+    std::vector<uint8_t> head((size_t)n_slots * kInlineBytes, 0);
+    std::vector<uint32_t> info((size_t)n_slots, 0);
+    std::vector<int32_t> tail_off((size_t)n_slots, 0), pos_of((size_t)V, 0);
+    std::vector<uint16_t> gstart((size_t)(K + 1), 0);
+    std::vector<uint32_t> units;
+    std::vector<int32_t> unit_off((size_t)nw + 1, 0);
+    int32_t max_units = 0;
+    std::vector<int16_t> eos_slot((size_t)nw, -1);
     std::vector<uint8_t> tail;
     std::vector<int32_t> ids;
     for (int32_t w = 0; w < nw; w++) {
@@ -139,29 +157,46 @@ int build_arena(domino_ctx* h) {
         ids.resize((size_t)(hi - lo));
         std::iota(ids.begin(), ids.end(), lo);
         std::sort(ids.begin(), ids.end(), less);
+        uint16_t* gs = gstart.data();
+        int c_next = 0;   // first class whose group start is still unset
         for (int32_t j = 0; j < hi - lo; j++) {
             int32_t t = ids[(size_t)j];
             int64_t p = (int64_t)lo + j;
             int32_t L = tlen(t);
-            orig[(size_t)p] = t;
-            len[(size_t)p] = (uint16_t)L;
+            info[(size_t)p] = (uint32_t)(t - lo) | kInfoValid | ((uint32_t)L << 16);
             pos_of[(size_t)t] = (int32_t)p;
+            if (t == h->eos_id) eos_slot[(size_t)w] = (int16_t)j;
             const uint8_t* c = cls.data() + h->tok_off[t];
-            std::memcpy(head.data() + p * kHeadBytes, c, (size_t)std::min(L, kHeadBytes));
-            if (L > kHeadBytes) {
+            if (L > 0) {
+                while (c_next <= c[0]) gs[c_next++] = (uint16_t)j;   // groups by first class
+            }
+            std::memcpy(head.data() + p * kInlineBytes, c, (size_t)std::min(L, kInlineBytes));
+            if (L > kInlineBytes) {
                 tail_off[(size_t)p] = (int32_t)tail.size();
-                tail.insert(tail.end(), c + kHeadBytes, c + L);
+                tail.insert(tail.end(), c + kInlineBytes, c + L);
             }
         }
+        while (c_next <= K) gs[c_next++] = (uint16_t)(hi - lo);
+        // work units: <= kUnitSlots consecutive slots of one first-class group
+        for (int c = 0; c < K; c++)
+            for (int b = gs[c]; b < gs[c + 1]; b += kUnitSlots) {
+                const int n = std::min(kUnitSlots, gs[c + 1] - b);
+                units.push_back((uint32_t)c | ((uint32_t)b << 8) | ((uint32_t)(n - 1) << 19));
+            }
+        unit_off[(size_t)w + 1] = (int32_t)units.size();
+        max_units = std::max(max_units, unit_off[(size_t)w + 1] - unit_off[(size_t)w]);
     }
     if (tail.size() > (size_t)INT32_MAX) return DOMINO_E_UNSUPPORTED;
     int rc;
     if ((rc = dev_upload(h->d_head, head.data(), head.size()))) return rc;
-    if ((rc = dev_upload(h->d_orig, orig.data(), orig.size() * 4))) return rc;
-    if ((rc = dev_upload(h->d_len, len.data(), len.size() * 2))) return rc;
+    if ((rc = dev_upload(h->d_info, info.data(), info.size() * 4))) return rc;
     if ((rc = dev_upload(h->d_tail_off, tail_off.data(), tail_off.size() * 4))) return rc;
     if ((rc = dev_upload(h->d_tail, tail.data(), tail.size()))) return rc;
     if ((rc = dev_upload(h->d_pos_of, pos_of.data(), pos_of.size() * 4))) return rc;
+    if ((rc = dev_upload(h->d_units, units.data(), units.size() * 4))) return rc;
+    if ((rc = dev_upload(h->d_unit_off, unit_off.data(), unit_off.size() * 4))) return rc;
+    h->max_units = max_units;
+    if ((rc = dev_upload(h->d_eos_slot, eos_slot.data(), eos_slot.size() * 2))) return rc;
     h->n_windows = nw;
     h->arena_ready = true;
     return DOMINO_OK;
@@ -170,35 +205,46 @@ int build_arena(domino_ctx* h) {
 StepView make_view(domino_ctx* h) {
     StepView v{};
     v.head = (const uint4*)h->d_head.p;
-    v.orig = (const int32_t*)h->d_orig.p;
-    v.len = (const uint16_t*)h->d_len.p;
+    v.info = (const uint32_t*)h->d_info.p;
     v.tail_off = (const int32_t*)h->d_tail_off.p;
     v.tail = (const uint8_t*)h->d_tail.p;
     v.pos_of = (const int32_t*)h->d_pos_of.p;
+    v.units = (const uint32_t*)h->d_units.p;
+    v.unit_off = (const int32_t*)h->d_unit_off.p;
+    v.max_units = h->max_units;
+    v.eos_slot = (const int16_t*)h->d_eos_slot.p;
     v.V = h->V;
     v.W = h->W;
     v.n_windows = h->n_windows;
     v.eos_id = h->eos_id;
-    v.t16 = (const uint16_t*)h->d_t16.p;
-    v.t32 = (const uint32_t*)h->d_t32.p;
-    v.ret = (const uint16_t*)h->d_ret.p;
+    const char* dense = (const char*)h->d_dense.p;
+    v.t16 = h->stack ? nullptr : (const uint16_t*)dense;
+    v.t32 = h->stack ? (const uint32_t*)dense : nullptr;
+    v.ret = dense ? (const uint16_t*)(dense + h->dense_ret_off) : nullptr;
+    v.sp_info = (const uint32_t*)h->d_sparse.p;
+    v.sp_tgt = h->d_sparse.p ? (const void*)((const char*)h->d_sparse.p + h->sp_tgt_off) : nullptr;
     v.accept_bits = (const uint32_t*)h->d_accept.p;
     v.Q = h->Q;
     v.K = h->K;
     v.start = h->start;
     v.max_depth = h->max_depth;
     v.n_ret = (int32_t)(h->ret.size() / 4);
-    size_t tb = h->stack ? h->t32.size() * 4 : h->t16.size() * 2;
-    tb = (tb + 15) / 16 * 16;
-    tb += (h->ret.size() * 2 + 15) / 16 * 16;
-    v.table_bytes = (int32_t)tb;
+    v.sp_nnz = h->sp_nnz;
     v.err = (uint32_t*)h->d_err.p;
     return v;
 }
 
-bool table_fits_smem(const domino_ctx* h, const StepView& v, bool next) {
-    if (h->env.max_smem_optin <= 0) return false;
-    return (int64_t)v.table_bytes + step_tile_smem_bytes(next) + 1024 <= (int64_t)h->env.max_smem_optin;
+// Table placement for the step kernel: dense in shared memory if it fits, else
+// the sparse live-class form, else dense through L1/L2.
+int choose_mode(const domino_ctx* h, const StepView& v, bool next) {
+    if (h->env.max_smem_optin <= 0) return kDenseGlobal;
+    const int64_t avail = (int64_t)h->env.max_smem_optin - step_fixed_smem_bytes(v, next) - 1024;
+    if (table_smem_bytes(v, h->stack, kDenseSmem) <= avail) return kDenseSmem;
+    if (h->sp_nnz > 0) {
+        const int mode = h->sp_words == 2 ? kSparse32Smem : kSparse64Smem;
+        if (table_smem_bytes(v, h->stack, mode) <= avail) return mode;
+    }
+    return kDenseGlobal;
 }
 
 int ready_for_compute(domino_ctx* h) {
@@ -252,7 +298,7 @@ int domino_create(domino_t* out, int32_t cuda_device) {
         cudaDeviceGetAttribute(&h->env.num_sms, cudaDevAttrMultiProcessorCount, h->device);
         cudaDeviceGetAttribute(&h->env.max_smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device);
         int rc = dev_reserve(h->d_err, 16);
-        if (!rc) rc = dev_reserve(h->d_partials, sizeof(float4) * (size_t)kMaxLogitRows * kMaxChunks);
+        if (!rc) rc = dev_reserve(h->d_partials, sizeof(float4) * (size_t)kMaxLogitRows * kMaxSegments);
         if (!rc) rc = dev_reserve(h->d_counters, sizeof(uint32_t) * (size_t)kMaxLogitRows);
         if (!rc) rc = dev_reserve(h->d_lse_tmp, sizeof(float) * (size_t)kMaxLogitRows);
         if (!rc && (cudaMemset(h->d_err.p, 0, 16) != cudaSuccess ||
@@ -274,8 +320,8 @@ int domino_destroy(domino_t h) {
     if (h->device >= 0) {
         DeviceGuard g(h->device);
         cudaDeviceSynchronize();
-        DevBuf* all[] = {&h->d_head, &h->d_orig, &h->d_len, &h->d_tail_off, &h->d_tail, &h->d_pos_of,
-                         &h->d_t16, &h->d_t32, &h->d_ret, &h->d_accept, &h->d_err, &h->d_partials,
+        DevBuf* all[] = {&h->d_head, &h->d_info, &h->d_tail_off, &h->d_tail, &h->d_pos_of, &h->d_units,
+                         &h->d_unit_off, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_err, &h->d_partials,
                          &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_states, &h->s_stacks,
                          &h->s_mask, &h->s_tokens, &h->s_lse};
         for (auto* b : all) dev_free(*b);
@@ -441,14 +487,68 @@ int domino_load_automaton(domino_t h, const int32_t* delta, int32_t n_states, co
         for (int64_t q = 0; q < Q; q++)
             if (accepting[q]) h->accept_bits[(size_t)(q / 32)] |= 1u << (q % 32);
     h->auto_loaded = true;
+    // dense image: [Q][K] entries | pop targets, each part 16-byte aligned
+    const size_t esz = stack ? 4 : 2;
+    auto a16 = [](size_t x) { return (x + 15) / 16 * 16; };
+    const size_t tab_bytes = (size_t)(Q * K) * esz;
+    h->dense_ret_off = (int64_t)a16(tab_bytes);
+    std::vector<uint8_t> dense_img(a16(tab_bytes) + a16(h->ret.size() * 2), 0);
+    std::memcpy(dense_img.data(), stack ? (const void*)h->t32.data() : (const void*)h->t16.data(), tab_bytes);
+    if (!h->ret.empty()) std::memcpy(dense_img.data() + h->dense_ret_off, h->ret.data(), h->ret.size() * 2);
+    // sparse image (K <= 64): per state {live-class mask, base} | live entries | pop targets
+    h->sp_nnz = 0;
+    h->sp_words = 0;
+    std::vector<uint8_t> sparse_img;
+    if (K <= 64) {
+        const int words = K <= 32 ? 2 : 4;
+        std::vector<uint32_t> rinfo((size_t)(Q * words), 0);
+        std::vector<uint32_t> tgt;
+        for (int64_t q = 0; q < Q; q++) {
+            uint64_t m = 0;
+            uint32_t base = (uint32_t)tgt.size();
+            for (int k = 0; k < K; k++) {
+                uint32_t e = stack ? h->t32[(size_t)(q * K + k)] : h->t16[(size_t)(q * K + k)];
+                if (e) {
+                    m |= 1ull << k;
+                    tgt.push_back(e);
+                }
+            }
+            if (words == 2) {
+                rinfo[(size_t)(q * 2)] = (uint32_t)m;
+                rinfo[(size_t)(q * 2 + 1)] = base;
+            } else {
+                rinfo[(size_t)(q * 4)] = (uint32_t)m;
+                rinfo[(size_t)(q * 4 + 1)] = (uint32_t)(m >> 32);
+                rinfo[(size_t)(q * 4 + 2)] = base;
+            }
+        }
+        if (!tgt.empty() && tgt.size() < (size_t)INT32_MAX) {
+            h->sp_nnz = (int32_t)tgt.size();
+            h->sp_words = words;
+            h->sp_tgt_off = (int64_t)a16(rinfo.size() * 4);
+            h->sp_ret_off = h->sp_tgt_off + (int64_t)a16(tgt.size() * esz);
+            sparse_img.assign((size_t)h->sp_ret_off + a16(h->ret.size() * 2), 0);
+            std::memcpy(sparse_img.data(), rinfo.data(), rinfo.size() * 4);
+            uint8_t* tp = sparse_img.data() + h->sp_tgt_off;
+            for (size_t i = 0; i < tgt.size(); i++) {
+                if (stack) {
+                    std::memcpy(tp + i * 4, &tgt[i], 4);
+                } else {
+                    uint16_t e16 = (uint16_t)tgt[i];
+                    std::memcpy(tp + i * 2, &e16, 2);
+                }
+            }
+            if (!h->ret.empty()) std::memcpy(sparse_img.data() + h->sp_ret_off, h->ret.data(), h->ret.size() * 2);
+        }
+    }
     if (is_host_only(h)) return DOMINO_OK;
     int rc;
-    if (stack) {
-        if ((rc = dev_upload(h->d_t32, h->t32.data(), h->t32.size() * 4))) return rc;
+    if ((rc = dev_upload(h->d_dense, dense_img.data(), dense_img.size()))) return rc;
+    if (!sparse_img.empty()) {
+        if ((rc = dev_upload(h->d_sparse, sparse_img.data(), sparse_img.size()))) return rc;
     } else {
-        if ((rc = dev_upload(h->d_t16, h->t16.data(), h->t16.size() * 2))) return rc;
+        dev_free(h->d_sparse);
     }
-    if ((rc = dev_upload(h->d_ret, h->ret.data(), h->ret.size() * 2))) return rc;
     if ((rc = dev_upload(h->d_accept, h->accept_bits.data(), h->accept_bits.size() * 4))) return rc;
     return build_arena(h);
 }
@@ -469,7 +569,7 @@ int domino_get_info(domino_t h, domino_info* out) {
     out->device = h->device;
     if (h->auto_loaded && h->device >= 0) {
         StepView v = make_view(h);
-        out->table_in_smem = table_fits_smem(h, v, false) ? 1 : 0;
+        out->table_in_smem = choose_mode(h, v, false) != kDenseGlobal ? 1 : 0;
     }
     out->device_bytes = dev_bytes(h);
     return DOMINO_OK;
@@ -490,8 +590,8 @@ int domino_step_mask(domino_t h, const int32_t* states_dev, const uint64_t* stac
     if (batch == 0) return DOMINO_OK;
     DeviceGuard g(h->device);
     StepView v = make_view(h);
-    bool smem = table_fits_smem(h, v, next_dev != nullptr);
-    return cuda_status(launch_step_mask(v, h->env, h->stack, smem, states_dev, stacks_dev, batch, false, mask_dev,
+    const int mode = choose_mode(h, v, next_dev != nullptr);
+    return cuda_status(launch_step_mask(v, h->env, h->stack, mode, states_dev, stacks_dev, batch, false, mask_dev,
                                         next_dev, (cudaStream_t)stream));
 }
 
@@ -502,8 +602,8 @@ int domino_precompute_table(domino_t h, int32_t* next_dev, uint32_t* mask_dev, v
     if (h->stack) return DOMINO_E_UNSUPPORTED;
     DeviceGuard g(h->device);
     StepView v = make_view(h);
-    bool smem = table_fits_smem(h, v, next_dev != nullptr);
-    return cuda_status(launch_step_mask(v, h->env, false, smem, nullptr, nullptr, h->Q, true, mask_dev, next_dev,
+    const int mode = choose_mode(h, v, next_dev != nullptr);
+    return cuda_status(launch_step_mask(v, h->env, false, mode, nullptr, nullptr, h->Q, true, mask_dev, next_dev,
                                         (cudaStream_t)stream));
 }
 
@@ -533,7 +633,8 @@ int domino_advance(domino_t h, const int32_t* states_dev, const uint64_t* stacks
     if (!states_dev || !tokens_dev || !states_out || (stacks_dev && !stacks_out)) return DOMINO_E_INVALID_ARG;
     DeviceGuard g(h->device);
     StepView v = make_view(h);
-    return cuda_status(launch_advance(v, h->stack, states_dev, stacks_dev, tokens_dev, batch, states_out,
+    const int mode = choose_mode(h, v, false);
+    return cuda_status(launch_advance(v, h->stack, mode, states_dev, stacks_dev, tokens_dev, batch, states_out,
                                       stacks_out, (cudaStream_t)stream));
 }
 

@@ -1,25 +1,35 @@
 // kernels.cu -- sm_103a kernels of the per-decode-step hot path.
 //
-//  step_kernel      C.mask() at k = infinity (Alg. 1; Sec. 3.5): every
-//                   (sequence, token) pair walks the token's byte classes
+//  step_kernel      C.mask() at lookahead k = infinity (Alg. 1; Sec. 3.5):
+//                   every (sequence, token) pair walks the token's byte classes
 //                   through the scanner table (and the bracket stack,
-//                   Sec. 3.4) with early exit on the dead state.  One CTA owns
-//                   one 1024-token vocabulary window (tokens kept in registers)
-//                   and a range of rows; the allowed bits are scattered from
-//                   prefix-sorted slot order to original ids in a
+//                   Sec. 3.4) with early exit on the dead state.  Persistent
+//                   CTAs (one per SM) hold the transition table in shared
+//                   memory (dense, or sparse per-state live-class masks) and
+//                   loop over tiles = (vocabulary window of 1024 tokens,
+//                   group of rows).  Inside a window tokens are sorted by
+//                   their class strings, so all tokens with the same first
+//                   class form one group: per row, the first transition is
+//                   taken once per class and only the groups whose first step
+//                   is live are walked (work proportional to the surviving
+//                   tokens).  Allowed bits are scattered to original ids in a
 //                   shared-memory tile and written out coalesced.  The same
 //                   kernel with row = state builds the state x token table
 //                   (Alg. 2's traversal, precomputed offline, Sec. 3.5).
-//  logits kernels   Alg. 1's v' = m (.) v and greedy decode: one streaming
-//                   pass (16-byte loads, masked vectors skipped) computes the
-//                   masked max / lowest-index argmax / sum of exp per chunk;
-//                   the last CTA of a row combines the chunks (atomic ticket,
-//                   no spinning).  Log-probs need a second pass over the row.
+//  logits kernels   Alg. 1's v' = m (.) v and greedy decode: a balanced flat
+//                   split of the batch x vocabulary logits over one wave of
+//                   CTAs; 16-byte loads (vectors with no allowed token are not
+//                   loaded), branch-free masked max / lowest-index argmax /
+//                   sum of exp per vector; per-row segments are combined by
+//                   the last CTA to finish (atomic ticket, no spinning).
+//                   Log-probs need a second pass over the row.
 //  advance_kernel   C.update(o): the chosen token's walk.
 #include <cuda_runtime.h>
 
 #include <climits>
 #include <cstdint>
+#include <algorithm>
+#include <type_traits>
 
 #include "domino_internal.h"
 
@@ -28,45 +38,70 @@ namespace domino {
 namespace {
 
 constexpr int kMaxDevices = 64;
-constexpr int kMaskTileBytes = 2 * kRowGroup * 32 * 4;
-constexpr int kNextTileBytes = 2 * kRowGroup * kWin * 4;
+static_assert(kStepThreads == kWin, "one thread per window slot");
+constexpr float kLog2e = 1.4426950408889634f;   // log2(e): exp(x) = 2^(x log2 e)
+
+__host__ __device__ constexpr int align16(int x) { return (x + 15) & ~15; }
+
+// Shared-memory layout of the step kernel (offsets in bytes).
+struct StepLayout {
+    int head, info, units, items, rows, ctrl, rowmask, cfg, mtile, ntile, accept, table, total;
+};
+
+__host__ __device__ inline StepLayout step_layout(int K, int R, bool next, bool stack, int max_units, int Q,
+                                                  int table_bytes) {
+    StepLayout L{};
+    int o = 0;
+    L.head = o;    o += kWin * 32;
+    L.info = o;    o += kWin * 4;
+    L.units = o;   o += align16(max_units * 4);
+    L.items = o;   o += align16(max_units * ((R + kWalkChains - 1) / kWalkChains) * 4);
+    L.rows = o;    o += R * 16;
+    L.ctrl = o;    o += 16;
+    L.rowmask = o; o += align16(K * 4);
+    L.cfg = o;     o += align16(R * K * (stack ? 16 : 4));
+    L.mtile = o;   o += align16(R * 32 * 4);
+    L.ntile = o;   o += next ? R * kWin * 4 : 0;
+    L.accept = o;  o += align16(((Q + 31) / 32) * 4);
+    L.table = o;   o += align16(table_bytes);
+    L.total = o;
+    return L;
+}
 
 __device__ __forceinline__ uint32_t head_byte(const uint4& h, int i) {
     uint32_t w = (i < 4) ? h.x : (i < 8) ? h.y : (i < 12) ? h.z : h.w;
     return (w >> (8 * (i & 3))) & 0xFFu;
 }
 
-template <bool SMEM, typename T>
-__device__ __forceinline__ T tload(const T* p, uint32_t i) {
-    if constexpr (SMEM) {
-        return p[i];
-    } else {
-        return __ldg(p + i);
+// Transition lookup for the four table modes.
+template <typename E, int MODE>
+struct Tab {
+    const E* dense;
+    const uint32_t* sp;
+    const E* tgt;
+    uint32_t K;
+    __device__ __forceinline__ uint32_t get(uint32_t s, uint32_t c) const {
+        if constexpr (MODE == kDenseSmem) {
+            return dense[s * K + c];
+        } else if constexpr (MODE == kDenseGlobal) {
+            return __ldg(dense + s * K + c);
+        } else if constexpr (MODE == kSparse32Smem) {
+            const uint2 ri = reinterpret_cast<const uint2*>(sp)[s];
+            if (!((ri.x >> c) & 1u)) return 0u;
+            return tgt[ri.y + __popc(ri.x & ((1u << c) - 1u))];
+        } else {
+            const uint4 ri = reinterpret_cast<const uint4*>(sp)[s];
+            const unsigned long long m = ((unsigned long long)ri.y << 32) | ri.x;
+            if (!((m >> c) & 1ull)) return 0u;
+            return tgt[ri.z + __popcll(m & ((1ull << c) - 1ull))];
+        }
     }
-}
-
-// DFA walk from s over the token's class string; 0 when the walk dies.
-template <bool SMEM>
-__device__ __forceinline__ uint32_t walk_dfa(const uint16_t* __restrict__ t, uint32_t K, uint32_t s, const uint4 h,
-                                             int len, const uint8_t* __restrict__ tail) {
-#pragma unroll
-    for (int i = 0; i < kHeadBytes; ++i) {
-        if (i >= len) return s;
-        s = tload<SMEM>(t, s * K + head_byte(h, i));
-        if (s == 0) return 0;
-    }
-    for (int i = kHeadBytes; i < len; ++i) {
-        s = tload<SMEM>(t, s * K + __ldg(tail + (i - kHeadBytes)));
-        if (s == 0) return 0;
-    }
-    return s;
-}
+};
 
 // One pushdown step for table entry e (bits 0..15 next, 16..17 kind, 18 sym,
 // 19..31 pop-target triple).  Returns the next state, 0 when rejected.
-template <bool SMEM>
-__device__ __forceinline__ uint32_t pda_step(uint32_t e, uint32_t& bits, uint32_t& depth, uint32_t max_depth,
-                                             const uint16_t* __restrict__ ret) {
+__device__ __forceinline__ uint32_t pda_apply(uint32_t e, uint32_t& bits, uint32_t& depth, uint32_t max_depth,
+                                              const uint16_t* ret) {
     const uint32_t kind = (e >> kKindShift) & 3u;
     if (kind == 0) return e & 0xFFFFu;
     const uint32_t sym = (e >> kSymShift) & 1u;
@@ -80,172 +115,333 @@ __device__ __forceinline__ uint32_t pda_step(uint32_t e, uint32_t& bits, uint32_
     bits >>= 1;
     --depth;
     const uint32_t revealed = depth == 0 ? 0u : 1u + (bits & 1u);
-    return tload<SMEM>(ret, (e >> kRetShift) * 4u + revealed);
+    return ret[(e >> kRetShift) * 4u + revealed];
 }
 
-template <bool SMEM>
-__device__ __forceinline__ uint32_t walk_pda(const uint32_t* __restrict__ t, const uint16_t* __restrict__ ret,
-                                             uint32_t K, uint32_t s, uint32_t& bits, uint32_t& depth,
-                                             uint32_t max_depth, const uint4 h, int len,
-                                             const uint8_t* __restrict__ tail) {
-#pragma unroll
-    for (int i = 0; i < kHeadBytes; ++i) {
-        if (i >= len) return s;
-        s = pda_step<SMEM>(tload<SMEM>(t, s * K + head_byte(h, i)), bits, depth, max_depth, ret);
+// One transition step (with the bracket rules for a pushdown table).
+template <bool STACK, typename T>
+__device__ __forceinline__ uint32_t step_once(const T& tab, const uint16_t* ret, uint32_t max_depth, uint32_t s,
+                                              uint32_t c, uint32_t& bits, uint32_t& depth) {
+    const uint32_t e = tab.get(s, c);
+    if constexpr (STACK) {
+        return pda_apply(e, bits, depth, max_depth, ret);
+    } else {
+        return e;
+    }
+}
+
+// Walk bytes FROM..len-1 of a token from state s; 0 when the walk dies.  The
+// first 32 class ids are at `head` (shared or global memory), bytes 32.. are in
+// `tail` (global memory, touched only by tokens that long).
+template <bool STACK, int FROM, typename T>
+__device__ __forceinline__ uint32_t walk(const T& tab, const uint16_t* ret, uint32_t max_depth, uint32_t s,
+                                         uint32_t& bits, uint32_t& depth, const uint8_t* head, int len,
+                                         const uint8_t* __restrict__ tail) {
+    const int n1 = min(len, kInlineBytes);
+#pragma unroll 1
+    for (int i = FROM; i < n1; ++i) {
+        s = step_once<STACK>(tab, ret, max_depth, s, head[i], bits, depth);
         if (s == 0) return 0;
     }
-    for (int i = kHeadBytes; i < len; ++i) {
-        s = pda_step<SMEM>(tload<SMEM>(t, s * K + __ldg(tail + (i - kHeadBytes))), bits, depth, max_depth, ret);
+#pragma unroll 1
+    for (int i = kInlineBytes; i < len; ++i) {
+        s = step_once<STACK>(tab, ret, max_depth, s, __ldg(tail + (i - kInlineBytes)), bits, depth);
         if (s == 0) return 0;
     }
     return s;
 }
 
-// Row configuration; invalid rows become the dead state and report once.
-struct RowCfg {
-    uint32_t s, bits, depth;
-    bool valid;
-};
-
-__device__ __forceinline__ RowCfg read_row(const StepView& v, const int32_t* __restrict__ states,
-                                           const uint64_t* __restrict__ stacks, int b, bool report) {
-    RowCfg c{0u, 0u, 0u, true};
-    const int32_t sv = __ldg(states + b);
-    uint32_t eb = 0;
-    if (sv < 0 || sv >= v.Q) {
-        c.valid = false;
-        eb |= DOMINO_DEVERR_BAD_STATE;
+template <bool STACK, int NW, typename T>
+__device__ __forceinline__ uint32_t chains_step(const T& tab, const uint16_t* ret, uint32_t max_depth,
+                                                uint32_t (&s)[NW], uint32_t (&bits)[NW], uint32_t (&depth)[NW],
+                                                uint32_t c) {
+    uint32_t alive = 0;
+#pragma unroll
+    for (int k = 0; k < NW; ++k) {
+        s[k] = step_once<STACK>(tab, ret, max_depth, s[k], c, bits[k], depth[k]);
+        alive |= s[k];
     }
-    if (stacks) {
-        const uint64_t w = __ldg(reinterpret_cast<const unsigned long long*>(stacks) + b);
-        const uint32_t depth = (uint32_t)(w >> 32) & 0xFFu;
-        const uint32_t bits = (uint32_t)w;
-        const bool ok = (w >> 40) == 0 && depth <= (uint32_t)v.max_depth && (depth >= 32u || (bits >> depth) == 0);
-        if (!ok) {
-            c.valid = false;
-            eb |= DOMINO_DEVERR_BAD_STACK;
-        }
-        c.bits = bits;
-        c.depth = depth;
-    }
-    if (c.valid) {
-        c.s = (uint32_t)sv;
-    } else {
-        c.bits = c.depth = 0;
-        if (report) atomicOr(v.err, eb);
-    }
-    return c;
+    return alive;
 }
 
-template <bool STACK, bool SMEM, bool NEXT>
-__global__ void __launch_bounds__(kStepThreads)
-    step_kernel(const StepView v, const int32_t* __restrict__ states, const uint64_t* __restrict__ stacks,
-                int32_t batch, int32_t rows_per_cta, int32_t row_is_state, uint32_t* __restrict__ mask,
-                int32_t* __restrict__ next) {
-    extern __shared__ __align__(16) unsigned char smem[];
-    uint32_t* mtile = reinterpret_cast<uint32_t*>(smem);
-    int32_t* ntile = reinterpret_cast<int32_t*>(smem + kMaskTileBytes);
-    unsigned char* tsm = smem + kMaskTileBytes + (NEXT ? kNextTileBytes : 0);
-
-    const int tid = threadIdx.x;
-    const int w = blockIdx.x;
-    const int row0 = blockIdx.y * rows_per_cta;
-    const int row1 = min(batch, row0 + rows_per_cta);
-    if (row0 >= row1) return;   // uniform over the CTA, before any barrier
-
-    const uint32_t K = (uint32_t)v.K;
-    const uint16_t* t16 = v.t16;
-    const uint32_t* t32 = v.t32;
-    const uint16_t* ret = v.ret;
-    if constexpr (SMEM) {
-        // stage the transition table (and pop targets) in shared memory; the
-        // device copies are padded to 16 bytes
-        const size_t esz = STACK ? 4 : 2;
-        const int n_tab = (int)(((size_t)v.Q * K * esz + 15) / 16);
-        const int n_ret = (int)(((size_t)v.n_ret * 8 + 15) / 16);
-        const uint4* src = STACK ? reinterpret_cast<const uint4*>(v.t32) : reinterpret_cast<const uint4*>(v.t16);
-        uint4* dst = reinterpret_cast<uint4*>(tsm);
-        for (int i = tid; i < n_tab; i += kStepThreads) dst[i] = __ldg(src + i);
-        const uint4* rsrc = reinterpret_cast<const uint4*>(v.ret);
-        for (int i = tid; i < n_ret; i += kStepThreads) dst[n_tab + i] = __ldg(rsrc + i);
-        t16 = reinterpret_cast<const uint16_t*>(tsm);
-        t32 = reinterpret_cast<const uint32_t*>(tsm);
-        ret = reinterpret_cast<const uint16_t*>(tsm + (size_t)n_tab * 16);
-    }
-    for (int i = tid; i < 2 * kRowGroup * 32; i += kStepThreads) mtile[i] = 0u;
-
-    // this thread's tokens (registers for the whole row range)
-    uint4 hd[kSlotsPerThread];
-    int ln[kSlotsPerThread], ol[kSlotsPerThread];
-    bool eos[kSlotsPerThread];
-    const uint8_t* tp[kSlotsPerThread];
-#pragma unroll
-    for (int j = 0; j < kSlotsPerThread; ++j) {
-        const int p = w * kWin + tid + j * kStepThreads;
-        const int o = __ldg(v.orig + p);
-        ol[j] = o >= 0 ? o - w * kWin : -1;
-        eos[j] = o >= 0 && o == v.eos_id;
-        ln[j] = __ldg(v.len + p);
-        hd[j] = __ldg(v.head + p);
-        tp[j] = ln[j] > kHeadBytes ? v.tail + __ldg(v.tail_off + p) : v.tail;
-    }
-    __syncthreads();
-
-    int buf = 0;
-    for (int g = row0; g < row1; g += kRowGroup, buf ^= 1) {
-        const int nr = min(kRowGroup, row1 - g);
-        uint32_t* mt = mtile + buf * kRowGroup * 32;
-        int32_t* nt = ntile + buf * kRowGroup * kWin;
+// NW independent walks of one token (bytes 1..len-1) from NW configurations;
+// a chain that dies stays 0 (row 0 of every table image is all zero).  `head`
+// is the token's first 32 class ids in shared memory.
+template <bool STACK, int NW, typename T>
+__device__ __forceinline__ void walk_chains(const T& tab, const uint16_t* ret, uint32_t max_depth,
+                                            uint32_t (&s)[NW], uint32_t (&bits)[NW], uint32_t (&depth)[NW],
+                                            const uint8_t* head, int len, const uint8_t* __restrict__ tail) {
+    const int n1 = min(len, kInlineBytes);
 #pragma unroll 1
-        for (int r = 0; r < nr; ++r) {
-            const int b = g + r;
-            RowCfg rc;
-            if (row_is_state) {
-                rc = RowCfg{(uint32_t)b, 0u, 0u, true};
-            } else {
-                rc = read_row(v, states, stacks, b, w == 0 && tid == 0);
+    for (int i = 1; i < n1; ++i)
+        if (!chains_step<STACK, NW>(tab, ret, max_depth, s, bits, depth, head[i])) return;
+#pragma unroll 1
+    for (int i = kInlineBytes; i < len; ++i)
+        if (!chains_step<STACK, NW>(tab, ret, max_depth, s, bits, depth, __ldg(tail + (i - kInlineBytes)))) return;
+}
+
+// Row configuration: x state, y stack bits, z depth, w flags (1 valid, 2 EOS allowed).
+// `sv` / `w` are the raw state and stack word of the row; accept bits may be
+// in shared or global memory.
+__device__ __forceinline__ uint4 decode_row(const StepView& v, int32_t sv, unsigned long long w, bool has_stack,
+                                            const uint32_t* accept_bits, bool report) {
+    uint32_t s = 0, bits = 0, depth = 0;
+    bool valid = true;
+    uint32_t eb = 0;
+    if (sv < 0 || sv >= v.Q) {
+        valid = false;
+        eb |= DOMINO_DEVERR_BAD_STATE;
+    }
+    if (has_stack) {
+        depth = (uint32_t)(w >> 32) & 0xFFu;
+        bits = (uint32_t)w;
+        const bool ok = (w >> 40) == 0 && depth <= (uint32_t)v.max_depth && (depth >= 32u || (bits >> depth) == 0);
+        if (!ok) {
+            valid = false;
+            eb |= DOMINO_DEVERR_BAD_STACK;
+        }
+    }
+    if (valid) {
+        s = (uint32_t)sv;
+    } else {
+        bits = depth = 0;
+        if (report) atomicOr(v.err, eb);
+    }
+    const bool eos_ok = valid && depth == 0 && ((accept_bits[s >> 5] >> (s & 31u)) & 1u);
+    return make_uint4(s, bits, depth, (valid ? 1u : 0u) | (eos_ok ? 2u : 0u));
+}
+
+__device__ __forceinline__ uint4 read_row(const StepView& v, const int32_t* __restrict__ states,
+                                          const uint64_t* __restrict__ stacks, int b, bool report) {
+    const int32_t sv = __ldg(states + b);
+    const unsigned long long w = stacks ? __ldg(reinterpret_cast<const unsigned long long*>(stacks) + b) : 0ull;
+    return decode_row(v, sv, w, stacks != nullptr, v.accept_bits, report);
+}
+
+template <bool STACK, int MODE, bool NEXT>
+__global__ void __launch_bounds__(kStepThreads, 1)
+    step_kernel(const StepView v, const uint4* __restrict__ img, int img_bytes, int img_tgt_off, int img_ret_off,
+                const int32_t* __restrict__ states, const uint64_t* __restrict__ stacks, int32_t batch,
+                int32_t R, int32_t n_row_tiles, int32_t n_tiles, int32_t row_is_state, uint32_t* __restrict__ mask,
+                int32_t* __restrict__ next) {
+    using E = typename std::conditional<STACK, uint32_t, uint16_t>::type;
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int K = v.K;
+    const StepLayout L = step_layout(K, R, NEXT, STACK, v.max_units, v.Q, MODE == kDenseGlobal ? 0 : img_bytes);
+    uint4* s_head = reinterpret_cast<uint4*>(smem + L.head);
+    uint32_t* s_info = reinterpret_cast<uint32_t*>(smem + L.info);
+    uint32_t* s_units = reinterpret_cast<uint32_t*>(smem + L.units);
+    uint32_t* s_items = reinterpret_cast<uint32_t*>(smem + L.items);   // unit | chain group << 16
+    uint4* s_rows = reinterpret_cast<uint4*>(smem + L.rows);
+    int* s_ctrl = reinterpret_cast<int*>(smem + L.ctrl);   // unit cursor, -, EOS slot, unit count
+    uint32_t* s_rowmask = reinterpret_cast<uint32_t*>(smem + L.rowmask);
+    uint32_t* s_cfg = reinterpret_cast<uint32_t*>(smem + L.cfg);   // [R][K] state (DFA)
+    uint4* s_cfg4 = reinterpret_cast<uint4*>(smem + L.cfg);        // [R][K] (state, bits, depth) (pushdown)
+    uint32_t* s_mtile = reinterpret_cast<uint32_t*>(smem + L.mtile);
+    int32_t* s_ntile = reinterpret_cast<int32_t*>(smem + L.ntile);
+    uint32_t* s_accept = reinterpret_cast<uint32_t*>(smem + L.accept);
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    for (int i = tid; i < (v.Q + 31) / 32; i += kStepThreads) s_accept[i] = __ldg(v.accept_bits + i);
+
+    Tab<E, MODE> tab;
+    tab.K = (uint32_t)K;
+    const uint16_t* ret;
+    if constexpr (MODE == kDenseGlobal) {
+        tab.dense = reinterpret_cast<const E*>(STACK ? (const void*)v.t32 : (const void*)v.t16);
+        ret = v.ret;
+    } else {
+        // stage the table image (dense or sparse, plus pop targets) once per CTA
+        uint4* dst = reinterpret_cast<uint4*>(smem + L.table);
+        for (int i = tid; i < img_bytes / 16; i += kStepThreads) dst[i] = __ldg(img + i);
+        const unsigned char* tb = smem + L.table;
+        tab.dense = reinterpret_cast<const E*>(tb);
+        tab.sp = reinterpret_cast<const uint32_t*>(tb);
+        tab.tgt = reinterpret_cast<const E*>(tb + img_tgt_off);
+        ret = reinterpret_cast<const uint16_t*>(tb + img_ret_off);
+    }
+    const uint32_t maxd = (uint32_t)v.max_depth;
+
+    const int t0 = (int)(((long long)blockIdx.x * n_tiles) / gridDim.x);
+    const int t1 = (int)(((long long)(blockIdx.x + 1) * n_tiles) / gridDim.x);
+    // the raw configuration of row r0+tid of the coming tile (threads < R),
+    // loaded one tile ahead so that its latency overlaps the walk
+    int32_t pf_s = 0;
+    unsigned long long pf_w = 0ull;
+    auto prefetch = [&](int t) {
+        if (t < t1 && tid < R && !row_is_state) {
+            const int wq = t / n_row_tiles;
+            const int b = (t - wq * n_row_tiles) * R + tid;
+            if (b < batch) {
+                pf_s = __ldg(states + b);
+                if (stacks) pf_w = __ldg(reinterpret_cast<const unsigned long long*>(stacks) + b);
             }
-            const bool eos_ok =
-                rc.valid && rc.depth == 0 && ((__ldg(v.accept_bits + (rc.s >> 5)) >> (rc.s & 31u)) & 1u);
-#pragma unroll
-            for (int j = 0; j < kSlotsPerThread; ++j) {
-                if (ol[j] < 0) continue;
-                uint32_t s;
-                if (ln[j] == 0) {
-                    s = (eos[j] && eos_ok) ? rc.s : 0u;
-                } else if constexpr (STACK) {
-                    uint32_t bits = rc.bits, depth = rc.depth;
-                    s = walk_pda<SMEM>(t32, ret, K, rc.s, bits, depth, (uint32_t)v.max_depth, hd[j], ln[j], tp[j]);
-                } else {
-                    s = walk_dfa<SMEM>(t16, K, rc.s, hd[j], ln[j], tp[j]);
+        }
+    };
+    prefetch(t0);
+    int cur_w = -1;
+    for (int t = t0; t < t1; ++t) {
+        const int w = t / n_row_tiles;
+        const int r0 = (t - w * n_row_tiles) * R;
+        const int nr = min(R, batch - r0);
+        __syncthreads();   // the previous tile is fully consumed
+        if (w != cur_w) {
+            s_head[2 * tid] = __ldg(v.head + 2 * ((size_t)w * kWin + tid));
+            s_head[2 * tid + 1] = __ldg(v.head + 2 * ((size_t)w * kWin + tid) + 1);
+            s_info[tid] = __ldg(v.info + (size_t)w * kWin + tid);
+            const int u0 = __ldg(v.unit_off + w), nu = __ldg(v.unit_off + w + 1) - u0;
+            for (int i = tid; i < nu; i += kStepThreads) s_units[i] = __ldg(v.units + u0 + i);
+            if (tid == 0) {
+                s_ctrl[2] = __ldg(v.eos_slot + w);
+                s_ctrl[3] = nu;
+            }
+            cur_w = w;
+        }
+        if (tid < nr) {
+            if (row_is_state) {
+                const uint32_t q = (uint32_t)(r0 + tid);
+                s_rows[tid] = make_uint4(q, 0u, 0u, 1u | (((s_accept[q >> 5] >> (q & 31u)) & 1u) ? 2u : 0u));
+            } else {
+                s_rows[tid] = decode_row(v, pf_s, pf_w, stacks != nullptr, s_accept, w == 0);
+            }
+        }
+        for (int i = tid; i < nr * 32; i += kStepThreads) s_mtile[i] = 0u;
+        if constexpr (NEXT) {
+            for (int i = tid; i < nr * (kWin / 4); i += kStepThreads)
+                reinterpret_cast<int4*>(s_ntile)[i] = make_int4(0, 0, 0, 0);
+        }
+        __syncthreads();
+
+        // first transition once per (row, first class): lane r of a warp takes
+        // row r, the ballot gives the class's live rows
+        for (int c = warp; c < K; c += kStepThreads / 32) {
+            uint32_t s = 0, bits = 0, depth = 0;
+            if (lane < nr) {
+                const uint4 row = s_rows[lane];
+                bits = row.y;
+                depth = row.z;
+                if (row.w & 1u) {
+                    const uint32_t e = tab.get(row.x, (uint32_t)c);
+                    if constexpr (STACK) {
+                        s = pda_apply(e, bits, depth, maxd, ret);
+                    } else {
+                        s = e;
+                    }
                 }
-                if (s) atomicOr(&mt[r * 32 + (ol[j] >> 5)], 1u << (ol[j] & 31));
-                if constexpr (NEXT) nt[r * kWin + ol[j]] = (int32_t)s;
+                if constexpr (STACK) {
+                    s_cfg4[lane * K + c] = make_uint4(s, bits, depth, 0u);
+                } else {
+                    s_cfg[lane * K + c] = s;
+                }
+            }
+            const uint32_t live = __ballot_sync(0xffffffffu, s != 0);
+            if (lane == 0) s_rowmask[c] = live;
+        }
+        const int eos_local = s_ctrl[2];
+        if (tid < nr && eos_local >= 0 && (s_rows[tid].w & 2u)) {
+            const int ol = (int)(s_info[eos_local] & 1023u);
+            atomicOr(&s_mtile[tid * 32 + (ol >> 5)], 1u << (ol & 31));
+            if constexpr (NEXT) s_ntile[tid * kWin + ol] = (int32_t)s_rows[tid].x;
+        }
+        __syncthreads();
+
+        prefetch(t + 1);
+        // work items: (unit, group of up to kWalkChains live rows), listed by
+        // warp 0 and dealt round-robin to the warps (items cost about the same)
+        const int nu = s_ctrl[3];
+        if (warp == 0) {
+            int base = 0;
+            for (int u0 = 0; u0 < nu; u0 += 32) {
+                const int u = u0 + lane;
+                int ng = 0;
+                if (u < nu) {
+                    const uint32_t rm = s_rowmask[s_units[u] & 0xFFu];
+                    const uint32_t unit = s_units[u];
+                    // a unit whose tokens all have one byte needs no walk beyond the first step
+                    ng = (__popc(rm) + kWalkChains - 1) / kWalkChains;
+                    (void)unit;
+                }
+                int incl = ng;
+#pragma unroll
+                for (int off = 1; off < 32; off <<= 1) {
+                    const int y = __shfl_up_sync(0xffffffffu, incl, off);
+                    if (lane >= off) incl += y;
+                }
+                for (int g = 0; g < ng; ++g) s_items[base + incl - ng + g] = (uint32_t)u | ((uint32_t)g << 16);
+                base += __shfl_sync(0xffffffffu, incl, 31);
+            }
+            if (lane == 0) s_ctrl[1] = base;
+        }
+        __syncthreads();
+        const int n_items = s_ctrl[1];
+        for (int it = warp; it < n_items; it += kStepThreads / 32) {
+            const uint32_t item = s_items[it];
+            const uint32_t unit = s_units[item & 0xFFFFu];
+            const int grp = (int)(item >> 16);
+            const int c = (int)(unit & 0xFFu);
+            uint32_t rm = s_rowmask[c];
+            for (int g = 0; g < grp * kWalkChains; ++g) rm &= rm - 1;   // skip earlier groups' rows
+            const int slot = (int)((unit >> 8) & 0x7FFu) + lane;
+            const bool active = lane <= (int)((unit >> 19) & 31u);
+            const uint32_t info = active ? s_info[slot] : 0u;
+            const uint8_t* hp = reinterpret_cast<const uint8_t*>(s_head + 2 * slot);
+            const int len = (int)(info >> 16);
+            const int ol = (int)(info & 1023u);
+            const uint8_t* tl = len > kInlineBytes ? v.tail + __ldg(v.tail_off + (size_t)w * kWin + slot) : v.tail;
+            {
+                int rr[kWalkChains];
+                uint32_t sv[kWalkChains], bv[kWalkChains], dv[kWalkChains];
+#pragma unroll
+                for (int k = 0; k < kWalkChains; ++k) {
+                    rr[k] = -1;
+                    sv[k] = bv[k] = dv[k] = 0u;
+                    if (rm) {
+                        rr[k] = __ffs(rm) - 1;
+                        rm &= rm - 1;
+                        if constexpr (STACK) {
+                            const uint4 cf = s_cfg4[rr[k] * K + c];
+                            sv[k] = cf.x;
+                            bv[k] = cf.y;
+                            dv[k] = cf.z;
+                        } else {
+                            sv[k] = s_cfg[rr[k] * K + c];
+                        }
+                    }
+                }
+                if (active) {
+                    walk_chains<STACK, kWalkChains>(tab, ret, maxd, sv, bv, dv, hp, len, tl);
+#pragma unroll
+                    for (int k = 0; k < kWalkChains; ++k) {
+                        if (rr[k] >= 0 && sv[k]) {
+                            atomicOr(&s_mtile[rr[k] * 32 + (ol >> 5)], 1u << (ol & 31));
+                            if constexpr (NEXT) s_ntile[rr[k] * kWin + ol] = (int32_t)sv[k];
+                        }
+                    }
+                }
             }
         }
         __syncthreads();
-        // write-out of this buffer (the other buffer is used by the next group;
-        // the barrier after that group orders this clear before its reuse)
-        for (int i = tid; i < nr * 32; i += kStepThreads) {
-            const int r = i >> 5, word = w * 32 + (i & 31);
-            if (mask && word < v.W) mask[(size_t)(g + r) * v.W + word] = mt[i];
-            mt[i] = 0u;
+
+        // coalesced write-out in original-id order
+        if (mask) {
+            for (int i = tid; i < nr * 32; i += kStepThreads) {
+                const int r = i >> 5, word = w * 32 + (i & 31);
+                if (word < v.W) mask[(size_t)(r0 + r) * v.W + word] = s_mtile[i];
+            }
         }
         if constexpr (NEXT) {
+            const int in_win = min(kWin, v.V - w * kWin);
             if (v.V % 4 == 0) {
-                const int per_row = min(kWin, v.V - w * kWin) / 4;
+                const int per_row = in_win / 4;
                 for (int i = tid; i < nr * (kWin / 4); i += kStepThreads) {
                     const int r = i / (kWin / 4), k4 = i % (kWin / 4);
-                    if (k4 < per_row) {
-                        const int4 val = reinterpret_cast<const int4*>(nt + r * kWin)[k4];
-                        __stcs(reinterpret_cast<int4*>(next + (size_t)(g + r) * v.V + (size_t)w * kWin) + k4, val);
-                    }
+                    if (k4 < per_row)
+                        __stcs(reinterpret_cast<int4*>(next + (size_t)(r0 + r) * v.V + (size_t)w * kWin) + k4,
+                               reinterpret_cast<const int4*>(s_ntile + r * kWin)[k4]);
                 }
             } else {
                 for (int i = tid; i < nr * kWin; i += kStepThreads) {
                     const int r = i / kWin, k = i % kWin;
-                    const int t = w * kWin + k;
-                    if (t < v.V) next[(size_t)(g + r) * v.V + t] = nt[i];
+                    if (k < in_win) next[(size_t)(r0 + r) * v.V + (size_t)w * kWin + k] = s_ntile[i];
                 }
             }
         }
@@ -255,18 +451,14 @@ __global__ void __launch_bounds__(kStepThreads)
 // ---------------------------------------------------------------------------
 // masked argmax / log-sum-exp
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ void acc_add(float& m, int& idx, float& s, float x, int t) {
-    if (x > m) {
-        s = s * __expf(m - x) + 1.0f;
-        m = x;
-        idx = t;
-    } else {
-        s += __expf(x - m);
-    }
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
 }
 
-// (m, idx, s) <- (m, idx, s) (+) (m2, i2, s2); the larger max wins, the lower
-// index on equal maxima; the loser's sum is rescaled to the winner's max.
+// (m, idx, s) <- (m, idx, s) (+) (m2, i2, s2): larger max wins, lower index on
+// equal maxima; the other sum is rescaled to the winner's max.
 __device__ __forceinline__ void acc_merge(float& m, int& idx, float& s, float m2, int i2, float s2) {
     if (m2 > m || (m2 == m && i2 < idx)) {
         const float tm = m, ts = s;
@@ -278,7 +470,20 @@ __device__ __forceinline__ void acc_merge(float& m, int& idx, float& s, float m2
         i2 = ti;
         s2 = ts;
     }
-    if (s2 != 0.0f) s += s2 * __expf(m2 - m);
+    if (s2 != 0.0f) s += s2 * ex2((m2 - m) * kLog2e);
+}
+
+// one allowed logit x at index t; mL = m * log2(e) is kept with m
+__device__ __forceinline__ void acc_add(float& m, float& mL, int& idx, float& s, float x, int t) {
+    if (x > m) {
+        const float xL = x * kLog2e;
+        s = s * ex2(mL - xL) + 1.0f;
+        m = x;
+        mL = xL;
+        idx = t;
+    } else {
+        s += ex2(fmaf(x, kLog2e, -mL));
+    }
 }
 
 __device__ __forceinline__ void warp_merge(float& m, int& idx, float& s) {
@@ -288,6 +493,27 @@ __device__ __forceinline__ void warp_merge(float& m, int& idx, float& s) {
         const int i2 = __shfl_xor_sync(0xffffffffu, idx, off);
         const float s2 = __shfl_xor_sync(0xffffffffu, s, off);
         acc_merge(m, idx, s, m2, i2, s2);
+    }
+}
+
+// CTA-wide (m, idx, s); the result is valid in thread 0.  Uses two barriers.
+__device__ __forceinline__ void block_merge(float& m, int& idx, float& s) {
+    __shared__ float sm_m[kLogitThreads / 32], sm_s[kLogitThreads / 32];
+    __shared__ int sm_i[kLogitThreads / 32];
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    warp_merge(m, idx, s);
+    __syncthreads();   // protect sm_* against the previous call's readers
+    if (lane == 0) {
+        sm_m[wid] = m;
+        sm_i[wid] = idx;
+        sm_s[wid] = s;
+    }
+    __syncthreads();
+    if (wid == 0) {
+        m = lane < kLogitThreads / 32 ? sm_m[lane] : -INFINITY;
+        idx = lane < kLogitThreads / 32 ? sm_i[lane] : INT_MAX;
+        s = lane < kLogitThreads / 32 ? sm_s[lane] : 0.0f;
+        warp_merge(m, idx, s);
     }
 }
 
@@ -303,16 +529,6 @@ __device__ __forceinline__ uint4 ld_vec(const uint4* p) {
     }
 }
 
-__device__ __forceinline__ uint32_t mask_bits8(const uint32_t* __restrict__ mrow, int v8) {
-    return (__ldg(mrow + (v8 >> 2)) >> ((v8 & 3) * 8)) & 0xFFu;
-}
-__device__ __forceinline__ uint32_t mask_bits4(const uint32_t* __restrict__ mrow, int v4) {
-    return (__ldg(mrow + (v4 >> 3)) >> ((v4 & 7) * 4)) & 0xFu;
-}
-__device__ __forceinline__ bool mask_bit(const uint32_t* __restrict__ mrow, int t) {
-    return (__ldg(mrow + (t >> 5)) >> (t & 31)) & 1u;
-}
-
 template <bool BF16>
 __device__ __forceinline__ float logit_at(const void* row, int t) {
     if constexpr (BF16) {
@@ -323,155 +539,157 @@ __device__ __forceinline__ float logit_at(const void* row, int t) {
     }
 }
 
-constexpr int kUnroll = 4;
-
-template <bool BF16, bool VEC, bool KEEP_L2>
-__global__ void __launch_bounds__(kLogitThreads)
-    logits_reduce_kernel(const void* __restrict__ logits, int64_t stride, const uint32_t* __restrict__ mask, int V,
-                         int W, int chunk, int S, float4* __restrict__ partials, uint32_t* __restrict__ counters,
-                         int32_t* __restrict__ argmax, float* __restrict__ lse) {
-    const int row = blockIdx.y, c = blockIdx.x, tid = threadIdx.x;
-    const int lo = c * chunk, hi = min(V, lo + chunk);
-    const uint32_t* mrow = mask + (size_t)row * W;
-    const char* lrow = reinterpret_cast<const char*>(logits) + (size_t)row * stride * (BF16 ? 2 : 4);
-    float m = -INFINITY, s = 0.0f;
-    int idx = INT_MAX;
-    int tail_lo = lo;
-    if constexpr (VEC) {
-        constexpr int E = BF16 ? 8 : 4;   // elements per 16-byte vector
-        const int v_lo = lo / E, v_hi = hi / E;
-        tail_lo = v_hi * E;
-        const uint4* vrow = reinterpret_cast<const uint4*>(lrow);
-        for (int v0 = v_lo + tid; v0 < v_hi; v0 += kUnroll * kLogitThreads) {
-            uint32_t mb[kUnroll];
-            uint4 raw[kUnroll];
+// Logits of the allowed tokens of mask word j of a row, handed to f(x, t) in
+// increasing t.  STAGE (bf16 rows on 16-byte boundaries): the word's 64 bytes
+// of logits are read as four 16-byte vectors (a vector with no allowed token is
+// not read) into this thread's shared-memory slot; otherwise, and for a partial
+// last word, each allowed logit is read on its own.
+template <bool BF16, bool STAGE, bool KEEP_L2, typename F>
+__device__ __forceinline__ void for_allowed(const char* lrow, uint32_t word, int j, int V, uint4* slot, F&& f) {
+    const int t0 = j * 32;
+    if (STAGE && t0 + 32 <= V) {
+        const uint4* src = reinterpret_cast<const uint4*>(lrow) + (size_t)j * 4;
+        uint4 d[4];
 #pragma unroll
-            for (int u = 0; u < kUnroll; ++u) {
-                const int vv = v0 + u * kLogitThreads;
-                mb[u] = vv < v_hi ? (BF16 ? mask_bits8(mrow, vv) : mask_bits4(mrow, vv)) : 0u;
-                raw[u] = mb[u] ? ld_vec<KEEP_L2>(vrow + vv) : make_uint4(0, 0, 0, 0);
-            }
+        for (int k = 0; k < 4; ++k)
+            if ((word >> (8 * k)) & 0xFFu) d[k] = ld_vec<KEEP_L2>(src + k);
 #pragma unroll
-            for (int u = 0; u < kUnroll; ++u) {
-                if (!mb[u]) continue;
-                const int t0 = (v0 + u * kLogitThreads) * E;
-                const uint32_t wd[4] = {raw[u].x, raw[u].y, raw[u].z, raw[u].w};
-#pragma unroll
-                for (int e = 0; e < E; ++e) {
-                    if ((mb[u] >> e) & 1u) {
-                        float x;
-                        if constexpr (BF16) {
-                            x = (e & 1) ? bf16_hi(wd[e >> 1]) : bf16_lo(wd[e >> 1]);
-                        } else {
-                            x = __uint_as_float(wd[e]);
-                        }
-                        acc_add(m, idx, s, x, t0 + e);
-                    }
-                }
-            }
+        for (int k = 0; k < 4; ++k)
+            if ((word >> (8 * k)) & 0xFFu) slot[k] = d[k];
+        const unsigned short* st = reinterpret_cast<const unsigned short*>(slot);
+        while (word) {
+            const int e = __ffs(word) - 1;
+            word &= word - 1;
+            f(__uint_as_float((uint32_t)st[e] << 16), t0 + e);
         }
-    }
-    for (int t = tail_lo + tid; t < hi; t += kLogitThreads)
-        if (mask_bit(mrow, t)) acc_add(m, idx, s, logit_at<BF16>(lrow, t), t);
-
-    // CTA reduction
-    __shared__ float sm_m[kLogitThreads / 32], sm_s[kLogitThreads / 32];
-    __shared__ int sm_i[kLogitThreads / 32];
-    __shared__ int sm_last;
-    warp_merge(m, idx, s);
-    const int lane = tid & 31, wid = tid >> 5;
-    if (lane == 0) {
-        sm_m[wid] = m;
-        sm_i[wid] = idx;
-        sm_s[wid] = s;
-    }
-    __syncthreads();
-    if (wid == 0) {
-        m = lane < kLogitThreads / 32 ? sm_m[lane] : -INFINITY;
-        idx = lane < kLogitThreads / 32 ? sm_i[lane] : INT_MAX;
-        s = lane < kLogitThreads / 32 ? sm_s[lane] : 0.0f;
-        warp_merge(m, idx, s);
-        if (lane == 0) {
-            if (S == 1) {
-                argmax[row] = m == -INFINITY ? -1 : idx;
-                if (lse) lse[row] = m == -INFINITY ? -INFINITY : m + logf(s);
-                sm_last = 0;
-            } else {
-                partials[(size_t)row * S + c] = make_float4(m, __int_as_float(idx), s, 0.0f);
-                __threadfence();
-                const unsigned ticket = atomicAdd(counters + row, 1u);
-                sm_last = ticket == (unsigned)(S - 1);
-            }
-        }
-    }
-    __syncthreads();
-    if (sm_last && wid == 0) {
-        // last CTA of this row: combine the S chunk partials (S <= 64)
-        __threadfence();
-        m = -INFINITY;
-        s = 0.0f;
-        idx = INT_MAX;
-        for (int k = lane; k < S; k += 32) {
-            const float4 p = __ldcg(partials + (size_t)row * S + k);
-            acc_merge(m, idx, s, p.x, __float_as_int(p.y), p.z);
-        }
-        warp_merge(m, idx, s);
-        if (lane == 0) {
-            argmax[row] = m == -INFINITY ? -1 : idx;
-            if (lse) lse[row] = m == -INFINITY ? -INFINITY : m + logf(s);
-            counters[row] = 0u;   // ready for the next launch (stream-ordered)
+    } else {
+        while (word) {
+            const int e = __ffs(word) - 1;
+            word &= word - 1;
+            if (t0 + e < V) f(logit_at<BF16>(lrow, t0 + e), t0 + e);
         }
     }
 }
 
+// Units are mask words (32 tokens); row r holds W units.  Each CTA takes a
+// contiguous range of the batch x W units; the CTAs sharing a row leave
+// (max, argmax, sum) partials and the last one to finish combines them.
+template <bool BF16, bool STAGE, bool KEEP_L2>
+__global__ void __launch_bounds__(kLogitThreads)
+    logits_reduce_kernel(const void* __restrict__ logits, int64_t stride, const uint32_t* __restrict__ mask, int V,
+                         int W, int B, long long per_cta, float4* __restrict__ partials,
+                         uint32_t* __restrict__ counters, int32_t* __restrict__ argmax, float* __restrict__ lse) {
+    __shared__ uint4 stage[STAGE ? kLogitThreads * 4 : 1];
+    __shared__ int sm_last;
+    const long long N = (long long)B * W;
+    const int tid = threadIdx.x;
+    uint4* slot = stage + (STAGE ? tid * 4 : 0);
+    long long u = (long long)blockIdx.x * per_cta;
+    const long long u_end = min(N, u + per_cta);
+    while (u < u_end) {
+        const int r = (int)(u / W);
+        const long long row_end = (long long)(r + 1) * W;
+        const long long seg_end = min(u_end, row_end);
+        const uint32_t* mrow = mask + (size_t)r * W;
+        const char* lrow = reinterpret_cast<const char*>(logits) + (size_t)r * stride * (BF16 ? 2 : 4);
+        const int j0 = (int)(u - (long long)r * W), j1 = (int)(seg_end - (long long)r * W);
+        float m = -INFINITY, mL = -INFINITY, s = 0.0f;
+        int idx = INT_MAX;
+        for (int j = j0 + tid; j < j1; j += kLogitThreads) {
+            const uint32_t word = __ldg(mrow + j);
+            if (word)
+                for_allowed<BF16, STAGE, KEEP_L2>(lrow, word, j, V, slot,
+                                                  [&](float x, int t) { acc_add(m, mL, idx, s, x, t); });
+        }
+        block_merge(m, idx, s);
+        const long long first = ((long long)r * W) / per_cta;
+        const long long last = (row_end - 1) / per_cta;
+        const int nseg = (int)(last - first + 1);
+        if (tid == 0) {
+            if (nseg == 1) {
+                argmax[r] = m == -INFINITY ? -1 : idx;
+                if (lse) lse[r] = m == -INFINITY ? -INFINITY : m + logf(s);
+                sm_last = 0;
+            } else {
+                partials[(size_t)r * kMaxSegments + (blockIdx.x - first)] =
+                    make_float4(m, __int_as_float(idx), s, 0.f);
+                __threadfence();
+                const unsigned ticket = atomicAdd(counters + r, 1u);
+                sm_last = ticket == (unsigned)(nseg - 1);
+            }
+        }
+        __syncthreads();
+        if (sm_last && tid < 32) {
+            // last CTA of the row: combine its segments
+            __threadfence();
+            m = -INFINITY;
+            s = 0.0f;
+            idx = INT_MAX;
+            for (int k = tid; k < nseg; k += 32) {
+                const float4 p = __ldcg(partials + (size_t)r * kMaxSegments + k);
+                acc_merge(m, idx, s, p.x, __float_as_int(p.y), p.z);
+            }
+            warp_merge(m, idx, s);
+            if (tid == 0) {
+                argmax[r] = m == -INFINITY ? -1 : idx;
+                if (lse) lse[r] = m == -INFINITY ? -INFINITY : m + logf(s);
+                counters[r] = 0u;   // ready for the next launch (stream-ordered)
+            }
+        }
+        u = seg_end;
+    }
+}
+
+// logprob[t] = logit[t] - lse for allowed t, -inf otherwise; one mask word (32
+// tokens) per thread, grid-stride over the batch x W words.  VEC: bf16 rows on
+// 16-byte boundaries and 16-byte aligned output rows (V % 4 == 0): four 16-byte
+// loads (skipped when no token of the vector is allowed) and eight float4
+// stores per word; otherwise one token at a time.
 template <bool BF16, bool VEC>
 __global__ void __launch_bounds__(kLogitThreads)
     logprobs_kernel(const void* __restrict__ logits, int64_t stride, const uint32_t* __restrict__ mask, int V, int W,
-                    int chunk, const float* __restrict__ lse, float* __restrict__ out) {
-    const int row = blockIdx.y, c = blockIdx.x, tid = threadIdx.x;
-    const int lo = c * chunk, hi = min(V, lo + chunk);
-    const uint32_t* mrow = mask + (size_t)row * W;
-    const char* lrow = reinterpret_cast<const char*>(logits) + (size_t)row * stride * (BF16 ? 2 : 4);
-    float* orow = out + (size_t)row * V;
-    const float l = __ldg(lse + row);
-    int tail_lo = lo;
-    if constexpr (VEC) {
-        constexpr int E = BF16 ? 8 : 4;
-        const int v_lo = lo / E, v_hi = hi / E;
-        tail_lo = v_hi * E;
-        const uint4* vrow = reinterpret_cast<const uint4*>(lrow);
-        for (int vv = v_lo + tid; vv < v_hi; vv += kLogitThreads) {
-            const uint32_t mb = BF16 ? mask_bits8(mrow, vv) : mask_bits4(mrow, vv);
-            const uint4 raw = mb ? __ldg(vrow + vv) : make_uint4(0, 0, 0, 0);
-            const uint32_t wd[4] = {raw.x, raw.y, raw.z, raw.w};
-            float r[E];
+                    int B, const float* __restrict__ lse, float* __restrict__ out) {
+    const long long N = (long long)B * W;
+    for (long long u = (long long)blockIdx.x * kLogitThreads + threadIdx.x; u < N;
+         u += (long long)gridDim.x * kLogitThreads) {
+        const int r = (int)(u / W), j = (int)(u - (long long)r * W);
+        const uint32_t word = __ldg(mask + u);
+        const char* lrow = reinterpret_cast<const char*>(logits) + (size_t)r * stride * (BF16 ? 2 : 4);
+        float* orow = out + (size_t)r * V + (size_t)j * 32;
+        const float l = __ldg(lse + r);
+        if (VEC && BF16 && j * 32 + 32 <= V) {
+            const uint4* src = reinterpret_cast<const uint4*>(lrow) + (size_t)j * 4;
+            uint4 d[4];
 #pragma unroll
-            for (int e = 0; e < E; ++e) {
-                float x;
-                if constexpr (BF16) {
-                    x = (e & 1) ? bf16_hi(wd[e >> 1]) : bf16_lo(wd[e >> 1]);
-                } else {
-                    x = __uint_as_float(wd[e]);
-                }
-                r[e] = ((mb >> e) & 1u) ? x - l : -INFINITY;
+            for (int k = 0; k < 4; ++k)
+                d[k] = ((word >> (8 * k)) & 0xFFu) ? __ldg(src + k) : make_uint4(0u, 0u, 0u, 0u);
+            float4* o4 = reinterpret_cast<float4*>(orow);
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const uint4& v8 = d[q >> 1];
+                const uint32_t w0 = (q & 1) ? v8.z : v8.x, w1 = (q & 1) ? v8.w : v8.y;
+                const float x[4] = {bf16_lo(w0), bf16_hi(w0), bf16_lo(w1), bf16_hi(w1)};
+                float o[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) o[e] = ((word >> (4 * q + e)) & 1u) ? x[e] - l : -INFINITY;
+                __stcs(o4 + q, make_float4(o[0], o[1], o[2], o[3]));
             }
-            float4* o4 = reinterpret_cast<float4*>(orow + (size_t)vv * E);
-            __stcs(o4, make_float4(r[0], r[1], r[2], r[3]));
-            if constexpr (BF16) __stcs(o4 + 1, make_float4(r[4], r[5], r[6], r[7]));
+        } else {
+            for (int e = 0; e < 32 && j * 32 + e < V; ++e)
+                orow[e] = ((word >> e) & 1u) ? logit_at<BF16>(lrow, j * 32 + e) - l : -INFINITY;
         }
     }
-    for (int t = tail_lo + tid; t < hi; t += kLogitThreads)
-        orow[t] = mask_bit(mrow, t) ? logit_at<BF16>(lrow, t) - l : -INFINITY;
 }
 
 // ---------------------------------------------------------------------------
 // advance
 // ---------------------------------------------------------------------------
-template <bool STACK>
+template <bool STACK, int MODE>
 __global__ void __launch_bounds__(kAdvanceThreads)
     advance_kernel(const StepView v, const int32_t* __restrict__ states, const uint64_t* __restrict__ stacks,
                    const int32_t* __restrict__ tokens, int32_t batch, int32_t* __restrict__ states_out,
                    uint64_t* __restrict__ stacks_out) {
+    using E = typename std::conditional<STACK, uint32_t, uint16_t>::type;
     const int b = blockIdx.x * kAdvanceThreads + threadIdx.x;
     if (b >= batch) return;
     const int32_t t = tokens[b];
@@ -481,21 +699,22 @@ __global__ void __launch_bounds__(kAdvanceThreads)
     } else if (t >= v.V) {
         atomicOr(v.err, DOMINO_DEVERR_BAD_TOKEN);
     } else {
-        const RowCfg rc = read_row(v, states, stacks, b, true);
-        if (rc.valid) {
+        const uint4 rc = read_row(v, states, stacks, b, true);
+        if (rc.w & 1u) {
+            // the table image the step kernel staged (L2-resident) read from global memory
+            Tab<E, MODE == kDenseSmem ? kDenseGlobal : MODE> tab;
+            tab.dense = reinterpret_cast<const E*>(STACK ? (const void*)v.t32 : (const void*)v.t16);
+            tab.sp = v.sp_info;
+            tab.tgt = reinterpret_cast<const E*>(v.sp_tgt);
+            tab.K = (uint32_t)v.K;
             const int p = __ldg(v.pos_of + t);
-            const int len = __ldg(v.len + p);
-            const uint4 h = __ldg(v.head + p);
-            const uint8_t* tail = len > kHeadBytes ? v.tail + __ldg(v.tail_off + p) : v.tail;
+            const int len = (int)(__ldg(v.info + p) >> 16);
+            const uint8_t* hp = reinterpret_cast<const uint8_t*>(v.head + 2 * (size_t)p);
+            const uint8_t* tail = len > kInlineBytes ? v.tail + __ldg(v.tail_off + p) : v.tail;
             if (len > 0) {
-                bits = rc.bits;
-                depth = rc.depth;
-                if constexpr (STACK) {
-                    s = walk_pda<false>(v.t32, v.ret, (uint32_t)v.K, rc.s, bits, depth, (uint32_t)v.max_depth, h,
-                                        len, tail);
-                } else {
-                    s = walk_dfa<false>(v.t16, (uint32_t)v.K, rc.s, h, len, tail);
-                }
+                bits = rc.y;
+                depth = rc.z;
+                s = walk<STACK, 0>(tab, v.ret, (uint32_t)v.max_depth, rc.x, bits, depth, hp, len, tail);
                 if (s == 0) bits = depth = 0;
             }
         }
@@ -504,65 +723,143 @@ __global__ void __launch_bounds__(kAdvanceThreads)
     if (stacks_out) stacks_out[b] = ((uint64_t)depth << 32) | bits;
 }
 
-template <bool STACK, bool SMEM, bool NEXT>
+// ---------------------------------------------------------------------------
+// launchers
+// ---------------------------------------------------------------------------
+// Rows per tile: as many as possible (<= 32, one ballot) while the tiles
+// still split evenly over one CTA per SM.
+int rows_per_tile(const StepView& v, const LaunchEnv& env, int batch, bool next) {
+    if (next) return kRowsPerTileNext;
+    int best = kRowsPerTile;
+    double best_waste = 1e9;
+    for (int R = kMaxRowsPerTile; R >= kRowsPerTile; R -= 4) {
+        const long long tiles = (long long)((batch + R - 1) / R) * v.n_windows;
+        const double per = (double)tiles / env.num_sms;
+        const double waste = tiles < env.num_sms ? 1.0 - per : (double)((tiles + env.num_sms - 1) / env.num_sms) / per - 1.0;
+        if (waste < 0.08) return R;
+        if (waste < best_waste) {
+            best_waste = waste;
+            best = R;
+        }
+    }
+    return best;
+}
+
+template <bool STACK, int MODE, bool NEXT>
 cudaError_t launch_step_t(const StepView& v, const LaunchEnv& env, const int32_t* states, const uint64_t* stacks,
                           int32_t batch, bool row_is_state, uint32_t* mask, int32_t* next, cudaStream_t st) {
-    const int smem = kMaskTileBytes + (NEXT ? kNextTileBytes : 0) + (SMEM ? v.table_bytes : 0);
-    auto kern = step_kernel<STACK, SMEM, NEXT>;
+    const int img_bytes = MODE == kDenseGlobal ? 0 : (int)table_smem_bytes(v, STACK, MODE);
+    const int R = rows_per_tile(v, env, batch, NEXT);
+    const StepLayout L = step_layout(v.K, R, NEXT, STACK, v.max_units, v.Q, img_bytes);
+    auto kern = step_kernel<STACK, MODE, NEXT>;
     // the dynamic shared-memory limit is raised once per device and size, so
     // that launches inside a stream capture make no attribute calls
     static int configured[kMaxDevices] = {0};
     int dev = 0;
     cudaGetDevice(&dev);
-    if (smem > 48 * 1024 && dev < kMaxDevices && configured[dev] < smem) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (L.total > 48 * 1024 && dev < kMaxDevices && configured[dev] < L.total) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L.total);
         if (e != cudaSuccess) return e;
-        configured[dev] = smem;
+        configured[dev] = L.total;
     }
-    const int row_groups = (batch + kRowGroup - 1) / kRowGroup;
-    int chunks = (4 * env.num_sms + v.n_windows - 1) / v.n_windows;
-    chunks = max(1, min(chunks, row_groups));
-    const int rows_per_cta = ((row_groups + chunks - 1) / chunks) * kRowGroup;
-    chunks = (batch + rows_per_cta - 1) / rows_per_cta;
-    dim3 grid((unsigned)v.n_windows, (unsigned)chunks);
-    kern<<<grid, kStepThreads, smem, st>>>(v, states, stacks, batch, rows_per_cta, row_is_state ? 1 : 0, mask,
-                                           next);
+    const int n_row_tiles = (batch + R - 1) / R;
+    const int n_tiles = n_row_tiles * v.n_windows;
+    const int grid = min(n_tiles, env.num_sms);
+    const uint4* img = nullptr;
+    int tgt_off = 0, ret_off = 0;
+    if constexpr (MODE != kDenseGlobal) {
+        const size_t esz = STACK ? 4 : 2;
+        if (MODE == kDenseSmem) {
+            img = reinterpret_cast<const uint4*>(STACK ? (const void*)v.t32 : (const void*)v.t16);
+            ret_off = align16((int)((size_t)v.Q * v.K * esz));
+        } else {
+            img = reinterpret_cast<const uint4*>(v.sp_info);
+            tgt_off = align16(v.Q * (MODE == kSparse32Smem ? 8 : 16));
+            ret_off = tgt_off + align16((int)((size_t)v.sp_nnz * esz));
+        }
+    }
+    kern<<<grid, kStepThreads, L.total, st>>>(v, img, img_bytes, tgt_off, ret_off, states, stacks, batch, R,
+                                              n_row_tiles, n_tiles, row_is_state ? 1 : 0, mask, next);
     return cudaGetLastError();
 }
 
-template <bool STACK, bool SMEM>
+template <bool STACK, int MODE>
 cudaError_t launch_step_n(const StepView& v, const LaunchEnv& env, const int32_t* states, const uint64_t* stacks,
                           int32_t batch, bool row_is_state, uint32_t* mask, int32_t* next, cudaStream_t st) {
-    if (next) return launch_step_t<STACK, SMEM, true>(v, env, states, stacks, batch, row_is_state, mask, next, st);
-    return launch_step_t<STACK, SMEM, false>(v, env, states, stacks, batch, row_is_state, mask, next, st);
+    if (next) return launch_step_t<STACK, MODE, true>(v, env, states, stacks, batch, row_is_state, mask, next, st);
+    return launch_step_t<STACK, MODE, false>(v, env, states, stacks, batch, row_is_state, mask, next, st);
 }
 
-template <bool BF16, bool VEC>
+template <bool STACK>
+cudaError_t launch_step_s(const StepView& v, const LaunchEnv& env, int mode, const int32_t* states,
+                          const uint64_t* stacks, int32_t batch, bool row_is_state, uint32_t* mask, int32_t* next,
+                          cudaStream_t st) {
+    switch (mode) {
+        case kDenseSmem:
+            return launch_step_n<STACK, kDenseSmem>(v, env, states, stacks, batch, row_is_state, mask, next, st);
+        case kSparse32Smem:
+            return launch_step_n<STACK, kSparse32Smem>(v, env, states, stacks, batch, row_is_state, mask, next, st);
+        case kSparse64Smem:
+            return launch_step_n<STACK, kSparse64Smem>(v, env, states, stacks, batch, row_is_state, mask, next, st);
+        default:
+            return launch_step_n<STACK, kDenseGlobal>(v, env, states, stacks, batch, row_is_state, mask, next, st);
+    }
+}
+
+// Resident CTAs per SM of one kernel, cached per (kernel, device).
+int occupancy(const void* kern, int threads) {
+    struct Entry {
+        const void* fn;
+        int dev, n;
+    };
+    static Entry cache[64];
+    static int used = 0;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    for (int i = 0; i < used; i++)
+        if (cache[i].fn == kern && cache[i].dev == dev) return cache[i].n;
+    int n = 1;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kern, threads, 0) != cudaSuccess || n < 1) {
+        cudaGetLastError();
+        n = 1;
+    }
+    if (used < 64) cache[used++] = Entry{kern, dev, n};
+    return n;
+}
+
+template <bool BF16, bool STAGE>
 cudaError_t launch_logits_t(const LaunchEnv& env, const void* logits, int32_t batch, int64_t stride, int32_t V,
                             const uint32_t* mask, int32_t* argmax, float* lse, float* logprobs, float4* partials,
-                            uint32_t* counters, float* lse_tmp, cudaStream_t st) {
+                            uint32_t* counters, float* lse_tmp, bool out_vec, cudaStream_t st) {
     const int W = (V + 31) / 32;
     const size_t esz = BF16 ? 2 : 4;
     for (int32_t r0 = 0; r0 < batch; r0 += kMaxLogitRows) {
         const int rows = min(kMaxLogitRows, batch - r0);
-        int S = (8 * env.num_sms + rows - 1) / rows;
-        S = max(1, min(S, min(kMaxChunks, (V + 2047) / 2048)));
-        const int chunk = (((V + S - 1) / S) + 7) / 8 * 8;
-        S = (V + chunk - 1) / chunk;
         const void* lg = reinterpret_cast<const char*>(logits) + (size_t)r0 * stride * esz;
         const uint32_t* mk = mask + (size_t)r0 * W;
         float* lse_rows = lse ? lse + r0 : (logprobs ? lse_tmp : nullptr);
-        dim3 grid((unsigned)S, (unsigned)rows);
+        const long long N = (long long)rows * W;
+        int grid = env.num_sms * (logprobs ? occupancy((const void*)logits_reduce_kernel<BF16, STAGE, true>, kLogitThreads)
+                                           : occupancy((const void*)logits_reduce_kernel<BF16, STAGE, false>, kLogitThreads));
+        grid = (int)std::min<long long>((long long)grid, (N + 2 * kLogitThreads - 1) / (2 * kLogitThreads));
+        grid = max(grid, 1);
+        long long per_cta = (N + grid - 1) / grid;
+        per_cta = std::max<long long>(per_cta, ((long long)W + kMaxSegments - 3) / (kMaxSegments - 2));
+        grid = (int)((N + per_cta - 1) / per_cta);
         if (logprobs) {
-            logits_reduce_kernel<BF16, VEC, true><<<grid, kLogitThreads, 0, st>>>(lg, stride, mk, V, W, chunk, S,
-                                                                                  partials, counters, argmax + r0,
-                                                                                  lse_rows);
-            logprobs_kernel<BF16, VEC><<<grid, kLogitThreads, 0, st>>>(lg, stride, mk, V, W, chunk, lse_rows,
-                                                                       logprobs + (size_t)r0 * V);
+            logits_reduce_kernel<BF16, STAGE, true><<<grid, kLogitThreads, 0, st>>>(
+                lg, stride, mk, V, W, rows, per_cta, partials, counters, argmax + r0, lse_rows);
+            int g2 = env.num_sms * occupancy((const void*)logprobs_kernel<BF16, true>, kLogitThreads);
+            g2 = (int)std::max<long long>(1, std::min<long long>((long long)g2, (N + kLogitThreads - 1) / kLogitThreads));
+            if (out_vec && STAGE)
+                logprobs_kernel<BF16, true><<<g2, kLogitThreads, 0, st>>>(lg, stride, mk, V, W, rows, lse_rows,
+                                                                         logprobs + (size_t)r0 * V);
+            else
+                logprobs_kernel<BF16, false><<<g2, kLogitThreads, 0, st>>>(lg, stride, mk, V, W, rows, lse_rows,
+                                                                          logprobs + (size_t)r0 * V);
         } else {
-            logits_reduce_kernel<BF16, VEC, false><<<grid, kLogitThreads, 0, st>>>(lg, stride, mk, V, W, chunk, S,
-                                                                                   partials, counters, argmax + r0,
-                                                                                   lse_rows);
+            logits_reduce_kernel<BF16, STAGE, false><<<grid, kLogitThreads, 0, st>>>(
+                lg, stride, mk, V, W, rows, per_cta, partials, counters, argmax + r0, lse_rows);
         }
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
@@ -572,17 +869,27 @@ cudaError_t launch_logits_t(const LaunchEnv& env, const void* logits, int32_t ba
 
 }  // namespace
 
-int step_tile_smem_bytes(bool next) { return kMaskTileBytes + (next ? kNextTileBytes : 0); }
-
-cudaError_t launch_step_mask(const StepView& v, const LaunchEnv& env, bool stack, bool smem_table,
-                             const int32_t* states, const uint64_t* stacks, int32_t batch, bool row_is_state,
-                             uint32_t* mask, int32_t* next, cudaStream_t st) {
-    if (stack) {
-        if (smem_table) return launch_step_n<true, true>(v, env, states, stacks, batch, row_is_state, mask, next, st);
-        return launch_step_n<true, false>(v, env, states, stacks, batch, row_is_state, mask, next, st);
+int64_t table_smem_bytes(const StepView& v, bool stack, int mode) {
+    const int64_t esz = stack ? 4 : 2;
+    const int64_t ret = align16(v.n_ret * 8);
+    switch (mode) {
+        case kDenseSmem: return align16((int)((int64_t)v.Q * v.K * esz)) + ret;
+        case kSparse32Smem: return align16(v.Q * 8) + align16((int)(v.sp_nnz * esz)) + ret;
+        case kSparse64Smem: return align16(v.Q * 16) + align16((int)(v.sp_nnz * esz)) + ret;
+        default: return 0;
     }
-    if (smem_table) return launch_step_n<false, true>(v, env, states, stacks, batch, row_is_state, mask, next, st);
-    return launch_step_n<false, false>(v, env, states, stacks, batch, row_is_state, mask, next, st);
+}
+
+int step_fixed_smem_bytes(const StepView& v, bool next) {
+    return step_layout(v.K, next ? kRowsPerTileNext : kMaxRowsPerTile, next, v.t32 != nullptr, v.max_units, v.Q, 0)
+        .total;
+}
+
+cudaError_t launch_step_mask(const StepView& v, const LaunchEnv& env, bool stack, int mode, const int32_t* states,
+                             const uint64_t* stacks, int32_t batch, bool row_is_state, uint32_t* mask,
+                             int32_t* next, cudaStream_t st) {
+    if (stack) return launch_step_s<true>(v, env, mode, states, stacks, batch, row_is_state, mask, next, st);
+    return launch_step_s<false>(v, env, mode, states, stacks, batch, row_is_state, mask, next, st);
 }
 
 cudaError_t launch_mask_logits(const LaunchEnv& env, const void* logits, int dtype, int32_t batch,
@@ -590,34 +897,45 @@ cudaError_t launch_mask_logits(const LaunchEnv& env, const void* logits, int dty
                                float* logprobs, float4* partials, uint32_t* counters, float* lse_tmp,
                                cudaStream_t st) {
     const bool bf16 = dtype == DOMINO_DTYPE_BF16;
-    const size_t esz = bf16 ? 2 : 4;
-    bool vec = (reinterpret_cast<uintptr_t>(logits) % 16 == 0) && ((size_t)row_stride * esz) % 16 == 0;
-    if (logprobs) vec = vec && (reinterpret_cast<uintptr_t>(logprobs) % 16 == 0) && (V % 4 == 0);
+    const bool out_vec = logprobs && (reinterpret_cast<uintptr_t>(logprobs) % 16 == 0) && (V % 4 == 0);
     if (bf16) {
-        if (vec)
+        const bool stage = (reinterpret_cast<uintptr_t>(logits) % 16 == 0) && ((size_t)row_stride * 2) % 16 == 0;
+        if (stage)
             return launch_logits_t<true, true>(env, logits, batch, row_stride, V, mask, argmax, lse, logprobs,
-                                               partials, counters, lse_tmp, st);
+                                               partials, counters, lse_tmp, out_vec, st);
         return launch_logits_t<true, false>(env, logits, batch, row_stride, V, mask, argmax, lse, logprobs, partials,
-                                            counters, lse_tmp, st);
+                                            counters, lse_tmp, out_vec, st);
     }
-    if (vec)
-        return launch_logits_t<false, true>(env, logits, batch, row_stride, V, mask, argmax, lse, logprobs, partials,
-                                            counters, lse_tmp, st);
     return launch_logits_t<false, false>(env, logits, batch, row_stride, V, mask, argmax, lse, logprobs, partials,
-                                         counters, lse_tmp, st);
+                                         counters, lse_tmp, out_vec, st);
 }
 
-cudaError_t launch_advance(const StepView& v, bool stack, const int32_t* states, const uint64_t* stacks,
+template <bool STACK>
+cudaError_t launch_advance_s(const StepView& v, int mode, const int32_t* states, const uint64_t* stacks,
+                             const int32_t* tokens, int32_t batch, int32_t* states_out, uint64_t* stacks_out,
+                             cudaStream_t st) {
+    const unsigned grid = (unsigned)((batch + kAdvanceThreads - 1) / kAdvanceThreads);
+    switch (mode) {
+        case kSparse32Smem:
+            advance_kernel<STACK, kSparse32Smem><<<grid, kAdvanceThreads, 0, st>>>(v, states, stacks, tokens, batch,
+                                                                                 states_out, stacks_out);
+            break;
+        case kSparse64Smem:
+            advance_kernel<STACK, kSparse64Smem><<<grid, kAdvanceThreads, 0, st>>>(v, states, stacks, tokens, batch,
+                                                                                 states_out, stacks_out);
+            break;
+        default:
+            advance_kernel<STACK, kDenseGlobal><<<grid, kAdvanceThreads, 0, st>>>(v, states, stacks, tokens, batch,
+                                                                                states_out, stacks_out);
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_advance(const StepView& v, bool stack, int mode, const int32_t* states, const uint64_t* stacks,
                            const int32_t* tokens, int32_t batch, int32_t* states_out, uint64_t* stacks_out,
                            cudaStream_t st) {
-    const unsigned grid = (unsigned)((batch + kAdvanceThreads - 1) / kAdvanceThreads);
-    if (stack)
-        advance_kernel<true><<<grid, kAdvanceThreads, 0, st>>>(v, states, stacks, tokens, batch, states_out,
-                                                               stacks_out);
-    else
-        advance_kernel<false><<<grid, kAdvanceThreads, 0, st>>>(v, states, stacks, tokens, batch, states_out,
-                                                                stacks_out);
-    return cudaGetLastError();
+    if (stack) return launch_advance_s<true>(v, mode, states, stacks, tokens, batch, states_out, stacks_out, st);
+    return launch_advance_s<false>(v, mode, states, stacks, tokens, batch, states_out, stacks_out, st);
 }
 
 }  // namespace domino
