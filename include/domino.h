@@ -192,6 +192,31 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
                             int32_t* states_host, uint64_t* stacks_host, int32_t* tokens_host, float* lse_host,
                             void* stream);
 
+/* domino_mask_logits without a handle and without allocating anything.
+ * Not a step of the paper (it has no counterpart there): it exists for callers
+ * that cannot call cudaMalloc -- for example code running while another
+ * component owns all of the device memory (a serving runtime whose caching
+ * allocator has reserved the GPU), or code on a path where an allocation's
+ * implicit device synchronisation is not acceptable -- and so cannot create a
+ * handle either.
+ *   Same arguments and results as domino_mask_logits, with the vocabulary size
+ *   n_tokens passed directly; batch <= 512 (larger batches return
+ *   DOMINO_E_INVALID_ARG: split them into calls of at most 512 rows).
+ *   Scratch: a fixed 516 KiB array inside libdomino.so (per-row partials,
+ *   tickets, temporary lse); every GPU that loads the library holds it until
+ *   the process exits.  Nothing is allocated by this call: no cudaMalloc,
+ *   cudaFree or allocating library routine.
+ *   The first call on a device looks up the array's device address with that
+ *   device current (the calling thread's current device); make that first
+ *   call before any stream capture.
+ *   All calls share the one array and each call clears the tickets it uses;
+ *   calls that overlap on the GPU (other streams or host threads without
+ *   ordering between them) race on it and corrupt each other's results, so
+ *   order them, e.g. on one stream. */
+int domino_mask_logits_noalloc(const void* logits_dev, int32_t dtype, int32_t batch, int32_t n_tokens,
+                               int64_t row_stride_elems, const uint32_t* mask_dev, int32_t* argmax_dev,
+                               float* lse_dev, float* logprobs_dev, void* stream);
+
 /* Synchronises `stream`, returns the sticky device error word (DOMINO_DEVERR_*
  * bits, 0 = none) in *code and clears it. */
 int domino_get_device_error(domino_t h, int32_t* code, void* stream);

@@ -65,6 +65,7 @@ _SIGS = {
     "domino_advance": [P, P, P, P, I32, P, P, P],
     "domino_decode_step_host": [P, P, I32, I32, P, P, P, P, P],
     "domino_get_device_error": [P, P, P],
+    "domino_mask_logits_noalloc": [P, I32, I32, I32, I64, P, P, P, P, P],
 }
 
 
@@ -208,6 +209,14 @@ def domino_decode_step_host(h: int, logits_host, dtype: int, batch: int, states_
     _check("domino_decode_step_host", lib().domino_decode_step_host(
         h, _ptr(logits_host), int(dtype), int(batch), _ptr(states_host), _ptr(stacks_host), _ptr(tokens_host),
         _ptr(lse_host), _stream(stream)))
+
+
+def domino_mask_logits_noalloc(logits_dev, dtype: int, batch: int, n_tokens: int, row_stride_elems: int, mask_dev,
+                               argmax_dev, lse_dev=None, logprobs_dev=None, stream=None) -> None:
+    """domino_mask_logits for callers that cannot allocate: no handle, fixed scratch, batch <= 512."""
+    _check("domino_mask_logits_noalloc", lib().domino_mask_logits_noalloc(
+        _ptr(logits_dev), int(dtype), int(batch), int(n_tokens), int(row_stride_elems), _ptr(mask_dev),
+        _ptr(argmax_dev), _ptr(lse_dev), _ptr(logprobs_dev), _stream(stream)))
 
 
 def domino_get_device_error(h: int, stream=None) -> int:

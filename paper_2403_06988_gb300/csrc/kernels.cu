@@ -28,6 +28,7 @@
 
 #include <climits>
 #include <cstdint>
+#include <mutex>
 #include <algorithm>
 #include <type_traits>
 
@@ -939,3 +940,87 @@ cudaError_t launch_advance(const StepView& v, bool stack, int mode, const int32_
 }
 
 }  // namespace domino
+
+// ---------------------------------------------------------------------------
+// domino_mask_logits_noalloc: the masked argmax / log-sum-exp for callers that
+// cannot allocate device memory.  Its scratch (per-row partials, tickets and a
+// temporary lse) is the fixed array below, part of this library's image, so
+// every GPU that loads the library holds it until the process exits.
+// ---------------------------------------------------------------------------
+namespace {
+
+constexpr int kNoAllocMaxRows = 512;
+constexpr int kNoAllocMaxDevices = 64;
+constexpr size_t kNoAllocPartialsBytes = sizeof(float4) * (size_t)kNoAllocMaxRows * domino::kMaxSegments;
+constexpr size_t kNoAllocCountersBytes = sizeof(uint32_t) * (size_t)kNoAllocMaxRows;
+constexpr size_t kNoAllocScratchBytes = kNoAllocPartialsBytes + kNoAllocCountersBytes + sizeof(float) * kNoAllocMaxRows;
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];   // 516 KiB
+
+struct NoAllocDevice {
+    bool ready;
+    unsigned char* scratch;   // device address of g_noalloc_scratch on this device
+    int num_sms;
+};
+NoAllocDevice g_noalloc_dev[kNoAllocMaxDevices];
+std::mutex g_noalloc_mu;
+
+// Once per device, with that device current: the array's device address.
+int noalloc_setup(int dev, NoAllocDevice* out) {
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    NoAllocDevice& d = g_noalloc_dev[dev];
+    if (!d.ready) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) {
+            cudaGetLastError();
+            return DOMINO_E_CUDA;
+        }
+        int sms = 0;
+        if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1) {
+            cudaGetLastError();
+            return DOMINO_E_CUDA;
+        }
+        d.scratch = static_cast<unsigned char*>(p);
+        d.num_sms = sms;
+        d.ready = true;
+    }
+    *out = d;
+    return DOMINO_OK;
+}
+
+}  // namespace
+
+extern "C" int domino_mask_logits_noalloc(const void* logits_dev, int32_t dtype, int32_t batch, int32_t n_tokens,
+                                          int64_t row_stride_elems, const uint32_t* mask_dev, int32_t* argmax_dev,
+                                          float* lse_dev, float* logprobs_dev, void* stream) {
+    if (dtype != DOMINO_DTYPE_F32 && dtype != DOMINO_DTYPE_BF16) return DOMINO_E_INVALID_ARG;
+    if (batch < 0 || batch > kNoAllocMaxRows || n_tokens < 1 || n_tokens > (1 << 24) || row_stride_elems < n_tokens)
+        return DOMINO_E_INVALID_ARG;
+    if (batch == 0) return DOMINO_OK;
+    if (!logits_dev || !mask_dev || !argmax_dev) return DOMINO_E_INVALID_ARG;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        return DOMINO_E_CUDA;
+    }
+    if (dev < 0 || dev >= kNoAllocMaxDevices) return DOMINO_E_UNSUPPORTED;
+    NoAllocDevice d{};
+    int rc = noalloc_setup(dev, &d);
+    if (rc != DOMINO_OK) return rc;
+    float4* partials = reinterpret_cast<float4*>(d.scratch);
+    uint32_t* counters = reinterpret_cast<uint32_t*>(d.scratch + kNoAllocPartialsBytes);
+    float* lse_tmp = reinterpret_cast<float*>(d.scratch + kNoAllocPartialsBytes + kNoAllocCountersBytes);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    // the tickets must start at zero; the array keeps whatever the last call left
+    cudaError_t e = cudaMemsetAsync(counters, 0, sizeof(uint32_t) * (size_t)batch, st);
+    if (e == cudaSuccess) {
+        domino::LaunchEnv env{d.num_sms, 0};
+        e = domino::launch_mask_logits(env, logits_dev, dtype, batch, row_stride_elems, n_tokens, mask_dev,
+                                       argmax_dev, lse_dev, logprobs_dev, partials, counters, lse_tmp, st);
+    }
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return DOMINO_E_CUDA;
+    }
+    return DOMINO_OK;
+}
