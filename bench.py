@@ -172,6 +172,36 @@ def measured_peaks():
 # ----------------------------------------------------------------------------
 # CPU oracle baseline (bounded sample of the same workload)
 # ----------------------------------------------------------------------------
+def walk_stats(name: str):
+    """Bytes the plain definition walks per check on this workload's trajectory,
+    stored by tests/golden/make_walk_stats.py (None when not stored)."""
+    p = os.path.join(ROOT, "tests", "golden", "walk_stats.json")
+    try:
+        with open(p) as f:
+            return float(json.load(f)[name]["walk_steps_per_check_mean"])
+    except (OSError, KeyError, ValueError):
+        return None
+
+
+def ncu_traffic(name: str) -> dict:
+    """DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from
+    the committed ncu summary, per kernel; a kernel whose source changed since
+    the capture maps to None."""
+    import hashlib
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    src = os.path.join(ROOT, "paper_2403_06988_gb300", "csrc", "kernels.cu")
+    try:
+        with open(p) as f:
+            rec = json.load(f)
+        with open(src, "rb") as f:
+            digest = hashlib.sha256(f.read()).hexdigest()[:16]
+    except (OSError, ValueError):
+        return {}
+    if rec.get("kernels_cu_sha256_16") != digest:
+        return {}
+    return {k: v for k, v in rec.get("per_launch_bytes", {}).get(name, {}).items()}
+
+
 def cpu_cores() -> int:
     try:
         return len(os.sched_getaffinity(0))
@@ -305,19 +335,11 @@ def run_domino(args, dist: Dist):
     p_logits = [t.data_ptr() for t in logits]
     launches_per_step = 3 + (1 if w.want_logprobs else 0)
 
-    def step(i, stream_ptr, ev=None):
-        if ev is not None:
-            ev[0].record()
+    def step(i, stream_ptr):
         rc = L.domino_step_mask(h, p_states, p_stacks, Bsz, p_mask, None, stream_ptr)
-        if ev is not None:
-            ev[1].record()
         rc |= L.domino_mask_logits(h, p_logits[i % nbuf], dtype_code, Bsz, V, p_mask, p_arg, p_lse, p_lp,
                                    stream_ptr)
-        if ev is not None:
-            ev[2].record()
         rc |= L.domino_advance(h, p_states, p_stacks, p_arg, Bsz, p_states, p_stacks, stream_ptr)
-        if ev is not None:
-            ev[3].record()
         if rc:
             raise RuntimeError(f"domino call failed ({rc})")
 
@@ -329,52 +351,75 @@ def run_domino(args, dist: Dist):
             step(i, sp)
     torch.cuda.synchronize()
 
-    try:
-        events = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(4)] for _ in range(K)]
-        have_ext = True
-    except TypeError:
-        events, have_ext = None, False
-    graph = None
-    if not args.no_graph:
-        graph = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(graph, stream=s, capture_error_mode="relaxed"):
+    def capture(n, body):
+        """A CUDA graph of n calls of body(i, stream) on stream s (None: eager)."""
+        if args.no_graph:
+            return None
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s, capture_error_mode="relaxed"):
             sp = torch.cuda.current_stream().cuda_stream
-            for i in range(K):
-                step(i, sp, events[i] if have_ext else None)
-        graph.replay()                      # upload + one untimed pass
+            for i in range(n):
+                body(i, sp)
+        g.replay()                          # upload + one untimed pass
         torch.cuda.synchronize()
+        return g
 
-    t_start = torch.cuda.Event(enable_timing=True)
-    t_end = torch.cuda.Event(enable_timing=True)
+    def timed(n, body, g, sampler=None):
+        """Device time (ms) of n calls, events on the launching stream, synchronized on both sides."""
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        dist.barrier()
+        torch.cuda.synchronize()
+        if sampler is not None:
+            sampler.start()
+        with torch.cuda.stream(s):
+            t0.record()
+            if g is not None:
+                g.replay()
+            else:
+                for i in range(n):
+                    body(i, s.cuda_stream)
+            t1.record()
+        torch.cuda.synchronize()
+        if sampler is not None:
+            sampler.stop()
+        dist.barrier()
+        return t0.elapsed_time(t1)
+
+    # ---- the timed region: K whole decode steps, nothing else in the graph ----
+    graph = capture(K, step)
     sampler = ClockSampler(dev_id)
-    dist.barrier()
-    torch.cuda.synchronize()
-    sampler.start()
-    with torch.cuda.stream(s):
-        t_start.record()
-        if graph is not None:
-            graph.replay()
-        else:
-            sp = s.cuda_stream
-            for i in range(K):
-                step(i, sp, events[i] if events else None)
-        t_end.record()
-    torch.cuda.synchronize()
-    sampler.stop()
-    dist.barrier()
-    ms = t_start.elapsed_time(t_end)
+    ms = timed(K, step, graph, sampler)
     ms_max = dist.max(ms)
     err = d.device_error()
     if err:
         raise RuntimeError(f"device error word {err}")
 
-    per_kernel = None
-    if events is not None and (graph is None or have_ext):
-        tk = [0.0, 0.0, 0.0]
-        for ev in events:
-            for j in range(3):
-                tk[j] += ev[j].elapsed_time(ev[j + 1])
-        per_kernel = {"step_mask": tk[0] / K, "mask_logits": tk[1] / K, "advance": tk[2] / K}
+    # ---- per-kernel average launch durations: each kernel alone, Kk launches
+    # back to back in its own graph on the same stream (its inputs as in a step)
+    Kk = min(K, 400)
+    st_tmp = torch.empty_like(states)
+    sk_tmp = torch.empty_like(stacks) if stack else None
+    p_st_tmp, p_sk_tmp = st_tmp.data_ptr(), (sk_tmp.data_ptr() if stack else None)
+
+    def k_step(i, sp):
+        if L.domino_step_mask(h, p_states, p_stacks, Bsz, p_mask, None, sp):
+            raise RuntimeError("step_mask failed")
+
+    def k_logits(i, sp):
+        if L.domino_mask_logits(h, p_logits[i % nbuf], dtype_code, Bsz, V, p_mask, p_arg, p_lse, p_lp, sp):
+            raise RuntimeError("mask_logits failed")
+
+    def k_adv(i, sp):
+        if L.domino_advance(h, p_states, p_stacks, p_arg, Bsz, p_st_tmp, p_sk_tmp, sp):
+            raise RuntimeError("advance failed")
+    per_kernel = {}
+    for name, body in (("step_mask", k_step), ("mask_logits", k_logits), ("advance", k_adv)):
+        g = capture(Kk, body)
+        per_kernel[name] = dist.max(timed(Kk, body, g)) / Kk      # ms per launch
+        del g
+    if d.device_error():
+        raise RuntimeError("device error after the per-kernel graphs")
 
     # ---- end to end through the host-buffer C entry point -------------------
     Ke = max(3, min(args.e2e_steps, K))
@@ -412,22 +457,38 @@ def run_domino(args, dist: Dist):
     value = n * Bsz * V * K / (ms_max / 1e3)
     peaks, peak_kind = measured_peaks()
     hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
-    kernels = {}
-    if per_kernel:
-        lg_bytes = Bsz * V * esz + Bsz * Wd * 4 + Bsz * 8 + (Bsz * V * 4 if w.want_logprobs else 0)
-        t_ml = per_kernel["mask_logits"] * 1e-3
-        kernels["mask_logits"] = {"us": per_kernel["mask_logits"] * 1e3, "bytes": lg_bytes,
-                                  "gbs": lg_bytes / t_ml / 1e9, "frac_hbm": lg_bytes / t_ml / 1e9 / hbm_peak}
-        t_sm = per_kernel["step_mask"] * 1e-3
-        kernels["step_mask"] = {"us": per_kernel["step_mask"] * 1e3, "checks_per_s": Bsz * V / t_sm,
-                                "mask_bytes": Bsz * Wd * 4}
-        kernels["advance"] = {"us": per_kernel["advance"] * 1e3}
-    roofline = None
-    if per_kernel:
-        km = kernels["mask_logits"]
-        roofline = {"kernel": "mask_logits", "bound": "hbm", "achieved": km["gbs"], "peak": hbm_peak,
-                    "unit": "GB/s", "frac": km["frac_hbm"], "traffic": None, "peak_source": peak_kind,
-                    "note": "dominant HBM-bound kernel; step_mask is reported in `kernels`"}
+    walk = walk_stats(w.name)
+    traffic = ncu_traffic(w.name)
+    lg_bytes = Bsz * V * esz + Bsz * Wd * 4 + Bsz * 8 + (Bsz * V * 4 if w.want_logprobs else 0)
+    t_ml = per_kernel["mask_logits"] * 1e-3
+    t_sm = per_kernel["step_mask"] * 1e-3
+    gbs = lg_bytes / t_ml / 1e9
+    kernels = {
+        "mask_logits": {"us": t_ml * 1e6, "algorithmic_bytes": lg_bytes, "gbs": gbs, "frac_hbm": gbs / hbm_peak,
+                        "dram_bytes_ncu": traffic.get("mask_logits")},
+        "step_mask": {"us": t_sm * 1e6, "checks_per_s": Bsz * V / t_sm, "mask_bytes": Bsz * Wd * 4,
+                      "dram_bytes_ncu": traffic.get("step_mask")},
+        "advance": {"us": per_kernel["advance"] * 1e3},
+        "timing": f"each kernel alone, {Kk} launches back to back in one CUDA graph, events on its stream",
+    }
+    # transition-lookup peak: one conflict-free 32-lane shared-memory gather per
+    # SM clock; every byte the definition walks is one table lookup
+    sm_clk = float(peaks.get("sm_max_mhz", 2070.0)) * 1e6
+    lookup_peak = torch.cuda.get_device_properties(dev_id).multi_processor_count * 32 * sm_clk / 1e9
+    if walk is not None:
+        trans = walk * Bsz * V
+        kernels["step_mask"].update({"walk_steps_per_check": walk, "gtransitions_per_s": trans / t_sm / 1e9,
+                                     "frac_lookup_peak": trans / t_sm / 1e9 / lookup_peak})
+    if t_sm >= t_ml and walk is not None:
+        roofline = {"kernel": "step_mask", "bound": "alu", "achieved": trans / t_sm / 1e9, "peak": lookup_peak,
+                    "unit": "Gtransitions/s", "frac": trans / t_sm / 1e9 / lookup_peak,
+                    "traffic": traffic.get("step_mask"), "algorithmic_units_per_launch": trans,
+                    "peak_source": f"{lookup_peak:.0f} G lookups/s = SMs x 32 lanes x {sm_clk / 1e6:.0f} MHz",
+                    "note": "walk bound by shared-memory gathers and issue, not HBM"}
+    else:
+        roofline = {"kernel": "mask_logits", "bound": "hbm", "achieved": gbs, "peak": hbm_peak, "unit": "GB/s",
+                    "frac": gbs / hbm_peak, "traffic": traffic.get("mask_logits"),
+                    "algorithmic_units_per_launch": lg_bytes, "peak_source": f"hbm_gbs {peak_kind}"}
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": n, "steps": K, "warmup": Wm,
         "ms_per_step": ms_max / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
@@ -442,6 +503,7 @@ def run_domino(args, dist: Dist):
         "e2e": {"value": n * Bsz * V * Ke / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "steps": Ke, "api": "domino_decode_step_host (pinned host buffers)"},
         "gpu_launches": K * launches_per_step,
+        "gpu_launches_note": "timed region only; per-kernel graphs and e2e are timed separately",
         "clocks": sampler.summary(),
     }
     if dist.rank == 0 and n == 1 and not args.no_cpu_baseline:

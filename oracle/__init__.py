@@ -64,6 +64,8 @@ def lib():
         L.oracle_mask_logits.restype = None
         L.oracle_mask_logits.argtypes = [P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64, P, P,
                                          P, P, ctypes.c_int32]
+        L.oracle_walk_steps.restype = ctypes.c_int64
+        L.oracle_walk_steps.argtypes = [P, P, P, ctypes.c_int32, ctypes.c_int32]
         L.oracle_advance.restype = ctypes.c_int64
         L.oracle_advance.argtypes = [P, P, P, P, ctypes.c_int32, ctypes.c_int32, P, P]
         _lib = L
@@ -137,6 +139,12 @@ class Problem:
         nxt = np.zeros((B, self.V), dtype=np.int32) if want_next else None
         bad = lib().oracle_step_mask(self._h, _ptr(states), _ptr(stacks), B, _ptr(mask), _ptr(nxt), int(n_threads))
         return mask, nxt, int(bad)
+
+    def walk_steps(self, states, stacks=None, n_threads=1) -> int:
+        """Bytes the plain definition walks to check every token from every row."""
+        states = np.ascontiguousarray(states, dtype=np.int32)
+        stacks = None if stacks is None else np.ascontiguousarray(stacks, dtype=np.uint64)
+        return int(lib().oracle_walk_steps(self._h, _ptr(states), _ptr(stacks), states.shape[0], int(n_threads)))
 
     def advance(self, states, stacks, tokens, start_state):
         states = np.ascontiguousarray(states, dtype=np.int32)

@@ -110,8 +110,10 @@ static int config_valid(const oracle_problem* p, int32_t state, uint64_t stack, 
 }
 
 /* Walk one token from (s, st); st is updated in place.  Returns 1 when the
- * token is allowed (Sec. 3.5 at k = infinity), with *end the state reached. */
-static int walk_token(const oracle_problem* p, int32_t s, stack_t_* st, int32_t t, int32_t* end) {
+ * token is allowed (Sec. 3.5 at k = infinity), with *end the state reached.
+ * *steps (when not NULL) counts the bytes taken, the last one included. */
+static int walk_token(const oracle_problem* p, int32_t s, stack_t_* st, int32_t t, int32_t* end,
+                      int64_t* steps) {
     int64_t lo = p->offsets[t], hi = p->offsets[t + 1];
     if (t == p->eos_id) {                         /* forced EOS: accepting and nothing left open */
         *end = s;
@@ -120,6 +122,7 @@ static int walk_token(const oracle_problem* p, int32_t s, stack_t_* st, int32_t 
     if (hi == lo) return 0;                       /* other empty tokens never advance the output */
     for (int64_t i = lo; i < hi; i++) {
         uint8_t c = p->bytes[i];
+        if (steps) (*steps)++;
         int32_t r = p->rule_at[(int64_t)s * 256 + c];
         if (r < 0) {
             s = p->delta[(int64_t)s * 256 + c];
@@ -145,7 +148,7 @@ int oracle_check_token(const oracle_problem* p, int32_t state, uint64_t stack, i
     stack_t_ st;
     if (!config_valid(p, state, stack, &st) || token < 0 || token >= p->n_tokens) return -1;
     int32_t end = 0;
-    if (!walk_token(p, state, &st, token, &end)) return 0;
+    if (!walk_token(p, state, &st, token, &end, NULL)) return 0;
     if (next_state) *next_state = end;
     if (next_stack) *next_stack = encode_stack(&st);
     return 1;
@@ -173,13 +176,34 @@ int64_t oracle_step_mask(const oracle_problem* p, const int32_t* states, const u
         for (int32_t t = 0; t < V; t++) {
             stack_t_ st = st0;
             int32_t end = 0;
-            if (walk_token(p, states[b], &st, t, &end)) {
+            if (walk_token(p, states[b], &st, t, &end, NULL)) {
                 mrow[t / 32] |= 1u << (t % 32);
                 if (nrow) nrow[t] = end;
             }
         }
     }
     return invalid;
+}
+
+int64_t oracle_walk_steps(const oracle_problem* p, const int32_t* states, const uint64_t* stacks,
+                          int32_t batch, int32_t n_threads) {
+    int64_t total = 0;
+#ifdef _OPENMP
+    if (n_threads < 1) n_threads = 1;
+#pragma omp parallel for schedule(dynamic, 1) num_threads(n_threads) reduction(+ : total)
+#endif
+    for (int32_t b = 0; b < batch; b++) {
+        stack_t_ st0;
+        if (!config_valid(p, states[b], stacks ? stacks[b] : 0, &st0)) continue;
+        int64_t n = 0;
+        for (int32_t t = 0; t < p->n_tokens; t++) {
+            stack_t_ st = st0;
+            int32_t end = 0;
+            walk_token(p, states[b], &st, t, &end, &n);
+        }
+        total += n;
+    }
+    return total;
 }
 
 static double logit_value(const void* logits, int32_t dtype, int64_t i) {
@@ -246,7 +270,7 @@ int64_t oracle_advance(const oracle_problem* p, const int32_t* states, const uin
                 invalid++;
             } else {
                 int32_t end = 0;
-                if (walk_token(p, s, &st, t, &end)) {
+                if (walk_token(p, s, &st, t, &end, NULL)) {
                     s_out = end;
                     w_out = encode_stack(&st);
                 }

@@ -74,6 +74,13 @@ int oracle_check_token(const oracle_problem* p, int32_t state, uint64_t stack, i
 int64_t oracle_step_mask(const oracle_problem* p, const int32_t* states, const uint64_t* stacks,
                          int32_t batch, uint32_t* mask, int32_t* next, int32_t n_threads);
 
+/* Work of the plain definition: the number of (byte, transition) steps that
+ * checking every token from every row takes, each walk counted up to and
+ * including the byte that rejects it (EOS and empty tokens take none).
+ * Invalid rows count 0.  Used to state the algorithmic work of a mask step. */
+int64_t oracle_walk_steps(const oracle_problem* p, const int32_t* states, const uint64_t* stacks,
+                          int32_t batch, int32_t n_threads);
+
 /* Per row of logits ([batch] rows of n_tokens values, row_stride elements
  * apart; dtype ORACLE_F32 or ORACLE_BF16 raw bits): argmax [batch] (-1 when
  * every token is masked), lse [batch] (NULL: skipped), logprobs

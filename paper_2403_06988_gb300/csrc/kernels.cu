@@ -29,6 +29,7 @@
 #include <climits>
 #include <cstdint>
 #include <mutex>
+#include <utility>
 #include <algorithm>
 #include <type_traits>
 
@@ -43,6 +44,31 @@ static_assert(kStepThreads == kWin, "one thread per window slot");
 constexpr float kLog2e = 1.4426950408889634f;   // log2(e): exp(x) = 2^(x log2 e)
 
 __host__ __device__ constexpr int align16(int x) { return (x + 15) & ~15; }
+
+// Programmatic dependent launch: a kernel may start while the previous kernel
+// of its stream drains; it runs only work that reads nothing the earlier
+// kernels write, then waits for them (griddepcontrol.wait returns at once when
+// the kernel was launched without the attribute).  Each kernel lets its
+// successor launch only after its own wait, so a chain of launches never runs
+// more than one kernel ahead.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+}
 
 // Shared-memory layout of the step kernel (offsets in bytes).
 struct StepLayout {
@@ -261,6 +287,8 @@ __global__ void __launch_bounds__(kStepThreads, 1)
         ret = reinterpret_cast<const uint16_t*>(tb + img_ret_off);
     }
     const uint32_t maxd = (uint32_t)v.max_depth;
+    pdl_wait();      // everything below may read what earlier kernels wrote
+    pdl_trigger();   // after the wait: at most two kernels of a stream overlap
 
     const int t0 = (int)(((long long)blockIdx.x * n_tiles) / gridDim.x);
     const int t1 = (int)(((long long)(blockIdx.x + 1) * n_tiles) / gridDim.x);
@@ -572,19 +600,40 @@ __device__ __forceinline__ void for_allowed(const char* lrow, uint32_t word, int
     }
 }
 
+// cp.async: 16 bytes global -> shared without a register round trip
+__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gmem_src) {
+    const unsigned dst = (unsigned)__cvta_generic_to_shared(smem_dst);
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(gmem_src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
+}
+
+constexpr int kReduceThreads = 32;            // one warp per CTA: no block barriers
+constexpr int kStageDepth = 3;                // 32-word batches in flight per warp
+
 // Units are mask words (32 tokens); row r holds W units.  Each CTA takes a
 // contiguous range of the batch x W units; the CTAs sharing a row leave
 // (max, argmax, sum) partials and the last one to finish combines them.
+// STAGE (bf16 rows on 16-byte boundaries): a warp takes 32 consecutive words
+// of its row at a time; the 16-byte logit vectors that hold an allowed token
+// are copied, fully coalesced, into the warp's double-buffered staging area
+// with cp.async (masks are read two batches ahead, logits one), and each lane
+// then folds its own word's allowed logits.  Otherwise each allowed logit is
+// read on its own.
 template <bool BF16, bool STAGE, bool KEEP_L2>
-__global__ void __launch_bounds__(kLogitThreads)
+__global__ void __launch_bounds__(kReduceThreads)
     logits_reduce_kernel(const void* __restrict__ logits, int64_t stride, const uint32_t* __restrict__ mask, int V,
                          int W, int B, long long per_cta, float4* __restrict__ partials,
                          uint32_t* __restrict__ counters, int32_t* __restrict__ argmax, float* __restrict__ lse) {
-    __shared__ uint4 stage[STAGE ? kLogitThreads * 4 : 1];
-    __shared__ int sm_last;
+    // [buffer][word][16-byte vector]
+    __shared__ __align__(16) uint4 stage[STAGE ? kStageDepth * 32 * 4 : 1];
+    pdl_wait();
+    pdl_trigger();
     const long long N = (long long)B * W;
-    const int tid = threadIdx.x;
-    uint4* slot = stage + (STAGE ? tid * 4 : 0);
+    const int lane = threadIdx.x;
     long long u = (long long)blockIdx.x * per_cta;
     const long long u_end = min(N, u + per_cta);
     while (u < u_end) {
@@ -596,42 +645,102 @@ __global__ void __launch_bounds__(kLogitThreads)
         const int j0 = (int)(u - (long long)r * W), j1 = (int)(seg_end - (long long)r * W);
         float m = -INFINITY, mL = -INFINITY, s = 0.0f;
         int idx = INT_MAX;
-        for (int j = j0 + tid; j < j1; j += kLogitThreads) {
-            const uint32_t word = __ldg(mrow + j);
-            if (word)
-                for_allowed<BF16, STAGE, KEEP_L2>(lrow, word, j, V, slot,
-                                                  [&](float x, int t) { acc_add(m, mL, idx, s, x, t); });
+        if constexpr (STAGE) {
+            const int nb = (j1 - j0 + 31) / 32;   // batches of 32 words
+            const int full_words = V / 32;       // words whose 64 bytes of logits lie inside the row
+            auto mask_of = [&](int b) -> uint32_t {
+                const int j = j0 + 32 * b + lane;
+                return (b < nb && j < j1) ? __ldg(mrow + j) : 0u;
+            };
+            auto issue = [&](int b, uint32_t mw) {
+                if (b < nb) {
+                    const char* base = lrow + (size_t)(j0 + 32 * b) * 64;
+                    uint4* dst = stage + (b % kStageDepth) * 128;
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        const int q = 32 * k + lane, wi = q >> 2, sub = q & 3;
+                        const uint32_t mq = __shfl_sync(0xffffffffu, mw, wi);
+                        if (((mq >> (8 * sub)) & 0xFFu) && j0 + 32 * b + wi < full_words)
+                            cp_async16(dst + q, base + (size_t)q * 16);
+                    }
+                }
+                cp_async_commit();
+            };
+            uint32_t mw[kStageDepth + 1];
+#pragma unroll
+            for (int k = 0; k <= kStageDepth; ++k) mw[k] = mask_of(k);
+#pragma unroll
+            for (int k = 0; k < kStageDepth - 1; ++k) issue(k, mw[k]);
+            for (int b = 0; b < nb; ++b) {
+                issue(b + kStageDepth - 1, mw[kStageDepth - 1]);
+                const uint32_t mw_far = mask_of(b + kStageDepth + 1);
+                cp_async_wait<kStageDepth - 1>();   // batch b has landed
+                __syncwarp();
+                const int j = j0 + 32 * b + lane;
+                uint32_t word = mw[0];
+                if (word) {
+                    const int t0 = j * 32;
+                    if (j < full_words) {
+                        const unsigned short* st =
+                            reinterpret_cast<const unsigned short*>(stage + (b % kStageDepth) * 128 + lane * 4);
+                        while (word) {
+                            const int e = __ffs(word) - 1;
+                            word &= word - 1;
+                            acc_add(m, mL, idx, s, __uint_as_float((uint32_t)st[e] << 16), t0 + e);
+                        }
+                    } else {   // the row's partial last word
+                        while (word) {
+                            const int e = __ffs(word) - 1;
+                            word &= word - 1;
+                            if (t0 + e < V) acc_add(m, mL, idx, s, logit_at<BF16>(lrow, t0 + e), t0 + e);
+                        }
+                    }
+                }
+                __syncwarp();   // this buffer is refilled by the next issue
+#pragma unroll
+                for (int k = 0; k < kStageDepth; ++k) mw[k] = mw[k + 1];
+                mw[kStageDepth] = mw_far;
+            }
+            cp_async_wait<0>();
+        } else {
+            for (int j = j0 + lane; j < j1; j += 32) {
+                uint32_t word = __ldg(mrow + j);
+                const int t0 = j * 32;
+                while (word) {
+                    const int e = __ffs(word) - 1;
+                    word &= word - 1;
+                    if (t0 + e < V) acc_add(m, mL, idx, s, logit_at<BF16>(lrow, t0 + e), t0 + e);
+                }
+            }
         }
-        block_merge(m, idx, s);
+        warp_merge(m, idx, s);
         const long long first = ((long long)r * W) / per_cta;
         const long long last = (row_end - 1) / per_cta;
         const int nseg = (int)(last - first + 1);
-        if (tid == 0) {
+        bool is_last = false;
+        if (lane == 0) {
             if (nseg == 1) {
                 argmax[r] = m == -INFINITY ? -1 : idx;
                 if (lse) lse[r] = m == -INFINITY ? -INFINITY : m + logf(s);
-                sm_last = 0;
             } else {
                 partials[(size_t)r * kMaxSegments + (blockIdx.x - first)] =
                     make_float4(m, __int_as_float(idx), s, 0.f);
                 __threadfence();
-                const unsigned ticket = atomicAdd(counters + r, 1u);
-                sm_last = ticket == (unsigned)(nseg - 1);
+                is_last = atomicAdd(counters + r, 1u) == (unsigned)(nseg - 1);
             }
         }
-        __syncthreads();
-        if (sm_last && tid < 32) {
+        if (__shfl_sync(0xffffffffu, is_last, 0)) {
             // last CTA of the row: combine its segments
             __threadfence();
             m = -INFINITY;
             s = 0.0f;
             idx = INT_MAX;
-            for (int k = tid; k < nseg; k += 32) {
+            for (int k = lane; k < nseg; k += 32) {
                 const float4 p = __ldcg(partials + (size_t)r * kMaxSegments + k);
                 acc_merge(m, idx, s, p.x, __float_as_int(p.y), p.z);
             }
             warp_merge(m, idx, s);
-            if (tid == 0) {
+            if (lane == 0) {
                 argmax[r] = m == -INFINITY ? -1 : idx;
                 if (lse) lse[r] = m == -INFINITY ? -INFINITY : m + logf(s);
                 counters[r] = 0u;   // ready for the next launch (stream-ordered)
@@ -650,6 +759,8 @@ template <bool BF16, bool VEC>
 __global__ void __launch_bounds__(kLogitThreads)
     logprobs_kernel(const void* __restrict__ logits, int64_t stride, const uint32_t* __restrict__ mask, int V, int W,
                     int B, const float* __restrict__ lse, float* __restrict__ out) {
+    pdl_wait();
+    pdl_trigger();
     const long long N = (long long)B * W;
     for (long long u = (long long)blockIdx.x * kLogitThreads + threadIdx.x; u < N;
          u += (long long)gridDim.x * kLogitThreads) {
@@ -691,6 +802,8 @@ __global__ void __launch_bounds__(kAdvanceThreads)
                    const int32_t* __restrict__ tokens, int32_t batch, int32_t* __restrict__ states_out,
                    uint64_t* __restrict__ stacks_out) {
     using E = typename std::conditional<STACK, uint32_t, uint16_t>::type;
+    pdl_wait();
+    pdl_trigger();
     const int b = blockIdx.x * kAdvanceThreads + threadIdx.x;
     if (b >= batch) return;
     const int32_t t = tokens[b];
@@ -779,9 +892,8 @@ cudaError_t launch_step_t(const StepView& v, const LaunchEnv& env, const int32_t
             ret_off = tgt_off + align16((int)((size_t)v.sp_nnz * esz));
         }
     }
-    kern<<<grid, kStepThreads, L.total, st>>>(v, img, img_bytes, tgt_off, ret_off, states, stacks, batch, R,
-                                              n_row_tiles, n_tiles, row_is_state ? 1 : 0, mask, next);
-    return cudaGetLastError();
+    return launch_pdl(kern, dim3(grid), dim3(kStepThreads), (size_t)L.total, st, v, img, img_bytes, tgt_off, ret_off,
+                      states, stacks, batch, R, n_row_tiles, n_tiles, row_is_state ? 1 : 0, mask, next);
 }
 
 template <bool STACK, int MODE>
@@ -840,27 +952,31 @@ cudaError_t launch_logits_t(const LaunchEnv& env, const void* logits, int32_t ba
         const uint32_t* mk = mask + (size_t)r0 * W;
         float* lse_rows = lse ? lse + r0 : (logprobs ? lse_tmp : nullptr);
         const long long N = (long long)rows * W;
-        int grid = env.num_sms * (logprobs ? occupancy((const void*)logits_reduce_kernel<BF16, STAGE, true>, kLogitThreads)
-                                           : occupancy((const void*)logits_reduce_kernel<BF16, STAGE, false>, kLogitThreads));
-        grid = (int)std::min<long long>((long long)grid, (N + 2 * kLogitThreads - 1) / (2 * kLogitThreads));
+        int grid = env.num_sms * (logprobs ? occupancy((const void*)logits_reduce_kernel<BF16, STAGE, true>, kReduceThreads)
+                                           : occupancy((const void*)logits_reduce_kernel<BF16, STAGE, false>, kReduceThreads));
+        grid = (int)std::min<long long>((long long)grid, (N + 127) / 128);   // at least 4 batches per warp
         grid = max(grid, 1);
         long long per_cta = (N + grid - 1) / grid;
         per_cta = std::max<long long>(per_cta, ((long long)W + kMaxSegments - 3) / (kMaxSegments - 2));
         grid = (int)((N + per_cta - 1) / per_cta);
         if (logprobs) {
-            logits_reduce_kernel<BF16, STAGE, true><<<grid, kLogitThreads, 0, st>>>(
-                lg, stride, mk, V, W, rows, per_cta, partials, counters, argmax + r0, lse_rows);
+            cudaError_t e0 = launch_pdl(logits_reduce_kernel<BF16, STAGE, true>, dim3(grid), dim3(kReduceThreads), 0, st,
+                                        lg, stride, mk, V, W, rows, per_cta, partials, counters, argmax + r0,
+                                        lse_rows);
+            if (e0 != cudaSuccess) return e0;
             int g2 = env.num_sms * occupancy((const void*)logprobs_kernel<BF16, true>, kLogitThreads);
             g2 = (int)std::max<long long>(1, std::min<long long>((long long)g2, (N + kLogitThreads - 1) / kLogitThreads));
-            if (out_vec && STAGE)
-                logprobs_kernel<BF16, true><<<g2, kLogitThreads, 0, st>>>(lg, stride, mk, V, W, rows, lse_rows,
-                                                                         logprobs + (size_t)r0 * V);
-            else
-                logprobs_kernel<BF16, false><<<g2, kLogitThreads, 0, st>>>(lg, stride, mk, V, W, rows, lse_rows,
-                                                                          logprobs + (size_t)r0 * V);
+            cudaError_t e1 = (out_vec && STAGE)
+                                 ? launch_pdl(logprobs_kernel<BF16, true>, dim3(g2), dim3(kLogitThreads), 0, st, lg,
+                                              stride, mk, V, W, rows, (const float*)lse_rows, logprobs + (size_t)r0 * V)
+                                 : launch_pdl(logprobs_kernel<BF16, false>, dim3(g2), dim3(kLogitThreads), 0, st, lg,
+                                              stride, mk, V, W, rows, (const float*)lse_rows, logprobs + (size_t)r0 * V);
+            if (e1 != cudaSuccess) return e1;
         } else {
-            logits_reduce_kernel<BF16, STAGE, false><<<grid, kLogitThreads, 0, st>>>(
-                lg, stride, mk, V, W, rows, per_cta, partials, counters, argmax + r0, lse_rows);
+            cudaError_t e0 = launch_pdl(logits_reduce_kernel<BF16, STAGE, false>, dim3(grid), dim3(kReduceThreads), 0,
+                                        st, lg, stride, mk, V, W, rows, per_cta, partials, counters, argmax + r0,
+                                        lse_rows);
+            if (e0 != cudaSuccess) return e0;
         }
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
@@ -918,16 +1034,16 @@ cudaError_t launch_advance_s(const StepView& v, int mode, const int32_t* states,
     const unsigned grid = (unsigned)((batch + kAdvanceThreads - 1) / kAdvanceThreads);
     switch (mode) {
         case kSparse32Smem:
-            advance_kernel<STACK, kSparse32Smem><<<grid, kAdvanceThreads, 0, st>>>(v, states, stacks, tokens, batch,
-                                                                                 states_out, stacks_out);
+            return launch_pdl(advance_kernel<STACK, kSparse32Smem>, dim3(grid), dim3(kAdvanceThreads), 0, st, v, states,
+                              stacks, tokens, batch, states_out, stacks_out);
             break;
         case kSparse64Smem:
-            advance_kernel<STACK, kSparse64Smem><<<grid, kAdvanceThreads, 0, st>>>(v, states, stacks, tokens, batch,
-                                                                                 states_out, stacks_out);
+            return launch_pdl(advance_kernel<STACK, kSparse64Smem>, dim3(grid), dim3(kAdvanceThreads), 0, st, v, states,
+                              stacks, tokens, batch, states_out, stacks_out);
             break;
         default:
-            advance_kernel<STACK, kDenseGlobal><<<grid, kAdvanceThreads, 0, st>>>(v, states, stacks, tokens, batch,
-                                                                                states_out, stacks_out);
+            return launch_pdl(advance_kernel<STACK, kDenseGlobal>, dim3(grid), dim3(kAdvanceThreads), 0, st, v, states,
+                              stacks, tokens, batch, states_out, stacks_out);
     }
     return cudaGetLastError();
 }
