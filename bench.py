@@ -35,7 +35,7 @@ METRIC = "token-checks/s and masked decode steps/s at 1 GB300; mask+logits HBM G
 UNIT = "token-checks/s"
 L2_BYTES = 129 * 1024 * 1024
 WORKLOAD_HELP = {1: "kv16_v1024_b1", 2: "kv200_v32000_b32", 3: "sparse5000_v128256_b256",
-                 5: "json300_pda_v152064_b128"}
+                 4: "precompute_sparse20000_v128256", 5: "json300_pda_v152064_b128"}
 
 
 def parse():
@@ -259,6 +259,8 @@ def run_reference(args, dist: Dist):
     w = synth.workload(args.workload)
     cores = cpu_cores()
     P = oracle.Problem.from_workload(w)
+    if w.config == 4:
+        return run_reference_precompute(args, w, P, cores)
     states, stacks = w.initial_configs()
     V = w.vocab.n_tokens
     rows = min(w.batch, max(1, cores))
@@ -289,6 +291,148 @@ def run_reference(args, dist: Dist):
                              "sample": f"{rows} of {w.batch} rows per step, full vocabulary"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+
+
+def precompute_sample(w, P, rows: int, cores: int, step: int = 0):
+    """The oracle's state x token table for `rows` states (next states and mask)."""
+    Q = w.automaton.n_states
+    states = ((np.arange(rows, dtype=np.int64) * 7919 + step * rows) % Q).astype(np.int32)
+    P.step_mask(states, None, want_next=True, n_threads=cores)
+
+
+def cpu_baseline_precompute(w, target_s: float):
+    import oracle
+    cores = cpu_cores()
+    P = oracle.Problem.from_workload(w)
+    rows = max(1, cores)
+    t0 = time.perf_counter()
+    precompute_sample(w, P, rows, cores)
+    reps = max(1, int(target_s / max(time.perf_counter() - t0, 1e-3)))
+    t0 = time.perf_counter()
+    for r in range(reps):
+        precompute_sample(w, P, rows, cores, r + 1)
+    dt = time.perf_counter() - t0
+    return {"value": rows * w.vocab.n_tokens * reps / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{reps} x {rows} of the {w.automaton.n_states} table rows (next states + mask), "
+                      f"OpenMP over rows"}
+
+
+def run_reference_precompute(args, w, P, cores):
+    V, Q = w.vocab.n_tokens, w.automaton.n_states
+    rows = max(1, cores)
+    t0 = time.perf_counter()
+    precompute_sample(w, P, rows, cores)
+    per = time.perf_counter() - t0
+    budget = 120.0 / max(1, args.steps + args.warmup)
+    rows = max(1, min(Q, int(rows * budget / max(per, 1e-4))))
+    for i in range(args.warmup):
+        precompute_sample(w, P, rows, cores, i)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        precompute_sample(w, P, rows, cores, i)
+    dt = time.perf_counter() - t0
+    value = rows * V * args.steps / dt
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3 / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int32",
+            "data": "synthetic", "config": {"workload": w.name, "states": Q, "vocab": V,
+                                            "sample_rows_per_step": rows},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": f"{rows} of {Q} table rows per step, full vocabulary"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_precompute(args, dist: Dist):
+    """Config 4: one step = the whole state x token table (next states int32 [Q][V] + mask)."""
+    import torch
+
+    from paper_2403_06988_gb300 import Domino, synth
+    from paper_2403_06988_gb300 import _binding as B
+
+    dev_id = dist.local
+    torch.cuda.set_device(dev_id)
+    dev = f"cuda:{dev_id}"
+    w = synth.workload(4)
+    d = Domino.from_parts(w.automaton, w.vocab, device=dev_id)
+    info = d.info()
+    Q, V, Wd = info["n_states"], info["n_tokens"], info["n_words"]
+    nxt = torch.empty((Q, V), dtype=torch.int32, device=dev)
+    mask = torch.empty((Q, Wd), dtype=torch.int32, device=dev)
+    L, h = B.lib(), d.h
+    p_n, p_m = nxt.data_ptr(), mask.data_ptr()
+    s = torch.cuda.Stream(device=dev)
+    K, Wm = args.steps, args.warmup
+
+    def step(i, sp):
+        if L.domino_precompute_table(h, p_n, p_m, sp):
+            raise RuntimeError("precompute failed")
+    with torch.cuda.stream(s):
+        for i in range(Wm):
+            step(i, s.cuda_stream)
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(dev_id)
+    dist.barrier()
+    torch.cuda.synchronize()
+    sampler.start()
+    with torch.cuda.stream(s):           # one launch per step, each far longer than a launch
+        t0.record()
+        for i in range(K):
+            step(i, s.cuda_stream)
+        t1.record()
+    torch.cuda.synchronize()
+    sampler.stop()
+    dist.barrier()
+    ms = dist.max(t0.elapsed_time(t1))
+    if d.device_error():
+        raise RuntimeError("device error word set")
+    # end to end: the table computed and read back into pinned host memory
+    host_n = torch.empty((Q, V), dtype=torch.int32).pin_memory()
+    host_m = torch.empty((Q, Wd), dtype=torch.int32).pin_memory()
+    Ke = max(1, min(2, K))
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    dist.barrier()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(s):
+        e0.record()
+        for i in range(Ke):
+            step(i, s.cuda_stream)
+            host_n.copy_(nxt, non_blocking=True)
+            host_m.copy_(mask, non_blocking=True)
+        e1.record()
+    torch.cuda.synchronize()
+    e2e_ms = dist.max(e0.elapsed_time(e1))
+    n = dist.world
+    out_bytes = Q * V * 4 + Q * Wd * 4
+    t = ms / K / 1e3
+    peaks, peak_kind = measured_peaks()
+    hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
+    traffic = ncu_traffic(w.name)
+    line = {
+        "metric": METRIC, "value": n * Q * V * K / (ms / 1e3), "unit": UNIT, "n_gpus": n, "steps": K,
+        "warmup": Wm, "ms_per_step": ms / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "int32", "data": "synthetic",
+        "config": {"workload": w.name, "states": Q, "vocab": V, "byte_classes": info["n_classes"],
+                   "table_in_smem": info["table_in_smem"], "output_bytes": out_bytes,
+                   "l2": f"each step writes {out_bytes / 2**30:.1f} GiB (> L2)", "parallelism": f"replicas x{n}"},
+        "roofline": {"kernel": "step_mask (row = state, next states written)", "bound": "hbm",
+                     "achieved": out_bytes / t / 1e9, "peak": hbm_peak, "unit": "GB/s",
+                     "frac": out_bytes / t / 1e9 / hbm_peak, "traffic": traffic.get("precompute"),
+                     "algorithmic_units_per_launch": out_bytes, "peak_source": f"hbm_gbs {peak_kind}"},
+        "e2e": {"value": n * Q * V * Ke / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": out_bytes, "steps": Ke,
+                "api": "domino_precompute_table + copy of the table to pinned host memory"},
+        "gpu_launches": K,
+        "clocks": sampler.summary(),
+    }
+    if dist.rank == 0 and n == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline_precompute(w, args.cpu_seconds)
+    if dist.rank == 0:
+        print(json.dumps(line), flush=True)
+    d.close()
 
 
 # ----------------------------------------------------------------------------
@@ -519,6 +663,8 @@ def main():
     try:
         if args.impl == "reference":
             run_reference(args, dist)
+        elif args.workload == 4:
+            run_precompute(args, dist)
         else:
             run_domino(args, dist)
     finally:

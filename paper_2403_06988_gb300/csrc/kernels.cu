@@ -842,8 +842,16 @@ __global__ void __launch_bounds__(kAdvanceThreads)
 // ---------------------------------------------------------------------------
 // Rows per tile: as many as possible (<= 32, one ballot) while the tiles
 // still split evenly over one CTA per SM.
-int rows_per_tile(const StepView& v, const LaunchEnv& env, int batch, bool next) {
-    if (next) return kRowsPerTileNext;
+// With next states, the [R][1024] staging tile of next states decides: as many
+// rows as shared memory holds (the table placement was chosen for R = 8).
+int rows_per_tile(const StepView& v, const LaunchEnv& env, int batch, bool next, bool stack, int img_bytes) {
+    if (next) {
+        for (int R = kMaxRowsPerTile; R > kRowsPerTileNext; R >>= 1)
+            if (step_layout(v.K, R, true, stack, v.max_units, v.Q, img_bytes).total <= env.max_smem_optin &&
+                (long long)((batch + R - 1) / R) * v.n_windows >= 4LL * env.num_sms)
+                return R;
+        return kRowsPerTileNext;
+    }
     int best = kRowsPerTile;
     double best_waste = 1e9;
     for (int R = kMaxRowsPerTile; R >= kRowsPerTile; R -= 4) {
@@ -863,7 +871,7 @@ template <bool STACK, int MODE, bool NEXT>
 cudaError_t launch_step_t(const StepView& v, const LaunchEnv& env, const int32_t* states, const uint64_t* stacks,
                           int32_t batch, bool row_is_state, uint32_t* mask, int32_t* next, cudaStream_t st) {
     const int img_bytes = MODE == kDenseGlobal ? 0 : (int)table_smem_bytes(v, STACK, MODE);
-    const int R = rows_per_tile(v, env, batch, NEXT);
+    const int R = rows_per_tile(v, env, batch, NEXT, STACK, img_bytes);
     const StepLayout L = step_layout(v.K, R, NEXT, STACK, v.max_units, v.Q, img_bytes);
     auto kern = step_kernel<STACK, MODE, NEXT>;
     // the dynamic shared-memory limit is raised once per device and size, so
