@@ -488,6 +488,7 @@ def run_domino(args, dist: Dist):
             raise RuntimeError(f"domino call failed ({rc})")
 
     K, Wm = args.steps, args.warmup
+    n_world = dist.world
     s = torch.cuda.Stream(device=dev)
     with torch.cuda.stream(s):
         sp = s.cuda_stream
@@ -564,6 +565,49 @@ def run_domino(args, dist: Dist):
         del g
     if d.device_error():
         raise RuntimeError("device error after the per-kernel graphs")
+
+    # ---- table-driven step (DFA only): masks and next states precomputed once
+    # for every state, then per step a mask-row lookup fused into the logits
+    # pass and one table read per sequence for the update
+    table_step = None
+    if not stack:
+        Q = info["n_states"]
+        t_next = torch.empty((Q, V), dtype=torch.int32, device=dev)
+        t_mask = torch.empty((Q, Wd), dtype=torch.int32, device=dev)
+        p_tn, p_tm = t_next.data_ptr(), t_mask.data_ptr()
+        pc0 = torch.cuda.Event(enable_timing=True)
+        pc1 = torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(s):
+            L.domino_precompute_table(h, p_tn, p_tm, s.cuda_stream)   # warm
+            pc0.record()
+            if L.domino_precompute_table(h, p_tn, p_tm, s.cuda_stream):
+                raise RuntimeError("precompute failed")
+            pc1.record()
+        torch.cuda.synchronize()
+        st_tab = torch.from_numpy(states0).to(dev)
+        p_st_tab = st_tab.data_ptr()
+
+        def t_step(i, sp):
+            rc = L.domino_mask_logits_table(h, p_logits[i % nbuf], dtype_code, Bsz, V, p_tm, p_st_tab, p_arg, p_lse,
+                                            p_lp, sp)
+            rc |= L.domino_advance_table(h, p_tn, p_st_tab, p_arg, Bsz, p_st_tab, sp)
+            if rc:
+                raise RuntimeError(f"table step failed ({rc})")
+        with torch.cuda.stream(s):
+            for i in range(Wm):
+                t_step(i, s.cuda_stream)
+        torch.cuda.synchronize()
+        g = capture(K, t_step)
+        ms_t = dist.max(timed(K, t_step, g))
+        del g
+        if d.device_error():
+            raise RuntimeError("device error in the table-driven step")
+        table_step = {"ms_per_step": ms_t / K, "token_checks_per_s": n_world * Bsz * V * K / (ms_t / 1e3),
+                      "masked_decode_steps_per_s": n_world * K / (ms_t / 1e3),
+                      "precompute_ms": pc0.elapsed_time(pc1), "table_bytes": Q * V * 4 + Q * Wd * 4,
+                      "note": "mask rows looked up from the precomputed [Q][W] table inside the logits pass; "
+                              "update = one read of next[s][t]"}
+        del t_next, t_mask
 
     # ---- end to end through the host-buffer C entry point -------------------
     Ke = max(3, min(args.e2e_steps, K))
@@ -643,7 +687,7 @@ def run_domino(args, dist: Dist):
                    "l2": f"logits rotate over {nbuf} buffers ({nbuf * logit_bytes / 2**20:.0f} MiB > 2x L2)",
                    "parallelism": f"replicas x{n}", "graph": graph is not None},
         "masked_decode_steps_per_s": n * K / (ms_max / 1e3),
-        "kernels": kernels, "roofline": roofline,
+        "kernels": kernels, "roofline": roofline, "table_driven_step": table_step,
         "e2e": {"value": n * Bsz * V * Ke / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "steps": Ke, "api": "domino_decode_step_host (pinned host buffers)"},
         "gpu_launches": K * launches_per_step,

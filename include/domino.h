@@ -181,6 +181,26 @@ int domino_mask_logits(domino_t h, const void* logits_dev, int32_t dtype, int32_
 int domino_advance(domino_t h, const int32_t* states_dev, const uint64_t* stacks_dev, const int32_t* tokens_dev,
                    int32_t batch, int32_t* states_out, uint64_t* stacks_out, void* stream);
 
+/* Table-driven decode step, mask and decode (Sec. 3.5: the per-state masks
+ * are computed before inference starts and looked up while decoding).  The
+ * same fused masked argmax / lse / log-probs as domino_mask_logits, with row
+ * b's mask taken from row states_dev[b] of table_mask_dev, the [Q][W] mask
+ * table written by domino_precompute_table for this handle's automaton and
+ * vocabulary.  A state outside [0, Q) reads as an empty row (argmax -1) and
+ * sets DOMINO_DEVERR_BAD_STATE.  Pushdown automata: DOMINO_E_UNSUPPORTED
+ * (their masks depend on the stack).  Uses the handle's scratch memory. */
+int domino_mask_logits_table(domino_t h, const void* logits_dev, int32_t dtype, int32_t batch,
+                             int64_t row_stride_elems, const uint32_t* table_mask_dev, const int32_t* states_dev,
+                             int32_t* argmax_dev, float* lse_dev, float* logprobs_dev, void* stream);
+
+/* Table-driven C.update() (Alg. 1): states_out[b] = table_next_dev[s][t] for
+ * s = states_dev[b], t = tokens_dev[b], from the [Q][V] next-state table of
+ * domino_precompute_table (0 for a rejected token).  t < 0 or t == eos_id:
+ * the start state.  t >= V or s outside [0, Q): 0 and the device error word.
+ * states_out may alias states_dev.  Pushdown automata: DOMINO_E_UNSUPPORTED. */
+int domino_advance_table(domino_t h, const int32_t* table_next_dev, const int32_t* states_dev,
+                         const int32_t* tokens_dev, int32_t batch, int32_t* states_out, void* stream);
+
 /* One whole decode step from HOST memory (end-to-end use): copies logits
  * (batch rows of V values, dense) and the configurations to the device,
  * runs step_mask -> mask_logits -> advance, copies tokens_host[b] (the

@@ -102,5 +102,27 @@ class Domino:
         B.domino_advance(self.h, states, stacks, tokens, b, so, wo, stream)
         return so, wo
 
+    def mask_logits_table(self, logits, table_mask, states, want_lse: bool = True, want_logprobs: bool = False,
+                          stream=None) -> Tuple:
+        """Table-driven mask + decode: row b's mask is table_mask[states[b]] (DFA only)."""
+        import torch
+        b = logits.shape[0]
+        V = self.info()["n_tokens"]
+        dtype = DTYPE_BF16 if logits.dtype == torch.bfloat16 else DTYPE_F32
+        if logits.stride(1) != 1:
+            raise ValueError("logits rows must be contiguous")
+        argmax = torch.empty(b, dtype=torch.int32, device=logits.device)
+        lse = torch.empty(b, dtype=torch.float32, device=logits.device) if want_lse else None
+        lp = torch.empty((b, V), dtype=torch.float32, device=logits.device) if want_logprobs else None
+        B.domino_mask_logits_table(self.h, logits, dtype, b, logits.stride(0), table_mask, states, argmax, lse, lp,
+                                   stream)
+        return argmax, lse, lp
+
+    def advance_table(self, table_next, states, tokens, states_out=None, stream=None):
+        """Table-driven update: states_out[b] = table_next[states[b], tokens[b]] (DFA only)."""
+        so = states if states_out is None else states_out
+        B.domino_advance_table(self.h, table_next, states, tokens, states.shape[0], so, stream)
+        return so
+
     def device_error(self, stream=None) -> int:
         return B.domino_get_device_error(self.h, stream)

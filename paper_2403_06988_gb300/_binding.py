@@ -66,6 +66,8 @@ _SIGS = {
     "domino_decode_step_host": [P, P, I32, I32, P, P, P, P, P],
     "domino_get_device_error": [P, P, P],
     "domino_mask_logits_noalloc": [P, I32, I32, I32, I64, P, P, P, P, P],
+    "domino_mask_logits_table": [P, P, I32, I32, I64, P, P, P, P, P, P],
+    "domino_advance_table": [P, P, P, P, I32, P, P],
 }
 
 
@@ -202,6 +204,19 @@ def domino_advance(h: int, states_dev, stacks_dev, tokens_dev, batch: int, state
                    stream=None) -> None:
     _check("domino_advance", lib().domino_advance(h, _ptr(states_dev), _ptr(stacks_dev), _ptr(tokens_dev),
                                                    int(batch), _ptr(states_out), _ptr(stacks_out), _stream(stream)))
+
+
+def domino_mask_logits_table(h: int, logits_dev, dtype: int, batch: int, row_stride_elems: int, table_mask_dev,
+                             states_dev, argmax_dev, lse_dev=None, logprobs_dev=None, stream=None) -> None:
+    _check("domino_mask_logits_table", lib().domino_mask_logits_table(
+        h, _ptr(logits_dev), int(dtype), int(batch), int(row_stride_elems), _ptr(table_mask_dev), _ptr(states_dev),
+        _ptr(argmax_dev), _ptr(lse_dev), _ptr(logprobs_dev), _stream(stream)))
+
+
+def domino_advance_table(h: int, table_next_dev, states_dev, tokens_dev, batch: int, states_out, stream=None) -> None:
+    _check("domino_advance_table", lib().domino_advance_table(h, _ptr(table_next_dev), _ptr(states_dev),
+                                                               _ptr(tokens_dev), int(batch), _ptr(states_out),
+                                                               _stream(stream)))
 
 
 def domino_decode_step_host(h: int, logits_host, dtype: int, batch: int, states_host, stacks_host, tokens_host,

@@ -87,14 +87,21 @@ cudaError_t launch_step_mask(const StepView& v, const LaunchEnv& env, bool stack
                              const uint64_t* stacks, int32_t batch, bool row_is_state, uint32_t* mask,
                              int32_t* next, cudaStream_t st);
 
+// row_state (table-driven step): row r's mask is row row_state[r] of the
+// [Q][W] table `mask`; out-of-range states read as empty rows and set `err`.
 cudaError_t launch_mask_logits(const LaunchEnv& env, const void* logits, int dtype, int32_t batch,
                                int64_t row_stride, int32_t V, const uint32_t* mask, int32_t* argmax, float* lse,
                                float* logprobs, float4* partials, uint32_t* counters, float* lse_tmp,
-                               cudaStream_t st);
+                               cudaStream_t st, const int32_t* row_state = nullptr, int32_t Q = 0,
+                               uint32_t* err = nullptr);
 
 // `mode` names the table image the step kernel reads (it is L2-resident after a step).
 cudaError_t launch_advance(const StepView& v, bool stack, int mode, const int32_t* states, const uint64_t* stacks,
                            const int32_t* tokens, int32_t batch, int32_t* states_out, uint64_t* stacks_out,
                            cudaStream_t st);
+
+cudaError_t launch_advance_table(const int32_t* table_next, int32_t Q, int32_t V, int32_t eos_id, int32_t start,
+                                 const int32_t* states, const int32_t* tokens, int32_t batch, int32_t* states_out,
+                                 uint32_t* err, cudaStream_t st);
 
 }  // namespace domino

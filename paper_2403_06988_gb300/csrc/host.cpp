@@ -638,6 +638,36 @@ int domino_advance(domino_t h, const int32_t* states_dev, const uint64_t* stacks
                                       stacks_out, (cudaStream_t)stream));
 }
 
+int domino_mask_logits_table(domino_t h, const void* logits_dev, int32_t dtype, int32_t batch,
+                             int64_t row_stride_elems, const uint32_t* table_mask_dev, const int32_t* states_dev,
+                             int32_t* argmax_dev, float* lse_dev, float* logprobs_dev, void* stream) {
+    int rc = ready_for_compute(h);
+    if (rc) return rc;
+    if (h->stack) return DOMINO_E_UNSUPPORTED;
+    if (dtype != DOMINO_DTYPE_F32 && dtype != DOMINO_DTYPE_BF16) return DOMINO_E_INVALID_ARG;
+    if (batch < 0 || row_stride_elems < h->V) return DOMINO_E_INVALID_ARG;
+    if (batch == 0) return DOMINO_OK;
+    if (!logits_dev || !table_mask_dev || !states_dev || !argmax_dev) return DOMINO_E_INVALID_ARG;
+    DeviceGuard g(h->device);
+    return cuda_status(launch_mask_logits(h->env, logits_dev, dtype, batch, row_stride_elems, h->V, table_mask_dev,
+                                          argmax_dev, lse_dev, logprobs_dev, (float4*)h->d_partials.p,
+                                          (uint32_t*)h->d_counters.p, (float*)h->d_lse_tmp.p, (cudaStream_t)stream,
+                                          states_dev, h->Q, (uint32_t*)h->d_err.p));
+}
+
+int domino_advance_table(domino_t h, const int32_t* table_next_dev, const int32_t* states_dev,
+                         const int32_t* tokens_dev, int32_t batch, int32_t* states_out, void* stream) {
+    int rc = ready_for_compute(h);
+    if (rc) return rc;
+    if (h->stack) return DOMINO_E_UNSUPPORTED;
+    if (batch < 0) return DOMINO_E_INVALID_ARG;
+    if (batch == 0) return DOMINO_OK;
+    if (!table_next_dev || !states_dev || !tokens_dev || !states_out) return DOMINO_E_INVALID_ARG;
+    DeviceGuard g(h->device);
+    return cuda_status(launch_advance_table(table_next_dev, h->Q, h->V, h->eos_id, h->start, states_dev, tokens_dev,
+                                            batch, states_out, (uint32_t*)h->d_err.p, (cudaStream_t)stream));
+}
+
 int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, int32_t batch,
                             int32_t* states_host, uint64_t* stacks_host, int32_t* tokens_host, float* lse_host,
                             void* stream) {

@@ -612,6 +612,26 @@ __device__ __forceinline__ void cp_async_wait() {
 }
 
 constexpr int kReduceThreads = 32;            // one warp per CTA: no block barriers
+
+// Where row r's mask words are: row r of `base` ([batch][W]), or, for the
+// table-driven step, row states[r] of a precomputed [Q][W] state table.  An
+// out-of-range state reads as an all-zero row (nothing allowed) and sets the
+// error word.
+struct MaskRows {
+    const uint32_t* base;
+    const int32_t* row_state;   // nullptr: base is [batch][W]
+    int32_t Q;
+    uint32_t* err;
+    __device__ __forceinline__ const uint32_t* row(int r, int W, bool report) const {
+        if (!row_state) return base + (size_t)r * W;
+        const int32_t q = __ldg(row_state + r);
+        if (q < 0 || q >= Q) {
+            if (report) atomicOr(err, DOMINO_DEVERR_BAD_STATE);
+            return nullptr;
+        }
+        return base + (size_t)q * W;
+    }
+};
 constexpr int kStageDepth = 3;                // 32-word batches in flight per warp
 
 // Units are mask words (32 tokens); row r holds W units.  Each CTA takes a
@@ -625,7 +645,7 @@ constexpr int kStageDepth = 3;                // 32-word batches in flight per w
 // read on its own.
 template <bool BF16, bool STAGE, bool KEEP_L2>
 __global__ void __launch_bounds__(kReduceThreads)
-    logits_reduce_kernel(const void* __restrict__ logits, int64_t stride, const uint32_t* __restrict__ mask, int V,
+    logits_reduce_kernel(const void* __restrict__ logits, int64_t stride, const MaskRows mask, int V,
                          int W, int B, long long per_cta, float4* __restrict__ partials,
                          uint32_t* __restrict__ counters, int32_t* __restrict__ argmax, float* __restrict__ lse) {
     // [buffer][word][16-byte vector]
@@ -640,9 +660,9 @@ __global__ void __launch_bounds__(kReduceThreads)
         const int r = (int)(u / W);
         const long long row_end = (long long)(r + 1) * W;
         const long long seg_end = min(u_end, row_end);
-        const uint32_t* mrow = mask + (size_t)r * W;
-        const char* lrow = reinterpret_cast<const char*>(logits) + (size_t)r * stride * (BF16 ? 2 : 4);
         const int j0 = (int)(u - (long long)r * W), j1 = (int)(seg_end - (long long)r * W);
+        const uint32_t* mrow = mask.row(r, W, lane == 0 && j0 == 0);
+        const char* lrow = reinterpret_cast<const char*>(logits) + (size_t)r * stride * (BF16 ? 2 : 4);
         float m = -INFINITY, mL = -INFINITY, s = 0.0f;
         int idx = INT_MAX;
         if constexpr (STAGE) {
@@ -650,7 +670,7 @@ __global__ void __launch_bounds__(kReduceThreads)
             const int full_words = V / 32;       // words whose 64 bytes of logits lie inside the row
             auto mask_of = [&](int b) -> uint32_t {
                 const int j = j0 + 32 * b + lane;
-                return (b < nb && j < j1) ? __ldg(mrow + j) : 0u;
+                return (b < nb && j < j1 && mrow) ? __ldg(mrow + j) : 0u;
             };
             auto issue = [&](int b, uint32_t mw) {
                 if (b < nb) {
@@ -703,7 +723,7 @@ __global__ void __launch_bounds__(kReduceThreads)
             }
             cp_async_wait<0>();
         } else {
-            for (int j = j0 + lane; j < j1; j += 32) {
+            for (int j = j0 + lane; j < j1 && mrow; j += 32) {
                 uint32_t word = __ldg(mrow + j);
                 const int t0 = j * 32;
                 while (word) {
@@ -757,7 +777,7 @@ __global__ void __launch_bounds__(kReduceThreads)
 // stores per word; otherwise one token at a time.
 template <bool BF16, bool VEC>
 __global__ void __launch_bounds__(kLogitThreads)
-    logprobs_kernel(const void* __restrict__ logits, int64_t stride, const uint32_t* __restrict__ mask, int V, int W,
+    logprobs_kernel(const void* __restrict__ logits, int64_t stride, const MaskRows mask, int V, int W,
                     int B, const float* __restrict__ lse, float* __restrict__ out) {
     pdl_wait();
     pdl_trigger();
@@ -765,7 +785,8 @@ __global__ void __launch_bounds__(kLogitThreads)
     for (long long u = (long long)blockIdx.x * kLogitThreads + threadIdx.x; u < N;
          u += (long long)gridDim.x * kLogitThreads) {
         const int r = (int)(u / W), j = (int)(u - (long long)r * W);
-        const uint32_t word = __ldg(mask + u);
+        const uint32_t* mrow = mask.row(r, W, false);
+        const uint32_t word = mrow ? __ldg(mrow + j) : 0u;
         const char* lrow = reinterpret_cast<const char*>(logits) + (size_t)r * stride * (BF16 ? 2 : 4);
         float* orow = out + (size_t)r * V + (size_t)j * 32;
         const float l = __ldg(lse + r);
@@ -835,6 +856,31 @@ __global__ void __launch_bounds__(kAdvanceThreads)
     }
     states_out[b] = (int32_t)s;
     if (stacks_out) stacks_out[b] = ((uint64_t)depth << 32) | bits;
+}
+
+// Alg. 1 update from the precomputed state x token table: one read of
+// next[s][t] per sequence (EOS or -1: the start state; a rejected token's
+// entry is 0, the dead state).
+__global__ void __launch_bounds__(kAdvanceThreads)
+    advance_table_kernel(const int32_t* __restrict__ table_next, int32_t Q, int32_t V, int32_t eos_id, int32_t start,
+                         const int32_t* __restrict__ states, const int32_t* __restrict__ tokens, int32_t batch,
+                         int32_t* __restrict__ states_out, uint32_t* __restrict__ err) {
+    pdl_wait();
+    pdl_trigger();
+    const int b = blockIdx.x * kAdvanceThreads + threadIdx.x;
+    if (b >= batch) return;
+    const int32_t t = tokens[b];
+    int32_t s = 0;
+    if (t < 0 || t == eos_id) {
+        s = start;
+    } else if (t >= V) {
+        atomicOr(err, DOMINO_DEVERR_BAD_TOKEN);
+    } else {
+        const int32_t q = states[b];
+        if (q < 0 || q >= Q) atomicOr(err, DOMINO_DEVERR_BAD_STATE);
+        else s = __ldg(table_next + (size_t)q * V + t);
+    }
+    states_out[b] = s;
 }
 
 // ---------------------------------------------------------------------------
@@ -950,14 +996,16 @@ int occupancy(const void* kern, int threads) {
 
 template <bool BF16, bool STAGE>
 cudaError_t launch_logits_t(const LaunchEnv& env, const void* logits, int32_t batch, int64_t stride, int32_t V,
-                            const uint32_t* mask, int32_t* argmax, float* lse, float* logprobs, float4* partials,
+                            const MaskRows& mask, int32_t* argmax, float* lse, float* logprobs, float4* partials,
                             uint32_t* counters, float* lse_tmp, bool out_vec, cudaStream_t st) {
     const int W = (V + 31) / 32;
     const size_t esz = BF16 ? 2 : 4;
     for (int32_t r0 = 0; r0 < batch; r0 += kMaxLogitRows) {
         const int rows = min(kMaxLogitRows, batch - r0);
         const void* lg = reinterpret_cast<const char*>(logits) + (size_t)r0 * stride * esz;
-        const uint32_t* mk = mask + (size_t)r0 * W;
+        MaskRows mk = mask;
+        if (mk.row_state) mk.row_state += r0;
+        else mk.base += (size_t)r0 * W;
         float* lse_rows = lse ? lse + r0 : (logprobs ? lse_tmp : nullptr);
         const long long N = (long long)rows * W;
         int grid = env.num_sms * (logprobs ? occupancy((const void*)logits_reduce_kernel<BF16, STAGE, true>, kReduceThreads)
@@ -1020,18 +1068,19 @@ cudaError_t launch_step_mask(const StepView& v, const LaunchEnv& env, bool stack
 cudaError_t launch_mask_logits(const LaunchEnv& env, const void* logits, int dtype, int32_t batch,
                                int64_t row_stride, int32_t V, const uint32_t* mask, int32_t* argmax, float* lse,
                                float* logprobs, float4* partials, uint32_t* counters, float* lse_tmp,
-                               cudaStream_t st) {
+                               cudaStream_t st, const int32_t* row_state, int32_t Q, uint32_t* err) {
+    const MaskRows mr{mask, row_state, Q, err};
     const bool bf16 = dtype == DOMINO_DTYPE_BF16;
     const bool out_vec = logprobs && (reinterpret_cast<uintptr_t>(logprobs) % 16 == 0) && (V % 4 == 0);
     if (bf16) {
         const bool stage = (reinterpret_cast<uintptr_t>(logits) % 16 == 0) && ((size_t)row_stride * 2) % 16 == 0;
         if (stage)
-            return launch_logits_t<true, true>(env, logits, batch, row_stride, V, mask, argmax, lse, logprobs,
+            return launch_logits_t<true, true>(env, logits, batch, row_stride, V, mr, argmax, lse, logprobs,
                                                partials, counters, lse_tmp, out_vec, st);
-        return launch_logits_t<true, false>(env, logits, batch, row_stride, V, mask, argmax, lse, logprobs, partials,
+        return launch_logits_t<true, false>(env, logits, batch, row_stride, V, mr, argmax, lse, logprobs, partials,
                                             counters, lse_tmp, out_vec, st);
     }
-    return launch_logits_t<false, false>(env, logits, batch, row_stride, V, mask, argmax, lse, logprobs, partials,
+    return launch_logits_t<false, false>(env, logits, batch, row_stride, V, mr, argmax, lse, logprobs, partials,
                                          counters, lse_tmp, out_vec, st);
 }
 
@@ -1061,6 +1110,14 @@ cudaError_t launch_advance(const StepView& v, bool stack, int mode, const int32_
                            cudaStream_t st) {
     if (stack) return launch_advance_s<true>(v, mode, states, stacks, tokens, batch, states_out, stacks_out, st);
     return launch_advance_s<false>(v, mode, states, stacks, tokens, batch, states_out, stacks_out, st);
+}
+
+cudaError_t launch_advance_table(const int32_t* table_next, int32_t Q, int32_t V, int32_t eos_id, int32_t start,
+                                 const int32_t* states, const int32_t* tokens, int32_t batch, int32_t* states_out,
+                                 uint32_t* err, cudaStream_t st) {
+    const unsigned grid = (unsigned)((batch + kAdvanceThreads - 1) / kAdvanceThreads);
+    return launch_pdl(advance_table_kernel, dim3(grid), dim3(kAdvanceThreads), 0, st, table_next, Q, V, eos_id, start,
+                      states, tokens, batch, states_out, err);
 }
 
 }  // namespace domino
