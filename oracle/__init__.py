@@ -66,6 +66,13 @@ def lib():
                                          P, P, ctypes.c_int32]
         L.oracle_walk_steps.restype = ctypes.c_int64
         L.oracle_walk_steps.argtypes = [P, P, P, ctypes.c_int32, ctypes.c_int32]
+        L.oracle_philox4x32_10.restype = None
+        L.oracle_philox4x32_10.argtypes = [P, ctypes.c_uint32, ctypes.c_uint32]
+        L.oracle_ln_f32.restype = ctypes.c_float
+        L.oracle_ln_f32.argtypes = [ctypes.c_float]
+        L.oracle_mask_sample.restype = None
+        L.oracle_mask_sample.argtypes = [P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64, P,
+                                         ctypes.c_float, ctypes.c_uint64, ctypes.c_uint64, P, ctypes.c_int32]
         L.oracle_advance.restype = ctypes.c_int64
         L.oracle_advance.argtypes = [P, P, P, P, ctypes.c_int32, ctypes.c_int32, P, P]
         _lib = L
@@ -174,6 +181,32 @@ def mask_logits(logits: np.ndarray, mask: np.ndarray, n_tokens: Optional[int] = 
     lib().oracle_mask_logits(_ptr(logits), dtype, B, V, stride, _ptr(mask), _ptr(arg), _ptr(lse), _ptr(lp),
                              int(n_threads))
     return arg, lse, lp
+
+
+def philox4x32_10(ctr, key0: int, key1: int) -> np.ndarray:
+    """Philox4x32-10 of one 4-word counter."""
+    c = np.ascontiguousarray(np.asarray(ctr, dtype=np.uint32).copy())
+    lib().oracle_philox4x32_10(_ptr(c), int(key0) & 0xFFFFFFFF, int(key1) & 0xFFFFFFFF)
+    return c
+
+
+def ln_f32(x: float) -> float:
+    return float(lib().oracle_ln_f32(float(x)))
+
+
+def mask_sample(logits: np.ndarray, mask: np.ndarray, temperature: float, seed: int, offset: int,
+                n_tokens: Optional[int] = None, n_threads: int = 1) -> np.ndarray:
+    """Gumbel-max draw per row over the allowed tokens (tokens int32 [batch], -1 when none)."""
+    batch = logits.shape[0]
+    V = logits.shape[1] if n_tokens is None else n_tokens
+    dtype = BF16 if logits.dtype == np.uint16 else F32
+    lg = np.ascontiguousarray(logits)
+    mask = np.ascontiguousarray(mask, dtype=np.uint32)
+    out = np.zeros(batch, dtype=np.int32)
+    lib().oracle_mask_sample(_ptr(lg), dtype, batch, V, lg.shape[1], _ptr(mask), float(temperature),
+                             int(seed) & 0xFFFFFFFFFFFFFFFF, int(offset) & 0xFFFFFFFFFFFFFFFF, _ptr(out),
+                             int(n_threads))
+    return out
 
 
 def bits_of(mask_row: np.ndarray, n_tokens: int) -> np.ndarray:

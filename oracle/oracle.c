@@ -252,6 +252,90 @@ void oracle_mask_logits(const void* logits, int32_t dtype, int32_t batch, int32_
     }
 }
 
+/* ---- sampling (Gumbel-max over the masked logits) ------------------------ */
+
+void oracle_philox4x32_10(uint32_t ctr[4], uint32_t key0, uint32_t key1) {
+    for (int round = 0; round < 10; round++) {
+        if (round > 0) {                          /* key schedule: add the Weyl constants */
+            key0 += 0x9E3779B9u;
+            key1 += 0xBB67AE85u;
+        }
+        uint64_t p0 = (uint64_t)0xD2511F53u * ctr[0];
+        uint64_t p1 = (uint64_t)0xCD9E8D57u * ctr[2];
+        uint32_t y0 = (uint32_t)(p1 >> 32) ^ ctr[1] ^ key0;
+        uint32_t y1 = (uint32_t)p1;
+        uint32_t y2 = (uint32_t)(p0 >> 32) ^ ctr[3] ^ key1;
+        uint32_t y3 = (uint32_t)p0;
+        ctr[0] = y0;
+        ctr[1] = y1;
+        ctr[2] = y2;
+        ctr[3] = y3;
+    }
+}
+
+float oracle_ln_f32(float x) {
+    uint32_t bits;
+    memcpy(&bits, &x, sizeof bits);
+    int32_t e = (int32_t)((bits >> 23) & 0xFFu) - 127;
+    uint32_t mb = (bits & 0x7FFFFFu) | 0x3F800000u;   /* mantissa in [1, 2) */
+    float m;
+    memcpy(&m, &mb, sizeof m);
+    if (m > 0x1.6a09e6p+0f) {                        /* move m into [sqrt(1/2), sqrt(2)) */
+        m = m * 0.5f;
+        e = e + 1;
+    }
+    float num = m - 1.0f;
+    float den = m + 1.0f;
+    float z = num / den;
+    float z2 = z * z;
+    float poly = 0x1.745d18p-4f;                    /* 1/11 */
+    poly = fmaf(poly, z2, 0x1.c71c72p-4f);           /* 1/9 */
+    poly = fmaf(poly, z2, 0x1.24924ap-3f);           /* 1/7 */
+    poly = fmaf(poly, z2, 0x1.99999ap-3f);           /* 1/5 */
+    poly = fmaf(poly, z2, 0x1.555556p-2f);           /* 1/3 */
+    poly = fmaf(poly, z2, 1.0f);
+    float two_z = z + z;
+    float r = two_z * poly;                          /* 2 atanh(z) = ln m */
+    float ef = (float)e;
+    float lo = fmaf(ef, -0x1.05c61p-29f, r);         /* e ln2 in two parts */
+    return fmaf(ef, 0x1.62e43p-1f, lo);
+}
+
+void oracle_mask_sample(const void* logits, int32_t dtype, int32_t batch, int32_t n_tokens, int64_t row_stride,
+                        const uint32_t* mask, float temperature, uint64_t seed, uint64_t offset, int32_t* tokens,
+                        int32_t n_threads) {
+    const int64_t W = ((int64_t)n_tokens + 31) / 32;
+    const float inv_t = 1.0f / temperature;
+    const uint32_t k0 = (uint32_t)seed, k1 = (uint32_t)(seed >> 32);
+#ifdef _OPENMP
+    if (n_threads < 1) n_threads = 1;
+#pragma omp parallel for schedule(dynamic, 1) num_threads(n_threads)
+#endif
+    for (int32_t b = 0; b < batch; b++) {
+        const uint32_t* mrow = mask + (int64_t)b * W;
+        const int64_t base = (int64_t)b * row_stride;
+        float best_score = -INFINITY;
+        int32_t best = -1;
+        for (int32_t t = 0; t < n_tokens; t++) {
+            if (!((mrow[t / 32] >> (t % 32)) & 1)) continue;
+            uint32_t c[4] = {(uint32_t)t / 4u, (uint32_t)b, (uint32_t)offset, (uint32_t)(offset >> 32)};
+            oracle_philox4x32_10(c, k0, k1);
+            uint32_t k = c[t % 4] >> 9;
+            float u = (float)(2u * k + 1u) * 0x1p-24f;       /* exact: an odd integer below 2^24 */
+            float e1 = -oracle_ln_f32(u);                    /* Exp(1) variate */
+            float g = -oracle_ln_f32(e1);                    /* Gumbel variate */
+            float x = (float)logit_value(logits, dtype, base + t);
+            float scaled = x * inv_t;
+            float score = scaled + g;
+            if (score > best_score) {
+                best_score = score;
+                best = t;
+            }
+        }
+        tokens[b] = best;
+    }
+}
+
 int64_t oracle_advance(const oracle_problem* p, const int32_t* states, const uint64_t* stacks,
                        const int32_t* tokens, int32_t batch, int32_t start_state, int32_t* states_out,
                        uint64_t* stacks_out) {

@@ -24,6 +24,11 @@
  *                 index on ties, log-sum-exp and log-probabilities in double.
  *   advance      (Alg. 1, C.update(o)): the chosen token's walk; EOS or "no
  *                 token" ends the sequence and the next one starts from init.
+ *   mask_sample  (Alg. 1, decode by sampling instead of the argmax): the
+ *                 Gumbel-max rule over the allowed tokens, with uniforms from
+ *                 the Philox4x32-10 counter-based generator (Salmon et al.,
+ *                 SC'11).  The score that decides the sample is formed in fp32
+ *                 with one fixed sequence of correctly rounded operations.
  *
  * All arrays are host memory owned by the caller.
  */
@@ -88,6 +93,28 @@ int64_t oracle_walk_steps(const oracle_problem* p, const int32_t* states, const 
 void oracle_mask_logits(const void* logits, int32_t dtype, int32_t batch, int32_t n_tokens,
                         int64_t row_stride, const uint32_t* mask, int32_t* argmax, double* lse,
                         double* logprobs, int32_t n_threads);
+
+/* Philox4x32-10: ten rounds on the 128-bit counter ctr under the 64-bit key
+ * (key0, key1); the four output words replace ctr. */
+void oracle_philox4x32_10(uint32_t ctr[4], uint32_t key0, uint32_t key1);
+
+/* Natural logarithm of a positive normal float: x = 2^e m with m in
+ * [sqrt(1/2), sqrt(2)), ln x = e ln 2 + 2 atanh((m - 1) / (m + 1)), atanh by
+ * its odd power series to the z^11 term, every step a correctly rounded fp32
+ * operation. */
+float oracle_ln_f32(float x);
+
+/* Sampling decode (Alg. 1 with the greedy argmax replaced by a draw from the
+ * masked softmax at temperature T): tokens[b] = argmax over allowed t of
+ * x_t * (1/T) + g_t, lowest index on ties, -1 when nothing is allowed.
+ * g_t = -ln(-ln(u_t)) (a Gumbel variate, so the argmax is distributed as
+ * softmax(x / T) over the allowed tokens); u_t = (2k + 1) / 2^24 with
+ * k = w >> 9 and w word (t mod 4) of Philox4x32-10 on the counter
+ * (t / 4, b, offset low, offset high) under the key (seed low, seed high).
+ * All arithmetic of the score is fp32.  temperature > 0. */
+void oracle_mask_sample(const void* logits, int32_t dtype, int32_t batch, int32_t n_tokens, int64_t row_stride,
+                        const uint32_t* mask, float temperature, uint64_t seed, uint64_t offset, int32_t* tokens,
+                        int32_t n_threads);
 
 /* Alg. 1 update: states_out/stacks_out may alias the inputs.  tokens[b] < 0 or
  * == eos_id: (start_state, empty).  A rejected token: (0, empty).  A token id

@@ -28,7 +28,13 @@ MUTANTS = {
     "bf16_wrong_shift": ("((const uint16_t*)logits)[i] << 16;", "((const uint16_t*)logits)[i] << 15;"),
     "stack_top_at_wrong_end": ("(uint8_t)((bits >> (st->depth - 1 - i)) & 1);", "(uint8_t)((bits >> i) & 1);"),
     "advance_eos_keeps_state": ("s_out = start_state;", "s_out = s;"),
+    "gumbel_sign_flipped": ("float g = -oracle_ln_f32(e1);", "float g = oracle_ln_f32(e1);"),
+    "temperature_multiplies": ("const float inv_t = 1.0f / temperature;", "const float inv_t = temperature;"),
+    "philox_word_ignores_token": ("uint32_t k = c[t % 4] >> 9;", "uint32_t k = c[0] >> 9;"),
+    "philox_rounds_short": ("for (int round = 0; round < 10; round++) {", "for (int round = 0; round < 9; round++) {"),
+    "ln_series_term_dropped": ("poly = fmaf(poly, z2, 0x1.99999ap-3f);           /* 1/5 */", "poly = poly;"),
 }
+PIN_FILES = ["test_oracle_pins.py", "test_oracle_sampling.py"]
 
 
 @pytest.mark.parametrize("name", sorted(MUTANTS))
@@ -45,6 +51,6 @@ def test_pins_catch_mutant(tmp_path, name):
                     "-lm"], check=True)
     env = dict(os.environ, DOMINO_ORACLE_SO=str(so))
     r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",
-                        os.path.join(ROOT, "tests", "test_oracle_pins.py")],
+                        *[os.path.join(ROOT, "tests", f) for f in PIN_FILES]],
                        cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
     assert r.returncode != 0, f"mutant {name} survived the pins:\n{r.stdout[-2000:]}"
