@@ -558,8 +558,13 @@ def run_domino(args, dist: Dist):
     def k_adv(i, sp):
         if L.domino_advance(h, p_states, p_stacks, p_arg, Bsz, p_st_tmp, p_sk_tmp, sp):
             raise RuntimeError("advance failed")
+    def k_sample(i, sp):
+        if L.domino_mask_sample(h, p_logits[i % nbuf], dtype_code, Bsz, V, p_mask, ctypes.c_float(1.0),
+                                ctypes.c_uint64(0x5EED), ctypes.c_uint64(i), p_arg, sp):
+            raise RuntimeError("mask_sample failed")
     per_kernel = {}
-    for name, body in (("step_mask", k_step), ("mask_logits", k_logits), ("advance", k_adv)):
+    for name, body in (("step_mask", k_step), ("mask_logits", k_logits), ("advance", k_adv),
+                       ("mask_sample", k_sample)):
         g = capture(Kk, body)
         per_kernel[name] = dist.max(timed(Kk, body, g)) / Kk      # ms per launch
         del g
@@ -657,6 +662,9 @@ def run_domino(args, dist: Dist):
         "step_mask": {"us": t_sm * 1e6, "checks_per_s": Bsz * V / t_sm, "mask_bytes": Bsz * Wd * 4,
                       "dram_bytes_ncu": traffic.get("step_mask")},
         "advance": {"us": per_kernel["advance"] * 1e3},
+        "mask_sample": {"us": per_kernel["mask_sample"] * 1e3,
+                        "gbs": (lg_bytes - Bsz * V * 4 * w.want_logprobs - Bsz * 4) / (per_kernel["mask_sample"] * 1e-3)
+                        / 1e9, "note": "Gumbel-max draw at T = 1 over the same masks (Philox per 4 allowed tokens)"},
         "timing": f"each kernel alone, {Kk} launches back to back in one CUDA graph, events on its stream",
     }
     # transition-lookup peak: one conflict-free 32-lane shared-memory gather per

@@ -181,6 +181,22 @@ int domino_mask_logits(domino_t h, const void* logits_dev, int32_t dtype, int32_
 int domino_advance(domino_t h, const int32_t* states_dev, const uint64_t* stacks_dev, const int32_t* tokens_dev,
                    int32_t batch, int32_t* states_out, uint64_t* stacks_out, void* stream);
 
+/* Alg. 1 with the greedy decode replaced by sampling: tokens_dev[b] is a draw
+ * from softmax(logits / temperature) restricted to the allowed tokens of
+ * mask_dev row b (-1 when nothing is allowed), by the Gumbel-max rule:
+ * the argmax over allowed t of x_t * (1/T) + g_t, lowest index on ties, with
+ * g_t = -ln(-ln(u_t)), u_t = (2k + 1) / 2^24, k = w >> 9, w = word (t mod 4)
+ * of Philox4x32-10 (Salmon et al., SC'11) on the counter
+ * (t / 4, b, offset low, offset high) under the key (seed low, seed high).
+ * 1/T is one fp32 division and the score is formed with correctly rounded
+ * fp32 operations (ln by the atanh series), so draws are reproducible bit for
+ * bit by an independent implementation.  A caller passes a new offset per
+ * decode step.  temperature must be finite and > 0.  Same logits and mask
+ * layout as domino_mask_logits; uses the handle's scratch memory. */
+int domino_mask_sample(domino_t h, const void* logits_dev, int32_t dtype, int32_t batch, int64_t row_stride_elems,
+                       const uint32_t* mask_dev, float temperature, uint64_t seed, uint64_t offset,
+                       int32_t* tokens_dev, void* stream);
+
 /* Table-driven decode step, mask and decode (Sec. 3.5: the per-state masks
  * are computed before inference starts and looked up while decoding).  The
  * same fused masked argmax / lse / log-probs as domino_mask_logits, with row

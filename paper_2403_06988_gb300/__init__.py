@@ -102,6 +102,18 @@ class Domino:
         B.domino_advance(self.h, states, stacks, tokens, b, so, wo, stream)
         return so, wo
 
+    def mask_sample(self, logits, mask, temperature: float, seed: int, offset: int, stream=None):
+        """Gumbel-max draw per row from softmax(logits / T) over the allowed tokens (-1: none allowed)."""
+        import torch
+        b = logits.shape[0]
+        dtype = DTYPE_BF16 if logits.dtype == torch.bfloat16 else DTYPE_F32
+        if logits.stride(1) != 1:
+            raise ValueError("logits rows must be contiguous")
+        tokens = torch.empty(b, dtype=torch.int32, device=logits.device)
+        B.domino_mask_sample(self.h, logits, dtype, b, logits.stride(0), mask, temperature, seed, offset, tokens,
+                             stream)
+        return tokens
+
     def mask_logits_table(self, logits, table_mask, states, want_lse: bool = True, want_logprobs: bool = False,
                           stream=None) -> Tuple:
         """Table-driven mask + decode: row b's mask is table_mask[states[b]] (DFA only)."""

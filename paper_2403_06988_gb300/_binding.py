@@ -68,6 +68,7 @@ _SIGS = {
     "domino_mask_logits_noalloc": [P, I32, I32, I32, I64, P, P, P, P, P],
     "domino_mask_logits_table": [P, P, I32, I32, I64, P, P, P, P, P, P],
     "domino_advance_table": [P, P, P, P, I32, P, P],
+    "domino_mask_sample": [P, P, I32, I32, I64, P, ctypes.c_float, ctypes.c_uint64, ctypes.c_uint64, P, P],
 }
 
 
@@ -204,6 +205,13 @@ def domino_advance(h: int, states_dev, stacks_dev, tokens_dev, batch: int, state
                    stream=None) -> None:
     _check("domino_advance", lib().domino_advance(h, _ptr(states_dev), _ptr(stacks_dev), _ptr(tokens_dev),
                                                    int(batch), _ptr(states_out), _ptr(stacks_out), _stream(stream)))
+
+
+def domino_mask_sample(h: int, logits_dev, dtype: int, batch: int, row_stride_elems: int, mask_dev,
+                       temperature: float, seed: int, offset: int, tokens_dev, stream=None) -> None:
+    _check("domino_mask_sample", lib().domino_mask_sample(
+        h, _ptr(logits_dev), int(dtype), int(batch), int(row_stride_elems), _ptr(mask_dev), float(temperature),
+        int(seed) & 0xFFFFFFFFFFFFFFFF, int(offset) & 0xFFFFFFFFFFFFFFFF, _ptr(tokens_dev), _stream(stream)))
 
 
 def domino_mask_logits_table(h: int, logits_dev, dtype: int, batch: int, row_stride_elems: int, table_mask_dev,

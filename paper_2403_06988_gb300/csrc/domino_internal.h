@@ -87,13 +87,28 @@ cudaError_t launch_step_mask(const StepView& v, const LaunchEnv& env, bool stack
                              const uint64_t* stacks, int32_t batch, bool row_is_state, uint32_t* mask,
                              int32_t* next, cudaStream_t st);
 
+// Sampling decode: Gumbel-max with Philox4x32-10 uniforms (kernels.cu).
+struct SampleArgs {
+    uint32_t key0, key1;     // the 64-bit seed
+    uint32_t off0, off1;     // the 64-bit offset (counter words 2 and 3)
+    float inv_t;             // 1 / temperature, rounded to fp32
+};
+
 // row_state (table-driven step): row r's mask is row row_state[r] of the
 // [Q][W] table `mask`; out-of-range states read as empty rows and set `err`.
+// sample: draw each row's token (into argmax) instead of the greedy argmax;
+// lse and logprobs must then be null.
 cudaError_t launch_mask_logits(const LaunchEnv& env, const void* logits, int dtype, int32_t batch,
                                int64_t row_stride, int32_t V, const uint32_t* mask, int32_t* argmax, float* lse,
                                float* logprobs, float4* partials, uint32_t* counters, float* lse_tmp,
                                cudaStream_t st, const int32_t* row_state = nullptr, int32_t Q = 0,
-                               uint32_t* err = nullptr);
+                               uint32_t* err = nullptr, const SampleArgs* sample = nullptr);
+
+// Fills the sampling arguments (1/T in fp32, seed and offset words).
+cudaError_t launch_mask_sample(const LaunchEnv& env, const void* logits, int dtype, int32_t batch,
+                               int64_t row_stride, int32_t V, const uint32_t* mask, float temperature,
+                               uint64_t seed, uint64_t offset, int32_t* tokens, float4* partials,
+                               uint32_t* counters, cudaStream_t st);
 
 // `mode` names the table image the step kernel reads (it is L2-resident after a step).
 cudaError_t launch_advance(const StepView& v, bool stack, int mode, const int32_t* states, const uint64_t* stacks,

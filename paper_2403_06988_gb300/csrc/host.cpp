@@ -4,6 +4,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cmath>
 #include <cstdint>
 #include <cstring>
 #include <new>
@@ -636,6 +637,24 @@ int domino_advance(domino_t h, const int32_t* states_dev, const uint64_t* stacks
     const int mode = choose_mode(h, v, false);
     return cuda_status(launch_advance(v, h->stack, mode, states_dev, stacks_dev, tokens_dev, batch, states_out,
                                       stacks_out, (cudaStream_t)stream));
+}
+
+int domino_mask_sample(domino_t h, const void* logits_dev, int32_t dtype, int32_t batch, int64_t row_stride_elems,
+                       const uint32_t* mask_dev, float temperature, uint64_t seed, uint64_t offset,
+                       int32_t* tokens_dev, void* stream) {
+    if (!h) return DOMINO_E_INVALID_ARG;
+    if (is_host_only(h)) return DOMINO_E_NO_DEVICE;
+    if (!h->vocab_loaded) return DOMINO_E_NOT_LOADED;
+    if (dtype != DOMINO_DTYPE_F32 && dtype != DOMINO_DTYPE_BF16) return DOMINO_E_INVALID_ARG;
+    if (!(temperature > 0.0f) || !std::isfinite(temperature) || !std::isfinite(1.0f / temperature))
+        return DOMINO_E_INVALID_ARG;
+    if (batch < 0 || row_stride_elems < h->V) return DOMINO_E_INVALID_ARG;
+    if (batch == 0) return DOMINO_OK;
+    if (!logits_dev || !mask_dev || !tokens_dev) return DOMINO_E_INVALID_ARG;
+    DeviceGuard g(h->device);
+    return cuda_status(launch_mask_sample(h->env, logits_dev, dtype, batch, row_stride_elems, h->V, mask_dev,
+                                          temperature, seed, offset, tokens_dev, (float4*)h->d_partials.p,
+                                          (uint32_t*)h->d_counters.p, (cudaStream_t)stream));
 }
 
 int domino_mask_logits_table(domino_t h, const void* logits_dev, int32_t dtype, int32_t batch,

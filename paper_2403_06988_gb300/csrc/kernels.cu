@@ -549,14 +549,6 @@ __device__ __forceinline__ void block_merge(float& m, int& idx, float& s) {
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
-template <bool KEEP_L2>
-__device__ __forceinline__ uint4 ld_vec(const uint4* p) {
-    if constexpr (KEEP_L2) {
-        return __ldg(p);
-    } else {
-        return __ldcs(p);
-    }
-}
 
 template <bool BF16>
 __device__ __forceinline__ float logit_at(const void* row, int t) {
@@ -568,37 +560,6 @@ __device__ __forceinline__ float logit_at(const void* row, int t) {
     }
 }
 
-// Logits of the allowed tokens of mask word j of a row, handed to f(x, t) in
-// increasing t.  STAGE (bf16 rows on 16-byte boundaries): the word's 64 bytes
-// of logits are read as four 16-byte vectors (a vector with no allowed token is
-// not read) into this thread's shared-memory slot; otherwise, and for a partial
-// last word, each allowed logit is read on its own.
-template <bool BF16, bool STAGE, bool KEEP_L2, typename F>
-__device__ __forceinline__ void for_allowed(const char* lrow, uint32_t word, int j, int V, uint4* slot, F&& f) {
-    const int t0 = j * 32;
-    if (STAGE && t0 + 32 <= V) {
-        const uint4* src = reinterpret_cast<const uint4*>(lrow) + (size_t)j * 4;
-        uint4 d[4];
-#pragma unroll
-        for (int k = 0; k < 4; ++k)
-            if ((word >> (8 * k)) & 0xFFu) d[k] = ld_vec<KEEP_L2>(src + k);
-#pragma unroll
-        for (int k = 0; k < 4; ++k)
-            if ((word >> (8 * k)) & 0xFFu) slot[k] = d[k];
-        const unsigned short* st = reinterpret_cast<const unsigned short*>(slot);
-        while (word) {
-            const int e = __ffs(word) - 1;
-            word &= word - 1;
-            f(__uint_as_float((uint32_t)st[e] << 16), t0 + e);
-        }
-    } else {
-        while (word) {
-            const int e = __ffs(word) - 1;
-            word &= word - 1;
-            if (t0 + e < V) f(logit_at<BF16>(lrow, t0 + e), t0 + e);
-        }
-    }
-}
 
 // cp.async: 16 bytes global -> shared without a register round trip
 __device__ __forceinline__ void cp_async16(void* smem_dst, const void* gmem_src) {
@@ -612,6 +573,65 @@ __device__ __forceinline__ void cp_async_wait() {
 }
 
 constexpr int kReduceThreads = 32;            // one warp per CTA: no block barriers
+
+// ---- sampling: Gumbel-max over the allowed logits --------------------------
+// Philox4x32-10 (Salmon, Moraes, Dror and Shaw, SC'11): ten rounds of two
+// 32x32 -> 64-bit products on the counter, the key advanced by the Weyl
+// constants between rounds.
+__device__ __forceinline__ uint4 philox10(uint4 c, uint32_t k0, uint32_t k1) {
+#pragma unroll
+    for (int i = 0; i < 10; ++i) {
+        const uint32_t lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
+        const uint32_t lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
+        c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+        k0 += 0x9E3779B9u;
+        k1 += 0xBB67AE85u;
+    }
+    return c;
+}
+
+// ln(x) for a positive normal float: x = 2^e m, m in [sqrt(1/2), sqrt(2)),
+// ln x = e ln 2 + 2 atanh(z), z = (m - 1) / (m + 1), with atanh's odd power
+// series up to z^11.  Every operation is an explicitly rounded fp32 intrinsic
+// (no contraction), so the value is reproducible bit for bit.
+__device__ __forceinline__ float ln_rn(float x) {
+    const uint32_t bits = __float_as_uint(x);
+    int e = (int)((bits >> 23) & 0xFFu) - 127;
+    float m = __uint_as_float((bits & 0x7FFFFFu) | 0x3F800000u);
+    if (m > 0x1.6a09e6p+0f) {
+        m = __fmul_rn(m, 0.5f);
+        e += 1;
+    }
+    const float z = __fdiv_rn(__fsub_rn(m, 1.0f), __fadd_rn(m, 1.0f));
+    const float z2 = __fmul_rn(z, z);
+    float p = 0x1.745d18p-4f;
+    p = __fmaf_rn(p, z2, 0x1.c71c72p-4f);
+    p = __fmaf_rn(p, z2, 0x1.24924ap-3f);
+    p = __fmaf_rn(p, z2, 0x1.99999ap-3f);
+    p = __fmaf_rn(p, z2, 0x1.555556p-2f);
+    p = __fmaf_rn(p, z2, 1.0f);
+    const float r = __fmul_rn(__fadd_rn(z, z), p);
+    const float ef = __int2float_rn(e);
+    return __fmaf_rn(ef, 0x1.62e43p-1f, __fmaf_rn(ef, -0x1.05c61p-29f, r));
+}
+
+// Gumbel variate of token t of row r: g_t = -ln(-ln(u_t)), u_t = (2k + 1) / 2^24,
+// k = (word t % 4 of Philox on (t / 4, r, offset)) >> 9.  `blk` / `rnd` cache
+// the last Philox block.
+__device__ __forceinline__ float gumbel(const SampleArgs& a, int r, int t, int& blk, uint4& rnd) {
+    if ((t >> 2) != blk) {
+        blk = t >> 2;
+        rnd = philox10(make_uint4((uint32_t)blk, (uint32_t)r, a.off0, a.off1), a.key0, a.key1);
+    }
+    const uint32_t w = (t & 2) ? ((t & 1) ? rnd.w : rnd.z) : ((t & 1) ? rnd.y : rnd.x);
+    const float u = __fmul_rn(__uint2float_rn(2u * (w >> 9) + 1u), 0x1p-24f);
+    return -ln_rn(-ln_rn(u));
+}
+
+// Every g_t is below this: u_t <= 1 - 2^-24 gives -ln(u_t) >= 5.96e-8 and
+// g_t <= 16.64.  A token with x / T + kGumbelMax below the best score so far
+// cannot win (rounding is monotonic), so its variate is never drawn.
+constexpr float kGumbelMax = 17.0f;
 
 // Where row r's mask words are: row r of `base` ([batch][W]), or, for the
 // table-driven step, row states[r] of a precomputed [Q][W] state table.  An
@@ -639,15 +659,16 @@ constexpr int kStageDepth = 3;                // 32-word batches in flight per w
 // (max, argmax, sum) partials and the last one to finish combines them.
 // STAGE (bf16 rows on 16-byte boundaries): a warp takes 32 consecutive words
 // of its row at a time; the 16-byte logit vectors that hold an allowed token
-// are copied, fully coalesced, into the warp's double-buffered staging area
-// with cp.async (masks are read two batches ahead, logits one), and each lane
+// are copied, fully coalesced, into the warp's three-deep staging area
+// with cp.async (masks are read four batches ahead, logits two), and each lane
 // then folds its own word's allowed logits.  Otherwise each allowed logit is
 // read on its own.
-template <bool BF16, bool STAGE, bool KEEP_L2>
+template <bool BF16, bool STAGE, bool SAMPLE>
 __global__ void __launch_bounds__(kReduceThreads)
     logits_reduce_kernel(const void* __restrict__ logits, int64_t stride, const MaskRows mask, int V,
                          int W, int B, long long per_cta, float4* __restrict__ partials,
-                         uint32_t* __restrict__ counters, int32_t* __restrict__ argmax, float* __restrict__ lse) {
+                         uint32_t* __restrict__ counters, int32_t* __restrict__ argmax, float* __restrict__ lse,
+                         const SampleArgs sa, int row0) {
     // [buffer][word][16-byte vector]
     __shared__ __align__(16) uint4 stage[STAGE ? kStageDepth * 32 * 4 : 1];
     pdl_wait();
@@ -665,6 +686,22 @@ __global__ void __launch_bounds__(kReduceThreads)
         const char* lrow = reinterpret_cast<const char*>(logits) + (size_t)r * stride * (BF16 ? 2 : 4);
         float m = -INFINITY, mL = -INFINITY, s = 0.0f;
         int idx = INT_MAX;
+        int blk = -1;                       // Philox block cached by gumbel_score
+        uint4 rnd = make_uint4(0u, 0u, 0u, 0u);
+        // one allowed logit x of token t (t increasing within a lane)
+        auto fold = [&](float x, int t) {
+            if constexpr (SAMPLE) {
+                const float sx = __fmul_rn(x, sa.inv_t);
+                if (__fadd_rn(sx, kGumbelMax) < m) return;
+                const float sc = __fadd_rn(sx, gumbel(sa, row0 + r, t, blk, rnd));
+                if (sc > m) {
+                    m = sc;
+                    idx = t;
+                }
+            } else {
+                acc_add(m, mL, idx, s, x, t);
+            }
+        };
         if constexpr (STAGE) {
             const int nb = (j1 - j0 + 31) / 32;   // batches of 32 words
             const int full_words = V / 32;       // words whose 64 bytes of logits lie inside the row
@@ -706,13 +743,13 @@ __global__ void __launch_bounds__(kReduceThreads)
                         while (word) {
                             const int e = __ffs(word) - 1;
                             word &= word - 1;
-                            acc_add(m, mL, idx, s, __uint_as_float((uint32_t)st[e] << 16), t0 + e);
+                            fold(__uint_as_float((uint32_t)st[e] << 16), t0 + e);
                         }
                     } else {   // the row's partial last word
                         while (word) {
                             const int e = __ffs(word) - 1;
                             word &= word - 1;
-                            if (t0 + e < V) acc_add(m, mL, idx, s, logit_at<BF16>(lrow, t0 + e), t0 + e);
+                            if (t0 + e < V) fold(logit_at<BF16>(lrow, t0 + e), t0 + e);
                         }
                     }
                 }
@@ -729,7 +766,7 @@ __global__ void __launch_bounds__(kReduceThreads)
                 while (word) {
                     const int e = __ffs(word) - 1;
                     word &= word - 1;
-                    if (t0 + e < V) acc_add(m, mL, idx, s, logit_at<BF16>(lrow, t0 + e), t0 + e);
+                    if (t0 + e < V) fold(logit_at<BF16>(lrow, t0 + e), t0 + e);
                 }
             }
         }
@@ -770,44 +807,48 @@ __global__ void __launch_bounds__(kReduceThreads)
     }
 }
 
-// logprob[t] = logit[t] - lse for allowed t, -inf otherwise; one mask word (32
-// tokens) per thread, grid-stride over the batch x W words.  VEC: bf16 rows on
-// 16-byte boundaries and 16-byte aligned output rows (V % 4 == 0): four 16-byte
-// loads (skipped when no token of the vector is allowed) and eight float4
-// stores per word; otherwise one token at a time.
+// logprob[t] = logit[t] - lse for allowed t, -inf otherwise.  VEC (bf16 rows on
+// 16-byte boundaries, V % 4 == 0): a thread takes 4 consecutive tokens, reads
+// their 8 bytes of logits (not at all when none is allowed) and writes one
+// float4, so a warp's stores cover 512 contiguous bytes; grid-stride over the
+// batch x V/4 quads.  Otherwise one mask word (32 tokens) per thread, one token
+// at a time.
 template <bool BF16, bool VEC>
 __global__ void __launch_bounds__(kLogitThreads)
     logprobs_kernel(const void* __restrict__ logits, int64_t stride, const MaskRows mask, int V, int W,
                     int B, const float* __restrict__ lse, float* __restrict__ out) {
     pdl_wait();
     pdl_trigger();
-    const long long N = (long long)B * W;
-    for (long long u = (long long)blockIdx.x * kLogitThreads + threadIdx.x; u < N;
-         u += (long long)gridDim.x * kLogitThreads) {
-        const int r = (int)(u / W), j = (int)(u - (long long)r * W);
-        const uint32_t* mrow = mask.row(r, W, false);
-        const uint32_t word = mrow ? __ldg(mrow + j) : 0u;
-        const char* lrow = reinterpret_cast<const char*>(logits) + (size_t)r * stride * (BF16 ? 2 : 4);
-        float* orow = out + (size_t)r * V + (size_t)j * 32;
-        const float l = __ldg(lse + r);
-        if (VEC && BF16 && j * 32 + 32 <= V) {
-            const uint4* src = reinterpret_cast<const uint4*>(lrow) + (size_t)j * 4;
-            uint4 d[4];
-#pragma unroll
-            for (int k = 0; k < 4; ++k)
-                d[k] = ((word >> (8 * k)) & 0xFFu) ? __ldg(src + k) : make_uint4(0u, 0u, 0u, 0u);
-            float4* o4 = reinterpret_cast<float4*>(orow);
-#pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                const uint4& v8 = d[q >> 1];
-                const uint32_t w0 = (q & 1) ? v8.z : v8.x, w1 = (q & 1) ? v8.w : v8.y;
-                const float x[4] = {bf16_lo(w0), bf16_hi(w0), bf16_lo(w1), bf16_hi(w1)};
-                float o[4];
-#pragma unroll
-                for (int e = 0; e < 4; ++e) o[e] = ((word >> (4 * q + e)) & 1u) ? x[e] - l : -INFINITY;
-                __stcs(o4 + q, make_float4(o[0], o[1], o[2], o[3]));
+    if constexpr (VEC && BF16) {
+        const int nq = V / 4;
+        const long long N = (long long)B * nq;
+        for (long long u = (long long)blockIdx.x * kLogitThreads + threadIdx.x; u < N;
+             u += (long long)gridDim.x * kLogitThreads) {
+            const int r = (int)(u / nq), qd = (int)(u - (long long)r * nq);
+            const uint32_t* mrow = mask.row(r, W, false);
+            const uint32_t nib = mrow ? (__ldg(mrow + (qd >> 3)) >> (4 * (qd & 7))) & 0xFu : 0u;
+            float4 o = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+            if (nib) {
+                const char* lrow = reinterpret_cast<const char*>(logits) + (size_t)r * stride * 2;
+                const uint2 v = __ldcs(reinterpret_cast<const uint2*>(lrow) + qd);
+                const float l = __ldg(lse + r);
+                if (nib & 1u) o.x = bf16_lo(v.x) - l;
+                if (nib & 2u) o.y = bf16_hi(v.x) - l;
+                if (nib & 4u) o.z = bf16_lo(v.y) - l;
+                if (nib & 8u) o.w = bf16_hi(v.y) - l;
             }
-        } else {
+            __stcs(reinterpret_cast<float4*>(out + (size_t)r * V) + qd, o);
+        }
+    } else {
+        const long long N = (long long)B * W;
+        for (long long u = (long long)blockIdx.x * kLogitThreads + threadIdx.x; u < N;
+             u += (long long)gridDim.x * kLogitThreads) {
+            const int r = (int)(u / W), j = (int)(u - (long long)r * W);
+            const uint32_t* mrow = mask.row(r, W, false);
+            const uint32_t word = mrow ? __ldg(mrow + j) : 0u;
+            const char* lrow = reinterpret_cast<const char*>(logits) + (size_t)r * stride * (BF16 ? 2 : 4);
+            float* orow = out + (size_t)r * V + (size_t)j * 32;
+            const float l = __ldg(lse + r);
             for (int e = 0; e < 32 && j * 32 + e < V; ++e)
                 orow[e] = ((word >> e) & 1u) ? logit_at<BF16>(lrow, j * 32 + e) - l : -INFINITY;
         }
@@ -997,9 +1038,12 @@ int occupancy(const void* kern, int threads) {
 template <bool BF16, bool STAGE>
 cudaError_t launch_logits_t(const LaunchEnv& env, const void* logits, int32_t batch, int64_t stride, int32_t V,
                             const MaskRows& mask, int32_t* argmax, float* lse, float* logprobs, float4* partials,
-                            uint32_t* counters, float* lse_tmp, bool out_vec, cudaStream_t st) {
+                            uint32_t* counters, float* lse_tmp, bool out_vec, const SampleArgs* sample,
+                            cudaStream_t st) {
     const int W = (V + 31) / 32;
     const size_t esz = BF16 ? 2 : 4;
+    const SampleArgs sa = sample ? *sample : SampleArgs{0u, 0u, 0u, 0u, 1.0f};
+    auto reduce = sample ? logits_reduce_kernel<BF16, STAGE, true> : logits_reduce_kernel<BF16, STAGE, false>;
     for (int32_t r0 = 0; r0 < batch; r0 += kMaxLogitRows) {
         const int rows = min(kMaxLogitRows, batch - r0);
         const void* lg = reinterpret_cast<const char*>(logits) + (size_t)r0 * stride * esz;
@@ -1008,34 +1052,28 @@ cudaError_t launch_logits_t(const LaunchEnv& env, const void* logits, int32_t ba
         else mk.base += (size_t)r0 * W;
         float* lse_rows = lse ? lse + r0 : (logprobs ? lse_tmp : nullptr);
         const long long N = (long long)rows * W;
-        int grid = env.num_sms * (logprobs ? occupancy((const void*)logits_reduce_kernel<BF16, STAGE, true>, kReduceThreads)
-                                           : occupancy((const void*)logits_reduce_kernel<BF16, STAGE, false>, kReduceThreads));
+        int grid = env.num_sms * occupancy((const void*)reduce, kReduceThreads);
         grid = (int)std::min<long long>((long long)grid, (N + 127) / 128);   // at least 4 batches per warp
         grid = max(grid, 1);
         long long per_cta = (N + grid - 1) / grid;
         per_cta = std::max<long long>(per_cta, ((long long)W + kMaxSegments - 3) / (kMaxSegments - 2));
         grid = (int)((N + per_cta - 1) / per_cta);
+        // a sampling pass draws row r of this chunk with counter row r0 + r
+        cudaError_t e0 = launch_pdl(reduce, dim3(grid), dim3(kReduceThreads), 0, st, lg, stride, mk, V, W, rows,
+                                    per_cta, partials, counters, argmax + r0, lse_rows, sa, r0);
+        if (e0 != cudaSuccess) return e0;
         if (logprobs) {
-            cudaError_t e0 = launch_pdl(logits_reduce_kernel<BF16, STAGE, true>, dim3(grid), dim3(kReduceThreads), 0, st,
-                                        lg, stride, mk, V, W, rows, per_cta, partials, counters, argmax + r0,
-                                        lse_rows);
-            if (e0 != cudaSuccess) return e0;
+            const long long n_items = (out_vec && STAGE) ? (long long)rows * (V / 4) : N;
             int g2 = env.num_sms * occupancy((const void*)logprobs_kernel<BF16, true>, kLogitThreads);
-            g2 = (int)std::max<long long>(1, std::min<long long>((long long)g2, (N + kLogitThreads - 1) / kLogitThreads));
+            g2 = (int)std::max<long long>(1, std::min<long long>((long long)g2,
+                                                                 (n_items + kLogitThreads - 1) / kLogitThreads));
             cudaError_t e1 = (out_vec && STAGE)
                                  ? launch_pdl(logprobs_kernel<BF16, true>, dim3(g2), dim3(kLogitThreads), 0, st, lg,
                                               stride, mk, V, W, rows, (const float*)lse_rows, logprobs + (size_t)r0 * V)
                                  : launch_pdl(logprobs_kernel<BF16, false>, dim3(g2), dim3(kLogitThreads), 0, st, lg,
                                               stride, mk, V, W, rows, (const float*)lse_rows, logprobs + (size_t)r0 * V);
             if (e1 != cudaSuccess) return e1;
-        } else {
-            cudaError_t e0 = launch_pdl(logits_reduce_kernel<BF16, STAGE, false>, dim3(grid), dim3(kReduceThreads), 0,
-                                        st, lg, stride, mk, V, W, rows, per_cta, partials, counters, argmax + r0,
-                                        lse_rows);
-            if (e0 != cudaSuccess) return e0;
         }
-        cudaError_t e = cudaGetLastError();
-        if (e != cudaSuccess) return e;
     }
     return cudaSuccess;
 }
@@ -1068,7 +1106,8 @@ cudaError_t launch_step_mask(const StepView& v, const LaunchEnv& env, bool stack
 cudaError_t launch_mask_logits(const LaunchEnv& env, const void* logits, int dtype, int32_t batch,
                                int64_t row_stride, int32_t V, const uint32_t* mask, int32_t* argmax, float* lse,
                                float* logprobs, float4* partials, uint32_t* counters, float* lse_tmp,
-                               cudaStream_t st, const int32_t* row_state, int32_t Q, uint32_t* err) {
+                               cudaStream_t st, const int32_t* row_state, int32_t Q, uint32_t* err,
+                               const SampleArgs* sample) {
     const MaskRows mr{mask, row_state, Q, err};
     const bool bf16 = dtype == DOMINO_DTYPE_BF16;
     const bool out_vec = logprobs && (reinterpret_cast<uintptr_t>(logprobs) % 16 == 0) && (V % 4 == 0);
@@ -1076,12 +1115,22 @@ cudaError_t launch_mask_logits(const LaunchEnv& env, const void* logits, int dty
         const bool stage = (reinterpret_cast<uintptr_t>(logits) % 16 == 0) && ((size_t)row_stride * 2) % 16 == 0;
         if (stage)
             return launch_logits_t<true, true>(env, logits, batch, row_stride, V, mr, argmax, lse, logprobs,
-                                               partials, counters, lse_tmp, out_vec, st);
+                                               partials, counters, lse_tmp, out_vec, sample, st);
         return launch_logits_t<true, false>(env, logits, batch, row_stride, V, mr, argmax, lse, logprobs, partials,
-                                            counters, lse_tmp, out_vec, st);
+                                            counters, lse_tmp, out_vec, sample, st);
     }
     return launch_logits_t<false, false>(env, logits, batch, row_stride, V, mr, argmax, lse, logprobs, partials,
-                                         counters, lse_tmp, out_vec, st);
+                                         counters, lse_tmp, out_vec, sample, st);
+}
+
+cudaError_t launch_mask_sample(const LaunchEnv& env, const void* logits, int dtype, int32_t batch,
+                               int64_t row_stride, int32_t V, const uint32_t* mask, float temperature,
+                               uint64_t seed, uint64_t offset, int32_t* tokens, float4* partials,
+                               uint32_t* counters, cudaStream_t st) {
+    const SampleArgs sa{(uint32_t)seed, (uint32_t)(seed >> 32), (uint32_t)offset, (uint32_t)(offset >> 32),
+                        1.0f / temperature};   // one correctly rounded fp32 division
+    return launch_mask_logits(env, logits, dtype, batch, row_stride, V, mask, tokens, nullptr, nullptr, partials,
+                              counters, nullptr, st, nullptr, 0, nullptr, &sa);
 }
 
 template <bool STACK>
