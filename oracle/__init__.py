@@ -73,6 +73,15 @@ def lib():
         L.oracle_mask_sample.restype = None
         L.oracle_mask_sample.argtypes = [P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64, P,
                                          ctypes.c_float, ctypes.c_uint64, ctypes.c_uint64, P, ctypes.c_int32]
+        L.oracle_spec_new.restype = P
+        L.oracle_spec_new.argtypes = [P]
+        L.oracle_spec_free.argtypes = [P]
+        L.oracle_spec_update.restype = None
+        L.oracle_spec_update.argtypes = [P, P, P, P, ctypes.c_int32]
+        L.oracle_spec_propose.restype = None
+        L.oracle_spec_propose.argtypes = [P, P, P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, P, P, P, P]
+        L.oracle_spec_accept.restype = None
+        L.oracle_spec_accept.argtypes = [P, P, P, ctypes.c_int32, ctypes.c_int32, P]
         L.oracle_advance.restype = ctypes.c_int64
         L.oracle_advance.argtypes = [P, P, P, P, ctypes.c_int32, ctypes.c_int32, P, P]
         _lib = L
@@ -163,6 +172,49 @@ class Problem:
         bad = lib().oracle_advance(self._h, _ptr(states), _ptr(stacks), _ptr(tokens), B, int(start_state),
                                    _ptr(so), _ptr(wo))
         return so, wo, int(bad)
+
+
+class Spec:
+    """Count-based speculative proposals (Sec. 3.6) over a Problem's automaton."""
+
+    def __init__(self, problem: "Problem"):
+        self.problem = problem                    # keeps the automaton alive
+        self._h = lib().oracle_spec_new(problem._h)
+
+    def __del__(self):
+        h = getattr(self, "_h", None)
+        if h and _lib is not None:
+            _lib.oracle_spec_free(h)
+            self._h = None
+
+    def update(self, states, stacks, tokens) -> None:
+        states = np.ascontiguousarray(states, dtype=np.int32)
+        stacks = None if stacks is None else np.ascontiguousarray(stacks, dtype=np.uint64)
+        tokens = np.ascontiguousarray(tokens, dtype=np.int32)
+        lib().oracle_spec_update(self._h, _ptr(states), _ptr(stacks), _ptr(tokens), states.shape[0])
+
+    def propose(self, states, stacks, s: int, min_permille: int):
+        """(proposals [B][s], n_prop [B], chain_states [B][s+1], chain_stacks [B][s+1] or None)."""
+        states = np.ascontiguousarray(states, dtype=np.int32)
+        B = states.shape[0]
+        stacks = None if stacks is None else np.ascontiguousarray(stacks, dtype=np.uint64)
+        prop = np.zeros((B, s), np.int32)
+        n = np.zeros(B, np.int32)
+        cs = np.zeros((B, s + 1), np.int32)
+        ck = np.zeros((B, s + 1), np.uint64) if stacks is not None else None
+        lib().oracle_spec_propose(self._h, _ptr(states), _ptr(stacks), B, int(s), int(min_permille), _ptr(prop),
+                                  _ptr(n), _ptr(cs), _ptr(ck))
+        return prop, n, cs, ck
+
+
+def spec_accept(proposals, n_prop, decoded) -> np.ndarray:
+    proposals = np.ascontiguousarray(proposals, dtype=np.int32)
+    n_prop = np.ascontiguousarray(n_prop, dtype=np.int32)
+    decoded = np.ascontiguousarray(decoded, dtype=np.int32)
+    B, s = proposals.shape
+    out = np.zeros(B, np.int32)
+    lib().oracle_spec_accept(_ptr(proposals), _ptr(n_prop), _ptr(decoded), B, s, _ptr(out))
+    return out
 
 
 def mask_logits(logits: np.ndarray, mask: np.ndarray, n_tokens: Optional[int] = None, want_lse=True,

@@ -18,7 +18,7 @@
 #define ORACLE_MAX_DEPTH 32
 
 struct oracle_problem {
-    int32_t n_tokens, eos_id, n_states, max_depth;
+    int32_t n_tokens, eos_id, n_states, max_depth, n_rules;
     uint8_t* bytes;      /* all token bytes */
     int64_t* offsets;    /* [n_tokens + 1] */
     int32_t* delta;      /* [n_states][256] */
@@ -47,6 +47,7 @@ oracle_problem* oracle_new(const uint8_t* bytes, const int64_t* offsets, int32_t
     p->eos_id = eos_id;
     p->n_states = n_states;
     p->max_depth = max_depth;
+    p->n_rules = n_rules > 0 ? n_rules : 0;
     p->offsets = (int64_t*)dup_bytes(offsets, sizeof(int64_t) * (size_t)(n_tokens + 1));
     p->bytes = (uint8_t*)dup_bytes(bytes, (size_t)offsets[n_tokens]);
     p->delta = (int32_t*)dup_bytes(delta, sizeof(int32_t) * (size_t)n_states * 256);
@@ -333,6 +334,138 @@ void oracle_mask_sample(const void* logits, int32_t dtype, int32_t batch, int32_
             }
         }
         tokens[b] = best;
+    }
+}
+
+/* ---- count-based speculation (Sec. 3.6) --------------------------------- */
+
+struct oracle_spec {
+    const oracle_problem* p;
+    int32_t n_keys;
+    int64_t* reached;     /* [n_keys] */
+    int32_t* len;         /* [n_keys]: distinct tokens seen */
+    int32_t* cap;
+    int32_t** tok;        /* [n_keys][len] token ids */
+    int64_t** cnt;        /* [n_keys][len] times chosen */
+};
+
+static int spec_key(const oracle_problem* p, int32_t state, const stack_t_* st) {
+    if (p->n_rules == 0) return state;
+    int top = st->depth == 0 ? 0 : 1 + st->sym[st->depth - 1];
+    return state * 3 + top;
+}
+
+oracle_spec* oracle_spec_new(const oracle_problem* p) {
+    oracle_spec* sp = (oracle_spec*)calloc(1, sizeof *sp);
+    if (!sp) return NULL;
+    sp->p = p;
+    sp->n_keys = p->n_rules == 0 ? p->n_states : p->n_states * 3;
+    sp->reached = (int64_t*)calloc((size_t)sp->n_keys, sizeof(int64_t));
+    sp->len = (int32_t*)calloc((size_t)sp->n_keys, sizeof(int32_t));
+    sp->cap = (int32_t*)calloc((size_t)sp->n_keys, sizeof(int32_t));
+    sp->tok = (int32_t**)calloc((size_t)sp->n_keys, sizeof(int32_t*));
+    sp->cnt = (int64_t**)calloc((size_t)sp->n_keys, sizeof(int64_t*));
+    return sp;
+}
+
+void oracle_spec_free(oracle_spec* sp) {
+    if (!sp) return;
+    for (int32_t k = 0; k < sp->n_keys; k++) {
+        free(sp->tok[k]);
+        free(sp->cnt[k]);
+    }
+    free(sp->reached);
+    free(sp->len);
+    free(sp->cap);
+    free(sp->tok);
+    free(sp->cnt);
+    free(sp);
+}
+
+void oracle_spec_update(oracle_spec* sp, const int32_t* states, const uint64_t* stacks, const int32_t* tokens,
+                        int32_t batch) {
+    const oracle_problem* p = sp->p;
+    for (int32_t b = 0; b < batch; b++) {
+        int32_t t = tokens[b];
+        stack_t_ st;
+        if (t < 0 || t >= p->n_tokens || !config_valid(p, states[b], stacks ? stacks[b] : 0, &st)) continue;
+        int key = spec_key(p, states[b], &st);
+        sp->reached[key]++;
+        int32_t i = 0;
+        while (i < sp->len[key] && sp->tok[key][i] != t) i++;
+        if (i == sp->len[key]) {                      /* first time t is chosen here */
+            if (sp->len[key] == sp->cap[key]) {
+                int32_t nc = sp->cap[key] ? 2 * sp->cap[key] : 4;
+                sp->tok[key] = (int32_t*)realloc(sp->tok[key], sizeof(int32_t) * (size_t)nc);
+                sp->cnt[key] = (int64_t*)realloc(sp->cnt[key], sizeof(int64_t) * (size_t)nc);
+                sp->cap[key] = nc;
+            }
+            sp->tok[key][i] = t;
+            sp->cnt[key][i] = 0;
+            sp->len[key]++;
+        }
+        sp->cnt[key][i]++;
+    }
+}
+
+void oracle_spec_propose(const oracle_spec* sp, const int32_t* states, const uint64_t* stacks, int32_t batch,
+                         int32_t s, int32_t min_permille, int32_t* proposals, int32_t* n_prop,
+                         int32_t* chain_states, uint64_t* chain_stacks) {
+    const oracle_problem* p = sp->p;
+    for (int32_t b = 0; b < batch; b++) {
+        int32_t state = states[b];
+        uint64_t word = stacks ? stacks[b] : 0;
+        int32_t n = 0;
+        stack_t_ st;
+        int ok = config_valid(p, state, word, &st);
+        while (ok && n < s) {
+            int key = spec_key(p, state, &st);
+            int64_t reached = sp->reached[key];
+            if (reached == 0) break;
+            int32_t best = -1;
+            int64_t best_c = 0;
+            for (int32_t i = 0; i < sp->len[key]; i++) {   /* most frequent, lowest id on ties */
+                if (sp->cnt[key][i] > best_c || (sp->cnt[key][i] == best_c && sp->tok[key][i] < best)) {
+                    best_c = sp->cnt[key][i];
+                    best = sp->tok[key][i];
+                }
+            }
+            if (best < 0 || best_c * 1000 < (int64_t)min_permille * reached) break;
+            if (best == p->eos_id) {                       /* EOS is proposed and ends the chain */
+                if (!(p->accepting[state] && st.depth == 0)) break;
+                proposals[(int64_t)b * s + n] = best;
+                chain_states[(int64_t)b * (s + 1) + n + 1] = state;
+                if (chain_stacks) chain_stacks[(int64_t)b * (s + 1) + n + 1] = encode_stack(&st);
+                n++;
+                break;
+            }
+            stack_t_ next = st;
+            int32_t end = 0;
+            if (!walk_token(p, state, &next, best, &end, NULL)) break;
+            proposals[(int64_t)b * s + n] = best;
+            state = end;
+            st = next;
+            n++;
+            chain_states[(int64_t)b * (s + 1) + n] = state;
+            if (chain_stacks) chain_stacks[(int64_t)b * (s + 1) + n] = encode_stack(&st);
+        }
+        n_prop[b] = n;
+        chain_states[(int64_t)b * (s + 1)] = states[b];
+        if (chain_stacks) chain_stacks[(int64_t)b * (s + 1)] = word;
+        for (int32_t i = n; i < s; i++) proposals[(int64_t)b * s + i] = -1;
+        for (int32_t i = n + 1; i <= s; i++) {
+            chain_states[(int64_t)b * (s + 1) + i] = chain_states[(int64_t)b * (s + 1) + n];
+            if (chain_stacks) chain_stacks[(int64_t)b * (s + 1) + i] = chain_stacks[(int64_t)b * (s + 1) + n];
+        }
+    }
+}
+
+void oracle_spec_accept(const int32_t* proposals, const int32_t* n_prop, const int32_t* decoded, int32_t batch,
+                        int32_t s, int32_t* n_accept) {
+    for (int32_t b = 0; b < batch; b++) {
+        int32_t k = 0;
+        while (k < n_prop[b] && decoded[(int64_t)b * (s + 1) + k] == proposals[(int64_t)b * s + k]) k++;
+        n_accept[b] = k;
     }
 }
 

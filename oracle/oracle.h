@@ -24,6 +24,12 @@
  *                 index on ties, log-sum-exp and log-probabilities in double.
  *   advance      (Alg. 1, C.update(o)): the chosen token's walk; EOS or "no
  *                 token" ends the sequence and the next one starts from init.
+ *   spec_*       (Sec. 3.6, count-based speculative proposals): counts of
+ *                 the tokens chosen in each (scanner state, parser sub-state);
+ *                 up to s tokens proposed by following the most frequent
+ *                 choice while its share is large enough; proposals accepted
+ *                 up to the first position where the constrained decode
+ *                 disagrees.
  *   mask_sample  (Alg. 1, decode by sampling instead of the argmax): the
  *                 Gumbel-max rule over the allowed tokens, with uniforms from
  *                 the Philox4x32-10 counter-based generator (Salmon et al.,
@@ -115,6 +121,39 @@ float oracle_ln_f32(float x);
 void oracle_mask_sample(const void* logits, int32_t dtype, int32_t batch, int32_t n_tokens, int64_t row_stride,
                         const uint32_t* mask, float temperature, uint64_t seed, uint64_t offset, int32_t* tokens,
                         int32_t n_threads);
+
+/* Count-based speculation (Sec. 3.6).  The count model is keyed by
+ * (alpha, beta) = (scanner state, top of the bracket stack): key = state for a
+ * plain DFA, state * 3 + top for a pushdown automaton, top = 0 for an empty
+ * stack, 1 + symbol otherwise. */
+typedef struct oracle_spec oracle_spec;
+oracle_spec* oracle_spec_new(const oracle_problem* p);
+void oracle_spec_free(oracle_spec* sp);
+
+/* After a decode step: the token tokens[b] (>= 0) was chosen from
+ * configuration b: #reached(key) += 1 and #chose(key, token) += 1.  Rows with
+ * a negative token or an invalid configuration are skipped. */
+void oracle_spec_update(oracle_spec* sp, const int32_t* states, const uint64_t* stacks, const int32_t* tokens,
+                        int32_t batch);
+
+/* Up to s proposals per row: from the row's configuration, repeatedly take
+ * the key's most frequent token (lowest id on equal counts) while
+ * count * 1000 >= min_permille * #reached(key) and #reached > 0; a proposed
+ * token must be allowed from the current configuration (the walk is taken and
+ * the configuration advanced); EOS is proposed and ends the chain.
+ *   proposals [batch][s] (-1 past n_prop[b]); n_prop [batch];
+ *   chain_states / chain_stacks [batch][s + 1]: entry i is the configuration
+ *   after the first i proposals (entries past n_prop[b] repeat the last one);
+ *   chain_stacks may be NULL. */
+void oracle_spec_propose(const oracle_spec* sp, const int32_t* states, const uint64_t* stacks, int32_t batch,
+                         int32_t s, int32_t min_permille, int32_t* proposals, int32_t* n_prop,
+                         int32_t* chain_states, uint64_t* chain_stacks);
+
+/* Verification: decoded [batch][s + 1] holds the constrained decode at each
+ * chain configuration; n_accept[b] = the number of leading proposals equal to
+ * it (at most n_prop[b]). */
+void oracle_spec_accept(const int32_t* proposals, const int32_t* n_prop, const int32_t* decoded, int32_t batch,
+                        int32_t s, int32_t* n_accept);
 
 /* Alg. 1 update: states_out/stacks_out may alias the inputs.  tokens[b] < 0 or
  * == eos_id: (start_state, empty).  A rejected token: (0, empty).  A token id

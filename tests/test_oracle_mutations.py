@@ -33,8 +33,13 @@ MUTANTS = {
     "philox_word_ignores_token": ("uint32_t k = c[t % 4] >> 9;", "uint32_t k = c[0] >> 9;"),
     "philox_rounds_short": ("for (int round = 0; round < 10; round++) {", "for (int round = 0; round < 9; round++) {"),
     "ln_series_term_dropped": ("poly = fmaf(poly, z2, 0x1.99999ap-3f);           /* 1/5 */", "poly = poly;"),
+    "spec_ties_highest_id": ("sp->tok[key][i] < best)) {", "sp->tok[key][i] > best)) {"),
+    "spec_threshold_strict": ("best_c * 1000 < (int64_t)min_permille * reached) break;",
+                              "best_c * 1000 <= (int64_t)min_permille * reached) break;"),
+    "spec_key_ignores_top": ("return state * 3 + top;", "return state * 3;"),
+    "spec_chain_not_advanced": ("            state = end;\n            st = next;", "            st = next;"),
 }
-PIN_FILES = ["test_oracle_pins.py", "test_oracle_sampling.py"]
+PIN_FILES = ["test_oracle_pins.py", "test_oracle_sampling.py", "test_oracle_spec.py"]
 
 
 @pytest.mark.parametrize("name", sorted(MUTANTS))
