@@ -571,6 +571,87 @@ def run_domino(args, dist: Dist):
     if d.device_error():
         raise RuntimeError("device error after the per-kernel graphs")
 
+    # ---- opportunistic masking on the same rows: the logits as generated
+    # (random: most proposals are rejected) and an obedient model's logits
+    # (+20 on every allowed token: proposals are accepted)
+    scratch = torch.empty((Bsz, Wd), dtype=torch.int32, device=dev)
+    n_fb = torch.zeros(1, dtype=torch.int32, device=dev)
+    p_scr, p_nfb = scratch.data_ptr(), n_fb.data_ptr()
+
+    def opp_body(bufs):
+        def body(i, sp):
+            if L.domino_opportunistic_step(h, bufs[i % len(bufs)], dtype_code, Bsz, V, p_states, p_stacks, p_scr,
+                                           p_arg, p_nfb, sp):
+                raise RuntimeError("opportunistic step failed")
+        return body
+    with torch.cuda.stream(s):
+        L.domino_step_mask(h, p_states, p_stacks, Bsz, p_mask, None, s.cuda_stream)
+    torch.cuda.synchronize()
+    bits = ((mask.view(torch.int32).unsqueeze(-1) >> torch.arange(32, device=dev, dtype=torch.int32)) & 1)
+    bits = bits.reshape(Bsz, Wd * 32)[:, :V].to(torch.float32)
+    obedient = [(t.to(torch.float32) + 20.0 * bits).to(t.dtype).contiguous() for t in logits]
+    del bits
+    opportunistic = {}
+    for name, bufs in (("random_logits", p_logits), ("obedient_logits", [t.data_ptr() for t in obedient])):
+        body = opp_body(bufs)
+        with torch.cuda.stream(s):
+            body(0, s.cuda_stream)
+        torch.cuda.synchronize()
+        g = capture(Kk, body)
+        ms_o = dist.max(timed(Kk, body, g))
+        del g
+        opportunistic[name] = {"us": ms_o / Kk * 1e3, "fallback_rows": int(n_fb.item()), "rows": Bsz}
+    opportunistic["masked_greedy_us"] = (per_kernel["step_mask"] + per_kernel["mask_logits"]) * 1e3
+    opportunistic["note"] = ("same rows, fixed states; tokens equal the masked greedy decode; obedient = +20 on "
+                             "every allowed logit")
+    del obedient, scratch
+    if d.device_error():
+        raise RuntimeError("device error in the opportunistic step")
+
+    # ---- count-based speculation: the model's update, s = 4 proposals and the
+    # acceptance, each alone (the verification is step_mask + mask_logits over
+    # batch x (s + 1) configurations, the kernels timed above)
+    n_keys = info["n_states"] * (3 if stack else 1)
+    S_SPEC = 4
+    counts = torch.zeros((n_keys, V), dtype=torch.int32, device=dev)
+    best = torch.zeros(n_keys, dtype=torch.int64, device=dev)
+    reached = torch.zeros(n_keys, dtype=torch.int32, device=dev)
+    prop = torch.empty((Bsz, S_SPEC), dtype=torch.int32, device=dev)
+    n_prop = torch.empty(Bsz, dtype=torch.int32, device=dev)
+    chain_s = torch.empty((Bsz, S_SPEC + 1), dtype=torch.int32, device=dev)
+    chain_k = torch.empty((Bsz, S_SPEC + 1), dtype=torch.int64, device=dev) if stack else None
+    decoded = torch.zeros((Bsz, S_SPEC + 1), dtype=torch.int32, device=dev)
+    n_acc = torch.empty(Bsz, dtype=torch.int32, device=dev)
+    pc, pb, pr = counts.data_ptr(), best.data_ptr(), reached.data_ptr()
+    pp, pn, pcs = prop.data_ptr(), n_prop.data_ptr(), chain_s.data_ptr()
+    pck = chain_k.data_ptr() if stack else None
+
+    def k_spec_update(i, sp):
+        if L.domino_spec_update(h, pc, pb, pr, p_states, p_stacks, p_arg, Bsz, sp):
+            raise RuntimeError("spec_update failed")
+
+    def k_spec_propose(i, sp):
+        if L.domino_spec_propose(h, pb, pr, p_states, p_stacks, Bsz, S_SPEC, 0, pp, pn, pcs, pck, sp):
+            raise RuntimeError("spec_propose failed")
+
+    def k_spec_accept(i, sp):
+        if L.domino_spec_accept(h, pp, pn, decoded.data_ptr(), pcs, pck, Bsz, S_SPEC, n_acc.data_ptr(), None, None,
+                                None, sp):
+            raise RuntimeError("spec_accept failed")
+    spec = {}
+    for name, body in (("update", k_spec_update), ("propose_s4", k_spec_propose), ("accept", k_spec_accept)):
+        with torch.cuda.stream(s):
+            body(0, s.cuda_stream)
+        torch.cuda.synchronize()
+        g = capture(Kk, body)
+        spec[name + "_us"] = dist.max(timed(Kk, body, g)) / Kk * 1e3
+        del g
+    spec["proposals_per_row"] = float(n_prop.float().mean().item())
+    spec["count_table_bytes"] = n_keys * V * 4
+    del counts
+    if d.device_error():
+        raise RuntimeError("device error in the speculation kernels")
+
     # ---- table-driven step (DFA only): masks and next states precomputed once
     # for every state, then per step a mask-row lookup fused into the logits
     # pass and one table read per sequence for the update
@@ -696,6 +777,7 @@ def run_domino(args, dist: Dist):
                    "parallelism": f"replicas x{n}", "graph": graph is not None},
         "masked_decode_steps_per_s": n * K / (ms_max / 1e3),
         "kernels": kernels, "roofline": roofline, "table_driven_step": table_step,
+        "opportunistic": opportunistic, "speculation": spec,
         "e2e": {"value": n * Bsz * V * Ke / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "steps": Ke, "api": "domino_decode_step_host (pinned host buffers)"},
         "gpu_launches": K * launches_per_step,

@@ -197,6 +197,65 @@ int domino_mask_sample(domino_t h, const void* logits_dev, int32_t dtype, int32_
                        const uint32_t* mask_dev, float temperature, uint64_t seed, uint64_t offset,
                        int32_t* tokens_dev, void* stream);
 
+/* Opportunistic masking (Sec. 3.5's speed-ups): the greedy token of a decode
+ * step without computing every mask.  Per row: the unmasked argmax (lowest
+ * index on ties) is proposed and checked with one walk from the row's
+ * configuration; if allowed it is the masked argmax.  Only the rows whose
+ * proposal is rejected get their full mask (domino_step_mask over the listed
+ * rows) and the masked argmax.  tokens_dev[b] equals what
+ * domino_step_mask + domino_mask_logits give (-1 when nothing is allowed).
+ *   mask_scratch_dev uint32 [batch][W]: caller-owned scratch; its first
+ *   n rows hold the masks of the fallback rows, in no fixed order.
+ *   n_fallback_dev int32 [1] or NULL: receives the number of fallback rows.
+ * No lse: the accepted rows' masks are never formed.  The first call with a
+ * batch larger than any before allocates scratch and synchronises `stream`.
+ * Invalid configurations behave as in domino_step_mask (error word, -1). */
+int domino_opportunistic_step(domino_t h, const void* logits_dev, int32_t dtype, int32_t batch,
+                              int64_t row_stride_elems, const int32_t* states_dev, const uint64_t* stacks_dev,
+                              uint32_t* mask_scratch_dev, int32_t* tokens_dev, int32_t* n_fallback_dev,
+                              void* stream);
+
+/* Count-based speculative proposals (Sec. 3.6).  The count model
+ * P(t | alpha, beta) = #chose(t) / #reached is keyed by the scanner state and
+ * the top of the bracket stack: n_keys = Q for a DFA, 3 Q for a pushdown
+ * automaton (key = state * 3 + top, top 0 for an empty stack, 1 + symbol
+ * otherwise).  The caller owns the model, zero-initialised:
+ *   counts_dev uint32 [n_keys][V]; best_dev uint64 [n_keys] (the most frequent
+ *   token of each key, packed as count << 32 | (0xFFFFFFFF - token));
+ *   reached_dev uint32 [n_keys].
+ * domino_spec_update: token tokens_dev[b] >= 0 was chosen from configuration
+ * b; rows with a negative token or an invalid configuration are skipped. */
+int domino_spec_update(domino_t h, uint32_t* counts_dev, uint64_t* best_dev, uint32_t* reached_dev,
+                       const int32_t* states_dev, const uint64_t* stacks_dev, const int32_t* tokens_dev,
+                       int32_t batch, void* stream);
+
+/* Up to s proposals per row: from the row's configuration, repeatedly the
+ * key's most frequent token (lowest id on equal counts) while
+ * count * 1000 >= min_permille * reached and reached > 0.  Each proposal is
+ * walked and must be allowed from the current configuration; EOS (accepting
+ * state, empty stack) is proposed and ends the chain.
+ *   proposals_dev int32 [batch][s] (-1 past the chain); n_prop_dev [batch];
+ *   chain_states_dev int32 [batch][s + 1], chain_stacks_dev uint64
+ *   [batch][s + 1] or NULL: entry i is the configuration after i proposals
+ *   (the last one repeated past the chain's end).  The verification is the
+ *   ordinary mask step + decode over these batch * (s + 1) configurations
+ *   (one LLM pass gives their logits). */
+int domino_spec_propose(domino_t h, const uint64_t* best_dev, const uint32_t* reached_dev,
+                        const int32_t* states_dev, const uint64_t* stacks_dev, int32_t batch, int32_t s,
+                        int32_t min_permille, int32_t* proposals_dev, int32_t* n_prop_dev,
+                        int32_t* chain_states_dev, uint64_t* chain_stacks_dev, void* stream);
+
+/* Acceptance: decoded_dev int32 [batch][s + 1] is the constrained decode at
+ * each chain configuration.  n_accept_dev[b] = the number of leading
+ * proposals equal to it; tokens_out_dev[b] = the decode right after them and
+ * states_out_dev / stacks_out_dev = the configuration it was decoded from
+ * (apply it with domino_advance).  Any output except n_accept_dev may be
+ * NULL. */
+int domino_spec_accept(domino_t h, const int32_t* proposals_dev, const int32_t* n_prop_dev,
+                       const int32_t* decoded_dev, const int32_t* chain_states_dev, const uint64_t* chain_stacks_dev,
+                       int32_t batch, int32_t s, int32_t* n_accept_dev, int32_t* tokens_out_dev,
+                       int32_t* states_out_dev, uint64_t* stacks_out_dev, void* stream);
+
 /* Table-driven decode step, mask and decode (Sec. 3.5: the per-state masks
  * are computed before inference starts and looked up while decoding).  The
  * same fused masked argmax / lse / log-probs as domino_mask_logits, with row

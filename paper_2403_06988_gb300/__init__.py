@@ -114,6 +114,21 @@ class Domino:
                              stream)
         return tokens
 
+    def opportunistic_step(self, logits, states, stacks=None, stream=None):
+        """Greedy tokens via opportunistic masking; returns (tokens, number of fallback rows as a tensor)."""
+        import torch
+        b = logits.shape[0]
+        dtype = DTYPE_BF16 if logits.dtype == torch.bfloat16 else DTYPE_F32
+        if logits.stride(1) != 1:
+            raise ValueError("logits rows must be contiguous")
+        W = self.info()["n_words"]
+        scratch = torch.empty((b, W), dtype=torch.int32, device=logits.device)
+        tokens = torch.empty(b, dtype=torch.int32, device=logits.device)
+        n_fb = torch.zeros(1, dtype=torch.int32, device=logits.device)
+        B.domino_opportunistic_step(self.h, logits, dtype, b, logits.stride(0), states, stacks, scratch, tokens, n_fb,
+                                    stream)
+        return tokens, n_fb
+
     def mask_logits_table(self, logits, table_mask, states, want_lse: bool = True, want_logprobs: bool = False,
                           stream=None) -> Tuple:
         """Table-driven mask + decode: row b's mask is table_mask[states[b]] (DFA only)."""

@@ -69,6 +69,10 @@ _SIGS = {
     "domino_mask_logits_table": [P, P, I32, I32, I64, P, P, P, P, P, P],
     "domino_advance_table": [P, P, P, P, I32, P, P],
     "domino_mask_sample": [P, P, I32, I32, I64, P, ctypes.c_float, ctypes.c_uint64, ctypes.c_uint64, P, P],
+    "domino_opportunistic_step": [P, P, I32, I32, I64, P, P, P, P, P, P],
+    "domino_spec_update": [P, P, P, P, P, P, P, I32, P],
+    "domino_spec_propose": [P, P, P, P, P, I32, I32, I32, P, P, P, P, P],
+    "domino_spec_accept": [P, P, P, P, P, P, I32, I32, P, P, P, P, P],
 }
 
 
@@ -212,6 +216,37 @@ def domino_mask_sample(h: int, logits_dev, dtype: int, batch: int, row_stride_el
     _check("domino_mask_sample", lib().domino_mask_sample(
         h, _ptr(logits_dev), int(dtype), int(batch), int(row_stride_elems), _ptr(mask_dev), float(temperature),
         int(seed) & 0xFFFFFFFFFFFFFFFF, int(offset) & 0xFFFFFFFFFFFFFFFF, _ptr(tokens_dev), _stream(stream)))
+
+
+def domino_opportunistic_step(h: int, logits_dev, dtype: int, batch: int, row_stride_elems: int, states_dev,
+                              stacks_dev, mask_scratch_dev, tokens_dev, n_fallback_dev=None, stream=None) -> None:
+    _check("domino_opportunistic_step", lib().domino_opportunistic_step(
+        h, _ptr(logits_dev), int(dtype), int(batch), int(row_stride_elems), _ptr(states_dev), _ptr(stacks_dev),
+        _ptr(mask_scratch_dev), _ptr(tokens_dev), _ptr(n_fallback_dev), _stream(stream)))
+
+
+def domino_spec_update(h: int, counts_dev, best_dev, reached_dev, states_dev, stacks_dev, tokens_dev, batch: int,
+                       stream=None) -> None:
+    _check("domino_spec_update", lib().domino_spec_update(h, _ptr(counts_dev), _ptr(best_dev), _ptr(reached_dev),
+                                                           _ptr(states_dev), _ptr(stacks_dev), _ptr(tokens_dev),
+                                                           int(batch), _stream(stream)))
+
+
+def domino_spec_propose(h: int, best_dev, reached_dev, states_dev, stacks_dev, batch: int, s: int, min_permille: int,
+                        proposals_dev, n_prop_dev, chain_states_dev, chain_stacks_dev=None, stream=None) -> None:
+    _check("domino_spec_propose", lib().domino_spec_propose(
+        h, _ptr(best_dev), _ptr(reached_dev), _ptr(states_dev), _ptr(stacks_dev), int(batch), int(s),
+        int(min_permille), _ptr(proposals_dev), _ptr(n_prop_dev), _ptr(chain_states_dev), _ptr(chain_stacks_dev),
+        _stream(stream)))
+
+
+def domino_spec_accept(h: int, proposals_dev, n_prop_dev, decoded_dev, chain_states_dev, chain_stacks_dev,
+                       batch: int, s: int, n_accept_dev, tokens_out_dev=None, states_out_dev=None,
+                       stacks_out_dev=None, stream=None) -> None:
+    _check("domino_spec_accept", lib().domino_spec_accept(
+        h, _ptr(proposals_dev), _ptr(n_prop_dev), _ptr(decoded_dev), _ptr(chain_states_dev), _ptr(chain_stacks_dev),
+        int(batch), int(s), _ptr(n_accept_dev), _ptr(tokens_out_dev), _ptr(states_out_dev), _ptr(stacks_out_dev),
+        _stream(stream)))
 
 
 def domino_mask_logits_table(h: int, logits_dev, dtype: int, batch: int, row_stride_elems: int, table_mask_dev,

@@ -83,9 +83,12 @@ int64_t table_smem_bytes(const StepView& v, bool stack, int mode);
 // Shared-memory bytes of the step kernel other than the table.
 int step_fixed_smem_bytes(const StepView& v, bool next);
 
+// row_ids / row_count (device): only rows row_ids[i], i < *row_count <= batch,
+// are walked; their masks are written to the compact rows i of `mask`.
 cudaError_t launch_step_mask(const StepView& v, const LaunchEnv& env, bool stack, int mode, const int32_t* states,
                              const uint64_t* stacks, int32_t batch, bool row_is_state, uint32_t* mask,
-                             int32_t* next, cudaStream_t st);
+                             int32_t* next, cudaStream_t st, const int32_t* row_ids = nullptr,
+                             const int32_t* row_count = nullptr);
 
 // Sampling decode: Gumbel-max with Philox4x32-10 uniforms (kernels.cu).
 struct SampleArgs {
@@ -97,12 +100,16 @@ struct SampleArgs {
 // row_state (table-driven step): row r's mask is row row_state[r] of the
 // [Q][W] table `mask`; out-of-range states read as empty rows and set `err`.
 // sample: draw each row's token (into argmax) instead of the greedy argmax;
-// lse and logprobs must then be null.
+// lse and logprobs must then be null.  mask == nullptr (no row_state): every
+// token allowed.  row_ids / row_count (device): only rows row_ids[i] for
+// i < *row_count are processed, their masks being the compact rows i of
+// `mask`; argmax and lse are indexed by batch row; no logprobs.
 cudaError_t launch_mask_logits(const LaunchEnv& env, const void* logits, int dtype, int32_t batch,
                                int64_t row_stride, int32_t V, const uint32_t* mask, int32_t* argmax, float* lse,
                                float* logprobs, float4* partials, uint32_t* counters, float* lse_tmp,
                                cudaStream_t st, const int32_t* row_state = nullptr, int32_t Q = 0,
-                               uint32_t* err = nullptr, const SampleArgs* sample = nullptr);
+                               uint32_t* err = nullptr, const SampleArgs* sample = nullptr,
+                               const int32_t* row_ids = nullptr, const int32_t* row_count = nullptr);
 
 // Fills the sampling arguments (1/T in fp32, seed and offset words).
 cudaError_t launch_mask_sample(const LaunchEnv& env, const void* logits, int dtype, int32_t batch,
@@ -118,5 +125,24 @@ cudaError_t launch_advance(const StepView& v, bool stack, int mode, const int32_
 cudaError_t launch_advance_table(const int32_t* table_next, int32_t Q, int32_t V, int32_t eos_id, int32_t start,
                                  const int32_t* states, const int32_t* tokens, int32_t batch, int32_t* states_out,
                                  uint32_t* err, cudaStream_t st);
+
+// Opportunistic masking: accepts row b's proposal into tokens_out[b] or
+// appends b to row_ids (counter *row_count, zeroed by the caller).
+cudaError_t launch_propose_check(const StepView& v, bool stack, int mode, const int32_t* states,
+                                 const uint64_t* stacks, const int32_t* proposals, int32_t batch, int32_t* tokens_out,
+                                 int32_t* row_ids, int32_t* row_count, cudaStream_t st);
+
+// Count-based speculation (Sec. 3.6): count update, proposals, acceptance.
+cudaError_t launch_spec_update(const StepView& v, bool stack, const int32_t* states, const uint64_t* stacks,
+                               const int32_t* tokens, int32_t batch, uint32_t* counts, unsigned long long* best,
+                               uint32_t* reached, cudaStream_t st);
+cudaError_t launch_spec_propose(const StepView& v, bool stack, int mode, const int32_t* states,
+                                const uint64_t* stacks, int32_t batch, int32_t s, int32_t min_permille,
+                                const unsigned long long* best, const uint32_t* reached, int32_t* proposals,
+                                int32_t* n_prop, int32_t* chain_states, uint64_t* chain_stacks, cudaStream_t st);
+cudaError_t launch_spec_accept(const int32_t* proposals, const int32_t* n_prop, const int32_t* decoded,
+                               const int32_t* chain_states, const uint64_t* chain_stacks, int32_t batch, int32_t s,
+                               int32_t* n_accept, int32_t* tokens_out, int32_t* states_out, uint64_t* stacks_out,
+                               cudaStream_t st);
 
 }  // namespace domino

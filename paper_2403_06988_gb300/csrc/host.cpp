@@ -58,6 +58,8 @@ struct domino_ctx {
     int32_t n_windows = 0;
     // staging for domino_decode_step_host
     DevBuf s_logits, s_states, s_stacks, s_mask, s_tokens, s_lse;
+    // opportunistic masking: proposals, the fallback row list and its length
+    DevBuf o_prop, o_rows, o_count;
 };
 
 namespace {
@@ -86,7 +88,7 @@ int64_t dev_bytes(const domino_ctx* h) {
     const DevBuf* all[] = {&h->d_head, &h->d_info, &h->d_tail_off, &h->d_tail, &h->d_pos_of, &h->d_units,
                            &h->d_unit_off, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_err, &h->d_partials,
                            &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_states, &h->s_stacks,
-                           &h->s_mask, &h->s_tokens, &h->s_lse};
+                           &h->s_mask, &h->s_tokens, &h->s_lse, &h->o_prop, &h->o_rows, &h->o_count};
     int64_t n = 0;
     for (auto* b : all) n += (int64_t)b->n;
     return n;
@@ -655,6 +657,97 @@ int domino_mask_sample(domino_t h, const void* logits_dev, int32_t dtype, int32_
     return cuda_status(launch_mask_sample(h->env, logits_dev, dtype, batch, row_stride_elems, h->V, mask_dev,
                                           temperature, seed, offset, tokens_dev, (float4*)h->d_partials.p,
                                           (uint32_t*)h->d_counters.p, (cudaStream_t)stream));
+}
+
+int domino_opportunistic_step(domino_t h, const void* logits_dev, int32_t dtype, int32_t batch,
+                              int64_t row_stride_elems, const int32_t* states_dev, const uint64_t* stacks_dev,
+                              uint32_t* mask_scratch_dev, int32_t* tokens_dev, int32_t* n_fallback_dev,
+                              void* stream) {
+    int rc = ready_for_compute(h);
+    if (rc) return rc;
+    if (dtype != DOMINO_DTYPE_F32 && dtype != DOMINO_DTYPE_BF16) return DOMINO_E_INVALID_ARG;
+    if (batch < 0 || row_stride_elems < h->V) return DOMINO_E_INVALID_ARG;
+    if (batch == 0) return DOMINO_OK;
+    if (!logits_dev || !states_dev || !mask_scratch_dev || !tokens_dev) return DOMINO_E_INVALID_ARG;
+    DeviceGuard g(h->device);
+    cudaStream_t st = (cudaStream_t)stream;
+    if (h->o_prop.n < (size_t)batch * 4 || h->o_rows.n < (size_t)batch * 4 || h->o_count.n < 16) {
+        if (cudaStreamSynchronize(st) != cudaSuccess) return cuda_status(cudaGetLastError());
+        if ((rc = dev_reserve(h->o_prop, (size_t)batch * 4))) return rc;
+        if ((rc = dev_reserve(h->o_rows, (size_t)batch * 4))) return rc;
+        if ((rc = dev_reserve(h->o_count, 16))) return rc;
+    }
+    int32_t* prop = (int32_t*)h->o_prop.p;
+    int32_t* rows = (int32_t*)h->o_rows.p;
+    int32_t* count = n_fallback_dev ? n_fallback_dev : (int32_t*)h->o_count.p;
+    StepView v = make_view(h);
+    const int mode = choose_mode(h, v, false);
+    cudaError_t e = cudaMemsetAsync(count, 0, sizeof(int32_t), st);
+    // 1. the unmasked argmax (every token allowed)
+    if (e == cudaSuccess)
+        e = launch_mask_logits(h->env, logits_dev, dtype, batch, row_stride_elems, h->V, nullptr, prop, nullptr,
+                               nullptr, (float4*)h->d_partials.p, (uint32_t*)h->d_counters.p, nullptr, st);
+    // 2. one walk per row: keep the proposal or list the row for the fallback
+    if (e == cudaSuccess)
+        e = launch_propose_check(v, h->stack, mode, states_dev, stacks_dev, prop, batch, tokens_dev, rows, count, st);
+    // 3. the listed rows only: their masks, then their masked argmax
+    if (e == cudaSuccess)
+        e = launch_step_mask(v, h->env, h->stack, mode, states_dev, stacks_dev, batch, false, mask_scratch_dev,
+                             nullptr, st, rows, count);
+    if (e == cudaSuccess)
+        e = launch_mask_logits(h->env, logits_dev, dtype, batch, row_stride_elems, h->V, mask_scratch_dev,
+                               tokens_dev, nullptr, nullptr, (float4*)h->d_partials.p, (uint32_t*)h->d_counters.p,
+                               nullptr, st, nullptr, 0, nullptr, nullptr, rows, count);
+    return cuda_status(e);
+}
+
+int domino_spec_update(domino_t h, uint32_t* counts_dev, uint64_t* best_dev, uint32_t* reached_dev,
+                       const int32_t* states_dev, const uint64_t* stacks_dev, const int32_t* tokens_dev,
+                       int32_t batch, void* stream) {
+    int rc = ready_for_compute(h);
+    if (rc) return rc;
+    if (batch < 0) return DOMINO_E_INVALID_ARG;
+    if (batch == 0) return DOMINO_OK;
+    if (!counts_dev || !best_dev || !reached_dev || !states_dev || !tokens_dev) return DOMINO_E_INVALID_ARG;
+    DeviceGuard g(h->device);
+    StepView v = make_view(h);
+    return cuda_status(launch_spec_update(v, h->stack, states_dev, stacks_dev, tokens_dev, batch, counts_dev,
+                                          (unsigned long long*)best_dev, reached_dev, (cudaStream_t)stream));
+}
+
+int domino_spec_propose(domino_t h, const uint64_t* best_dev, const uint32_t* reached_dev,
+                        const int32_t* states_dev, const uint64_t* stacks_dev, int32_t batch, int32_t s,
+                        int32_t min_permille, int32_t* proposals_dev, int32_t* n_prop_dev,
+                        int32_t* chain_states_dev, uint64_t* chain_stacks_dev, void* stream) {
+    int rc = ready_for_compute(h);
+    if (rc) return rc;
+    if (batch < 0 || s < 1 || min_permille < 0 || min_permille > 1000) return DOMINO_E_INVALID_ARG;
+    if (batch == 0) return DOMINO_OK;
+    if (!best_dev || !reached_dev || !states_dev || !proposals_dev || !n_prop_dev || !chain_states_dev)
+        return DOMINO_E_INVALID_ARG;
+    if (stacks_dev && !chain_stacks_dev) return DOMINO_E_INVALID_ARG;
+    DeviceGuard g(h->device);
+    StepView v = make_view(h);
+    const int mode = choose_mode(h, v, false);
+    return cuda_status(launch_spec_propose(v, h->stack, mode, states_dev, stacks_dev, batch, s, min_permille,
+                                           (const unsigned long long*)best_dev, reached_dev, proposals_dev,
+                                           n_prop_dev, chain_states_dev, chain_stacks_dev, (cudaStream_t)stream));
+}
+
+int domino_spec_accept(domino_t h, const int32_t* proposals_dev, const int32_t* n_prop_dev,
+                       const int32_t* decoded_dev, const int32_t* chain_states_dev, const uint64_t* chain_stacks_dev,
+                       int32_t batch, int32_t s, int32_t* n_accept_dev, int32_t* tokens_out_dev,
+                       int32_t* states_out_dev, uint64_t* stacks_out_dev, void* stream) {
+    if (!h) return DOMINO_E_INVALID_ARG;
+    if (is_host_only(h)) return DOMINO_E_NO_DEVICE;
+    if (batch < 0 || s < 1) return DOMINO_E_INVALID_ARG;
+    if (batch == 0) return DOMINO_OK;
+    if (!proposals_dev || !n_prop_dev || !decoded_dev || !n_accept_dev) return DOMINO_E_INVALID_ARG;
+    if ((states_out_dev && !chain_states_dev) || (stacks_out_dev && !chain_stacks_dev)) return DOMINO_E_INVALID_ARG;
+    DeviceGuard g(h->device);
+    return cuda_status(launch_spec_accept(proposals_dev, n_prop_dev, decoded_dev, chain_states_dev, chain_stacks_dev,
+                                          batch, s, n_accept_dev, tokens_out_dev, states_out_dev, stacks_out_dev,
+                                          (cudaStream_t)stream));
 }
 
 int domino_mask_logits_table(domino_t h, const void* logits_dev, int32_t dtype, int32_t batch,

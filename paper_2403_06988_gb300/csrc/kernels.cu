@@ -70,6 +70,20 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t sme
     return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
 }
 
+// A compacted list of the rows to process (opportunistic masking's rejected
+// rows): entry i of the pass is row ids[i] of the batch, and only the first
+// *count - base entries of this pass exist (the count is device memory).
+struct RowList {
+    const int32_t* ids;     // nullptr: rows are 0..B-1
+    const int32_t* count;
+    int32_t base;           // first list entry of this pass
+    __device__ __forceinline__ int rows(int cap) const {
+        if (!ids) return cap;
+        return max(0, min(cap, __ldg(count) - base));
+    }
+    __device__ __forceinline__ int row(int i) const { return ids ? __ldg(ids + base + i) : i; }
+};
+
 // Shared-memory layout of the step kernel (offsets in bytes).
 struct StepLayout {
     int head, info, units, items, rows, ctrl, rowmask, cfg, mtile, ntile, accept, table, total;
@@ -250,7 +264,7 @@ __global__ void __launch_bounds__(kStepThreads, 1)
     step_kernel(const StepView v, const uint4* __restrict__ img, int img_bytes, int img_tgt_off, int img_ret_off,
                 const int32_t* __restrict__ states, const uint64_t* __restrict__ stacks, int32_t batch,
                 int32_t R, int32_t n_row_tiles, int32_t n_tiles, int32_t row_is_state, uint32_t* __restrict__ mask,
-                int32_t* __restrict__ next) {
+                int32_t* __restrict__ next, const RowList list) {
     using E = typename std::conditional<STACK, uint32_t, uint16_t>::type;
     extern __shared__ __align__(16) unsigned char smem[];
     const int K = v.K;
@@ -268,6 +282,11 @@ __global__ void __launch_bounds__(kStepThreads, 1)
     int32_t* s_ntile = reinterpret_cast<int32_t*>(smem + L.ntile);
     uint32_t* s_accept = reinterpret_cast<uint32_t*>(smem + L.accept);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    if (list.ids) {   // a row list may be empty: learn its length before staging anything
+        pdl_wait();
+        pdl_trigger();
+        if (list.rows(batch) == 0) return;
+    }
     for (int i = tid; i < (v.Q + 31) / 32; i += kStepThreads) s_accept[i] = __ldg(v.accept_bits + i);
 
     Tab<E, MODE> tab;
@@ -289,6 +308,11 @@ __global__ void __launch_bounds__(kStepThreads, 1)
     const uint32_t maxd = (uint32_t)v.max_depth;
     pdl_wait();      // everything below may read what earlier kernels wrote
     pdl_trigger();   // after the wait: at most two kernels of a stream overlap
+    if (list.ids) {  // a compacted row list: its length is known only now
+        batch = list.rows(batch);
+        n_row_tiles = (batch + R - 1) / R;
+        n_tiles = n_row_tiles * v.n_windows;
+    }
 
     const int t0 = (int)(((long long)blockIdx.x * n_tiles) / gridDim.x);
     const int t1 = (int)(((long long)(blockIdx.x + 1) * n_tiles) / gridDim.x);
@@ -301,8 +325,9 @@ __global__ void __launch_bounds__(kStepThreads, 1)
             const int wq = t / n_row_tiles;
             const int b = (t - wq * n_row_tiles) * R + tid;
             if (b < batch) {
-                pf_s = __ldg(states + b);
-                if (stacks) pf_w = __ldg(reinterpret_cast<const unsigned long long*>(stacks) + b);
+                const int rb = list.row(b);
+                pf_s = __ldg(states + rb);
+                if (stacks) pf_w = __ldg(reinterpret_cast<const unsigned long long*>(stacks) + rb);
             }
         }
     };
@@ -638,11 +663,13 @@ constexpr float kGumbelMax = 17.0f;
 // out-of-range state reads as an all-zero row (nothing allowed) and sets the
 // error word.
 struct MaskRows {
-    const uint32_t* base;
+    const uint32_t* base;       // nullptr (and no row_state): every token allowed
     const int32_t* row_state;   // nullptr: base is [batch][W]
     int32_t Q;
     uint32_t* err;
+    __device__ __forceinline__ bool all() const { return base == nullptr; }
     __device__ __forceinline__ const uint32_t* row(int r, int W, bool report) const {
+        if (all()) return nullptr;
         if (!row_state) return base + (size_t)r * W;
         const int32_t q = __ldg(row_state + r);
         if (q < 0 || q >= Q) {
@@ -651,7 +678,12 @@ struct MaskRows {
         }
         return base + (size_t)q * W;
     }
+    // word j of a row given by row(); all-allowed rows read as all ones
+    __device__ __forceinline__ uint32_t word(const uint32_t* mrow, int j) const {
+        return all() ? 0xFFFFFFFFu : (mrow ? __ldg(mrow + j) : 0u);
+    }
 };
+
 constexpr int kStageDepth = 3;                // 32-word batches in flight per warp
 
 // Units are mask words (32 tokens); row r holds W units.  Each CTA takes a
@@ -663,17 +695,24 @@ constexpr int kStageDepth = 3;                // 32-word batches in flight per w
 // with cp.async (masks are read four batches ahead, logits two), and each lane
 // then folds its own word's allowed logits.  Otherwise each allowed logit is
 // read on its own.
-template <bool BF16, bool STAGE, bool SAMPLE>
+// What a row's allowed logits are folded into.
+enum Fold : int {
+    kFoldLse = 0,      // max, lowest-index argmax and sum of exp (log-sum-exp)
+    kFoldMax = 1,      // max and lowest-index argmax only (no lse requested)
+    kFoldSample = 2,   // Gumbel-max draw
+};
+
+template <bool BF16, bool STAGE, int FOLD>
 __global__ void __launch_bounds__(kReduceThreads)
     logits_reduce_kernel(const void* __restrict__ logits, int64_t stride, const MaskRows mask, int V,
                          int W, int B, long long per_cta, float4* __restrict__ partials,
                          uint32_t* __restrict__ counters, int32_t* __restrict__ argmax, float* __restrict__ lse,
-                         const SampleArgs sa, int row0) {
+                         const SampleArgs sa, int row0, const RowList list) {
     // [buffer][word][16-byte vector]
     __shared__ __align__(16) uint4 stage[STAGE ? kStageDepth * 32 * 4 : 1];
     pdl_wait();
     pdl_trigger();
-    const long long N = (long long)B * W;
+    const long long N = (long long)list.rows(B) * W;
     const int lane = threadIdx.x;
     long long u = (long long)blockIdx.x * per_cta;
     const long long u_end = min(N, u + per_cta);
@@ -683,19 +722,25 @@ __global__ void __launch_bounds__(kReduceThreads)
         const long long seg_end = min(u_end, row_end);
         const int j0 = (int)(u - (long long)r * W), j1 = (int)(seg_end - (long long)r * W);
         const uint32_t* mrow = mask.row(r, W, lane == 0 && j0 == 0);
-        const char* lrow = reinterpret_cast<const char*>(logits) + (size_t)r * stride * (BF16 ? 2 : 4);
+        const int orow = list.row(r);   // the batch row: logits, outputs and the sampling counter
+        const char* lrow = reinterpret_cast<const char*>(logits) + (size_t)orow * stride * (BF16 ? 2 : 4);
         float m = -INFINITY, mL = -INFINITY, s = 0.0f;
         int idx = INT_MAX;
         int blk = -1;                       // Philox block cached by gumbel_score
         uint4 rnd = make_uint4(0u, 0u, 0u, 0u);
         // one allowed logit x of token t (t increasing within a lane)
         auto fold = [&](float x, int t) {
-            if constexpr (SAMPLE) {
+            if constexpr (FOLD == kFoldSample) {
                 const float sx = __fmul_rn(x, sa.inv_t);
                 if (__fadd_rn(sx, kGumbelMax) < m) return;
-                const float sc = __fadd_rn(sx, gumbel(sa, row0 + r, t, blk, rnd));
+                const float sc = __fadd_rn(sx, gumbel(sa, row0 + orow, t, blk, rnd));
                 if (sc > m) {
                     m = sc;
+                    idx = t;
+                }
+            } else if constexpr (FOLD == kFoldMax) {
+                if (x > m) {
+                    m = x;
                     idx = t;
                 }
             } else {
@@ -707,7 +752,7 @@ __global__ void __launch_bounds__(kReduceThreads)
             const int full_words = V / 32;       // words whose 64 bytes of logits lie inside the row
             auto mask_of = [&](int b) -> uint32_t {
                 const int j = j0 + 32 * b + lane;
-                return (b < nb && j < j1 && mrow) ? __ldg(mrow + j) : 0u;
+                return (b < nb && j < j1) ? mask.word(mrow, j) : 0u;
             };
             auto issue = [&](int b, uint32_t mw) {
                 if (b < nb) {
@@ -737,7 +782,25 @@ __global__ void __launch_bounds__(kReduceThreads)
                 uint32_t word = mw[0];
                 if (word) {
                     const int t0 = j * 32;
-                    if (j < full_words) {
+                    if (FOLD == kFoldMax && j < full_words && __popc(word) > 12) {
+                        // a dense word: every token compared in order, no bit scan
+                        const uint4* sv = stage + (b % kStageDepth) * 128 + lane * 4;
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            if ((word >> (8 * k)) & 0xFFu) {
+                                const uint4 q = sv[k];
+                                const uint32_t qs[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+                                for (int hh = 0; hh < 8; ++hh) {
+                                    const float x = (hh & 1) ? bf16_hi(qs[hh >> 1]) : bf16_lo(qs[hh >> 1]);
+                                    if (((word >> (8 * k + hh)) & 1u) && x > m) {
+                                        m = x;
+                                        idx = t0 + 8 * k + hh;
+                                    }
+                                }
+                            }
+                        }
+                    } else if (j < full_words) {
                         const unsigned short* st =
                             reinterpret_cast<const unsigned short*>(stage + (b % kStageDepth) * 128 + lane * 4);
                         while (word) {
@@ -760,8 +823,8 @@ __global__ void __launch_bounds__(kReduceThreads)
             }
             cp_async_wait<0>();
         } else {
-            for (int j = j0 + lane; j < j1 && mrow; j += 32) {
-                uint32_t word = __ldg(mrow + j);
+            for (int j = j0 + lane; j < j1; j += 32) {
+                uint32_t word = mask.word(mrow, j);
                 const int t0 = j * 32;
                 while (word) {
                     const int e = __ffs(word) - 1;
@@ -777,8 +840,8 @@ __global__ void __launch_bounds__(kReduceThreads)
         bool is_last = false;
         if (lane == 0) {
             if (nseg == 1) {
-                argmax[r] = m == -INFINITY ? -1 : idx;
-                if (lse) lse[r] = m == -INFINITY ? -INFINITY : m + logf(s);
+                argmax[orow] = m == -INFINITY ? -1 : idx;
+                if (lse) lse[orow] = m == -INFINITY ? -INFINITY : m + logf(s);
             } else {
                 partials[(size_t)r * kMaxSegments + (blockIdx.x - first)] =
                     make_float4(m, __int_as_float(idx), s, 0.f);
@@ -798,8 +861,8 @@ __global__ void __launch_bounds__(kReduceThreads)
             }
             warp_merge(m, idx, s);
             if (lane == 0) {
-                argmax[r] = m == -INFINITY ? -1 : idx;
-                if (lse) lse[r] = m == -INFINITY ? -INFINITY : m + logf(s);
+                argmax[orow] = m == -INFINITY ? -1 : idx;
+                if (lse) lse[orow] = m == -INFINITY ? -INFINITY : m + logf(s);
                 counters[r] = 0u;   // ready for the next launch (stream-ordered)
             }
         }
@@ -826,7 +889,7 @@ __global__ void __launch_bounds__(kLogitThreads)
              u += (long long)gridDim.x * kLogitThreads) {
             const int r = (int)(u / nq), qd = (int)(u - (long long)r * nq);
             const uint32_t* mrow = mask.row(r, W, false);
-            const uint32_t nib = mrow ? (__ldg(mrow + (qd >> 3)) >> (4 * (qd & 7))) & 0xFu : 0u;
+            const uint32_t nib = (mask.word(mrow, qd >> 3) >> (4 * (qd & 7))) & 0xFu;
             float4 o = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
             if (nib) {
                 const char* lrow = reinterpret_cast<const char*>(logits) + (size_t)r * stride * 2;
@@ -845,7 +908,7 @@ __global__ void __launch_bounds__(kLogitThreads)
              u += (long long)gridDim.x * kLogitThreads) {
             const int r = (int)(u / W), j = (int)(u - (long long)r * W);
             const uint32_t* mrow = mask.row(r, W, false);
-            const uint32_t word = mrow ? __ldg(mrow + j) : 0u;
+            const uint32_t word = mask.word(mrow, j);
             const char* lrow = reinterpret_cast<const char*>(logits) + (size_t)r * stride * (BF16 ? 2 : 4);
             float* orow = out + (size_t)r * V + (size_t)j * 32;
             const float l = __ldg(lse + r);
@@ -897,6 +960,177 @@ __global__ void __launch_bounds__(kAdvanceThreads)
     }
     states_out[b] = (int32_t)s;
     if (stacks_out) stacks_out[b] = ((uint64_t)depth << 32) | bits;
+}
+
+// Opportunistic masking, the check: is row b's proposal (its unmasked argmax)
+// allowed from the row's configuration?  The same rule as the mask: the walk
+// stays live; EOS needs an accepting state and an empty stack; other empty
+// tokens never pass.  Allowed proposals are the row's decoded token; rejected
+// (and invalid) rows are appended to the fallback list.
+template <bool STACK, int MODE>
+__global__ void __launch_bounds__(kAdvanceThreads)
+    propose_check_kernel(const StepView v, const int32_t* __restrict__ states, const uint64_t* __restrict__ stacks,
+                         const int32_t* __restrict__ proposals, int32_t batch, int32_t* __restrict__ tokens_out,
+                         int32_t* __restrict__ row_ids, int32_t* __restrict__ row_count) {
+    using E = typename std::conditional<STACK, uint32_t, uint16_t>::type;
+    pdl_wait();
+    pdl_trigger();
+    const int b = blockIdx.x * kAdvanceThreads + threadIdx.x;
+    if (b >= batch) return;
+    const int32_t t = proposals[b];
+    bool ok = false;
+    if (t >= 0 && t < v.V) {
+        const uint4 rc = read_row(v, states, stacks, b, false);   // the fallback reports invalid rows
+        if (rc.w & 1u) {
+            if (t == v.eos_id) {
+                ok = (rc.w & 2u) != 0u;
+            } else {
+                Tab<E, MODE == kDenseSmem ? kDenseGlobal : MODE> tab;
+                tab.dense = reinterpret_cast<const E*>(STACK ? (const void*)v.t32 : (const void*)v.t16);
+                tab.sp = v.sp_info;
+                tab.tgt = reinterpret_cast<const E*>(v.sp_tgt);
+                tab.K = (uint32_t)v.K;
+                const int p = __ldg(v.pos_of + t);
+                const int len = (int)(__ldg(v.info + p) >> 16);
+                if (len > 0) {
+                    const uint8_t* hp = reinterpret_cast<const uint8_t*>(v.head + 2 * (size_t)p);
+                    const uint8_t* tail = len > kInlineBytes ? v.tail + __ldg(v.tail_off + p) : v.tail;
+                    uint32_t bits = rc.y, depth = rc.z;
+                    ok = walk<STACK, 0>(tab, v.ret, (uint32_t)v.max_depth, rc.x, bits, depth, hp, len, tail) != 0u;
+                }
+            }
+        }
+    }
+    if (ok) {
+        tokens_out[b] = t;
+    } else {
+        row_ids[atomicAdd(row_count, 1)] = b;
+    }
+}
+
+// ---- count-based speculation (Sec. 3.6) ------------------------------------
+// The count model is keyed by (scanner state, top of the bracket stack):
+// key = state for a DFA, state * 3 + top for a pushdown automaton (top 0: empty
+// stack, 1 + symbol otherwise).  best[key] packs the largest count with the
+// complement of its token id, so atomicMax keeps the most frequent token and,
+// on equal counts, the lowest id, whatever order the updates come in.
+__device__ __forceinline__ uint32_t spec_key(bool stack, uint32_t s, uint32_t bits, uint32_t depth) {
+    if (!stack) return s;
+    return s * 3u + (depth == 0 ? 0u : 1u + (bits & 1u));
+}
+
+template <bool STACK>
+__global__ void __launch_bounds__(kAdvanceThreads)
+    spec_update_kernel(const StepView v, const int32_t* __restrict__ states, const uint64_t* __restrict__ stacks,
+                       const int32_t* __restrict__ tokens, int32_t batch, uint32_t* __restrict__ counts,
+                       unsigned long long* __restrict__ best, uint32_t* __restrict__ reached) {
+    pdl_wait();
+    pdl_trigger();
+    const int b = blockIdx.x * kAdvanceThreads + threadIdx.x;
+    if (b >= batch) return;
+    const int32_t t = tokens[b];
+    if (t < 0 || t >= v.V) return;
+    const uint4 rc = read_row(v, states, stacks, b, false);
+    if (!(rc.w & 1u)) return;
+    const uint32_t key = spec_key(STACK, rc.x, rc.y, rc.z);
+    atomicAdd(reached + key, 1u);
+    const uint32_t c = atomicAdd(counts + (size_t)key * v.V + t, 1u) + 1u;
+    atomicMax(best + key, ((unsigned long long)c << 32) | (0xFFFFFFFFu - (uint32_t)t));
+}
+
+// Up to s proposals per row, each the key's most frequent token while
+// count * 1000 >= min_permille * reached; a proposal must be allowed from the
+// chain's configuration (walked; EOS needs an accepting state and an empty
+// stack, and ends the chain).  chain_* [batch][s + 1]: configurations after
+// 0..s proposals, the last one repeated past the chain's end.
+template <bool STACK, int MODE>
+__global__ void __launch_bounds__(kAdvanceThreads)
+    spec_propose_kernel(const StepView v, const int32_t* __restrict__ states, const uint64_t* __restrict__ stacks,
+                        int32_t batch, int32_t s, int32_t min_permille, const unsigned long long* __restrict__ best,
+                        const uint32_t* __restrict__ reached, int32_t* __restrict__ proposals,
+                        int32_t* __restrict__ n_prop, int32_t* __restrict__ chain_states,
+                        uint64_t* __restrict__ chain_stacks) {
+    using E = typename std::conditional<STACK, uint32_t, uint16_t>::type;
+    pdl_wait();
+    pdl_trigger();
+    const int b = blockIdx.x * kAdvanceThreads + threadIdx.x;
+    if (b >= batch) return;
+    Tab<E, MODE == kDenseSmem ? kDenseGlobal : MODE> tab;
+    tab.dense = reinterpret_cast<const E*>(STACK ? (const void*)v.t32 : (const void*)v.t16);
+    tab.sp = v.sp_info;
+    tab.tgt = reinterpret_cast<const E*>(v.sp_tgt);
+    tab.K = (uint32_t)v.K;
+    const int32_t sv = __ldg(states + b);
+    const unsigned long long wv = stacks ? __ldg(reinterpret_cast<const unsigned long long*>(stacks) + b) : 0ull;
+    const uint4 rc = decode_row(v, sv, wv, stacks != nullptr, v.accept_bits, false);
+    uint32_t q = rc.x, bits = rc.y, depth = rc.z;
+    int n = 0;
+    int32_t* prow = proposals + (size_t)b * s;
+    int32_t* crow = chain_states + (size_t)b * (s + 1);
+    uint64_t* krow = chain_stacks ? chain_stacks + (size_t)b * (s + 1) : nullptr;
+    crow[0] = sv;
+    if (krow) krow[0] = wv;
+    bool go = (rc.w & 1u) != 0u;
+    while (go && n < s) {
+        const uint32_t key = spec_key(STACK, q, bits, depth);
+        const uint32_t R = __ldg(reached + key);
+        const unsigned long long bk = __ldg(best + key);
+        const uint32_t c = (uint32_t)(bk >> 32);
+        const int32_t t = (int32_t)(0xFFFFFFFFu - (uint32_t)bk);
+        if (R == 0u || c == 0u || (unsigned long long)c * 1000ull < (unsigned long long)min_permille * R) break;
+        if (t == v.eos_id) {
+            const bool acc = depth == 0 && ((__ldg(v.accept_bits + (q >> 5)) >> (q & 31u)) & 1u);
+            if (!acc) break;
+            prow[n] = t;
+            ++n;
+            crow[n] = (int32_t)q;
+            if (krow) krow[n] = ((uint64_t)depth << 32) | bits;
+            break;
+        }
+        const int p = __ldg(v.pos_of + t);
+        const int len = (int)(__ldg(v.info + p) >> 16);
+        if (len == 0) break;
+        const uint8_t* hp = reinterpret_cast<const uint8_t*>(v.head + 2 * (size_t)p);
+        const uint8_t* tail = len > kInlineBytes ? v.tail + __ldg(v.tail_off + p) : v.tail;
+        uint32_t nb = bits, nd = depth;
+        const uint32_t nq = walk<STACK, 0>(tab, v.ret, (uint32_t)v.max_depth, q, nb, nd, hp, len, tail);
+        if (nq == 0u) break;
+        prow[n] = t;
+        q = nq;
+        bits = nb;
+        depth = nd;
+        ++n;
+        crow[n] = (int32_t)q;
+        if (krow) krow[n] = ((uint64_t)depth << 32) | bits;
+    }
+    n_prop[b] = n;
+    for (int i = n; i < s; ++i) prow[i] = -1;
+    for (int i = n + 1; i <= s; ++i) {
+        crow[i] = crow[n];
+        if (krow) krow[i] = krow[n];
+    }
+}
+
+// n_accept[b]: leading proposals equal to the constrained decode at their
+// chain configuration; tokens_out[b] the decode after them and
+// states_out / stacks_out the chain configuration it is decoded from.
+__global__ void __launch_bounds__(kAdvanceThreads)
+    spec_accept_kernel(const int32_t* __restrict__ proposals, const int32_t* __restrict__ n_prop,
+                       const int32_t* __restrict__ decoded, const int32_t* __restrict__ chain_states,
+                       const uint64_t* __restrict__ chain_stacks, int32_t batch, int32_t s,
+                       int32_t* __restrict__ n_accept, int32_t* __restrict__ tokens_out,
+                       int32_t* __restrict__ states_out, uint64_t* __restrict__ stacks_out) {
+    pdl_wait();
+    pdl_trigger();
+    const int b = blockIdx.x * kAdvanceThreads + threadIdx.x;
+    if (b >= batch) return;
+    const int n = n_prop[b];
+    int k = 0;
+    while (k < n && decoded[(size_t)b * (s + 1) + k] == proposals[(size_t)b * s + k]) ++k;
+    n_accept[b] = k;
+    if (tokens_out) tokens_out[b] = decoded[(size_t)b * (s + 1) + k];
+    if (states_out) states_out[b] = chain_states[(size_t)b * (s + 1) + k];
+    if (stacks_out && chain_stacks) stacks_out[b] = chain_stacks[(size_t)b * (s + 1) + k];
 }
 
 // Alg. 1 update from the precomputed state x token table: one read of
@@ -956,7 +1190,8 @@ int rows_per_tile(const StepView& v, const LaunchEnv& env, int batch, bool next,
 
 template <bool STACK, int MODE, bool NEXT>
 cudaError_t launch_step_t(const StepView& v, const LaunchEnv& env, const int32_t* states, const uint64_t* stacks,
-                          int32_t batch, bool row_is_state, uint32_t* mask, int32_t* next, cudaStream_t st) {
+                          int32_t batch, bool row_is_state, uint32_t* mask, int32_t* next, const RowList& list,
+                          cudaStream_t st) {
     const int img_bytes = MODE == kDenseGlobal ? 0 : (int)table_smem_bytes(v, STACK, MODE);
     const int R = rows_per_tile(v, env, batch, NEXT, STACK, img_bytes);
     const StepLayout L = step_layout(v.K, R, NEXT, STACK, v.max_units, v.Q, img_bytes);
@@ -988,29 +1223,31 @@ cudaError_t launch_step_t(const StepView& v, const LaunchEnv& env, const int32_t
         }
     }
     return launch_pdl(kern, dim3(grid), dim3(kStepThreads), (size_t)L.total, st, v, img, img_bytes, tgt_off, ret_off,
-                      states, stacks, batch, R, n_row_tiles, n_tiles, row_is_state ? 1 : 0, mask, next);
+                      states, stacks, batch, R, n_row_tiles, n_tiles, row_is_state ? 1 : 0, mask, next, list);
 }
 
 template <bool STACK, int MODE>
 cudaError_t launch_step_n(const StepView& v, const LaunchEnv& env, const int32_t* states, const uint64_t* stacks,
-                          int32_t batch, bool row_is_state, uint32_t* mask, int32_t* next, cudaStream_t st) {
-    if (next) return launch_step_t<STACK, MODE, true>(v, env, states, stacks, batch, row_is_state, mask, next, st);
-    return launch_step_t<STACK, MODE, false>(v, env, states, stacks, batch, row_is_state, mask, next, st);
+                          int32_t batch, bool row_is_state, uint32_t* mask, int32_t* next, const RowList& list,
+                          cudaStream_t st) {
+    if (next)
+        return launch_step_t<STACK, MODE, true>(v, env, states, stacks, batch, row_is_state, mask, next, list, st);
+    return launch_step_t<STACK, MODE, false>(v, env, states, stacks, batch, row_is_state, mask, next, list, st);
 }
 
 template <bool STACK>
 cudaError_t launch_step_s(const StepView& v, const LaunchEnv& env, int mode, const int32_t* states,
                           const uint64_t* stacks, int32_t batch, bool row_is_state, uint32_t* mask, int32_t* next,
-                          cudaStream_t st) {
+                          const RowList& list, cudaStream_t st) {
     switch (mode) {
         case kDenseSmem:
-            return launch_step_n<STACK, kDenseSmem>(v, env, states, stacks, batch, row_is_state, mask, next, st);
+            return launch_step_n<STACK, kDenseSmem>(v, env, states, stacks, batch, row_is_state, mask, next, list, st);
         case kSparse32Smem:
-            return launch_step_n<STACK, kSparse32Smem>(v, env, states, stacks, batch, row_is_state, mask, next, st);
+            return launch_step_n<STACK, kSparse32Smem>(v, env, states, stacks, batch, row_is_state, mask, next, list, st);
         case kSparse64Smem:
-            return launch_step_n<STACK, kSparse64Smem>(v, env, states, stacks, batch, row_is_state, mask, next, st);
+            return launch_step_n<STACK, kSparse64Smem>(v, env, states, stacks, batch, row_is_state, mask, next, list, st);
         default:
-            return launch_step_n<STACK, kDenseGlobal>(v, env, states, stacks, batch, row_is_state, mask, next, st);
+            return launch_step_n<STACK, kDenseGlobal>(v, env, states, stacks, batch, row_is_state, mask, next, list, st);
     }
 }
 
@@ -1039,18 +1276,24 @@ template <bool BF16, bool STAGE>
 cudaError_t launch_logits_t(const LaunchEnv& env, const void* logits, int32_t batch, int64_t stride, int32_t V,
                             const MaskRows& mask, int32_t* argmax, float* lse, float* logprobs, float4* partials,
                             uint32_t* counters, float* lse_tmp, bool out_vec, const SampleArgs* sample,
-                            cudaStream_t st) {
+                            const RowList& list, cudaStream_t st) {
     const int W = (V + 31) / 32;
     const size_t esz = BF16 ? 2 : 4;
     const SampleArgs sa = sample ? *sample : SampleArgs{0u, 0u, 0u, 0u, 1.0f};
-    auto reduce = sample ? logits_reduce_kernel<BF16, STAGE, true> : logits_reduce_kernel<BF16, STAGE, false>;
+    auto reduce = sample ? logits_reduce_kernel<BF16, STAGE, kFoldSample>
+                         : (lse || logprobs) ? logits_reduce_kernel<BF16, STAGE, kFoldLse>
+                                             : logits_reduce_kernel<BF16, STAGE, kFoldMax>;
     for (int32_t r0 = 0; r0 < batch; r0 += kMaxLogitRows) {
         const int rows = min(kMaxLogitRows, batch - r0);
-        const void* lg = reinterpret_cast<const char*>(logits) + (size_t)r0 * stride * esz;
+        // a row list addresses batch rows itself: logits and outputs stay unshifted
+        const size_t shift = list.ids ? 0 : (size_t)r0;
+        const void* lg = reinterpret_cast<const char*>(logits) + shift * stride * esz;
         MaskRows mk = mask;
         if (mk.row_state) mk.row_state += r0;
-        else mk.base += (size_t)r0 * W;
-        float* lse_rows = lse ? lse + r0 : (logprobs ? lse_tmp : nullptr);
+        else if (mk.base) mk.base += (size_t)r0 * W;
+        RowList lst = list;
+        lst.base = r0;
+        float* lse_rows = lse ? lse + shift : (logprobs ? lse_tmp : nullptr);
         const long long N = (long long)rows * W;
         int grid = env.num_sms * occupancy((const void*)reduce, kReduceThreads);
         grid = (int)std::min<long long>((long long)grid, (N + 127) / 128);   // at least 4 batches per warp
@@ -1060,7 +1303,7 @@ cudaError_t launch_logits_t(const LaunchEnv& env, const void* logits, int32_t ba
         grid = (int)((N + per_cta - 1) / per_cta);
         // a sampling pass draws row r of this chunk with counter row r0 + r
         cudaError_t e0 = launch_pdl(reduce, dim3(grid), dim3(kReduceThreads), 0, st, lg, stride, mk, V, W, rows,
-                                    per_cta, partials, counters, argmax + r0, lse_rows, sa, r0);
+                                    per_cta, partials, counters, argmax + shift, lse_rows, sa, (int)shift, lst);
         if (e0 != cudaSuccess) return e0;
         if (logprobs) {
             const long long n_items = (out_vec && STAGE) ? (long long)rows * (V / 4) : N;
@@ -1098,29 +1341,31 @@ int step_fixed_smem_bytes(const StepView& v, bool next) {
 
 cudaError_t launch_step_mask(const StepView& v, const LaunchEnv& env, bool stack, int mode, const int32_t* states,
                              const uint64_t* stacks, int32_t batch, bool row_is_state, uint32_t* mask,
-                             int32_t* next, cudaStream_t st) {
-    if (stack) return launch_step_s<true>(v, env, mode, states, stacks, batch, row_is_state, mask, next, st);
-    return launch_step_s<false>(v, env, mode, states, stacks, batch, row_is_state, mask, next, st);
+                             int32_t* next, cudaStream_t st, const int32_t* row_ids, const int32_t* row_count) {
+    const RowList list{row_ids, row_count, 0};
+    if (stack) return launch_step_s<true>(v, env, mode, states, stacks, batch, row_is_state, mask, next, list, st);
+    return launch_step_s<false>(v, env, mode, states, stacks, batch, row_is_state, mask, next, list, st);
 }
 
 cudaError_t launch_mask_logits(const LaunchEnv& env, const void* logits, int dtype, int32_t batch,
                                int64_t row_stride, int32_t V, const uint32_t* mask, int32_t* argmax, float* lse,
                                float* logprobs, float4* partials, uint32_t* counters, float* lse_tmp,
                                cudaStream_t st, const int32_t* row_state, int32_t Q, uint32_t* err,
-                               const SampleArgs* sample) {
+                               const SampleArgs* sample, const int32_t* row_ids, const int32_t* row_count) {
     const MaskRows mr{mask, row_state, Q, err};
+    const RowList list{row_ids, row_count, 0};
     const bool bf16 = dtype == DOMINO_DTYPE_BF16;
     const bool out_vec = logprobs && (reinterpret_cast<uintptr_t>(logprobs) % 16 == 0) && (V % 4 == 0);
     if (bf16) {
         const bool stage = (reinterpret_cast<uintptr_t>(logits) % 16 == 0) && ((size_t)row_stride * 2) % 16 == 0;
         if (stage)
             return launch_logits_t<true, true>(env, logits, batch, row_stride, V, mr, argmax, lse, logprobs,
-                                               partials, counters, lse_tmp, out_vec, sample, st);
+                                               partials, counters, lse_tmp, out_vec, sample, list, st);
         return launch_logits_t<true, false>(env, logits, batch, row_stride, V, mr, argmax, lse, logprobs, partials,
-                                            counters, lse_tmp, out_vec, sample, st);
+                                            counters, lse_tmp, out_vec, sample, list, st);
     }
     return launch_logits_t<false, false>(env, logits, batch, row_stride, V, mr, argmax, lse, logprobs, partials,
-                                         counters, lse_tmp, out_vec, sample, st);
+                                         counters, lse_tmp, out_vec, sample, list, st);
 }
 
 cudaError_t launch_mask_sample(const LaunchEnv& env, const void* logits, int dtype, int32_t batch,
@@ -1167,6 +1412,63 @@ cudaError_t launch_advance_table(const int32_t* table_next, int32_t Q, int32_t V
     const unsigned grid = (unsigned)((batch + kAdvanceThreads - 1) / kAdvanceThreads);
     return launch_pdl(advance_table_kernel, dim3(grid), dim3(kAdvanceThreads), 0, st, table_next, Q, V, eos_id, start,
                       states, tokens, batch, states_out, err);
+}
+
+cudaError_t launch_propose_check(const StepView& v, bool stack, int mode, const int32_t* states,
+                                 const uint64_t* stacks, const int32_t* proposals, int32_t batch, int32_t* tokens_out,
+                                 int32_t* row_ids, int32_t* row_count, cudaStream_t st) {
+    const unsigned grid = (unsigned)((batch + kAdvanceThreads - 1) / kAdvanceThreads);
+    auto pick = [&](auto kern) {
+        return launch_pdl(kern, dim3(grid), dim3(kAdvanceThreads), 0, st, v, states, stacks, proposals, batch,
+                          tokens_out, row_ids, row_count);
+    };
+    if (stack) {
+        if (mode == kSparse32Smem) return pick(propose_check_kernel<true, kSparse32Smem>);
+        if (mode == kSparse64Smem) return pick(propose_check_kernel<true, kSparse64Smem>);
+        return pick(propose_check_kernel<true, kDenseGlobal>);
+    }
+    if (mode == kSparse32Smem) return pick(propose_check_kernel<false, kSparse32Smem>);
+    if (mode == kSparse64Smem) return pick(propose_check_kernel<false, kSparse64Smem>);
+    return pick(propose_check_kernel<false, kDenseGlobal>);
+}
+
+cudaError_t launch_spec_update(const StepView& v, bool stack, const int32_t* states, const uint64_t* stacks,
+                               const int32_t* tokens, int32_t batch, uint32_t* counts, unsigned long long* best,
+                               uint32_t* reached, cudaStream_t st) {
+    const unsigned grid = (unsigned)((batch + kAdvanceThreads - 1) / kAdvanceThreads);
+    if (stack)
+        return launch_pdl(spec_update_kernel<true>, dim3(grid), dim3(kAdvanceThreads), 0, st, v, states, stacks,
+                          tokens, batch, counts, best, reached);
+    return launch_pdl(spec_update_kernel<false>, dim3(grid), dim3(kAdvanceThreads), 0, st, v, states, stacks, tokens,
+                      batch, counts, best, reached);
+}
+
+cudaError_t launch_spec_propose(const StepView& v, bool stack, int mode, const int32_t* states,
+                                const uint64_t* stacks, int32_t batch, int32_t s, int32_t min_permille,
+                                const unsigned long long* best, const uint32_t* reached, int32_t* proposals,
+                                int32_t* n_prop, int32_t* chain_states, uint64_t* chain_stacks, cudaStream_t st) {
+    const unsigned grid = (unsigned)((batch + kAdvanceThreads - 1) / kAdvanceThreads);
+    auto pick = [&](auto kern) {
+        return launch_pdl(kern, dim3(grid), dim3(kAdvanceThreads), 0, st, v, states, stacks, batch, s, min_permille,
+                          best, reached, proposals, n_prop, chain_states, chain_stacks);
+    };
+    if (stack) {
+        if (mode == kSparse32Smem) return pick(spec_propose_kernel<true, kSparse32Smem>);
+        if (mode == kSparse64Smem) return pick(spec_propose_kernel<true, kSparse64Smem>);
+        return pick(spec_propose_kernel<true, kDenseGlobal>);
+    }
+    if (mode == kSparse32Smem) return pick(spec_propose_kernel<false, kSparse32Smem>);
+    if (mode == kSparse64Smem) return pick(spec_propose_kernel<false, kSparse64Smem>);
+    return pick(spec_propose_kernel<false, kDenseGlobal>);
+}
+
+cudaError_t launch_spec_accept(const int32_t* proposals, const int32_t* n_prop, const int32_t* decoded,
+                               const int32_t* chain_states, const uint64_t* chain_stacks, int32_t batch, int32_t s,
+                               int32_t* n_accept, int32_t* tokens_out, int32_t* states_out, uint64_t* stacks_out,
+                               cudaStream_t st) {
+    const unsigned grid = (unsigned)((batch + kAdvanceThreads - 1) / kAdvanceThreads);
+    return launch_pdl(spec_accept_kernel, dim3(grid), dim3(kAdvanceThreads), 0, st, proposals, n_prop, decoded,
+                      chain_states, chain_stacks, batch, s, n_accept, tokens_out, states_out, stacks_out);
 }
 
 }  // namespace domino
