@@ -782,23 +782,50 @@ __global__ void __launch_bounds__(kReduceThreads)
                 uint32_t word = mw[0];
                 if (word) {
                     const int t0 = j * 32;
-                    if (FOLD == kFoldMax && j < full_words && __popc(word) > 12) {
-                        // a dense word: every token compared in order, no bit scan
+                    if (FOLD != kFoldSample && j < full_words && __popc(word) > 12) {
+                        // a dense word: the word's maximum first (every token compared in
+                        // order, no bit scan), then, for the log-sum-exp, one rescale and
+                        // the sum of the word's terms
                         const uint4* sv = stage + (b % kStageDepth) * 128 + lane * 4;
+                        uint32_t qs[16];
 #pragma unroll
                         for (int k = 0; k < 4; ++k) {
-                            if ((word >> (8 * k)) & 0xFFu) {
-                                const uint4 q = sv[k];
-                                const uint32_t qs[4] = {q.x, q.y, q.z, q.w};
+                            const uint4 q = ((word >> (8 * k)) & 0xFFu) ? sv[k] : make_uint4(0u, 0u, 0u, 0u);
+                            qs[4 * k] = q.x;
+                            qs[4 * k + 1] = q.y;
+                            qs[4 * k + 2] = q.z;
+                            qs[4 * k + 3] = q.w;
+                        }
+                        float wm = -INFINITY;
+                        int wi = 0;
 #pragma unroll
-                                for (int hh = 0; hh < 8; ++hh) {
-                                    const float x = (hh & 1) ? bf16_hi(qs[hh >> 1]) : bf16_lo(qs[hh >> 1]);
-                                    if (((word >> (8 * k + hh)) & 1u) && x > m) {
-                                        m = x;
-                                        idx = t0 + 8 * k + hh;
-                                    }
-                                }
+                        for (int e = 0; e < 32; ++e) {
+                            const float x = (e & 1) ? bf16_hi(qs[e >> 1]) : bf16_lo(qs[e >> 1]);
+                            if (((word >> e) & 1u) && x > wm) {
+                                wm = x;
+                                wi = e;
                             }
+                        }
+                        if constexpr (FOLD == kFoldMax) {
+                            if (wm > m) {
+                                m = wm;
+                                idx = t0 + wi;
+                            }
+                        } else {
+                            if (wm > m) {   // earlier words hold lower ids: equal maxima keep idx
+                                const float wL = wm * kLog2e;
+                                s = s == 0.0f ? 0.0f : s * ex2(mL - wL);
+                                m = wm;
+                                mL = wL;
+                                idx = t0 + wi;
+                            }
+                            float acc = 0.0f;
+#pragma unroll
+                            for (int e = 0; e < 32; ++e) {
+                                const float x = (e & 1) ? bf16_hi(qs[e >> 1]) : bf16_lo(qs[e >> 1]);
+                                acc += ((word >> e) & 1u) ? ex2(fmaf(x, kLog2e, -mL)) : 0.0f;
+                            }
+                            s += acc;
                         }
                     } else if (j < full_words) {
                         const unsigned short* st =
@@ -871,18 +898,62 @@ __global__ void __launch_bounds__(kReduceThreads)
 }
 
 // logprob[t] = logit[t] - lse for allowed t, -inf otherwise.  VEC (bf16 rows on
-// 16-byte boundaries, V % 4 == 0): a thread takes 4 consecutive tokens, reads
-// their 8 bytes of logits (not at all when none is allowed) and writes one
-// float4, so a warp's stores cover 512 contiguous bytes; grid-stride over the
-// batch x V/4 quads.  Otherwise one mask word (32 tokens) per thread, one token
-// at a time.
+// 16-byte boundaries, V % 4 == 0): a thread takes 16 consecutive tokens when
+// V % 16 == 0 (32 bytes of logits read unconditionally, four float4 stores),
+// else 4 (their 8 bytes read only when one is allowed, one float4 store);
+// grid-stride over the batch's groups.  Otherwise one mask word (32 tokens) per
+// thread, one token at a time.
 template <bool BF16, bool VEC>
 __global__ void __launch_bounds__(kLogitThreads)
     logprobs_kernel(const void* __restrict__ logits, int64_t stride, const MaskRows mask, int V, int W,
-                    int B, const float* __restrict__ lse, float* __restrict__ out) {
+                    int B, const float* __restrict__ lse, float* __restrict__ out, int wide) {
     pdl_wait();
     pdl_trigger();
-    if constexpr (VEC && BF16) {
+    if (VEC && BF16 && V % 16 == 0) {
+        // 16 tokens per thread: two 16-byte logit loads and the mask half-word,
+        // all independent, then four float4 stores
+        const int ng = V / 16;
+        const long long N = (long long)B * ng;
+        for (long long u = (long long)blockIdx.x * kLogitThreads + threadIdx.x; u < N;
+             u += (long long)gridDim.x * kLogitThreads) {
+            const int r = (int)(u / ng), g = (int)(u - (long long)r * ng);
+            const uint32_t* mrow = mask.row(r, W, false);
+            const char* lrow = reinterpret_cast<const char*>(logits) + (size_t)r * stride * 2;
+            const uint4* src = reinterpret_cast<const uint4*>(lrow) + 2 * (size_t)g;
+            uint32_t ws[8];
+            if (wide) {   // one 32-byte load (32-byte aligned rows)
+                asm volatile("ld.global.cs.v8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                             : "=r"(ws[0]), "=r"(ws[1]), "=r"(ws[2]), "=r"(ws[3]), "=r"(ws[4]), "=r"(ws[5]),
+                               "=r"(ws[6]), "=r"(ws[7])
+                             : "l"(src));
+            } else {
+                const uint4 a = __ldcs(src), c = __ldcs(src + 1);
+                ws[0] = a.x; ws[1] = a.y; ws[2] = a.z; ws[3] = a.w;
+                ws[4] = c.x; ws[5] = c.y; ws[6] = c.z; ws[7] = c.w;
+            }
+            const uint32_t bits = (mask.word(mrow, g >> 1) >> (16 * (g & 1))) & 0xFFFFu;
+            const float l = __ldg(lse + r);
+            float o[16];
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                const float x = (e & 1) ? bf16_hi(ws[e >> 1]) : bf16_lo(ws[e >> 1]);
+                o[e] = ((bits >> e) & 1u) ? x - l : -INFINITY;
+            }
+            float* dst = out + (size_t)r * V + 16 * (size_t)g;
+            if (wide) {   // two 32-byte stores
+#pragma unroll
+                for (int h = 0; h < 2; ++h)
+                    asm volatile("st.global.cs.v8.f32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"l"(dst + 8 * h),
+                                 "f"(o[8 * h]), "f"(o[8 * h + 1]), "f"(o[8 * h + 2]), "f"(o[8 * h + 3]),
+                                 "f"(o[8 * h + 4]), "f"(o[8 * h + 5]), "f"(o[8 * h + 6]), "f"(o[8 * h + 7])
+                                 : "memory");
+            } else {
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    __stcs(reinterpret_cast<float4*>(dst) + q, make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]));
+            }
+        }
+    } else if constexpr (VEC && BF16) {
         const int nq = V / 4;
         const long long N = (long long)B * nq;
         for (long long u = (long long)blockIdx.x * kLogitThreads + threadIdx.x; u < N;
@@ -1306,15 +1377,19 @@ cudaError_t launch_logits_t(const LaunchEnv& env, const void* logits, int32_t ba
                                     per_cta, partials, counters, argmax + shift, lse_rows, sa, (int)shift, lst);
         if (e0 != cudaSuccess) return e0;
         if (logprobs) {
-            const long long n_items = (out_vec && STAGE) ? (long long)rows * (V / 4) : N;
+            const long long n_items = (out_vec && STAGE) ? (long long)rows * (V % 16 == 0 ? V / 16 : V / 4) : N;
             int g2 = env.num_sms * occupancy((const void*)logprobs_kernel<BF16, true>, kLogitThreads);
             g2 = (int)std::max<long long>(1, std::min<long long>((long long)g2,
                                                                  (n_items + kLogitThreads - 1) / kLogitThreads));
+            // 32-byte vector loads and stores where rows start on 32-byte boundaries
+            float* lp = logprobs + (size_t)r0 * V;
+            const int wide = (reinterpret_cast<uintptr_t>(lg) % 32 == 0) && ((size_t)stride * esz) % 32 == 0 &&
+                             (reinterpret_cast<uintptr_t>(lp) % 32 == 0) && V % 16 == 0;
             cudaError_t e1 = (out_vec && STAGE)
                                  ? launch_pdl(logprobs_kernel<BF16, true>, dim3(g2), dim3(kLogitThreads), 0, st, lg,
-                                              stride, mk, V, W, rows, (const float*)lse_rows, logprobs + (size_t)r0 * V)
+                                              stride, mk, V, W, rows, (const float*)lse_rows, lp, wide)
                                  : launch_pdl(logprobs_kernel<BF16, false>, dim3(g2), dim3(kLogitThreads), 0, st, lg,
-                                              stride, mk, V, W, rows, (const float*)lse_rows, logprobs + (size_t)r0 * V);
+                                              stride, mk, V, W, rows, (const float*)lse_rows, lp, 0);
             if (e1 != cudaSuccess) return e1;
         }
     }
