@@ -60,6 +60,11 @@ struct domino_ctx {
     DevBuf s_logits, s_states, s_stacks, s_mask, s_tokens, s_lse;
     // opportunistic masking: proposals, the fallback row list and its length
     DevBuf o_prop, o_rows, o_count;
+    // domino_decode_step_host: a copy stream and the events that hand each
+    // chunk of rows from the copies to the kernels
+    cudaStream_t cp_stream = nullptr;
+    cudaEvent_t ev_cfg = nullptr;
+    cudaEvent_t ev_chunk[8] = {};
 };
 
 namespace {
@@ -326,8 +331,12 @@ int domino_destroy(domino_t h) {
         DevBuf* all[] = {&h->d_head, &h->d_info, &h->d_tail_off, &h->d_tail, &h->d_pos_of, &h->d_units,
                          &h->d_unit_off, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_err, &h->d_partials,
                          &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_states, &h->s_stacks,
-                         &h->s_mask, &h->s_tokens, &h->s_lse};
+                         &h->s_mask, &h->s_tokens, &h->s_lse, &h->o_prop, &h->o_rows, &h->o_count};
         for (auto* b : all) dev_free(*b);
+        for (cudaEvent_t& e : h->ev_chunk)
+            if (e) cudaEventDestroy(e);
+        if (h->ev_cfg) cudaEventDestroy(h->ev_cfg);
+        if (h->cp_stream) cudaStreamDestroy(h->cp_stream);
         cudaGetLastError();
     }
     delete h;
@@ -792,8 +801,9 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
     DeviceGuard g(h->device);
     cudaStream_t st = (cudaStream_t)stream;
     const size_t esz = dtype == DOMINO_DTYPE_BF16 ? 2 : 4;
-    const size_t logit_bytes = (size_t)batch * (size_t)h->V * esz;
-    if (h->s_logits.n < logit_bytes || h->s_states.n < (size_t)batch * 4) {
+    const size_t row_bytes = (size_t)h->V * esz;
+    const size_t logit_bytes = (size_t)batch * row_bytes;
+    if (h->s_logits.n < logit_bytes || h->s_states.n < (size_t)batch * 4 || !h->cp_stream) {
         if (cudaStreamSynchronize(st) != cudaSuccess) return cuda_status(cudaGetLastError());
     }
     if ((rc = dev_reserve(h->s_logits, logit_bytes))) return rc;
@@ -802,23 +812,49 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
     if ((rc = dev_reserve(h->s_mask, (size_t)batch * (size_t)h->W * 4))) return rc;
     if ((rc = dev_reserve(h->s_tokens, (size_t)batch * 4))) return rc;
     if ((rc = dev_reserve(h->s_lse, (size_t)batch * 4))) return rc;
+    if (!h->cp_stream) {
+        cudaError_t e = cudaStreamCreateWithFlags(&h->cp_stream, cudaStreamNonBlocking);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_cfg, cudaEventDisableTiming);
+        for (cudaEvent_t& ev : h->ev_chunk)
+            if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+        if (e != cudaSuccess) return cuda_status(e);
+    }
     int32_t* d_states = (int32_t*)h->s_states.p;
     uint64_t* d_stacks = stacks_host ? (uint64_t*)h->s_stacks.p : nullptr;
-    cudaError_t e = cudaMemcpyAsync(h->s_logits.p, logits_host, logit_bytes, cudaMemcpyHostToDevice, st);
-    if (e == cudaSuccess)
-        e = cudaMemcpyAsync(d_states, states_host, (size_t)batch * 4, cudaMemcpyHostToDevice, st);
+    uint32_t* d_mask = (uint32_t*)h->s_mask.p;
+    int32_t* d_tok = (int32_t*)h->s_tokens.p;
+    float* d_lse = (float*)h->s_lse.p;
+    // The logits arrive in up to 8 chunks of rows on the copy stream; the mask
+    // step runs while they copy, and each chunk's masked argmax starts as soon
+    // as its rows have landed.
+    const int n_chunks = (int)std::max<size_t>(1, std::min<size_t>({(size_t)8, (size_t)batch, logit_bytes >> 23}));
+    cudaError_t e = cudaEventRecord(h->ev_cfg, st);   // the caller's earlier work on `stream` comes first
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(h->cp_stream, h->ev_cfg, 0);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(d_states, states_host, (size_t)batch * 4, cudaMemcpyHostToDevice, h->cp_stream);
     if (e == cudaSuccess && d_stacks)
-        e = cudaMemcpyAsync(d_stacks, stacks_host, (size_t)batch * 8, cudaMemcpyHostToDevice, st);
+        e = cudaMemcpyAsync(d_stacks, stacks_host, (size_t)batch * 8, cudaMemcpyHostToDevice, h->cp_stream);
+    if (e == cudaSuccess) e = cudaEventRecord(h->ev_cfg, h->cp_stream);
+    std::vector<int32_t> r0s((size_t)n_chunks + 1);
+    for (int k = 0; k <= n_chunks; ++k) r0s[(size_t)k] = (int32_t)(((int64_t)batch * k) / n_chunks);
+    for (int k = 0; k < n_chunks && e == cudaSuccess; ++k) {
+        const size_t off = (size_t)r0s[(size_t)k] * row_bytes, n = (size_t)(r0s[(size_t)k + 1] - r0s[(size_t)k]) * row_bytes;
+        e = cudaMemcpyAsync((char*)h->s_logits.p + off, (const char*)logits_host + off, n, cudaMemcpyHostToDevice,
+                            h->cp_stream);
+        if (e == cudaSuccess) e = cudaEventRecord(h->ev_chunk[k], h->cp_stream);
+    }
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(st, h->ev_cfg, 0);
     if (e != cudaSuccess) return cuda_status(e);
-    if ((rc = domino_step_mask(h, d_states, d_stacks, batch, (uint32_t*)h->s_mask.p, nullptr, stream))) return rc;
-    if ((rc = domino_mask_logits(h, h->s_logits.p, dtype, batch, h->V, (uint32_t*)h->s_mask.p,
-                                 (int32_t*)h->s_tokens.p, (float*)h->s_lse.p, nullptr, stream)))
-        return rc;
-    if ((rc = domino_advance(h, d_states, d_stacks, (int32_t*)h->s_tokens.p, batch, d_states, d_stacks, stream)))
-        return rc;
-    e = cudaMemcpyAsync(tokens_host, h->s_tokens.p, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
-    if (e == cudaSuccess && lse_host)
-        e = cudaMemcpyAsync(lse_host, h->s_lse.p, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
+    if ((rc = domino_step_mask(h, d_states, d_stacks, batch, d_mask, nullptr, stream))) return rc;
+    for (int k = 0; k < n_chunks; ++k) {
+        const int32_t r0 = r0s[(size_t)k], rows = r0s[(size_t)k + 1] - r0;
+        if ((e = cudaStreamWaitEvent(st, h->ev_chunk[k], 0)) != cudaSuccess) return cuda_status(e);
+        if ((rc = domino_mask_logits(h, (const char*)h->s_logits.p + (size_t)r0 * row_bytes, dtype, rows, h->V,
+                                     d_mask + (size_t)r0 * h->W, d_tok + r0, d_lse + r0, nullptr, stream)))
+            return rc;
+    }
+    if ((rc = domino_advance(h, d_states, d_stacks, d_tok, batch, d_states, d_stacks, stream))) return rc;
+    e = cudaMemcpyAsync(tokens_host, d_tok, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess && lse_host) e = cudaMemcpyAsync(lse_host, d_lse, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess) e = cudaMemcpyAsync(states_host, d_states, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess && d_stacks)
         e = cudaMemcpyAsync(stacks_host, d_stacks, (size_t)batch * 8, cudaMemcpyDeviceToHost, st);

@@ -280,6 +280,34 @@ def test_decode_loop_parity(config, steps):
             assert (sk.cpu().numpy().view(np.uint64) == k_o).all(), i
 
 
+@pytest.mark.parametrize("config", [3, 5])
+def test_decode_step_host_in_chunks_matches_oracle(config):
+    """The host-buffer step copies the logits in chunks of rows and decodes each
+    chunk as it lands; tokens, lse and new configurations match the oracle."""
+    import oracle
+    w = workload(config)
+    states, stacks = configs(config)
+    has_stack = w.automaton.rules is not None
+    d = handle(config)
+    lg = w.logits(5)
+    s_host = states.copy()
+    k_host = stacks.copy() if has_stack else None
+    tok = np.zeros(len(states), np.int32)
+    lse_h = np.zeros(len(states), np.float32)
+    dt = B.DTYPE_BF16 if lg.dtype == np.uint16 else B.DTYPE_F32
+    B.domino_decode_step_host(d.h, lg, dt, len(states), s_host, k_host, tok, lse_h, stream=0)
+    P = problem(config)
+    m, _, _ = P.step_mask(states, stacks if has_stack else None, n_threads=NT)
+    a_o, l_o, _ = oracle.mask_logits(lg, m)
+    s_o, k_o, _ = P.advance(states, stacks if has_stack else None, a_o, w.automaton.start)
+    assert (tok == a_o).all()
+    fin = np.isfinite(l_o)
+    assert np.abs(lse_h[fin] - l_o[fin]).max(initial=0) < TOL
+    assert (s_host == s_o).all()
+    if has_stack:
+        assert (k_host == k_o).all()
+
+
 def test_decode_step_host_matches_device_path():
     w = workload(2)
     states, _ = configs(2)
