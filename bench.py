@@ -779,7 +779,9 @@ def run_domino(args, dist: Dist):
         "kernels": kernels, "roofline": roofline, "table_driven_step": table_step,
         "opportunistic": opportunistic, "speculation": spec,
         "e2e": {"value": n * Bsz * V * Ke / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h, "steps": Ke, "api": "domino_decode_step_host (pinned host buffers)"},
+                "d2h_bytes_per_step": d2h, "steps": Ke, "api": "domino_decode_step_host with pinned host buffers",
+                "h2d_note": "h2d_bytes_per_step counts the whole logits tensor; the masked pass reads pinned logits "
+                            "in place, so only the 16-byte vectors holding an allowed token cross the link"},
         "gpu_launches": K * launches_per_step,
         "gpu_launches_note": "timed region only; per-kernel graphs and e2e are timed separately",
         "clocks": sampler.summary(),

@@ -65,6 +65,9 @@ struct domino_ctx {
     cudaStream_t cp_stream = nullptr;
     cudaEvent_t ev_cfg = nullptr;
     cudaEvent_t ev_chunk[8] = {};
+    DevBuf s_count;                 // non-zero mask bytes of the last step
+    uint64_t* h_count = nullptr;    // its pinned host copy
+    double vec_density = 0.0;       // share of logit vectors the last step's masks allowed
 };
 
 namespace {
@@ -93,7 +96,8 @@ int64_t dev_bytes(const domino_ctx* h) {
     const DevBuf* all[] = {&h->d_head, &h->d_info, &h->d_tail_off, &h->d_tail, &h->d_pos_of, &h->d_units,
                            &h->d_unit_off, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_err, &h->d_partials,
                            &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_states, &h->s_stacks,
-                           &h->s_mask, &h->s_tokens, &h->s_lse, &h->o_prop, &h->o_rows, &h->o_count};
+                           &h->s_mask, &h->s_tokens, &h->s_lse, &h->o_prop, &h->o_rows, &h->o_count,
+                           &h->s_count};
     int64_t n = 0;
     for (auto* b : all) n += (int64_t)b->n;
     return n;
@@ -331,12 +335,14 @@ int domino_destroy(domino_t h) {
         DevBuf* all[] = {&h->d_head, &h->d_info, &h->d_tail_off, &h->d_tail, &h->d_pos_of, &h->d_units,
                          &h->d_unit_off, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_err, &h->d_partials,
                          &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_states, &h->s_stacks,
-                         &h->s_mask, &h->s_tokens, &h->s_lse, &h->o_prop, &h->o_rows, &h->o_count};
+                         &h->s_mask, &h->s_tokens, &h->s_lse, &h->o_prop, &h->o_rows, &h->o_count,
+                           &h->s_count};
         for (auto* b : all) dev_free(*b);
         for (cudaEvent_t& e : h->ev_chunk)
             if (e) cudaEventDestroy(e);
         if (h->ev_cfg) cudaEventDestroy(h->ev_cfg);
         if (h->cp_stream) cudaStreamDestroy(h->cp_stream);
+        if (h->h_count) cudaFreeHost(h->h_count);
         cudaGetLastError();
     }
     delete h;
@@ -789,44 +795,23 @@ int domino_advance_table(domino_t h, const int32_t* table_next_dev, const int32_
                                             batch, states_out, (uint32_t*)h->d_err.p, (cudaStream_t)stream));
 }
 
-int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, int32_t batch,
-                            int32_t* states_host, uint64_t* stacks_host, int32_t* tokens_host, float* lse_host,
-                            void* stream) {
-    int rc = ready_for_compute(h);
-    if (rc) return rc;
-    if (dtype != DOMINO_DTYPE_F32 && dtype != DOMINO_DTYPE_BF16) return DOMINO_E_INVALID_ARG;
-    if (batch < 0) return DOMINO_E_INVALID_ARG;
-    if (batch == 0) return DOMINO_OK;
-    if (!logits_host || !states_host || !tokens_host) return DOMINO_E_INVALID_ARG;
-    DeviceGuard g(h->device);
-    cudaStream_t st = (cudaStream_t)stream;
+namespace {
+
+// Pageable logits: the configurations and then the logits are copied in up
+// to 8 chunks of rows on the copy stream; the mask step runs while they copy,
+// and each chunk's masked argmax starts as soon as its rows have landed.
+int copy_and_decode_chunks(domino_ctx* h, const void* logits_host, int32_t dtype, int32_t batch,
+                           const int32_t* states_host, const uint64_t* stacks_host, cudaStream_t st) {
+    int rc;
+    void* stream = (void*)st;
     const size_t esz = dtype == DOMINO_DTYPE_BF16 ? 2 : 4;
     const size_t row_bytes = (size_t)h->V * esz;
     const size_t logit_bytes = (size_t)batch * row_bytes;
-    if (h->s_logits.n < logit_bytes || h->s_states.n < (size_t)batch * 4 || !h->cp_stream) {
-        if (cudaStreamSynchronize(st) != cudaSuccess) return cuda_status(cudaGetLastError());
-    }
-    if ((rc = dev_reserve(h->s_logits, logit_bytes))) return rc;
-    if ((rc = dev_reserve(h->s_states, (size_t)batch * 4))) return rc;
-    if ((rc = dev_reserve(h->s_stacks, (size_t)batch * 8))) return rc;
-    if ((rc = dev_reserve(h->s_mask, (size_t)batch * (size_t)h->W * 4))) return rc;
-    if ((rc = dev_reserve(h->s_tokens, (size_t)batch * 4))) return rc;
-    if ((rc = dev_reserve(h->s_lse, (size_t)batch * 4))) return rc;
-    if (!h->cp_stream) {
-        cudaError_t e = cudaStreamCreateWithFlags(&h->cp_stream, cudaStreamNonBlocking);
-        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_cfg, cudaEventDisableTiming);
-        for (cudaEvent_t& ev : h->ev_chunk)
-            if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
-        if (e != cudaSuccess) return cuda_status(e);
-    }
     int32_t* d_states = (int32_t*)h->s_states.p;
     uint64_t* d_stacks = stacks_host ? (uint64_t*)h->s_stacks.p : nullptr;
     uint32_t* d_mask = (uint32_t*)h->s_mask.p;
     int32_t* d_tok = (int32_t*)h->s_tokens.p;
     float* d_lse = (float*)h->s_lse.p;
-    // The logits arrive in up to 8 chunks of rows on the copy stream; the mask
-    // step runs while they copy, and each chunk's masked argmax starts as soon
-    // as its rows have landed.
     const int n_chunks = (int)std::max<size_t>(1, std::min<size_t>({(size_t)8, (size_t)batch, logit_bytes >> 23}));
     cudaError_t e = cudaEventRecord(h->ev_cfg, st);   // the caller's earlier work on `stream` comes first
     if (e == cudaSuccess) e = cudaStreamWaitEvent(h->cp_stream, h->ev_cfg, 0);
@@ -852,15 +837,88 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
                                      d_mask + (size_t)r0 * h->W, d_tok + r0, d_lse + r0, nullptr, stream)))
             return rc;
     }
+    return DOMINO_OK;
+}
+
+}  // namespace
+
+int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, int32_t batch,
+                            int32_t* states_host, uint64_t* stacks_host, int32_t* tokens_host, float* lse_host,
+                            void* stream) {
+    int rc = ready_for_compute(h);
+    if (rc) return rc;
+    if (dtype != DOMINO_DTYPE_F32 && dtype != DOMINO_DTYPE_BF16) return DOMINO_E_INVALID_ARG;
+    if (batch < 0) return DOMINO_E_INVALID_ARG;
+    if (batch == 0) return DOMINO_OK;
+    if (!logits_host || !states_host || !tokens_host) return DOMINO_E_INVALID_ARG;
+    DeviceGuard g(h->device);
+    cudaStream_t st = (cudaStream_t)stream;
+    const size_t esz = dtype == DOMINO_DTYPE_BF16 ? 2 : 4;
+    const size_t row_bytes = (size_t)h->V * esz;
+    const size_t logit_bytes = (size_t)batch * row_bytes;
+    // Pinned (page-locked, mapped) logits are read where they are: the masked
+    // pass pulls only the 16-byte logit vectors that hold an allowed token
+    // across the host link, so masked-out logits never travel.  When the last
+    // step's masks allowed most vectors (and for fp32 rows) the chunked copy is
+    // used instead: it moves as many bytes but overlaps the mask step.
+    cudaPointerAttributes pa{};
+    const bool pinned = cudaPointerGetAttributes(&pa, logits_host) == cudaSuccess && pa.type == cudaMemoryTypeHost &&
+                        pa.devicePointer != nullptr;
+    if (!pinned) cudaGetLastError();
+    const bool mapped = pinned && dtype == DOMINO_DTYPE_BF16 && h->vec_density < 0.5;
+    if ((!mapped && h->s_logits.n < logit_bytes) || h->s_states.n < (size_t)batch * 4 || !h->cp_stream) {
+        if (cudaStreamSynchronize(st) != cudaSuccess) return cuda_status(cudaGetLastError());
+    }
+    if (!mapped && (rc = dev_reserve(h->s_logits, logit_bytes))) return rc;
+    if ((rc = dev_reserve(h->s_states, (size_t)batch * 4))) return rc;
+    if ((rc = dev_reserve(h->s_stacks, (size_t)batch * 8))) return rc;
+    if ((rc = dev_reserve(h->s_mask, (size_t)batch * (size_t)h->W * 4))) return rc;
+    if ((rc = dev_reserve(h->s_tokens, (size_t)batch * 4))) return rc;
+    if ((rc = dev_reserve(h->s_lse, (size_t)batch * 4))) return rc;
+    if ((rc = dev_reserve(h->s_count, 16))) return rc;
+    if (!h->cp_stream) {
+        if (cudaMallocHost((void**)&h->h_count, sizeof(uint64_t)) != cudaSuccess) {
+            cudaGetLastError();
+            h->h_count = nullptr;
+            return DOMINO_E_OOM;
+        }
+        cudaError_t e = cudaStreamCreateWithFlags(&h->cp_stream, cudaStreamNonBlocking);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_cfg, cudaEventDisableTiming);
+        for (cudaEvent_t& ev : h->ev_chunk)
+            if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+        if (e != cudaSuccess) return cuda_status(e);
+    }
+    int32_t* d_states = (int32_t*)h->s_states.p;
+    uint64_t* d_stacks = stacks_host ? (uint64_t*)h->s_stacks.p : nullptr;
+    uint32_t* d_mask = (uint32_t*)h->s_mask.p;
+    int32_t* d_tok = (int32_t*)h->s_tokens.p;
+    float* d_lse = (float*)h->s_lse.p;
+    if (mapped) {
+        cudaError_t e = cudaMemcpyAsync(d_states, states_host, (size_t)batch * 4, cudaMemcpyHostToDevice, st);
+        if (e == cudaSuccess && d_stacks)
+            e = cudaMemcpyAsync(d_stacks, stacks_host, (size_t)batch * 8, cudaMemcpyHostToDevice, st);
+        if (e != cudaSuccess) return cuda_status(e);
+        if ((rc = domino_step_mask(h, d_states, d_stacks, batch, d_mask, nullptr, stream))) return rc;
+        if ((rc = domino_mask_logits(h, pa.devicePointer, dtype, batch, h->V, d_mask, d_tok, d_lse, nullptr, stream)))
+            return rc;
+    } else {
+        if ((rc = copy_and_decode_chunks(h, logits_host, dtype, batch, states_host, stacks_host, st))) return rc;
+    }
     if ((rc = domino_advance(h, d_states, d_stacks, d_tok, batch, d_states, d_stacks, stream))) return rc;
-    e = cudaMemcpyAsync(tokens_host, d_tok, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
+    cudaError_t e = cudaMemsetAsync(h->s_count.p, 0, sizeof(uint64_t), st);
+    if (e == cudaSuccess)
+        e = launch_mask_vector_count(h->env, d_mask, (long long)batch * h->W, (unsigned long long*)h->s_count.p, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(h->h_count, h->s_count.p, sizeof(uint64_t), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(tokens_host, d_tok, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess && lse_host) e = cudaMemcpyAsync(lse_host, d_lse, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess) e = cudaMemcpyAsync(states_host, d_states, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess && d_stacks)
         e = cudaMemcpyAsync(stacks_host, d_stacks, (size_t)batch * 8, cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e == cudaSuccess) h->vec_density = (double)*h->h_count / ((double)batch * h->W * 4.0);
     return cuda_status(e);
 }
+
 
 int domino_get_device_error(domino_t h, int32_t* code, void* stream) {
     if (!h || !code) return DOMINO_E_INVALID_ARG;

@@ -280,16 +280,21 @@ def test_decode_loop_parity(config, steps):
             assert (sk.cpu().numpy().view(np.uint64) == k_o).all(), i
 
 
+@pytest.mark.parametrize("pinned", [False, True])
 @pytest.mark.parametrize("config", [3, 5])
-def test_decode_step_host_in_chunks_matches_oracle(config):
-    """The host-buffer step copies the logits in chunks of rows and decodes each
-    chunk as it lands; tokens, lse and new configurations match the oracle."""
+def test_decode_step_host_matches_oracle(config, pinned):
+    """Pageable logits are copied in chunks of rows and each chunk is decoded as
+    it lands; pinned logits are read in place.  Tokens, lse and the new
+    configurations match the oracle either way."""
     import oracle
     w = workload(config)
     states, stacks = configs(config)
     has_stack = w.automaton.rules is not None
     d = handle(config)
     lg = w.logits(5)
+    if pinned:
+        lg = torch.from_numpy(lg.view(np.int16) if lg.dtype == np.uint16 else lg).pin_memory().numpy()
+        lg = lg.view(np.uint16) if lg.dtype == np.int16 else lg
     s_host = states.copy()
     k_host = stacks.copy() if has_stack else None
     tok = np.zeros(len(states), np.int32)
