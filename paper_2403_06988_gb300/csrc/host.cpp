@@ -68,6 +68,9 @@ struct domino_ctx {
     DevBuf s_count;                 // non-zero mask bytes of the last step
     uint64_t* h_count = nullptr;    // its pinned host copy
     double vec_density = 0.0;       // share of logit vectors the last step's masks allowed
+    cudaEvent_t ev_t[4] = {};       // timing: mask step (0, 1) and logits copy (2, 3)
+    double t_step_ms = 0.0;         // last mask-step time
+    double link_gbs = 0.0;          // host link rate seen by the last chunked copy (0: none yet)
 };
 
 namespace {
@@ -339,6 +342,8 @@ int domino_destroy(domino_t h) {
                            &h->s_count};
         for (auto* b : all) dev_free(*b);
         for (cudaEvent_t& e : h->ev_chunk)
+            if (e) cudaEventDestroy(e);
+        for (cudaEvent_t& e : h->ev_t)
             if (e) cudaEventDestroy(e);
         if (h->ev_cfg) cudaEventDestroy(h->ev_cfg);
         if (h->cp_stream) cudaStreamDestroy(h->cp_stream);
@@ -821,15 +826,19 @@ int copy_and_decode_chunks(domino_ctx* h, const void* logits_host, int32_t dtype
     if (e == cudaSuccess) e = cudaEventRecord(h->ev_cfg, h->cp_stream);
     std::vector<int32_t> r0s((size_t)n_chunks + 1);
     for (int k = 0; k <= n_chunks; ++k) r0s[(size_t)k] = (int32_t)(((int64_t)batch * k) / n_chunks);
+    if (e == cudaSuccess) e = cudaEventRecord(h->ev_t[2], h->cp_stream);
     for (int k = 0; k < n_chunks && e == cudaSuccess; ++k) {
         const size_t off = (size_t)r0s[(size_t)k] * row_bytes, n = (size_t)(r0s[(size_t)k + 1] - r0s[(size_t)k]) * row_bytes;
         e = cudaMemcpyAsync((char*)h->s_logits.p + off, (const char*)logits_host + off, n, cudaMemcpyHostToDevice,
                             h->cp_stream);
         if (e == cudaSuccess) e = cudaEventRecord(h->ev_chunk[k], h->cp_stream);
     }
+    if (e == cudaSuccess) e = cudaEventRecord(h->ev_t[3], h->cp_stream);
     if (e == cudaSuccess) e = cudaStreamWaitEvent(st, h->ev_cfg, 0);
+    if (e == cudaSuccess) e = cudaEventRecord(h->ev_t[0], st);
     if (e != cudaSuccess) return cuda_status(e);
     if ((rc = domino_step_mask(h, d_states, d_stacks, batch, d_mask, nullptr, stream))) return rc;
+    if ((e = cudaEventRecord(h->ev_t[1], st)) != cudaSuccess) return cuda_status(e);
     for (int k = 0; k < n_chunks; ++k) {
         const int32_t r0 = r0s[(size_t)k], rows = r0s[(size_t)k + 1] - r0;
         if ((e = cudaStreamWaitEvent(st, h->ev_chunk[k], 0)) != cudaSuccess) return cuda_status(e);
@@ -858,14 +867,20 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
     const size_t logit_bytes = (size_t)batch * row_bytes;
     // Pinned (page-locked, mapped) logits are read where they are: the masked
     // pass pulls only the 16-byte logit vectors that hold an allowed token
-    // across the host link, so masked-out logits never travel.  When the last
-    // step's masks allowed most vectors (and for fp32 rows) the chunked copy is
-    // used instead: it moves as many bytes but overlaps the mask step.
+    // across the host link, so masked-out logits never travel, but it starts
+    // after the mask step.  The chunked copy moves every byte while the mask
+    // step runs.  The choice compares the two with the last step's mask
+    // density, mask-step time and link rate:
+    //   in place: t_step + density * bytes / rate;  copy: max(bytes / rate, t_step).
     cudaPointerAttributes pa{};
     const bool pinned = cudaPointerGetAttributes(&pa, logits_host) == cudaSuccess && pa.type == cudaMemoryTypeHost &&
                         pa.devicePointer != nullptr;
     if (!pinned) cudaGetLastError();
-    const bool mapped = pinned && dtype == DOMINO_DTYPE_BF16 && h->vec_density < 0.5;
+    bool mapped = pinned && dtype == DOMINO_DTYPE_BF16;
+    if (mapped && h->link_gbs > 0.0) {
+        const double t_copy = (double)logit_bytes / (h->link_gbs * 1e6);   // ms
+        mapped = h->t_step_ms + h->vec_density * t_copy < std::max(t_copy, h->t_step_ms);
+    }
     if ((!mapped && h->s_logits.n < logit_bytes) || h->s_states.n < (size_t)batch * 4 || !h->cp_stream) {
         if (cudaStreamSynchronize(st) != cudaSuccess) return cuda_status(cudaGetLastError());
     }
@@ -886,6 +901,8 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_cfg, cudaEventDisableTiming);
         for (cudaEvent_t& ev : h->ev_chunk)
             if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+        for (cudaEvent_t& ev : h->ev_t)
+            if (e == cudaSuccess) e = cudaEventCreate(&ev);
         if (e != cudaSuccess) return cuda_status(e);
     }
     int32_t* d_states = (int32_t*)h->s_states.p;
@@ -897,10 +914,14 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
         cudaError_t e = cudaMemcpyAsync(d_states, states_host, (size_t)batch * 4, cudaMemcpyHostToDevice, st);
         if (e == cudaSuccess && d_stacks)
             e = cudaMemcpyAsync(d_stacks, stacks_host, (size_t)batch * 8, cudaMemcpyHostToDevice, st);
+        if (e == cudaSuccess) e = cudaEventRecord(h->ev_t[0], st);
         if (e != cudaSuccess) return cuda_status(e);
         if ((rc = domino_step_mask(h, d_states, d_stacks, batch, d_mask, nullptr, stream))) return rc;
+        if ((e = cudaEventRecord(h->ev_t[1], st)) != cudaSuccess) return cuda_status(e);
+        if ((e = cudaEventRecord(h->ev_t[2], st)) != cudaSuccess) return cuda_status(e);
         if ((rc = domino_mask_logits(h, pa.devicePointer, dtype, batch, h->V, d_mask, d_tok, d_lse, nullptr, stream)))
             return rc;
+        if ((e = cudaEventRecord(h->ev_t[3], st)) != cudaSuccess) return cuda_status(e);
     } else {
         if ((rc = copy_and_decode_chunks(h, logits_host, dtype, batch, states_host, stacks_host, st))) return rc;
     }
@@ -915,7 +936,17 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
     if (e == cudaSuccess && d_stacks)
         e = cudaMemcpyAsync(stacks_host, d_stacks, (size_t)batch * 8, cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
-    if (e == cudaSuccess) h->vec_density = (double)*h->h_count / ((double)batch * h->W * 4.0);
+    if (e == cudaSuccess) {
+        h->vec_density = (double)*h->h_count / ((double)batch * h->W * 4.0);
+        float ms = 0.f;
+        if (cudaEventElapsedTime(&ms, h->ev_t[0], h->ev_t[1]) == cudaSuccess) h->t_step_ms = ms;
+        // the link rate: bytes copied over the copy time, or the vectors read in
+        // place over the in-place pass's time (that pass is bound by the link)
+        const double moved = mapped ? h->vec_density * (double)logit_bytes : (double)logit_bytes;
+        if (moved > (double)(1 << 20) && cudaEventElapsedTime(&ms, h->ev_t[2], h->ev_t[3]) == cudaSuccess && ms > 0.f)
+            h->link_gbs = moved / ((double)ms * 1e6);
+        cudaGetLastError();
+    }
     return cuda_status(e);
 }
 
