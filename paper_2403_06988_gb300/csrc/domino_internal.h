@@ -17,7 +17,7 @@ namespace domino {
 // bits are scattered back to original ids in shared memory.
 constexpr int kWin = 1024;
 constexpr int kStepThreads = 1024;             // step kernel CTA size (one CTA per SM)
-constexpr int kRowsPerTile = 16;               // fewest rows per tile (mask only)
+constexpr int kRowsPerTile = 4;                // fewest rows per tile (mask only; small batches)
 constexpr int kMaxRowsPerTile = 32;            // most rows per tile (one warp ballot)
 constexpr int kRowsPerTileNext = 8;            // rows per tile when next states are written
 constexpr int kUnitSlots = 32;                 // slots per work unit (one per lane)
