@@ -1385,8 +1385,11 @@ cudaError_t launch_logits_t(const LaunchEnv& env, const void* logits, int32_t ba
         lst.base = r0;
         float* lse_rows = lse ? lse + shift : (logprobs ? lse_tmp : nullptr);
         const long long N = (long long)rows * W;
-        int grid = env.num_sms * occupancy((const void*)reduce, kReduceThreads);
-        grid = (int)std::min<long long>((long long)grid, (N + 127) / 128);   // at least 4 batches per warp
+        // at least 4 batches of 32 words per warp; a pass too small to fill the
+        // GPU that way gives each warp fewer (down to one batch) instead
+        const int slots = env.num_sms * occupancy((const void*)reduce, kReduceThreads);
+        int grid = (int)std::min<long long>((long long)slots, (N + 127) / 128);
+        if (grid < slots) grid = (int)std::min<long long>((long long)slots, (N + 31) / 32);
         grid = max(grid, 1);
         long long per_cta = (N + grid - 1) / grid;
         per_cta = std::max<long long>(per_cta, ((long long)W + kMaxSegments - 3) / (kMaxSegments - 2));
