@@ -120,3 +120,22 @@ def test_opportunistic_invalid_rows():
     assert (t[:3] == -1).all()
     assert int(n_fb.item()) >= 3
     assert d.device_error() == B.DEVERR_BAD_STATE
+
+
+def test_opportunistic_more_rows_than_one_logits_pass():
+    """4100 rows: the fallback list spans two passes of the logits kernel."""
+    import oracle
+    w = workload(1)
+    P = oracle.Problem.from_workload(w)
+    d = handle(1)
+    rng = np.random.default_rng(11)
+    states = rng.choice(np.nonzero(w.automaton.live)[0], size=4100).astype(np.int32)
+    x = (rng.standard_normal((4100, w.vocab.n_tokens)) * 2).astype(np.float32)
+    m, _, _ = P.step_mask(states, None, n_threads=NT)
+    allowed_rows = np.unpackbits(m.view(np.uint8), axis=1, bitorder="little")[:, :w.vocab.n_tokens].sum(axis=0)
+    x[:, int(np.argmin(allowed_rows))] += 50.0          # a token almost never allowed wins every proposal
+    want, _, _ = oracle.mask_logits(x, m)
+    tok, n_fb = d.opportunistic_step(dev(x), dev(states))
+    assert (tok.cpu().numpy() == want).all()
+    assert int(n_fb.item()) > 4096
+
