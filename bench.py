@@ -769,8 +769,8 @@ def run_domino(args, dist: Dist):
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": n, "steps": K, "warmup": Wm,
         "ms_per_step": ms_max / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": w.logits_dtype, "data": "synthetic",
-        "config": {"workload": w.name, "batch": Bsz, "vocab": V, "states": a.n_states,
+        "dtype": "int32+f32", "data": "synthetic",
+        "config": {"workload": w.name, "batch": Bsz, "vocab": V, "states": a.n_states, "logits_dtype": w.logits_dtype,
                    "byte_classes": info["n_classes"], "table_in_smem": info["table_in_smem"],
                    "logprobs": w.want_logprobs,
                    "l2": f"logits rotate over {nbuf} buffers ({nbuf * logit_bytes / 2**20:.0f} MiB > 2x L2)",
