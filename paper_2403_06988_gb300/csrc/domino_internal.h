@@ -58,6 +58,7 @@ struct StepView {
     // packed as class (bits 0..7) | first slot (bits 8..18) | count-1 (bits 19..23)
     const uint32_t* units;    // all windows' units, window w at [unit_off[w], unit_off[w+1])
     const int32_t* unit_off;  // [n_windows + 1]
+    const uint16_t* cls_units; // [n_windows][K + 1]: window-local first unit of each first class
     const int16_t* eos_slot;  // [n_windows] window-local slot of EOS, -1 if not in the window
     int32_t max_units;        // max units of one window
     int32_t V, W, n_windows, eos_id;

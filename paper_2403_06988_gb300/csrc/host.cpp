@@ -50,7 +50,7 @@ struct domino_ctx {
     int64_t dense_ret_off = 0, sp_tgt_off = 0, sp_ret_off = 0;
 
     // ---- device copies
-    DevBuf d_head, d_info, d_tail_off, d_tail, d_pos_of, d_units, d_unit_off, d_eos_slot;
+    DevBuf d_head, d_info, d_tail_off, d_tail, d_pos_of, d_units, d_unit_off, d_cls_units, d_eos_slot;
     int32_t max_units = 0;
     DevBuf d_dense, d_sparse, d_accept;
     DevBuf d_err, d_partials, d_counters, d_lse_tmp;
@@ -97,7 +97,7 @@ void dev_free(DevBuf& b) {
 
 int64_t dev_bytes(const domino_ctx* h) {
     const DevBuf* all[] = {&h->d_head, &h->d_info, &h->d_tail_off, &h->d_tail, &h->d_pos_of, &h->d_units,
-                           &h->d_unit_off, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_err, &h->d_partials,
+                           &h->d_unit_off, &h->d_cls_units, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_err, &h->d_partials,
                            &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_states, &h->s_stacks,
                            &h->s_mask, &h->s_tokens, &h->s_lse, &h->o_prop, &h->o_rows, &h->o_count,
                            &h->s_count};
@@ -163,6 +163,7 @@ int build_arena(domino_ctx* h) {
     std::vector<uint16_t> gstart((size_t)(K + 1), 0);
     std::vector<uint32_t> units;
     std::vector<int32_t> unit_off((size_t)nw + 1, 0);
+    std::vector<uint16_t> cls_units((size_t)nw * (size_t)(h->K + 1), 0);   // [window][class]: first unit
     int32_t max_units = 0;
     std::vector<int16_t> eos_slot((size_t)nw, -1);
     std::vector<uint8_t> tail;
@@ -192,12 +193,16 @@ int build_arena(domino_ctx* h) {
             }
         }
         while (c_next <= K) gs[c_next++] = (uint16_t)(hi - lo);
-        // work units: <= kUnitSlots consecutive slots of one first-class group
-        for (int c = 0; c < K; c++)
+        // work units: <= kUnitSlots consecutive slots of one first-class group;
+        // each class's units are contiguous, from cls_units[w][c] on
+        for (int c = 0; c < K; c++) {
+            cls_units[(size_t)w * (K + 1) + c] = (uint16_t)(units.size() - (size_t)unit_off[(size_t)w]);
             for (int b = gs[c]; b < gs[c + 1]; b += kUnitSlots) {
                 const int n = std::min(kUnitSlots, gs[c + 1] - b);
                 units.push_back((uint32_t)c | ((uint32_t)b << 8) | ((uint32_t)(n - 1) << 19));
             }
+        }
+        cls_units[(size_t)w * (K + 1) + K] = (uint16_t)(units.size() - (size_t)unit_off[(size_t)w]);
         unit_off[(size_t)w + 1] = (int32_t)units.size();
         max_units = std::max(max_units, unit_off[(size_t)w + 1] - unit_off[(size_t)w]);
     }
@@ -210,6 +215,7 @@ int build_arena(domino_ctx* h) {
     if ((rc = dev_upload(h->d_pos_of, pos_of.data(), pos_of.size() * 4))) return rc;
     if ((rc = dev_upload(h->d_units, units.data(), units.size() * 4))) return rc;
     if ((rc = dev_upload(h->d_unit_off, unit_off.data(), unit_off.size() * 4))) return rc;
+    if ((rc = dev_upload(h->d_cls_units, cls_units.data(), cls_units.size() * 2))) return rc;
     h->max_units = max_units;
     if ((rc = dev_upload(h->d_eos_slot, eos_slot.data(), eos_slot.size() * 2))) return rc;
     h->n_windows = nw;
@@ -226,6 +232,7 @@ StepView make_view(domino_ctx* h) {
     v.pos_of = (const int32_t*)h->d_pos_of.p;
     v.units = (const uint32_t*)h->d_units.p;
     v.unit_off = (const int32_t*)h->d_unit_off.p;
+    v.cls_units = (const uint16_t*)h->d_cls_units.p;
     v.max_units = h->max_units;
     v.eos_slot = (const int16_t*)h->d_eos_slot.p;
     v.V = h->V;
@@ -336,7 +343,7 @@ int domino_destroy(domino_t h) {
         DeviceGuard g(h->device);
         cudaDeviceSynchronize();
         DevBuf* all[] = {&h->d_head, &h->d_info, &h->d_tail_off, &h->d_tail, &h->d_pos_of, &h->d_units,
-                         &h->d_unit_off, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_err, &h->d_partials,
+                         &h->d_unit_off, &h->d_cls_units, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_err, &h->d_partials,
                          &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_states, &h->s_stacks,
                          &h->s_mask, &h->s_tokens, &h->s_lse, &h->o_prop, &h->o_rows, &h->o_count,
                            &h->s_count};

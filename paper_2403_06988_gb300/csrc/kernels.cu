@@ -86,7 +86,7 @@ struct RowList {
 
 // Shared-memory layout of the step kernel (offsets in bytes).
 struct StepLayout {
-    int head, info, units, items, rows, ctrl, rowmask, cfg, mtile, ntile, accept, table, total;
+    int head, info, units, cls, items, rows, ctrl, rowmask, cfg, mtile, ntile, accept, table, total;
 };
 
 __host__ __device__ inline StepLayout step_layout(int K, int R, bool next, bool stack, int max_units, int Q,
@@ -96,6 +96,7 @@ __host__ __device__ inline StepLayout step_layout(int K, int R, bool next, bool 
     L.head = o;    o += kWin * 32;
     L.info = o;    o += kWin * 4;
     L.units = o;   o += align16(max_units * 4);
+    L.cls = o;     o += align16((K + 1) * 2);
     L.items = o;   o += align16(max_units * ((R + kWalkChains - 1) / kWalkChains) * 4);
     L.rows = o;    o += R * 16;
     L.ctrl = o;    o += 16;
@@ -272,6 +273,7 @@ __global__ void __launch_bounds__(kStepThreads, 1)
     uint4* s_head = reinterpret_cast<uint4*>(smem + L.head);
     uint32_t* s_info = reinterpret_cast<uint32_t*>(smem + L.info);
     uint32_t* s_units = reinterpret_cast<uint32_t*>(smem + L.units);
+    uint16_t* s_cls = reinterpret_cast<uint16_t*>(smem + L.cls);      // [K + 1] first unit of each first class
     uint32_t* s_items = reinterpret_cast<uint32_t*>(smem + L.items);   // unit | chain group << 16
     uint4* s_rows = reinterpret_cast<uint4*>(smem + L.rows);
     int* s_ctrl = reinterpret_cast<int*>(smem + L.ctrl);   // unit cursor, -, EOS slot, unit count
@@ -344,6 +346,7 @@ __global__ void __launch_bounds__(kStepThreads, 1)
             s_info[tid] = __ldg(v.info + (size_t)w * kWin + tid);
             const int u0 = __ldg(v.unit_off + w), nu = __ldg(v.unit_off + w + 1) - u0;
             for (int i = tid; i < nu; i += kStepThreads) s_units[i] = __ldg(v.units + u0 + i);
+            for (int i = tid; i <= K; i += kStepThreads) s_cls[i] = __ldg(v.cls_units + (size_t)w * (K + 1) + i);
             if (tid == 0) {
                 s_ctrl[2] = __ldg(v.eos_slot + w);
                 s_ctrl[3] = nu;
@@ -358,6 +361,7 @@ __global__ void __launch_bounds__(kStepThreads, 1)
                 s_rows[tid] = decode_row(v, pf_s, pf_w, stacks != nullptr, s_accept, w == 0);
             }
         }
+        if (tid == 0) s_ctrl[1] = 0;   // items listed so far
         for (int i = tid; i < nr * 32; i += kStepThreads) s_mtile[i] = 0u;
         if constexpr (NEXT) {
             for (int i = tid; i < nr * (kWin / 4); i += kStepThreads)
@@ -366,7 +370,9 @@ __global__ void __launch_bounds__(kStepThreads, 1)
         __syncthreads();
 
         // first transition once per (row, first class): lane r of a warp takes
-        // row r, the ballot gives the class's live rows
+        // row r, the ballot gives the class's live rows; the warp then lists
+        // the work items of the class's units, (unit, group of up to
+        // kWalkChains live rows), for the warps to walk
         for (int c = warp; c < K; c += kStepThreads / 32) {
             uint32_t s = 0, bits = 0, depth = 0;
             if (lane < nr) {
@@ -389,6 +395,15 @@ __global__ void __launch_bounds__(kStepThreads, 1)
             }
             const uint32_t live = __ballot_sync(0xffffffffu, s != 0);
             if (lane == 0) s_rowmask[c] = live;
+            const int ub = s_cls[c], g = (__popc(live) + kWalkChains - 1) / kWalkChains;
+            const int n = (s_cls[c + 1] - ub) * g;
+            if (n > 0) {
+                int base = 0;
+                if (lane == 0) base = atomicAdd(&s_ctrl[1], n);
+                base = __shfl_sync(0xffffffffu, base, 0);
+                for (int k = lane; k < n; k += 32)
+                    s_items[base + k] = (uint32_t)(ub + k / g) | ((uint32_t)(k % g) << 16);
+            }
         }
         const int eos_local = s_ctrl[2];
         if (tid < nr && eos_local >= 0 && (s_rows[tid].w & 2u)) {
@@ -399,33 +414,6 @@ __global__ void __launch_bounds__(kStepThreads, 1)
         __syncthreads();
 
         prefetch(t + 1);
-        // work items: (unit, group of up to kWalkChains live rows), listed by
-        // warp 0 and dealt round-robin to the warps (items cost about the same)
-        const int nu = s_ctrl[3];
-        if (warp == 0) {
-            int base = 0;
-            for (int u0 = 0; u0 < nu; u0 += 32) {
-                const int u = u0 + lane;
-                int ng = 0;
-                if (u < nu) {
-                    const uint32_t rm = s_rowmask[s_units[u] & 0xFFu];
-                    const uint32_t unit = s_units[u];
-                    // a unit whose tokens all have one byte needs no walk beyond the first step
-                    ng = (__popc(rm) + kWalkChains - 1) / kWalkChains;
-                    (void)unit;
-                }
-                int incl = ng;
-#pragma unroll
-                for (int off = 1; off < 32; off <<= 1) {
-                    const int y = __shfl_up_sync(0xffffffffu, incl, off);
-                    if (lane >= off) incl += y;
-                }
-                for (int g = 0; g < ng; ++g) s_items[base + incl - ng + g] = (uint32_t)u | ((uint32_t)g << 16);
-                base += __shfl_sync(0xffffffffu, incl, 31);
-            }
-            if (lane == 0) s_ctrl[1] = base;
-        }
-        __syncthreads();
         const int n_items = s_ctrl[1];
         for (int it = warp; it < n_items; it += kStepThreads / 32) {
             const uint32_t item = s_items[it];
