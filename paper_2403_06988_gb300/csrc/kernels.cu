@@ -15,15 +15,23 @@
 //                   tokens).  Allowed bits are scattered to original ids in a
 //                   shared-memory tile and written out coalesced.  The same
 //                   kernel with row = state builds the state x token table
-//                   (Alg. 2's traversal, precomputed offline, Sec. 3.5).
-//  logits kernels   Alg. 1's v' = m (.) v and greedy decode: a balanced flat
-//                   split of the batch x vocabulary logits over one wave of
-//                   CTAs; 16-byte loads (vectors with no allowed token are not
-//                   loaded), branch-free masked max / lowest-index argmax /
-//                   sum of exp per vector; per-row segments are combined by
-//                   the last CTA to finish (atomic ticket, no spinning).
-//                   Log-probs need a second pass over the row.
-//  advance_kernel   C.update(o): the chosen token's walk.
+//                   (Alg. 2's traversal, precomputed offline, Sec. 3.5), and,
+//                   over a device-side row list, masks only the rows that
+//                   opportunistic masking rejected.
+//  logits_reduce    Alg. 1's v' = m (.) v and decode: a balanced flat split of
+//                   the batch x mask words over one-warp CTAs; the 16-byte
+//                   logit vectors that hold an allowed token are staged with
+//                   cp.async (the others are never read); a lane folds its
+//                   word into a masked max / lowest-index argmax / sum of
+//                   exp, or a Gumbel-max draw (sampling); per-row segments are
+//                   combined by the last CTA to finish (atomic ticket, no
+//                   spinning).  Rows may come from a precomputed mask table
+//                   (table-driven step) or a device-side row list.
+//  logprobs         the second pass for log-probabilities.
+//  advance          C.update(o): the chosen token's walk (or one read of the
+//                   precomputed next-state table).
+//  propose_check,   opportunistic masking's one-walk check, and count-based
+//  spec_*           speculation (Sec. 3.6): count update, proposals, acceptance.
 #include <cuda_runtime.h>
 
 #include <climits>
@@ -276,7 +284,7 @@ __global__ void __launch_bounds__(kStepThreads, 1)
     uint16_t* s_cls = reinterpret_cast<uint16_t*>(smem + L.cls);      // [K + 1] first unit of each first class
     uint32_t* s_items = reinterpret_cast<uint32_t*>(smem + L.items);   // unit | chain group << 16
     uint4* s_rows = reinterpret_cast<uint4*>(smem + L.rows);
-    int* s_ctrl = reinterpret_cast<int*>(smem + L.ctrl);   // unit cursor, -, EOS slot, unit count
+    int* s_ctrl = reinterpret_cast<int*>(smem + L.ctrl);   // -, items listed, EOS slot, unit count
     uint32_t* s_rowmask = reinterpret_cast<uint32_t*>(smem + L.rowmask);
     uint32_t* s_cfg = reinterpret_cast<uint32_t*>(smem + L.cfg);   // [R][K] state (DFA)
     uint4* s_cfg4 = reinterpret_cast<uint4*>(smem + L.cfg);        // [R][K] (state, bits, depth) (pushdown)
