@@ -69,6 +69,10 @@ struct StepView {
     const void* sp_tgt;       // sparse live entries (uint16 or uint32)
     const uint16_t* ret;      // [n_ret][4]
     const uint32_t* accept_bits;
+    // self loops (nullptr when not used): per state the classes that keep it,
+    // per slot the classes of the token's bytes after the first
+    const unsigned long long* self_mask;  // [Q]
+    const unsigned long long* tok_cls;    // [n_slots]
     int32_t Q, K, start, max_depth, n_ret, sp_nnz;
     uint32_t* err;            // sticky device error word
 };

@@ -45,6 +45,7 @@ struct domino_ctx {
     std::vector<uint32_t> t32;
     std::vector<uint16_t> ret;
     std::vector<uint32_t> accept_bits;
+    std::vector<uint64_t> self_mask;   // [Q]: classes that keep the state (no stack action); empty if unused
     int32_t sp_nnz = 0;       // live entries of the sparse table (0: no sparse image)
     int32_t sp_words = 0;     // uint32 words per state in the sparse row info (2 or 4)
     int64_t dense_ret_off = 0, sp_tgt_off = 0, sp_ret_off = 0;
@@ -52,7 +53,7 @@ struct domino_ctx {
     // ---- device copies
     DevBuf d_head, d_info, d_tail_off, d_tail, d_pos_of, d_units, d_unit_off, d_cls_units, d_eos_slot;
     int32_t max_units = 0;
-    DevBuf d_dense, d_sparse, d_accept;
+    DevBuf d_dense, d_sparse, d_accept, d_self, d_tok_cls;
     DevBuf d_err, d_partials, d_counters, d_lse_tmp;
     bool arena_ready = false;
     int32_t n_windows = 0;
@@ -97,7 +98,7 @@ void dev_free(DevBuf& b) {
 
 int64_t dev_bytes(const domino_ctx* h) {
     const DevBuf* all[] = {&h->d_head, &h->d_info, &h->d_tail_off, &h->d_tail, &h->d_pos_of, &h->d_units,
-                           &h->d_unit_off, &h->d_cls_units, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_err, &h->d_partials,
+                           &h->d_unit_off, &h->d_cls_units, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_self, &h->d_tok_cls, &h->d_err, &h->d_partials,
                            &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_states, &h->s_stacks,
                            &h->s_mask, &h->s_tokens, &h->s_lse, &h->o_prop, &h->o_rows, &h->o_count,
                            &h->s_count};
@@ -158,6 +159,8 @@ int build_arena(domino_ctx* h) {
     };
     const int K = h->K;
     std::vector<uint8_t> head((size_t)n_slots * kInlineBytes, 0);
+    const bool self = !h->self_mask.empty();
+    std::vector<uint64_t> tok_cls(self ? (size_t)n_slots : 0, 0);   // classes of bytes 1.. of each slot
     std::vector<uint32_t> info((size_t)n_slots, 0);
     std::vector<int32_t> tail_off((size_t)n_slots, 0), pos_of((size_t)V, 0);
     std::vector<uint16_t> gstart((size_t)(K + 1), 0);
@@ -187,6 +190,8 @@ int build_arena(domino_ctx* h) {
                 while (c_next <= c[0]) gs[c_next++] = (uint16_t)j;   // groups by first class
             }
             std::memcpy(head.data() + p * kInlineBytes, c, (size_t)std::min(L, kInlineBytes));
+            if (self)
+                for (int32_t i = 1; i < L; i++) tok_cls[(size_t)p] |= 1ull << c[i];
             if (L > kInlineBytes) {
                 tail_off[(size_t)p] = (int32_t)tail.size();
                 tail.insert(tail.end(), c + kInlineBytes, c + L);
@@ -216,6 +221,11 @@ int build_arena(domino_ctx* h) {
     if ((rc = dev_upload(h->d_units, units.data(), units.size() * 4))) return rc;
     if ((rc = dev_upload(h->d_unit_off, unit_off.data(), unit_off.size() * 4))) return rc;
     if ((rc = dev_upload(h->d_cls_units, cls_units.data(), cls_units.size() * 2))) return rc;
+    if (self) {
+        if ((rc = dev_upload(h->d_tok_cls, tok_cls.data(), tok_cls.size() * 8))) return rc;
+    } else {
+        dev_free(h->d_tok_cls);
+    }
     h->max_units = max_units;
     if ((rc = dev_upload(h->d_eos_slot, eos_slot.data(), eos_slot.size() * 2))) return rc;
     h->n_windows = nw;
@@ -246,6 +256,8 @@ StepView make_view(domino_ctx* h) {
     v.sp_info = (const uint32_t*)h->d_sparse.p;
     v.sp_tgt = h->d_sparse.p ? (const void*)((const char*)h->d_sparse.p + h->sp_tgt_off) : nullptr;
     v.accept_bits = (const uint32_t*)h->d_accept.p;
+    v.self_mask = h->self_mask.empty() ? nullptr : (const unsigned long long*)h->d_self.p;
+    v.tok_cls = h->self_mask.empty() ? nullptr : (const unsigned long long*)h->d_tok_cls.p;
     v.Q = h->Q;
     v.K = h->K;
     v.start = h->start;
@@ -343,7 +355,7 @@ int domino_destroy(domino_t h) {
         DeviceGuard g(h->device);
         cudaDeviceSynchronize();
         DevBuf* all[] = {&h->d_head, &h->d_info, &h->d_tail_off, &h->d_tail, &h->d_pos_of, &h->d_units,
-                         &h->d_unit_off, &h->d_cls_units, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_err, &h->d_partials,
+                         &h->d_unit_off, &h->d_cls_units, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_self, &h->d_tok_cls, &h->d_err, &h->d_partials,
                          &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_states, &h->s_stacks,
                          &h->s_mask, &h->s_tokens, &h->s_lse, &h->o_prop, &h->o_rows, &h->o_count,
                            &h->s_count};
@@ -512,6 +524,23 @@ int domino_load_automaton(domino_t h, const int32_t* delta, int32_t n_states, co
             for (int k = 0; k < K; k++) h->t16[(size_t)(q * K + k)] = (uint16_t)col[(size_t)rep[k] * Q + q];
     }
     h->ret = ret;
+    // Self loops: class k keeps state q (with no stack action).  A token whose
+    // remaining classes all keep the row's state leaves it unchanged, so the
+    // walk can skip it.  Used when some state loops on at least a quarter of
+    // the classes: the string, number and whitespace states of real grammars.
+    h->self_mask.clear();
+    if (K <= 64) {
+        std::vector<uint64_t> sm((size_t)Q, 0);
+        bool wide = false;
+        for (int64_t q = 1; q < Q; q++) {
+            for (int k = 0; k < K; k++) {
+                const uint32_t e = stack ? h->t32[(size_t)(q * K + k)] : h->t16[(size_t)(q * K + k)];
+                if (e == (uint32_t)q) sm[(size_t)q] |= 1ull << k;   // next state q, kind 0 (no push or pop)
+            }
+            wide = wide || 4 * __builtin_popcountll(sm[(size_t)q]) >= K;
+        }
+        if (wide) h->self_mask.swap(sm);
+    }
     h->accept_bits.assign((size_t)((Q + 31) / 32), 0u);
     if (accepting)
         for (int64_t q = 0; q < Q; q++)
@@ -580,6 +609,11 @@ int domino_load_automaton(domino_t h, const int32_t* delta, int32_t n_states, co
         dev_free(h->d_sparse);
     }
     if ((rc = dev_upload(h->d_accept, h->accept_bits.data(), h->accept_bits.size() * 4))) return rc;
+    if (!h->self_mask.empty()) {
+        if ((rc = dev_upload(h->d_self, h->self_mask.data(), h->self_mask.size() * 8))) return rc;
+    } else {
+        dev_free(h->d_self);
+    }
     return build_arena(h);
 }
 

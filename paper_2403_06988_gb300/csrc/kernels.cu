@@ -94,17 +94,18 @@ struct RowList {
 
 // Shared-memory layout of the step kernel (offsets in bytes).
 struct StepLayout {
-    int head, info, units, cls, items, rows, ctrl, rowmask, cfg, mtile, ntile, accept, table, total;
+    int head, info, units, cls, tokcls, items, rows, ctrl, rowmask, cfg, mtile, ntile, accept, self, table, total;
 };
 
 __host__ __device__ inline StepLayout step_layout(int K, int R, bool next, bool stack, int max_units, int Q,
-                                                  int table_bytes) {
+                                                  int table_bytes, bool self) {
     StepLayout L{};
     int o = 0;
     L.head = o;    o += kWin * 32;
     L.info = o;    o += kWin * 4;
     L.units = o;   o += align16(max_units * 4);
     L.cls = o;     o += align16((K + 1) * 2);
+    L.tokcls = o;  o += self ? kWin * 8 : 0;
     L.items = o;   o += align16(max_units * ((R + kWalkChains - 1) / kWalkChains) * 4);
     L.rows = o;    o += R * 16;
     L.ctrl = o;    o += 16;
@@ -113,6 +114,7 @@ __host__ __device__ inline StepLayout step_layout(int K, int R, bool next, bool 
     L.mtile = o;   o += align16(R * 32 * 4);
     L.ntile = o;   o += next ? R * kWin * 4 : 0;
     L.accept = o;  o += align16(((Q + 31) / 32) * 4);
+    L.self = o;    o += self ? align16(Q * 8) : 0;
     L.table = o;   o += align16(table_bytes);
     L.total = o;
     return L;
@@ -277,7 +279,9 @@ __global__ void __launch_bounds__(kStepThreads, 1)
     using E = typename std::conditional<STACK, uint32_t, uint16_t>::type;
     extern __shared__ __align__(16) unsigned char smem[];
     const int K = v.K;
-    const StepLayout L = step_layout(K, R, NEXT, STACK, v.max_units, v.Q, MODE == kDenseGlobal ? 0 : img_bytes);
+    const bool use_self = v.self_mask != nullptr;
+    const StepLayout L = step_layout(K, R, NEXT, STACK, v.max_units, v.Q, MODE == kDenseGlobal ? 0 : img_bytes,
+                                     use_self);
     uint4* s_head = reinterpret_cast<uint4*>(smem + L.head);
     uint32_t* s_info = reinterpret_cast<uint32_t*>(smem + L.info);
     uint32_t* s_units = reinterpret_cast<uint32_t*>(smem + L.units);
@@ -291,6 +295,8 @@ __global__ void __launch_bounds__(kStepThreads, 1)
     uint32_t* s_mtile = reinterpret_cast<uint32_t*>(smem + L.mtile);
     int32_t* s_ntile = reinterpret_cast<int32_t*>(smem + L.ntile);
     uint32_t* s_accept = reinterpret_cast<uint32_t*>(smem + L.accept);
+    unsigned long long* s_self = reinterpret_cast<unsigned long long*>(smem + L.self);       // [Q]
+    unsigned long long* s_tokcls = reinterpret_cast<unsigned long long*>(smem + L.tokcls);   // [kWin]
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     if (list.ids) {   // a row list may be empty: learn its length before staging anything
         pdl_wait();
@@ -298,6 +304,8 @@ __global__ void __launch_bounds__(kStepThreads, 1)
         if (list.rows(batch) == 0) return;
     }
     for (int i = tid; i < (v.Q + 31) / 32; i += kStepThreads) s_accept[i] = __ldg(v.accept_bits + i);
+    if (use_self)
+        for (int i = tid; i < v.Q; i += kStepThreads) s_self[i] = __ldg(v.self_mask + i);
 
     Tab<E, MODE> tab;
     tab.K = (uint32_t)K;
@@ -352,6 +360,7 @@ __global__ void __launch_bounds__(kStepThreads, 1)
             s_head[2 * tid] = __ldg(v.head + 2 * ((size_t)w * kWin + tid));
             s_head[2 * tid + 1] = __ldg(v.head + 2 * ((size_t)w * kWin + tid) + 1);
             s_info[tid] = __ldg(v.info + (size_t)w * kWin + tid);
+            if (use_self) s_tokcls[tid] = __ldg(v.tok_cls + (size_t)w * kWin + tid);
             const int u0 = __ldg(v.unit_off + w), nu = __ldg(v.unit_off + w + 1) - u0;
             for (int i = tid; i < nu; i += kStepThreads) s_units[i] = __ldg(v.units + u0 + i);
             for (int i = tid; i <= K; i += kStepThreads) s_cls[i] = __ldg(v.cls_units + (size_t)w * (K + 1) + i);
@@ -458,7 +467,16 @@ __global__ void __launch_bounds__(kStepThreads, 1)
                     }
                 }
                 if (active) {
-                    walk_chains<STACK, kWalkChains>(tab, ret, maxd, sv, bv, dv, hp, len, tl);
+                    // a token whose later classes all keep every chain's state
+                    // leaves the chains as they are: no walk
+                    bool keep = use_self;
+                    if (use_self) {
+                        const unsigned long long tc = s_tokcls[slot];
+#pragma unroll
+                        for (int k = 0; k < kWalkChains; ++k)
+                            if (sv[k] && (tc & ~s_self[sv[k]])) keep = false;
+                    }
+                    if (!keep) walk_chains<STACK, kWalkChains>(tab, ret, maxd, sv, bv, dv, hp, len, tl);
 #pragma unroll
                     for (int k = 0; k < kWalkChains; ++k) {
                         if (rr[k] >= 0 && sv[k]) {
@@ -1254,7 +1272,8 @@ __global__ void __launch_bounds__(kAdvanceThreads)
 int rows_per_tile(const StepView& v, const LaunchEnv& env, int batch, bool next, bool stack, int img_bytes) {
     if (next) {
         for (int R = kMaxRowsPerTile; R > kRowsPerTileNext; R >>= 1)
-            if (step_layout(v.K, R, true, stack, v.max_units, v.Q, img_bytes).total <= env.max_smem_optin &&
+            if (step_layout(v.K, R, true, stack, v.max_units, v.Q, img_bytes, v.self_mask != nullptr).total <=
+                    env.max_smem_optin &&
                 (long long)((batch + R - 1) / R) * v.n_windows >= 4LL * env.num_sms)
                 return R;
         return kRowsPerTileNext;
@@ -1280,7 +1299,7 @@ cudaError_t launch_step_t(const StepView& v, const LaunchEnv& env, const int32_t
                           cudaStream_t st) {
     const int img_bytes = MODE == kDenseGlobal ? 0 : (int)table_smem_bytes(v, STACK, MODE);
     const int R = rows_per_tile(v, env, batch, NEXT, STACK, img_bytes);
-    const StepLayout L = step_layout(v.K, R, NEXT, STACK, v.max_units, v.Q, img_bytes);
+    const StepLayout L = step_layout(v.K, R, NEXT, STACK, v.max_units, v.Q, img_bytes, v.self_mask != nullptr);
     auto kern = step_kernel<STACK, MODE, NEXT>;
     // the dynamic shared-memory limit is raised once per device and size, so
     // that launches inside a stream capture make no attribute calls
@@ -1428,7 +1447,8 @@ int64_t table_smem_bytes(const StepView& v, bool stack, int mode) {
 }
 
 int step_fixed_smem_bytes(const StepView& v, bool next) {
-    return step_layout(v.K, next ? kRowsPerTileNext : kMaxRowsPerTile, next, v.t32 != nullptr, v.max_units, v.Q, 0)
+    return step_layout(v.K, next ? kRowsPerTileNext : kMaxRowsPerTile, next, v.t32 != nullptr, v.max_units, v.Q, 0,
+                       v.self_mask != nullptr)
         .total;
 }
 
