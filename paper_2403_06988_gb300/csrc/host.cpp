@@ -72,6 +72,16 @@ struct domino_ctx {
     cudaEvent_t ev_t[4] = {};       // timing: mask step (0, 1) and logits copy (2, 3)
     double t_step_ms = 0.0;         // last mask-step time
     double link_gbs = 0.0;          // host link rate seen by the last chunked copy (0: none yet)
+    // Recorded host-buffer steps: a call whose buffers, sizes and path match an
+    // earlier one replays that call's CUDA graph instead of issuing each copy
+    // and launch again.  Cleared when an automaton or vocabulary is loaded.
+    struct HostGraph {
+        const void* key[16];
+        cudaGraphExec_t exec;
+        uint64_t used;
+    };
+    std::vector<HostGraph> host_graphs;
+    uint64_t host_calls = 0;
 };
 
 namespace {
@@ -129,6 +139,11 @@ int dev_upload(DevBuf& b, const void* src, size_t n) {
 int dev_reserve(DevBuf& b, size_t n) { return dev_upload(b, nullptr, n); }
 
 bool is_host_only(const domino_ctx* h) { return h->device < 0; }
+
+void clear_host_graphs(domino_ctx* h) {
+    for (auto& g : h->host_graphs) cudaGraphExecDestroy(g.exec);
+    h->host_graphs.clear();
+}
 
 // Byte-class strings of every token, the window sort and the slot arrays.
 int build_arena(domino_ctx* h) {
@@ -367,6 +382,7 @@ int domino_destroy(domino_t h) {
         if (h->ev_cfg) cudaEventDestroy(h->ev_cfg);
         if (h->cp_stream) cudaStreamDestroy(h->cp_stream);
         if (h->h_count) cudaFreeHost(h->h_count);
+        clear_host_graphs(h);
         cudaGetLastError();
     }
     delete h;
@@ -375,6 +391,7 @@ int domino_destroy(domino_t h) {
 
 int domino_load_vocab(domino_t h, const uint8_t* bytes, const int64_t* offsets, int32_t n_tokens,
                       int32_t eos_id) {
+    if (h) clear_host_graphs(h);
     if (!h || !offsets || n_tokens < 1 || n_tokens > (1 << 24)) return DOMINO_E_INVALID_ARG;
     if (eos_id < -1 || eos_id >= n_tokens || offsets[0] != 0) return DOMINO_E_INVALID_ARG;
     int32_t max_len = 0;
@@ -503,6 +520,7 @@ int domino_load_automaton(domino_t h, const int32_t* delta, int32_t n_states, co
         cls[c] = (uint8_t)found;
     }
     DeviceGuard g(h->device);
+    clear_host_graphs(h);
     h->auto_loaded = false;
     h->arena_ready = false;
     h->Q = n_states;
@@ -887,9 +905,51 @@ int copy_and_decode_chunks(domino_ctx* h, const void* logits_host, int32_t dtype
                                      d_mask + (size_t)r0 * h->W, d_tok + r0, d_lse + r0, nullptr, stream)))
             return rc;
     }
-    return DOMINO_OK;
+    // every copy-stream node rejoins `stream` (a recorded graph needs it; the
+    // copies are done by now anyway)
+    return cuda_status(cudaStreamWaitEvent(st, h->ev_t[3], 0));
 }
 
+
+// The host-buffer step's copies and launches on `st` (and the copy stream),
+// without the final synchronisation.
+int enqueue_host_step(domino_ctx* h, const void* logits_host, void* logits_mapped, bool mapped, int32_t dtype,
+                      int32_t batch, int32_t* states_host, uint64_t* stacks_host, int32_t* tokens_host,
+                      float* lse_host, cudaStream_t st) {
+    int rc;
+    void* stream = (void*)st;
+    int32_t* d_states = (int32_t*)h->s_states.p;
+    uint64_t* d_stacks = stacks_host ? (uint64_t*)h->s_stacks.p : nullptr;
+    uint32_t* d_mask = (uint32_t*)h->s_mask.p;
+    int32_t* d_tok = (int32_t*)h->s_tokens.p;
+    float* d_lse = (float*)h->s_lse.p;
+    if (mapped) {
+        cudaError_t e = cudaMemcpyAsync(d_states, states_host, (size_t)batch * 4, cudaMemcpyHostToDevice, st);
+        if (e == cudaSuccess && d_stacks)
+            e = cudaMemcpyAsync(d_stacks, stacks_host, (size_t)batch * 8, cudaMemcpyHostToDevice, st);
+        if (e == cudaSuccess) e = cudaEventRecord(h->ev_t[0], st);
+        if (e != cudaSuccess) return cuda_status(e);
+        if ((rc = domino_step_mask(h, d_states, d_stacks, batch, d_mask, nullptr, stream))) return rc;
+        if ((e = cudaEventRecord(h->ev_t[1], st)) != cudaSuccess) return cuda_status(e);
+        if ((e = cudaEventRecord(h->ev_t[2], st)) != cudaSuccess) return cuda_status(e);
+        if ((rc = domino_mask_logits(h, logits_mapped, dtype, batch, h->V, d_mask, d_tok, d_lse, nullptr, stream)))
+            return rc;
+        if ((e = cudaEventRecord(h->ev_t[3], st)) != cudaSuccess) return cuda_status(e);
+    } else {
+        if ((rc = copy_and_decode_chunks(h, logits_host, dtype, batch, states_host, stacks_host, st))) return rc;
+    }
+    if ((rc = domino_advance(h, d_states, d_stacks, d_tok, batch, d_states, d_stacks, stream))) return rc;
+    cudaError_t e = cudaMemsetAsync(h->s_count.p, 0, sizeof(uint64_t), st);
+    if (e == cudaSuccess)
+        e = launch_mask_vector_count(h->env, d_mask, (long long)batch * h->W, (unsigned long long*)h->s_count.p, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(h->h_count, h->s_count.p, sizeof(uint64_t), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(tokens_host, d_tok, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess && lse_host) e = cudaMemcpyAsync(lse_host, d_lse, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(states_host, d_states, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess && d_stacks)
+        e = cudaMemcpyAsync(stacks_host, d_stacks, (size_t)batch * 8, cudaMemcpyDeviceToHost, st);
+    return cuda_status(e);
+}
 }  // namespace
 
 int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, int32_t batch,
@@ -946,36 +1006,57 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
             if (e == cudaSuccess) e = cudaEventCreate(&ev);
         if (e != cudaSuccess) return cuda_status(e);
     }
-    int32_t* d_states = (int32_t*)h->s_states.p;
-    uint64_t* d_stacks = stacks_host ? (uint64_t*)h->s_stacks.p : nullptr;
-    uint32_t* d_mask = (uint32_t*)h->s_mask.p;
-    int32_t* d_tok = (int32_t*)h->s_tokens.p;
-    float* d_lse = (float*)h->s_lse.p;
-    if (mapped) {
-        cudaError_t e = cudaMemcpyAsync(d_states, states_host, (size_t)batch * 4, cudaMemcpyHostToDevice, st);
-        if (e == cudaSuccess && d_stacks)
-            e = cudaMemcpyAsync(d_stacks, stacks_host, (size_t)batch * 8, cudaMemcpyHostToDevice, st);
-        if (e == cudaSuccess) e = cudaEventRecord(h->ev_t[0], st);
+    // The step's copies and launches, recorded once per set of buffers on a
+    // non-default stream (the default stream cannot be captured) and replayed
+    // afterwards.  The first two calls of a handle run them directly: the
+    // first sets kernel attributes, the second times the mask step and the
+    // link for the path choice warm (replays update the mask density only).
+    const void* key[16] = {logits_host, states_host, stacks_host, tokens_host, lse_host,
+                           (const void*)(intptr_t)batch, (const void*)(intptr_t)(dtype * 2 + (mapped ? 1 : 0)),
+                           h->s_logits.p, h->s_states.p, h->s_stacks.p, h->s_mask.p, h->s_tokens.p, h->s_lse.p,
+                           h->s_count.p, (const void*)h->h_count, (const void*)st};
+    cudaGraphExec_t exec = nullptr;
+    for (auto& hg : h->host_graphs)
+        if (std::equal(std::begin(key), std::end(key), std::begin(hg.key))) {
+            exec = hg.exec;
+            hg.used = h->host_calls;
+        }
+    cudaError_t e = cudaSuccess;
+    if (!exec && st != nullptr && h->host_calls > 1) {
+        cudaGraph_t gr = nullptr;
+        e = cudaStreamBeginCapture(st, cudaStreamCaptureModeRelaxed);
         if (e != cudaSuccess) return cuda_status(e);
-        if ((rc = domino_step_mask(h, d_states, d_stacks, batch, d_mask, nullptr, stream))) return rc;
-        if ((e = cudaEventRecord(h->ev_t[1], st)) != cudaSuccess) return cuda_status(e);
-        if ((e = cudaEventRecord(h->ev_t[2], st)) != cudaSuccess) return cuda_status(e);
-        if ((rc = domino_mask_logits(h, pa.devicePointer, dtype, batch, h->V, d_mask, d_tok, d_lse, nullptr, stream)))
-            return rc;
-        if ((e = cudaEventRecord(h->ev_t[3], st)) != cudaSuccess) return cuda_status(e);
-    } else {
-        if ((rc = copy_and_decode_chunks(h, logits_host, dtype, batch, states_host, stacks_host, st))) return rc;
+        rc = enqueue_host_step(h, logits_host, pa.devicePointer, mapped, dtype, batch, states_host, stacks_host,
+                               tokens_host, lse_host, st);
+        e = cudaStreamEndCapture(st, &gr);
+        if (rc || e != cudaSuccess) {
+            if (gr) cudaGraphDestroy(gr);
+            return rc ? rc : cuda_status(e);
+        }
+        e = cudaGraphInstantiate(&exec, gr, 0);
+        cudaGraphDestroy(gr);
+        if (e != cudaSuccess) return cuda_status(e);
+        if (h->host_graphs.size() >= 8) {   // keep the 8 most recently used
+            auto lru = std::min_element(h->host_graphs.begin(), h->host_graphs.end(),
+                                        [](const domino_ctx::HostGraph& x, const domino_ctx::HostGraph& y) {
+                                            return x.used < y.used;
+                                        });
+            cudaGraphExecDestroy(lru->exec);
+            h->host_graphs.erase(lru);
+        }
+        domino_ctx::HostGraph hg{};
+        std::copy(std::begin(key), std::end(key), std::begin(hg.key));
+        hg.exec = exec;
+        hg.used = h->host_calls;
+        h->host_graphs.push_back(hg);
     }
-    if ((rc = domino_advance(h, d_states, d_stacks, d_tok, batch, d_states, d_stacks, stream))) return rc;
-    cudaError_t e = cudaMemsetAsync(h->s_count.p, 0, sizeof(uint64_t), st);
-    if (e == cudaSuccess)
-        e = launch_mask_vector_count(h->env, d_mask, (long long)batch * h->W, (unsigned long long*)h->s_count.p, st);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(h->h_count, h->s_count.p, sizeof(uint64_t), cudaMemcpyDeviceToHost, st);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(tokens_host, d_tok, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
-    if (e == cudaSuccess && lse_host) e = cudaMemcpyAsync(lse_host, d_lse, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(states_host, d_states, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
-    if (e == cudaSuccess && d_stacks)
-        e = cudaMemcpyAsync(stacks_host, d_stacks, (size_t)batch * 8, cudaMemcpyDeviceToHost, st);
+    if (exec) {
+        e = cudaGraphLaunch(exec, st);
+    } else if ((rc = enqueue_host_step(h, logits_host, pa.devicePointer, mapped, dtype, batch, states_host,
+                                       stacks_host, tokens_host, lse_host, st))) {
+        return rc;
+    }
+    h->host_calls++;
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
     if (e == cudaSuccess) {
         h->vec_density = (double)*h->h_count / ((double)batch * h->W * 4.0);

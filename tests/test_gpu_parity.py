@@ -313,6 +313,46 @@ def test_decode_step_host_matches_oracle(config, pinned):
         assert (k_host == k_o).all()
 
 
+@pytest.mark.parametrize("config", [2, 5])
+def test_decode_step_host_replayed_steps_match_oracle(config):
+    """On a non-default stream the host-buffer step is recorded once per set of
+    buffers and replayed: a multi-step loop over two alternating pinned logits
+    buffers and one pageable one gives the oracle's tokens and configurations
+    every step."""
+    import oracle
+    w = workload(config)
+    has_stack = w.automaton.rules is not None
+    d = Domino.from_parts(w.automaton, w.vocab, device=0)
+    P = problem(config)
+    states, stacks = w.initial_configs()
+    s_host = torch.from_numpy(states.copy()).pin_memory()
+    k_host = torch.from_numpy(stacks.view(np.int64).copy()).pin_memory() if has_stack else None
+    tok = torch.empty(len(states), dtype=torch.int32).pin_memory()
+    lse_h = torch.empty(len(states), dtype=torch.float32).pin_memory()
+    bufs = [torch.from_numpy(w.logits(40 + i).view(np.int16)).pin_memory() for i in range(2)]
+    bufs.append(torch.from_numpy(w.logits(42).view(np.int16)))          # pageable: the copy path
+    s_o, k_o = states.copy(), stacks.copy()
+    st = torch.cuda.Stream()
+    for i in range(7):
+        b = bufs[i % 3]
+        B.domino_decode_step_host(d.h, b.data_ptr(), B.DTYPE_BF16, len(states), s_host.data_ptr(),
+                                  k_host.data_ptr() if has_stack else None, tok.data_ptr(), lse_h.data_ptr(),
+                                  stream=st.cuda_stream)
+        lg = b.numpy().view(np.uint16)
+        m, _, _ = P.step_mask(s_o, k_o if has_stack else None, n_threads=NT)
+        a_o, l_o, _ = oracle.mask_logits(lg, m)
+        s_o, k_o2, _ = P.advance(s_o, k_o if has_stack else None, a_o, w.automaton.start)
+        k_o = k_o2 if has_stack else k_o
+        assert (tok.numpy() == a_o).all(), i
+        fin = np.isfinite(l_o)
+        assert np.abs(lse_h.numpy()[fin] - l_o[fin]).max(initial=0) < TOL
+        assert (s_host.numpy() == s_o).all(), i
+        if has_stack:
+            assert (k_host.numpy().view(np.uint64) == k_o).all(), i
+    assert d.device_error() == 0
+    d.close()
+
+
 def test_decode_step_host_matches_device_path():
     w = workload(2)
     states, _ = configs(2)
