@@ -58,7 +58,11 @@ struct domino_ctx {
     bool arena_ready = false;
     int32_t n_windows = 0;
     // staging for domino_decode_step_host
-    DevBuf s_logits, s_states, s_stacks, s_mask, s_tokens, s_lse;
+    // s_io packs the step's small inputs and outputs (see io_layout) so that
+    // each direction takes one copy through the pinned staging buffer h_io
+    DevBuf s_logits, s_mask, s_io;
+    void* h_io = nullptr;
+    size_t h_io_n = 0;
     // opportunistic masking: proposals, the fallback row list and its length
     DevBuf o_prop, o_rows, o_count;
     // domino_decode_step_host: a copy stream and the events that hand each
@@ -66,8 +70,6 @@ struct domino_ctx {
     cudaStream_t cp_stream = nullptr;
     cudaEvent_t ev_cfg = nullptr;
     cudaEvent_t ev_chunk[8] = {};
-    DevBuf s_count;                 // non-zero mask bytes of the last step
-    uint64_t* h_count = nullptr;    // its pinned host copy
     double vec_density = 0.0;       // share of logit vectors the last step's masks allowed
     cudaEvent_t ev_t[4] = {};       // timing: mask step (0, 1) and logits copy (2, 3)
     double t_step_ms = 0.0;         // last mask-step time
@@ -109,9 +111,8 @@ void dev_free(DevBuf& b) {
 int64_t dev_bytes(const domino_ctx* h) {
     const DevBuf* all[] = {&h->d_head, &h->d_info, &h->d_tail_off, &h->d_tail, &h->d_pos_of, &h->d_units,
                            &h->d_unit_off, &h->d_cls_units, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_self, &h->d_tok_cls, &h->d_err, &h->d_partials,
-                           &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_states, &h->s_stacks,
-                           &h->s_mask, &h->s_tokens, &h->s_lse, &h->o_prop, &h->o_rows, &h->o_count,
-                           &h->s_count};
+                           &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_mask, &h->s_io,
+                           &h->o_prop, &h->o_rows, &h->o_count};
     int64_t n = 0;
     for (auto* b : all) n += (int64_t)b->n;
     return n;
@@ -371,9 +372,8 @@ int domino_destroy(domino_t h) {
         cudaDeviceSynchronize();
         DevBuf* all[] = {&h->d_head, &h->d_info, &h->d_tail_off, &h->d_tail, &h->d_pos_of, &h->d_units,
                          &h->d_unit_off, &h->d_cls_units, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_self, &h->d_tok_cls, &h->d_err, &h->d_partials,
-                         &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_states, &h->s_stacks,
-                         &h->s_mask, &h->s_tokens, &h->s_lse, &h->o_prop, &h->o_rows, &h->o_count,
-                           &h->s_count};
+                         &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_mask, &h->s_io,
+                         &h->o_prop, &h->o_rows, &h->o_count};
         for (auto* b : all) dev_free(*b);
         for (cudaEvent_t& e : h->ev_chunk)
             if (e) cudaEventDestroy(e);
@@ -381,7 +381,7 @@ int domino_destroy(domino_t h) {
             if (e) cudaEventDestroy(e);
         if (h->ev_cfg) cudaEventDestroy(h->ev_cfg);
         if (h->cp_stream) cudaStreamDestroy(h->cp_stream);
-        if (h->h_count) cudaFreeHost(h->h_count);
+        if (h->h_io) cudaFreeHost(h->h_io);
         clear_host_graphs(h);
         cudaGetLastError();
     }
@@ -861,27 +861,46 @@ int domino_advance_table(domino_t h, const int32_t* table_next_dev, const int32_
 
 namespace {
 
+// The host-buffer step's small inputs and outputs in one buffer (device s_io,
+// pinned host h_io): [count of non-zero mask bytes | tokens | lse | states |
+// stacks], each part on a 16-byte boundary.  States and stacks go up in one
+// copy, everything comes back in one.
+struct IoLayout {
+    size_t cnt, tok, lse, st, sk, in_end;
+};
+IoLayout io_layout(int32_t batch, bool stacks) {
+    auto a16 = [](size_t x) { return (x + 15) / 16 * 16; };
+    IoLayout L{};
+    L.cnt = 0;
+    L.tok = 16;
+    L.lse = a16(L.tok + (size_t)batch * 4);
+    L.st = a16(L.lse + (size_t)batch * 4);
+    L.sk = a16(L.st + (size_t)batch * 4);
+    L.in_end = stacks ? L.sk + (size_t)batch * 8 : L.st + (size_t)batch * 4;
+    return L;
+}
+
 // Pageable logits: the configurations and then the logits are copied in up
 // to 8 chunks of rows on the copy stream; the mask step runs while they copy,
 // and each chunk's masked argmax starts as soon as its rows have landed.
-int copy_and_decode_chunks(domino_ctx* h, const void* logits_host, int32_t dtype, int32_t batch,
-                           const int32_t* states_host, const uint64_t* stacks_host, cudaStream_t st) {
+int copy_and_decode_chunks(domino_ctx* h, const void* logits_host, int32_t dtype, int32_t batch, bool stacks,
+                           const IoLayout& L, cudaStream_t st) {
     int rc;
     void* stream = (void*)st;
     const size_t esz = dtype == DOMINO_DTYPE_BF16 ? 2 : 4;
     const size_t row_bytes = (size_t)h->V * esz;
     const size_t logit_bytes = (size_t)batch * row_bytes;
-    int32_t* d_states = (int32_t*)h->s_states.p;
-    uint64_t* d_stacks = stacks_host ? (uint64_t*)h->s_stacks.p : nullptr;
+    char* io = (char*)h->s_io.p;
+    int32_t* d_states = (int32_t*)(io + L.st);
+    uint64_t* d_stacks = stacks ? (uint64_t*)(io + L.sk) : nullptr;
     uint32_t* d_mask = (uint32_t*)h->s_mask.p;
-    int32_t* d_tok = (int32_t*)h->s_tokens.p;
-    float* d_lse = (float*)h->s_lse.p;
+    int32_t* d_tok = (int32_t*)(io + L.tok);
+    float* d_lse = (float*)(io + L.lse);
     const int n_chunks = (int)std::max<size_t>(1, std::min<size_t>({(size_t)8, (size_t)batch, logit_bytes >> 23}));
     cudaError_t e = cudaEventRecord(h->ev_cfg, st);   // the caller's earlier work on `stream` comes first
     if (e == cudaSuccess) e = cudaStreamWaitEvent(h->cp_stream, h->ev_cfg, 0);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(d_states, states_host, (size_t)batch * 4, cudaMemcpyHostToDevice, h->cp_stream);
-    if (e == cudaSuccess && d_stacks)
-        e = cudaMemcpyAsync(d_stacks, stacks_host, (size_t)batch * 8, cudaMemcpyHostToDevice, h->cp_stream);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(io + L.st, (char*)h->h_io + L.st, L.in_end - L.st, cudaMemcpyHostToDevice, h->cp_stream);
     if (e == cudaSuccess) e = cudaEventRecord(h->ev_cfg, h->cp_stream);
     std::vector<int32_t> r0s((size_t)n_chunks + 1);
     for (int k = 0; k <= n_chunks; ++k) r0s[(size_t)k] = (int32_t)(((int64_t)batch * k) / n_chunks);
@@ -910,23 +929,22 @@ int copy_and_decode_chunks(domino_ctx* h, const void* logits_host, int32_t dtype
     return cuda_status(cudaStreamWaitEvent(st, h->ev_t[3], 0));
 }
 
-
 // The host-buffer step's copies and launches on `st` (and the copy stream),
-// without the final synchronisation.
+// without the final synchronisation.  The states and stacks are already in
+// h_io; the outputs land there.
 int enqueue_host_step(domino_ctx* h, const void* logits_host, void* logits_mapped, bool mapped, int32_t dtype,
-                      int32_t batch, int32_t* states_host, uint64_t* stacks_host, int32_t* tokens_host,
-                      float* lse_host, cudaStream_t st) {
+                      int32_t batch, bool stacks, const IoLayout& L, cudaStream_t st) {
     int rc;
     void* stream = (void*)st;
-    int32_t* d_states = (int32_t*)h->s_states.p;
-    uint64_t* d_stacks = stacks_host ? (uint64_t*)h->s_stacks.p : nullptr;
+    char* io = (char*)h->s_io.p;
+    int32_t* d_states = (int32_t*)(io + L.st);
+    uint64_t* d_stacks = stacks ? (uint64_t*)(io + L.sk) : nullptr;
     uint32_t* d_mask = (uint32_t*)h->s_mask.p;
-    int32_t* d_tok = (int32_t*)h->s_tokens.p;
-    float* d_lse = (float*)h->s_lse.p;
+    int32_t* d_tok = (int32_t*)(io + L.tok);
+    float* d_lse = (float*)(io + L.lse);
     if (mapped) {
-        cudaError_t e = cudaMemcpyAsync(d_states, states_host, (size_t)batch * 4, cudaMemcpyHostToDevice, st);
-        if (e == cudaSuccess && d_stacks)
-            e = cudaMemcpyAsync(d_stacks, stacks_host, (size_t)batch * 8, cudaMemcpyHostToDevice, st);
+        cudaError_t e =
+            cudaMemcpyAsync(io + L.st, (char*)h->h_io + L.st, L.in_end - L.st, cudaMemcpyHostToDevice, st);
         if (e == cudaSuccess) e = cudaEventRecord(h->ev_t[0], st);
         if (e != cudaSuccess) return cuda_status(e);
         if ((rc = domino_step_mask(h, d_states, d_stacks, batch, d_mask, nullptr, stream))) return rc;
@@ -936,20 +954,16 @@ int enqueue_host_step(domino_ctx* h, const void* logits_host, void* logits_mappe
             return rc;
         if ((e = cudaEventRecord(h->ev_t[3], st)) != cudaSuccess) return cuda_status(e);
     } else {
-        if ((rc = copy_and_decode_chunks(h, logits_host, dtype, batch, states_host, stacks_host, st))) return rc;
+        if ((rc = copy_and_decode_chunks(h, logits_host, dtype, batch, stacks, L, st))) return rc;
     }
     if ((rc = domino_advance(h, d_states, d_stacks, d_tok, batch, d_states, d_stacks, stream))) return rc;
-    cudaError_t e = cudaMemsetAsync(h->s_count.p, 0, sizeof(uint64_t), st);
+    cudaError_t e = cudaMemsetAsync(io + L.cnt, 0, sizeof(uint64_t), st);
     if (e == cudaSuccess)
-        e = launch_mask_vector_count(h->env, d_mask, (long long)batch * h->W, (unsigned long long*)h->s_count.p, st);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(h->h_count, h->s_count.p, sizeof(uint64_t), cudaMemcpyDeviceToHost, st);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(tokens_host, d_tok, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
-    if (e == cudaSuccess && lse_host) e = cudaMemcpyAsync(lse_host, d_lse, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(states_host, d_states, (size_t)batch * 4, cudaMemcpyDeviceToHost, st);
-    if (e == cudaSuccess && d_stacks)
-        e = cudaMemcpyAsync(stacks_host, d_stacks, (size_t)batch * 8, cudaMemcpyDeviceToHost, st);
+        e = launch_mask_vector_count(h->env, d_mask, (long long)batch * h->W, (unsigned long long*)(io + L.cnt), st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(h->h_io, io, L.in_end, cudaMemcpyDeviceToHost, st);
     return cuda_status(e);
 }
+
 }  // namespace
 
 int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, int32_t batch,
@@ -966,6 +980,8 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
     const size_t esz = dtype == DOMINO_DTYPE_BF16 ? 2 : 4;
     const size_t row_bytes = (size_t)h->V * esz;
     const size_t logit_bytes = (size_t)batch * row_bytes;
+    const bool stacks = stacks_host != nullptr;
+    const IoLayout L = io_layout(batch, stacks);
     // Pinned (page-locked, mapped) logits are read where they are: the masked
     // pass pulls only the 16-byte logit vectors that hold an allowed token
     // across the host link, so masked-out logits never travel, but it starts
@@ -982,22 +998,27 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
         const double t_copy = (double)logit_bytes / (h->link_gbs * 1e6);   // ms
         mapped = h->t_step_ms + h->vec_density * t_copy < std::max(t_copy, h->t_step_ms);
     }
-    if ((!mapped && h->s_logits.n < logit_bytes) || h->s_states.n < (size_t)batch * 4 || !h->cp_stream) {
+    const bool grow = (!mapped && h->s_logits.n < logit_bytes) || h->s_io.n < L.in_end ||
+                      h->s_mask.n < (size_t)batch * (size_t)h->W * 4 || h->h_io_n < L.in_end || !h->cp_stream;
+    if (grow) {   // buffers may move: recorded steps that use them are dropped
         if (cudaStreamSynchronize(st) != cudaSuccess) return cuda_status(cudaGetLastError());
+        clear_host_graphs(h);
     }
     if (!mapped && (rc = dev_reserve(h->s_logits, logit_bytes))) return rc;
-    if ((rc = dev_reserve(h->s_states, (size_t)batch * 4))) return rc;
-    if ((rc = dev_reserve(h->s_stacks, (size_t)batch * 8))) return rc;
     if ((rc = dev_reserve(h->s_mask, (size_t)batch * (size_t)h->W * 4))) return rc;
-    if ((rc = dev_reserve(h->s_tokens, (size_t)batch * 4))) return rc;
-    if ((rc = dev_reserve(h->s_lse, (size_t)batch * 4))) return rc;
-    if ((rc = dev_reserve(h->s_count, 16))) return rc;
-    if (!h->cp_stream) {
-        if (cudaMallocHost((void**)&h->h_count, sizeof(uint64_t)) != cudaSuccess) {
+    if ((rc = dev_reserve(h->s_io, L.in_end))) return rc;
+    if (h->h_io_n < L.in_end) {
+        if (h->h_io) cudaFreeHost(h->h_io);
+        h->h_io = nullptr;
+        h->h_io_n = 0;
+        if (cudaMallocHost(&h->h_io, L.in_end) != cudaSuccess) {
             cudaGetLastError();
-            h->h_count = nullptr;
+            h->h_io = nullptr;
             return DOMINO_E_OOM;
         }
+        h->h_io_n = L.in_end;
+    }
+    if (!h->cp_stream) {
         cudaError_t e = cudaStreamCreateWithFlags(&h->cp_stream, cudaStreamNonBlocking);
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_cfg, cudaEventDisableTiming);
         for (cudaEvent_t& ev : h->ev_chunk)
@@ -1006,15 +1027,17 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
             if (e == cudaSuccess) e = cudaEventCreate(&ev);
         if (e != cudaSuccess) return cuda_status(e);
     }
+    std::memcpy((char*)h->h_io + L.st, states_host, (size_t)batch * 4);
+    if (stacks) std::memcpy((char*)h->h_io + L.sk, stacks_host, (size_t)batch * 8);
     // The step's copies and launches, recorded once per set of buffers on a
     // non-default stream (the default stream cannot be captured) and replayed
     // afterwards.  The first two calls of a handle run them directly: the
     // first sets kernel attributes, the second times the mask step and the
     // link for the path choice warm (replays update the mask density only).
-    const void* key[16] = {logits_host, states_host, stacks_host, tokens_host, lse_host,
-                           (const void*)(intptr_t)batch, (const void*)(intptr_t)(dtype * 2 + (mapped ? 1 : 0)),
-                           h->s_logits.p, h->s_states.p, h->s_stacks.p, h->s_mask.p, h->s_tokens.p, h->s_lse.p,
-                           h->s_count.p, (const void*)h->h_count, (const void*)st};
+    const void* key[16] = {logits_host, (const void*)(intptr_t)batch,
+                           (const void*)(intptr_t)(dtype * 4 + (mapped ? 1 : 0) + (stacks ? 2 : 0)), h->s_logits.p,
+                           h->s_mask.p, h->s_io.p, h->h_io, (const void*)st, nullptr, nullptr, nullptr, nullptr,
+                           nullptr, nullptr, nullptr, nullptr};
     cudaGraphExec_t exec = nullptr;
     for (auto& hg : h->host_graphs)
         if (std::equal(std::begin(key), std::end(key), std::begin(hg.key))) {
@@ -1026,8 +1049,7 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
         cudaGraph_t gr = nullptr;
         e = cudaStreamBeginCapture(st, cudaStreamCaptureModeRelaxed);
         if (e != cudaSuccess) return cuda_status(e);
-        rc = enqueue_host_step(h, logits_host, pa.devicePointer, mapped, dtype, batch, states_host, stacks_host,
-                               tokens_host, lse_host, st);
+        rc = enqueue_host_step(h, logits_host, pa.devicePointer, mapped, dtype, batch, stacks, L, st);
         e = cudaStreamEndCapture(st, &gr);
         if (rc || e != cudaSuccess) {
             if (gr) cudaGraphDestroy(gr);
@@ -1052,24 +1074,29 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
     }
     if (exec) {
         e = cudaGraphLaunch(exec, st);
-    } else if ((rc = enqueue_host_step(h, logits_host, pa.devicePointer, mapped, dtype, batch, states_host,
-                                       stacks_host, tokens_host, lse_host, st))) {
+    } else if ((rc = enqueue_host_step(h, logits_host, pa.devicePointer, mapped, dtype, batch, stacks, L, st))) {
         return rc;
     }
     h->host_calls++;
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
-    if (e == cudaSuccess) {
-        h->vec_density = (double)*h->h_count / ((double)batch * h->W * 4.0);
-        float ms = 0.f;
-        if (cudaEventElapsedTime(&ms, h->ev_t[0], h->ev_t[1]) == cudaSuccess) h->t_step_ms = ms;
-        // the link rate: bytes copied over the copy time, or the vectors read in
-        // place over the in-place pass's time (that pass is bound by the link)
-        const double moved = mapped ? h->vec_density * (double)logit_bytes : (double)logit_bytes;
-        if (moved > (double)(1 << 20) && cudaEventElapsedTime(&ms, h->ev_t[2], h->ev_t[3]) == cudaSuccess && ms > 0.f)
-            h->link_gbs = moved / ((double)ms * 1e6);
-        cudaGetLastError();
-    }
-    return cuda_status(e);
+    if (e != cudaSuccess) return cuda_status(e);
+    const char* io = (const char*)h->h_io;
+    std::memcpy(tokens_host, io + L.tok, (size_t)batch * 4);
+    if (lse_host) std::memcpy(lse_host, io + L.lse, (size_t)batch * 4);
+    std::memcpy(states_host, io + L.st, (size_t)batch * 4);
+    if (stacks) std::memcpy(stacks_host, io + L.sk, (size_t)batch * 8);
+    uint64_t count = 0;
+    std::memcpy(&count, io + L.cnt, sizeof(count));
+    h->vec_density = (double)count / ((double)batch * h->W * 4.0);
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, h->ev_t[0], h->ev_t[1]) == cudaSuccess) h->t_step_ms = ms;
+    // the link rate: bytes copied over the copy time, or the vectors read in
+    // place over the in-place pass's time (that pass is bound by the link)
+    const double moved = mapped ? h->vec_density * (double)logit_bytes : (double)logit_bytes;
+    if (moved > (double)(1 << 20) && cudaEventElapsedTime(&ms, h->ev_t[2], h->ev_t[3]) == cudaSuccess && ms > 0.f)
+        h->link_gbs = moved / ((double)ms * 1e6);
+    cudaGetLastError();
+    return DOMINO_OK;
 }
 
 
