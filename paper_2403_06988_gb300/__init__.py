@@ -65,6 +65,25 @@ class Domino:
         B.domino_step_mask(self.h, states, stacks, b, mask, nxt, stream)
         return mask, nxt
 
+    def step_decode(self, states, stacks, logits, want_logprobs: bool = False, out_mask=None, stream=None):
+        """Mask step fused with the masked greedy decode: returns (mask, argmax, lse, logprobs or None)."""
+        import torch
+        b = states.shape[0]
+        dtype = DTYPE_BF16 if logits.dtype == torch.bfloat16 else DTYPE_F32
+        if dtype == DTYPE_F32 and logits.dtype != torch.float32:
+            raise TypeError("logits must be float32 or bfloat16")
+        if logits.stride(1) != 1:
+            raise ValueError("logits rows must be contiguous")
+        mask = out_mask if out_mask is not None else torch.empty((b, self.info()["n_words"]), dtype=torch.int32,
+                                                                 device=states.device)
+        argmax = torch.empty(b, dtype=torch.int32, device=states.device)
+        lse = torch.empty(b, dtype=torch.float32, device=states.device)
+        lp = torch.empty((b, self.info()["n_tokens"]), dtype=torch.float32, device=states.device) if want_logprobs \
+            else None
+        B.domino_step_decode(self.h, states, stacks, b, logits.data_ptr(), dtype, logits.stride(0), mask, argmax, lse,
+                             lp, stream)
+        return mask, argmax, lse, lp
+
     def precompute_table(self, want_next: bool = True, want_mask: bool = True, stream=None):
         import torch
         info = self.info()

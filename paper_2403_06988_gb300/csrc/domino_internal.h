@@ -93,7 +93,19 @@ int step_fixed_smem_bytes(const StepView& v, bool next);
 cudaError_t launch_step_mask(const StepView& v, const LaunchEnv& env, bool stack, int mode, const int32_t* states,
                              const uint64_t* stacks, int32_t batch, bool row_is_state, uint32_t* mask,
                              int32_t* next, cudaStream_t st, const int32_t* row_ids = nullptr,
-                             const int32_t* row_count = nullptr);
+                             const int32_t* row_count = nullptr, const void* fuse_logits = nullptr,
+                             int64_t fuse_stride = 0, float4* fuse_part = nullptr, bool fuse_prefetch = false);
+
+// The mask step fused with the masked decode (bf16 logits, rows on 16-byte
+// boundaries): fuse_part [batch][n_windows] receives per-window partials,
+// merged into argmax / lse by launch_fused_combine.
+cudaError_t launch_fused_combine(const float4* part, int32_t batch, int32_t n_windows, int32_t* argmax, float* lse,
+                                 cudaStream_t st);
+
+// Log-probabilities only (bf16 logits, rows on 16-byte boundaries), given the
+// rows' lse: logprobs[b][t] = logit - lse[b] for allowed t, -inf else.
+cudaError_t launch_logprobs_bf16(const LaunchEnv& env, const void* logits, int32_t batch, int64_t row_stride,
+                                 int32_t V, const uint32_t* mask, const float* lse, float* logprobs, cudaStream_t st);
 
 // Sampling decode: Gumbel-max with Philox4x32-10 uniforms (kernels.cu).
 struct SampleArgs {

@@ -54,7 +54,7 @@ struct domino_ctx {
     DevBuf d_head, d_info, d_tail_off, d_tail, d_pos_of, d_units, d_unit_off, d_cls_units, d_eos_slot;
     int32_t max_units = 0;
     DevBuf d_dense, d_sparse, d_accept, d_self, d_tok_cls;
-    DevBuf d_err, d_partials, d_counters, d_lse_tmp;
+    DevBuf d_err, d_partials, d_counters, d_lse_tmp, d_fpart;
     bool arena_ready = false;
     int32_t n_windows = 0;
     // staging for domino_decode_step_host
@@ -110,7 +110,7 @@ void dev_free(DevBuf& b) {
 
 int64_t dev_bytes(const domino_ctx* h) {
     const DevBuf* all[] = {&h->d_head, &h->d_info, &h->d_tail_off, &h->d_tail, &h->d_pos_of, &h->d_units,
-                           &h->d_unit_off, &h->d_cls_units, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_self, &h->d_tok_cls, &h->d_err, &h->d_partials,
+                           &h->d_unit_off, &h->d_cls_units, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_self, &h->d_tok_cls, &h->d_err, &h->d_fpart, &h->d_partials,
                            &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_mask, &h->s_io,
                            &h->o_prop, &h->o_rows, &h->o_count};
     int64_t n = 0;
@@ -371,7 +371,7 @@ int domino_destroy(domino_t h) {
         DeviceGuard g(h->device);
         cudaDeviceSynchronize();
         DevBuf* all[] = {&h->d_head, &h->d_info, &h->d_tail_off, &h->d_tail, &h->d_pos_of, &h->d_units,
-                         &h->d_unit_off, &h->d_cls_units, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_self, &h->d_tok_cls, &h->d_err, &h->d_partials,
+                         &h->d_unit_off, &h->d_cls_units, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_self, &h->d_tok_cls, &h->d_err, &h->d_fpart, &h->d_partials,
                          &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_mask, &h->s_io,
                          &h->o_prop, &h->o_rows, &h->o_count};
         for (auto* b : all) dev_free(*b);
@@ -718,6 +718,49 @@ int domino_advance(domino_t h, const int32_t* states_dev, const uint64_t* stacks
     const int mode = choose_mode(h, v, false);
     return cuda_status(launch_advance(v, h->stack, mode, states_dev, stacks_dev, tokens_dev, batch, states_out,
                                       stacks_out, (cudaStream_t)stream));
+}
+
+int domino_step_decode(domino_t h, const int32_t* states_dev, const uint64_t* stacks_dev, int32_t batch,
+                       const void* logits_dev, int32_t dtype, int64_t row_stride_elems, uint32_t* mask_dev,
+                       int32_t* argmax_dev, float* lse_dev, float* logprobs_dev, void* stream) {
+    int rc = ready_for_compute(h);
+    if (rc) return rc;
+    if (dtype != DOMINO_DTYPE_F32 && dtype != DOMINO_DTYPE_BF16) return DOMINO_E_INVALID_ARG;
+    if (batch < 0 || row_stride_elems < h->V) return DOMINO_E_INVALID_ARG;
+    if (batch == 0) return DOMINO_OK;
+    if (!states_dev || !logits_dev || !mask_dev || !argmax_dev || (logprobs_dev && !lse_dev))
+        return DOMINO_E_INVALID_ARG;
+    DeviceGuard g(h->device);
+    cudaStream_t st = (cudaStream_t)stream;
+    const bool fusable = dtype == DOMINO_DTYPE_BF16 && reinterpret_cast<uintptr_t>(logits_dev) % 16 == 0 &&
+                         ((size_t)row_stride_elems * 2) % 16 == 0 &&
+                         (int64_t)batch * h->n_windows < (int64_t)INT32_MAX;   // partial slots are int
+    if (!fusable) {   // the two kernels one after the other
+        if ((rc = domino_step_mask(h, states_dev, stacks_dev, batch, mask_dev, nullptr, stream))) return rc;
+        return domino_mask_logits(h, logits_dev, dtype, batch, row_stride_elems, mask_dev, argmax_dev, lse_dev,
+                                  logprobs_dev, stream);
+    }
+    const size_t part_bytes = (size_t)batch * (size_t)h->n_windows * sizeof(float4);
+    if (h->d_fpart.n < part_bytes) {
+        if (cudaStreamSynchronize(st) != cudaSuccess) return cuda_status(cudaGetLastError());
+        if ((rc = dev_reserve(h->d_fpart, part_bytes))) return rc;
+    }
+    // logits in device memory are pulled into L2 a tile ahead of their fold;
+    // host-resident logits are read only where the mask allows a token
+    cudaPointerAttributes pa{};
+    const bool on_device = cudaPointerGetAttributes(&pa, logits_dev) == cudaSuccess && pa.type == cudaMemoryTypeDevice;
+    if (!on_device) cudaGetLastError();
+    StepView v = make_view(h);
+    const int mode = choose_mode(h, v, false);
+    cudaError_t e = launch_step_mask(v, h->env, h->stack, mode, states_dev, stacks_dev, batch, false, mask_dev, nullptr,
+                                     st, nullptr, nullptr, logits_dev, row_stride_elems, (float4*)h->d_fpart.p,
+                                     on_device);
+    if (e == cudaSuccess)
+        e = launch_fused_combine((const float4*)h->d_fpart.p, batch, h->n_windows, argmax_dev, lse_dev, st);
+    if (e == cudaSuccess && logprobs_dev)
+        e = launch_logprobs_bf16(h->env, logits_dev, batch, row_stride_elems, h->V, mask_dev, lse_dev, logprobs_dev,
+                                 st);
+    return cuda_status(e);
 }
 
 int domino_mask_sample(domino_t h, const void* logits_dev, int32_t dtype, int32_t batch, int64_t row_stride_elems,

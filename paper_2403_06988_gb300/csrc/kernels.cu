@@ -92,6 +92,116 @@ struct RowList {
     __device__ __forceinline__ int row(int i) const { return ids ? __ldg(ids + base + i) : i; }
 };
 
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// (m, idx, s) <- (m, idx, s) (+) (m2, i2, s2): larger max wins, lower index on
+// equal maxima; the other sum is rescaled to the winner's max.
+__device__ __forceinline__ void acc_merge(float& m, int& idx, float& s, float m2, int i2, float s2) {
+    if (m2 > m || (m2 == m && i2 < idx)) {
+        const float tm = m, ts = s;
+        const int ti = idx;
+        m = m2;
+        idx = i2;
+        s = s2;
+        m2 = tm;
+        i2 = ti;
+        s2 = ts;
+    }
+    if (s2 != 0.0f) s += s2 * ex2((m2 - m) * kLog2e);
+}
+
+// one allowed logit x at index t; mL = m * log2(e) is kept with m
+__device__ __forceinline__ void acc_add(float& m, float& mL, int& idx, float& s, float x, int t) {
+    if (x > m) {
+        const float xL = x * kLog2e;
+        s = s * ex2(mL - xL) + 1.0f;
+        m = x;
+        mL = xL;
+        idx = t;
+    } else {
+        s += ex2(fmaf(x, kLog2e, -mL));
+    }
+}
+
+__device__ __forceinline__ void warp_merge(float& m, int& idx, float& s) {
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+        const int i2 = __shfl_xor_sync(0xffffffffu, idx, off);
+        const float s2 = __shfl_xor_sync(0xffffffffu, s, off);
+        acc_merge(m, idx, s, m2, i2, s2);
+    }
+}
+
+// CTA-wide (m, idx, s); the result is valid in thread 0.  Uses two barriers.
+__device__ __forceinline__ void block_merge(float& m, int& idx, float& s) {
+    __shared__ float sm_m[kLogitThreads / 32], sm_s[kLogitThreads / 32];
+    __shared__ int sm_i[kLogitThreads / 32];
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    warp_merge(m, idx, s);
+    __syncthreads();   // protect sm_* against the previous call's readers
+    if (lane == 0) {
+        sm_m[wid] = m;
+        sm_i[wid] = idx;
+        sm_s[wid] = s;
+    }
+    __syncthreads();
+    if (wid == 0) {
+        m = lane < kLogitThreads / 32 ? sm_m[lane] : -INFINITY;
+        idx = lane < kLogitThreads / 32 ? sm_i[lane] : INT_MAX;
+        s = lane < kLogitThreads / 32 ? sm_s[lane] : 0.0f;
+        warp_merge(m, idx, s);
+    }
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+
+// The mask step fused with the masked decode: after each tile's walk, warp r
+// folds row r's allowed bf16 logits of the tile's window into a (max, argmax,
+// sum of exp) partial per (row, window); a combine kernel merges a row's
+// windows.  A window with at most 32 allowed tokens lists them one per lane,
+// loads their logits and folds them after the next tile's walk; a denser
+// window is folded at once, lane j over mask word j.  `logits` may point to
+// device memory or to pinned host memory.
+__device__ __forceinline__ void prefetch_l2(const void* p) {
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+
+// Folds one row window whose allowed tokens (at most 32) were listed one per
+// lane: t = INT_MAX marks an empty lane, raw the lane's bf16 logit.  Writes
+// (max, lowest index of the max, sum of exp against the max) to part[slot].
+__device__ __forceinline__ void fold_pending(float4* part, int slot, unsigned short raw, int t, int lane) {
+    const float x = t != INT_MAX ? __uint_as_float((uint32_t)raw << 16) : -INFINITY;
+    float m = x;
+    int idx = t;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+        const int i2 = __shfl_xor_sync(0xffffffffu, idx, off);
+        if (m2 > m || (m2 == m && i2 < idx)) {
+            m = m2;
+            idx = i2;
+        }
+    }
+    float e = t != INT_MAX ? ex2(fmaf(x, kLog2e, -m * kLog2e)) : 0.0f;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) e += __shfl_xor_sync(0xffffffffu, e, off);
+    if (lane == 0) part[slot] = make_float4(m, __int_as_float(idx), e, 0.f);
+}
+
+struct FuseArgs {
+    const void* logits;   // nullptr: no fusion
+    int64_t stride;       // row stride in elements
+    float4* part;         // [batch][n_windows] partials
+    int prefetch;         // logits in device memory: pull each tile's rows into L2 ahead of the fold
+};
+
 // Shared-memory layout of the step kernel (offsets in bytes).
 struct StepLayout {
     int head, info, units, cls, tokcls, items, rows, ctrl, rowmask, cfg, mtile, ntile, accept, self, table, total;
@@ -275,7 +385,7 @@ __global__ void __launch_bounds__(kStepThreads, 1)
     step_kernel(const StepView v, const uint4* __restrict__ img, int img_bytes, int img_tgt_off, int img_ret_off,
                 const int32_t* __restrict__ states, const uint64_t* __restrict__ stacks, int32_t batch,
                 int32_t R, int32_t n_row_tiles, int32_t n_tiles, int32_t row_is_state, uint32_t* __restrict__ mask,
-                int32_t* __restrict__ next, const RowList list) {
+                int32_t* __restrict__ next, const RowList list, const FuseArgs fuse) {
     using E = typename std::conditional<STACK, uint32_t, uint16_t>::type;
     extern __shared__ __align__(16) unsigned char smem[];
     const int K = v.K;
@@ -351,6 +461,10 @@ __global__ void __launch_bounds__(kStepThreads, 1)
     };
     prefetch(t0);
     int cur_w = -1;
+    // a sparse fold in flight (fused decode): partial slot (-1: none), the
+    // lane's token (INT_MAX: none) and its raw bf16 logit
+    int p_slot = -1, p_t = INT_MAX;
+    unsigned short p_raw = 0;
     for (int t = t0; t < t1; ++t) {
         const int w = t / n_row_tiles;
         const int r0 = (t - w * n_row_tiles) * R;
@@ -380,6 +494,17 @@ __global__ void __launch_bounds__(kStepThreads, 1)
         }
         if (tid == 0) s_ctrl[1] = 0;   // items listed so far
         for (int i = tid; i < nr * 32; i += kStepThreads) s_mtile[i] = 0u;
+        if (fuse.prefetch) {
+            // the tile's logits head for L2 while the walk runs: one 128-byte
+            // line per thread, every line start inside the row's window slice
+            const int win_bytes = min(kWin, v.V - w * kWin) * 2;
+            for (int i = tid; i < nr * (kWin * 2 / 128); i += kStepThreads) {
+                const int r = i / (kWin * 2 / 128), off = (i % (kWin * 2 / 128)) * 128;
+                if (off < win_bytes)
+                    prefetch_l2(reinterpret_cast<const char*>(fuse.logits) + (size_t)(r0 + r) * fuse.stride * 2 +
+                                (size_t)w * kWin * 2 + off);
+            }
+        }
         if constexpr (NEXT) {
             for (int i = tid; i < nr * (kWin / 4); i += kStepThreads)
                 reinterpret_cast<int4*>(s_ntile)[i] = make_int4(0, 0, 0, 0);
@@ -496,6 +621,170 @@ __global__ void __launch_bounds__(kStepThreads, 1)
                 if (word < v.W) mask[(size_t)(r0 + r) * v.W + word] = s_mtile[i];
             }
         }
+        if constexpr (!NEXT) {
+            if (fuse.logits) {
+                if (p_slot >= 0) {   // the previous tile's sparse fold, its loads landed
+                    fold_pending(fuse.part, p_slot, p_raw, p_t, lane);
+                    p_slot = -1;
+                }
+                // the masked decode of this tile: warp r folds row r of the window
+                // (the write-out above gave row r's words to warp r alone, so
+                // the warp may reuse that row of the tile as scratch)
+                const int full_words = v.V / 32;
+                for (int r = warp; r < nr; r += kStepThreads / 32) {
+                    const int j = w * 32 + lane;
+                    const uint32_t word = j < v.W ? s_mtile[r * 32 + lane] : 0u;
+                    const int c = __popc(word);
+                    const int n = __reduce_add_sync(0xffffffffu, c);
+                    const char* lrow = reinterpret_cast<const char*>(fuse.logits) + (size_t)(r0 + r) * fuse.stride * 2;
+                    const unsigned short* u = reinterpret_cast<const unsigned short*>(lrow);
+                    // exclusive offset of the lane's tokens in the row window's list
+                    // (lane order, then bit order)
+                    int o = 0;
+                    if (n <= 128) {
+                        o = c;
+#pragma unroll
+                        for (int d = 1; d < 32; d <<= 1) {
+                            const int y = __shfl_up_sync(0xffffffffu, o, d);
+                            if (lane >= d) o += y;
+                        }
+                        o -= c;
+                    }
+                    if (n <= 32) {
+                        // few allowed tokens: listed one per lane, the logit loaded
+                        // now and folded after the next tile's walk (fold_pending),
+                        // which hides the load's latency
+                        __syncwarp();
+                        uint32_t wd = word;
+                        int oo = o;
+                        while (wd) {
+                            const int e = __ffs(wd) - 1;
+                            wd &= wd - 1;
+                            s_mtile[r * 32 + oo++] = (uint32_t)(lane * 32 + e);
+                        }
+                        __syncwarp();
+                        p_t = INT_MAX;
+                        if (lane < n) {
+                            p_t = w * kWin + (int)s_mtile[r * 32 + lane];
+                            p_raw = __ldcs(u + p_t);
+                        }
+                        p_slot = (r0 + r) * v.n_windows + w;
+                    } else if (n <= 128) {
+                        // up to four tokens per lane: listed (16-bit entries, two
+                        // rounds of 64) and loaded together, then a lane-local
+                        // maximum, the warp's argmax and the warp's sum
+                        unsigned short* lst = reinterpret_cast<unsigned short*>(s_mtile + r * 32);
+                        int tk[4];
+                        unsigned short raw[4];
+                        uint32_t wd = word;
+                        int oo = o;
+#pragma unroll
+                        for (int h = 0; h < 2; ++h) {
+                            __syncwarp();
+                            while (wd && oo < 64 * (h + 1)) {
+                                const int e = __ffs(wd) - 1;
+                                wd &= wd - 1;
+                                lst[oo++ - 64 * h] = (unsigned short)(lane * 32 + e);
+                            }
+                            __syncwarp();
+#pragma unroll
+                            for (int q = 0; q < 2; ++q) {
+                                const int k = 64 * h + 32 * q + lane;
+                                tk[2 * h + q] = k < n ? w * kWin + (int)lst[k - 64 * h] : INT_MAX;
+                                raw[2 * h + q] = k < n ? __ldcs(u + tk[2 * h + q]) : (unsigned short)0;
+                            }
+                        }
+                        float m = -INFINITY;
+                        int idx = INT_MAX;
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {   // tokens ascend with q
+                            const float x = __uint_as_float((uint32_t)raw[q] << 16);
+                            if (tk[q] != INT_MAX && x > m) {
+                                m = x;
+                                idx = tk[q];
+                            }
+                        }
+#pragma unroll
+                        for (int off = 16; off > 0; off >>= 1) {
+                            const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+                            const int i2 = __shfl_xor_sync(0xffffffffu, idx, off);
+                            if (m2 > m || (m2 == m && i2 < idx)) {
+                                m = m2;
+                                idx = i2;
+                            }
+                        }
+                        const float mL = m * kLog2e;
+                        float sum = 0.0f;
+#pragma unroll
+                        for (int q = 0; q < 4; ++q)
+                            if (tk[q] != INT_MAX) sum += ex2(fmaf(__uint_as_float((uint32_t)raw[q] << 16), kLog2e, -mL));
+#pragma unroll
+                        for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+                        if (lane == 0)
+                            fuse.part[(size_t)(r0 + r) * v.n_windows + w] = make_float4(m, __int_as_float(idx), sum, 0.f);
+                    } else {
+                        float m = -INFINITY, mL = -INFINITY, sum = 0.0f;
+                        int idx = INT_MAX;
+                        uint32_t wd = word;
+                        const int t0 = j * 32;
+                        if (wd && j < full_words) {
+                            // many allowed tokens: each lane folds its own word, the
+                            // word's four 16-byte vectors loaded at once; compact
+                            // loops, since where masks are sparse this path runs
+                            // rarely and its code is fetched cold
+                            const uint4* src = reinterpret_cast<const uint4*>(lrow) + (size_t)j * 4;
+                            const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+                            const uint4 q0 = (wd & 0xFFu) ? __ldcs(src) : z;
+                            const uint4 q1 = (wd & 0xFF00u) ? __ldcs(src + 1) : z;
+                            const uint4 q2 = (wd & 0xFF0000u) ? __ldcs(src + 2) : z;
+                            const uint4 q3 = (wd & 0xFF000000u) ? __ldcs(src + 3) : z;
+                            // the word's maximum (lowest index on ties), then the sum of
+                            // its terms: no dependence chain through the exponentials
+                            int wi = 0;
+#pragma unroll 1
+                            for (int k = 0; k < 4; ++k) {
+                                const uint32_t bits = (wd >> (8 * k)) & 0xFFu;
+                                const uint4 q = k == 0 ? q0 : k == 1 ? q1 : k == 2 ? q2 : q3;
+                                const uint32_t qs[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+                                for (int e = 0; e < 8; ++e) {
+                                    const float x = (e & 1) ? bf16_hi(qs[e >> 1]) : bf16_lo(qs[e >> 1]);
+                                    if (((bits >> e) & 1u) && x > m) {
+                                        m = x;
+                                        wi = 8 * k + e;
+                                    }
+                                }
+                            }
+                            mL = m * kLog2e;
+                            idx = t0 + wi;
+#pragma unroll 1
+                            for (int k = 0; k < 4; ++k) {
+                                const uint32_t bits = (wd >> (8 * k)) & 0xFFu;
+                                const uint4 q = k == 0 ? q0 : k == 1 ? q1 : k == 2 ? q2 : q3;
+                                const uint32_t qs[4] = {q.x, q.y, q.z, q.w};
+                                float acc = 0.0f;
+#pragma unroll
+                                for (int e = 0; e < 8; ++e) {
+                                    const float x = (e & 1) ? bf16_hi(qs[e >> 1]) : bf16_lo(qs[e >> 1]);
+                                    acc += ((bits >> e) & 1u) ? ex2(fmaf(x, kLog2e, -mL)) : 0.0f;
+                                }
+                                sum += acc;
+                            }
+                        } else {   // the row's partial last word
+                            while (wd) {
+                                const int e = __ffs(wd) - 1;
+                                wd &= wd - 1;
+                                if (t0 + e < v.V)
+                                    acc_add(m, mL, idx, sum, __uint_as_float((uint32_t)__ldcs(u + t0 + e) << 16), t0 + e);
+                            }
+                        }
+                        warp_merge(m, idx, sum);
+                        if (lane == 0)
+                            fuse.part[(size_t)(r0 + r) * v.n_windows + w] = make_float4(m, __int_as_float(idx), sum, 0.f);
+                    }
+                }
+            }
+        }
         if constexpr (NEXT) {
             const int in_win = min(kWin, v.V - w * kWin);
             if (v.V % 4 == 0) {
@@ -514,81 +803,14 @@ __global__ void __launch_bounds__(kStepThreads, 1)
             }
         }
     }
+    if constexpr (!NEXT) {
+        if (p_slot >= 0) fold_pending(fuse.part, p_slot, p_raw, p_t, lane);
+    }
 }
 
 // ---------------------------------------------------------------------------
 // masked argmax / log-sum-exp
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ float ex2(float x) {
-    float y;
-    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-    return y;
-}
-
-// (m, idx, s) <- (m, idx, s) (+) (m2, i2, s2): larger max wins, lower index on
-// equal maxima; the other sum is rescaled to the winner's max.
-__device__ __forceinline__ void acc_merge(float& m, int& idx, float& s, float m2, int i2, float s2) {
-    if (m2 > m || (m2 == m && i2 < idx)) {
-        const float tm = m, ts = s;
-        const int ti = idx;
-        m = m2;
-        idx = i2;
-        s = s2;
-        m2 = tm;
-        i2 = ti;
-        s2 = ts;
-    }
-    if (s2 != 0.0f) s += s2 * ex2((m2 - m) * kLog2e);
-}
-
-// one allowed logit x at index t; mL = m * log2(e) is kept with m
-__device__ __forceinline__ void acc_add(float& m, float& mL, int& idx, float& s, float x, int t) {
-    if (x > m) {
-        const float xL = x * kLog2e;
-        s = s * ex2(mL - xL) + 1.0f;
-        m = x;
-        mL = xL;
-        idx = t;
-    } else {
-        s += ex2(fmaf(x, kLog2e, -mL));
-    }
-}
-
-__device__ __forceinline__ void warp_merge(float& m, int& idx, float& s) {
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-        const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
-        const int i2 = __shfl_xor_sync(0xffffffffu, idx, off);
-        const float s2 = __shfl_xor_sync(0xffffffffu, s, off);
-        acc_merge(m, idx, s, m2, i2, s2);
-    }
-}
-
-// CTA-wide (m, idx, s); the result is valid in thread 0.  Uses two barriers.
-__device__ __forceinline__ void block_merge(float& m, int& idx, float& s) {
-    __shared__ float sm_m[kLogitThreads / 32], sm_s[kLogitThreads / 32];
-    __shared__ int sm_i[kLogitThreads / 32];
-    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-    warp_merge(m, idx, s);
-    __syncthreads();   // protect sm_* against the previous call's readers
-    if (lane == 0) {
-        sm_m[wid] = m;
-        sm_i[wid] = idx;
-        sm_s[wid] = s;
-    }
-    __syncthreads();
-    if (wid == 0) {
-        m = lane < kLogitThreads / 32 ? sm_m[lane] : -INFINITY;
-        idx = lane < kLogitThreads / 32 ? sm_i[lane] : INT_MAX;
-        s = lane < kLogitThreads / 32 ? sm_s[lane] : 0.0f;
-        warp_merge(m, idx, s);
-    }
-}
-
-__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
-
-
 template <bool BF16>
 __device__ __forceinline__ float logit_at(const void* row, int t) {
     if constexpr (BF16) {
@@ -1296,7 +1518,7 @@ int rows_per_tile(const StepView& v, const LaunchEnv& env, int batch, bool next,
 template <bool STACK, int MODE, bool NEXT>
 cudaError_t launch_step_t(const StepView& v, const LaunchEnv& env, const int32_t* states, const uint64_t* stacks,
                           int32_t batch, bool row_is_state, uint32_t* mask, int32_t* next, const RowList& list,
-                          cudaStream_t st) {
+                          const FuseArgs& fuse, cudaStream_t st) {
     const int img_bytes = MODE == kDenseGlobal ? 0 : (int)table_smem_bytes(v, STACK, MODE);
     const int R = rows_per_tile(v, env, batch, NEXT, STACK, img_bytes);
     const StepLayout L = step_layout(v.K, R, NEXT, STACK, v.max_units, v.Q, img_bytes, v.self_mask != nullptr);
@@ -1328,31 +1550,32 @@ cudaError_t launch_step_t(const StepView& v, const LaunchEnv& env, const int32_t
         }
     }
     return launch_pdl(kern, dim3(grid), dim3(kStepThreads), (size_t)L.total, st, v, img, img_bytes, tgt_off, ret_off,
-                      states, stacks, batch, R, n_row_tiles, n_tiles, row_is_state ? 1 : 0, mask, next, list);
+                      states, stacks, batch, R, n_row_tiles, n_tiles, row_is_state ? 1 : 0, mask, next, list, fuse);
 }
 
 template <bool STACK, int MODE>
 cudaError_t launch_step_n(const StepView& v, const LaunchEnv& env, const int32_t* states, const uint64_t* stacks,
                           int32_t batch, bool row_is_state, uint32_t* mask, int32_t* next, const RowList& list,
-                          cudaStream_t st) {
+                          const FuseArgs& fuse, cudaStream_t st) {
     if (next)
-        return launch_step_t<STACK, MODE, true>(v, env, states, stacks, batch, row_is_state, mask, next, list, st);
-    return launch_step_t<STACK, MODE, false>(v, env, states, stacks, batch, row_is_state, mask, next, list, st);
+        return launch_step_t<STACK, MODE, true>(v, env, states, stacks, batch, row_is_state, mask, next, list, fuse,
+                                                st);
+    return launch_step_t<STACK, MODE, false>(v, env, states, stacks, batch, row_is_state, mask, next, list, fuse, st);
 }
 
 template <bool STACK>
 cudaError_t launch_step_s(const StepView& v, const LaunchEnv& env, int mode, const int32_t* states,
                           const uint64_t* stacks, int32_t batch, bool row_is_state, uint32_t* mask, int32_t* next,
-                          const RowList& list, cudaStream_t st) {
+                          const RowList& list, const FuseArgs& fuse, cudaStream_t st) {
     switch (mode) {
         case kDenseSmem:
-            return launch_step_n<STACK, kDenseSmem>(v, env, states, stacks, batch, row_is_state, mask, next, list, st);
+            return launch_step_n<STACK, kDenseSmem>(v, env, states, stacks, batch, row_is_state, mask, next, list, fuse, st);
         case kSparse32Smem:
-            return launch_step_n<STACK, kSparse32Smem>(v, env, states, stacks, batch, row_is_state, mask, next, list, st);
+            return launch_step_n<STACK, kSparse32Smem>(v, env, states, stacks, batch, row_is_state, mask, next, list, fuse, st);
         case kSparse64Smem:
-            return launch_step_n<STACK, kSparse64Smem>(v, env, states, stacks, batch, row_is_state, mask, next, list, st);
+            return launch_step_n<STACK, kSparse64Smem>(v, env, states, stacks, batch, row_is_state, mask, next, list, fuse, st);
         default:
-            return launch_step_n<STACK, kDenseGlobal>(v, env, states, stacks, batch, row_is_state, mask, next, list, st);
+            return launch_step_n<STACK, kDenseGlobal>(v, env, states, stacks, batch, row_is_state, mask, next, list, fuse, st);
     }
 }
 
@@ -1454,10 +1677,63 @@ int step_fixed_smem_bytes(const StepView& v, bool next) {
 
 cudaError_t launch_step_mask(const StepView& v, const LaunchEnv& env, bool stack, int mode, const int32_t* states,
                              const uint64_t* stacks, int32_t batch, bool row_is_state, uint32_t* mask,
-                             int32_t* next, cudaStream_t st, const int32_t* row_ids, const int32_t* row_count) {
+                             int32_t* next, cudaStream_t st, const int32_t* row_ids, const int32_t* row_count,
+                             const void* fuse_logits, int64_t fuse_stride, float4* fuse_part, bool fuse_prefetch) {
     const RowList list{row_ids, row_count, 0};
-    if (stack) return launch_step_s<true>(v, env, mode, states, stacks, batch, row_is_state, mask, next, list, st);
-    return launch_step_s<false>(v, env, mode, states, stacks, batch, row_is_state, mask, next, list, st);
+    const FuseArgs fuse{fuse_logits, fuse_stride, fuse_part, fuse_logits && fuse_prefetch ? 1 : 0};
+    if (stack)
+        return launch_step_s<true>(v, env, mode, states, stacks, batch, row_is_state, mask, next, list, fuse, st);
+    return launch_step_s<false>(v, env, mode, states, stacks, batch, row_is_state, mask, next, list, fuse, st);
+}
+
+// Merges each row's per-window partials of the fused step: one warp per row.
+__global__ void __launch_bounds__(kLogitThreads)
+    fused_combine_kernel(const float4* __restrict__ part, int32_t batch, int32_t n_windows,
+                         int32_t* __restrict__ argmax, float* __restrict__ lse) {
+    pdl_wait();
+    pdl_trigger();
+    const int r = blockIdx.x * (kLogitThreads / 32) + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+    if (r >= batch) return;
+    float m = -INFINITY, s = 0.0f;
+    int idx = INT_MAX;
+    for (int k = lane; k < n_windows; k += 32) {
+        const float4 p = __ldcg(part + (size_t)r * n_windows + k);
+        acc_merge(m, idx, s, p.x, __float_as_int(p.y), p.z);
+    }
+    warp_merge(m, idx, s);
+    if (lane == 0) {
+        argmax[r] = m == -INFINITY ? -1 : idx;
+        if (lse) lse[r] = m == -INFINITY ? -INFINITY : m + logf(s);
+    }
+}
+
+cudaError_t launch_fused_combine(const float4* part, int32_t batch, int32_t n_windows, int32_t* argmax, float* lse,
+                                 cudaStream_t st) {
+    const unsigned grid = (unsigned)((batch + kLogitThreads / 32 - 1) / (kLogitThreads / 32));
+    return launch_pdl(fused_combine_kernel, dim3(grid), dim3(kLogitThreads), 0, st, part, batch, n_windows, argmax, lse);
+}
+
+cudaError_t launch_logprobs_bf16(const LaunchEnv& env, const void* logits, int32_t batch, int64_t row_stride,
+                                 int32_t V, const uint32_t* mask, const float* lse, float* logprobs, cudaStream_t st) {
+    const int W = (V + 31) / 32;
+    const bool out_vec = (reinterpret_cast<uintptr_t>(logprobs) % 16 == 0) && (V % 4 == 0);
+    for (int32_t r0 = 0; r0 < batch; r0 += kMaxLogitRows) {
+        const int rows = min(kMaxLogitRows, batch - r0);
+        const void* lg = reinterpret_cast<const char*>(logits) + (size_t)r0 * row_stride * 2;
+        const MaskRows mk{mask + (size_t)r0 * W, nullptr, 0, nullptr};
+        const long long n_items = out_vec ? (long long)rows * (V % 16 == 0 ? V / 16 : V / 4) : (long long)rows * W;
+        int g = env.num_sms * occupancy((const void*)logprobs_kernel<true, true>, kLogitThreads);
+        g = (int)std::max<long long>(1, std::min<long long>((long long)g, (n_items + kLogitThreads - 1) / kLogitThreads));
+        float* lp = logprobs + (size_t)r0 * V;
+        const int wide = (reinterpret_cast<uintptr_t>(lg) % 32 == 0) && ((size_t)row_stride * 2) % 32 == 0 &&
+                         (reinterpret_cast<uintptr_t>(lp) % 32 == 0) && V % 16 == 0;
+        cudaError_t e = out_vec ? launch_pdl(logprobs_kernel<true, true>, dim3(g), dim3(kLogitThreads), 0, st, lg,
+                                             row_stride, mk, V, W, rows, lse + r0, lp, wide)
+                                : launch_pdl(logprobs_kernel<true, false>, dim3(g), dim3(kLogitThreads), 0, st, lg,
+                                             row_stride, mk, V, W, rows, lse + r0, lp, 0);
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
 cudaError_t launch_mask_logits(const LaunchEnv& env, const void* logits, int dtype, int32_t batch,

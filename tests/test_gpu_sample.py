@@ -85,7 +85,8 @@ def test_sample_ragged_and_unaligned(V, stride, dtype):
     m = packed(bits)
     want = oracle.mask_sample(x, m, 0.9, 99, 3, n_tokens=V)
     tok = torch.empty(B_, dtype=torch.int32, device="cuda")
-    B.domino_mask_sample(d.h, logits_tensor(x).data_ptr(), B.DTYPE_BF16 if dtype == "bf16" else B.DTYPE_F32, B_,
+    lg = logits_tensor(x)   # held across the call: nothing else may reuse its memory
+    B.domino_mask_sample(d.h, lg.data_ptr(), B.DTYPE_BF16 if dtype == "bf16" else B.DTYPE_F32, B_,
                          stride, dev(m.view(np.int32)), 0.9, 99, 3, tok)
     got = tok.cpu().numpy()
     assert (got == want).all() and got[0] == -1
