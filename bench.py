@@ -719,7 +719,7 @@ def run_domino(args, dist: Dist):
                                            sp)
             if rc:
                 raise RuntimeError(f"decode_step_host failed ({rc})")
-        for i in range(3):
+        for i in range(8):   # warm-up: the handle times its two host paths on its first calls
             e2e_step(i)
         dist.barrier()
         torch.cuda.synchronize()
@@ -791,8 +791,8 @@ def run_domino(args, dist: Dist):
         "opportunistic": opportunistic, "speculation": spec,
         "e2e": {"value": n * Bsz * V * Ke / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "steps": Ke, "api": "domino_decode_step_host with pinned host buffers",
-                "h2d_note": "h2d_bytes_per_step counts the whole logits tensor; the masked pass reads pinned logits "
-                            "in place, so only the 16-byte vectors holding an allowed token cross the link"},
+                "h2d_note": "h2d_bytes_per_step counts the whole logits tensor; on the in-place path only the "
+                            "allowed logits cross the link (the handle times both paths and uses the faster)"},
         "gpu_launches": K * launches_per_step,
         "gpu_launches_note": "timed region only; per-kernel graphs and e2e are timed separately",
         "clocks": sampler.summary(),

@@ -297,14 +297,18 @@ int domino_advance_table(domino_t h, const int32_t* table_next_dev, const int32_
 
 /* One whole decode step from HOST memory (end-to-end use): logits (batch
  * rows of V values, dense) and the configurations come from host memory,
- * step_mask -> mask_logits -> advance run on the device, and tokens_host[b]
- * (the argmax), lse_host (may be NULL) and the new configurations are
- * written back into states_host / stacks_host (stacks_host may be NULL for a
- * DFA); `stream` is synchronised before the call returns.
- *   Pinned (page-locked) logits are read in place by the masked pass: only
- *   the 16-byte vectors that hold an allowed token cross the host link.
- *   Pageable logits are copied in chunks of rows on a copy stream owned by
- *   the handle, overlapped with the mask step and each chunk's decode.
+ * the mask step, the greedy decode and advance run on the device, and
+ * tokens_host[b] (the argmax), lse_host (may be NULL) and the new
+ * configurations are written back into states_host / stacks_host
+ * (stacks_host may be NULL for a DFA); `stream` is synchronised before the
+ * call returns.
+ *   Logits are either copied in chunks of rows on a copy stream owned by the
+ *   handle, overlapped with the mask step and each chunk's decode, or, when
+ *   they are pinned (page-locked) bf16, possibly read in place by the mask
+ *   step itself (domino_step_decode), so that only allowed logits cross the
+ *   host link, during the walk.  For pinned bf16 logits the handle times both
+ *   paths on its own calls and takes the faster, retiming the other every
+ *   64th call; pageable or fp32 logits are always copied.
  * Device staging buffers are owned by the handle and grown on demand. */
 int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, int32_t batch,
                             int32_t* states_host, uint64_t* stacks_host, int32_t* tokens_host, float* lse_host,

@@ -162,8 +162,5 @@ cudaError_t launch_spec_accept(const int32_t* proposals, const int32_t* n_prop, 
                                int32_t* n_accept, int32_t* tokens_out, int32_t* states_out, uint64_t* stacks_out,
                                cudaStream_t st);
 
-// Adds the number of non-zero mask bytes of n_words words to *count.
-cudaError_t launch_mask_vector_count(const LaunchEnv& env, const uint32_t* mask, long long n_words,
-                                     unsigned long long* count, cudaStream_t st);
 
 }  // namespace domino

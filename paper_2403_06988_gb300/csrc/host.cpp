@@ -4,6 +4,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <chrono>
 #include <cmath>
 #include <cstdint>
 #include <cstring>
@@ -70,10 +71,10 @@ struct domino_ctx {
     cudaStream_t cp_stream = nullptr;
     cudaEvent_t ev_cfg = nullptr;
     cudaEvent_t ev_chunk[8] = {};
-    double vec_density = 0.0;       // share of logit vectors the last step's masks allowed
-    cudaEvent_t ev_t[4] = {};       // timing: mask step (0, 1) and logits copy (2, 3)
-    double t_step_ms = 0.0;         // last mask-step time
-    double link_gbs = 0.0;          // host link rate seen by the last chunked copy (0: none yet)
+    cudaEvent_t ev_t[4] = {};       // the chunked copy's start and end (2, 3)
+    // host wall time of the last settled call of each path for pinned bf16
+    // logits: [0] the chunked copy, [1] the in-place read (0: not yet seen)
+    double t_wall_ms[2] = {0.0, 0.0};
     // Recorded host-buffer steps: a call whose buffers, sizes and path match an
     // earlier one replays that call's CUDA graph instead of issuing each copy
     // and launch again.  Cleared when an automaton or vocabulary is loaded.
@@ -144,6 +145,7 @@ bool is_host_only(const domino_ctx* h) { return h->device < 0; }
 void clear_host_graphs(domino_ctx* h) {
     for (auto& g : h->host_graphs) cudaGraphExecDestroy(g.exec);
     h->host_graphs.clear();
+    h->t_wall_ms[0] = h->t_wall_ms[1] = 0.0;   // the paths are timed afresh
 }
 
 // Byte-class strings of every token, the window sort and the slot arrays.
@@ -909,13 +911,12 @@ namespace {
 // stacks], each part on a 16-byte boundary.  States and stacks go up in one
 // copy, everything comes back in one.
 struct IoLayout {
-    size_t cnt, tok, lse, st, sk, in_end;
+    size_t tok, lse, st, sk, in_end;
 };
 IoLayout io_layout(int32_t batch, bool stacks) {
     auto a16 = [](size_t x) { return (x + 15) / 16 * 16; };
     IoLayout L{};
-    L.cnt = 0;
-    L.tok = 16;
+    L.tok = 0;
     L.lse = a16(L.tok + (size_t)batch * 4);
     L.st = a16(L.lse + (size_t)batch * 4);
     L.sk = a16(L.st + (size_t)batch * 4);
@@ -956,10 +957,8 @@ int copy_and_decode_chunks(domino_ctx* h, const void* logits_host, int32_t dtype
     }
     if (e == cudaSuccess) e = cudaEventRecord(h->ev_t[3], h->cp_stream);
     if (e == cudaSuccess) e = cudaStreamWaitEvent(st, h->ev_cfg, 0);
-    if (e == cudaSuccess) e = cudaEventRecord(h->ev_t[0], st);
     if (e != cudaSuccess) return cuda_status(e);
     if ((rc = domino_step_mask(h, d_states, d_stacks, batch, d_mask, nullptr, stream))) return rc;
-    if ((e = cudaEventRecord(h->ev_t[1], st)) != cudaSuccess) return cuda_status(e);
     for (int k = 0; k < n_chunks; ++k) {
         const int32_t r0 = r0s[(size_t)k], rows = r0s[(size_t)k + 1] - r0;
         if ((e = cudaStreamWaitEvent(st, h->ev_chunk[k], 0)) != cudaSuccess) return cuda_status(e);
@@ -985,26 +984,18 @@ int enqueue_host_step(domino_ctx* h, const void* logits_host, void* logits_mappe
     uint32_t* d_mask = (uint32_t*)h->s_mask.p;
     int32_t* d_tok = (int32_t*)(io + L.tok);
     float* d_lse = (float*)(io + L.lse);
-    if (mapped) {
+    if (mapped) {   // the mask step folds the pinned logits it allows, read in place
         cudaError_t e =
             cudaMemcpyAsync(io + L.st, (char*)h->h_io + L.st, L.in_end - L.st, cudaMemcpyHostToDevice, st);
-        if (e == cudaSuccess) e = cudaEventRecord(h->ev_t[0], st);
         if (e != cudaSuccess) return cuda_status(e);
-        if ((rc = domino_step_mask(h, d_states, d_stacks, batch, d_mask, nullptr, stream))) return rc;
-        if ((e = cudaEventRecord(h->ev_t[1], st)) != cudaSuccess) return cuda_status(e);
-        if ((e = cudaEventRecord(h->ev_t[2], st)) != cudaSuccess) return cuda_status(e);
-        if ((rc = domino_mask_logits(h, logits_mapped, dtype, batch, h->V, d_mask, d_tok, d_lse, nullptr, stream)))
+        if ((rc = domino_step_decode(h, d_states, d_stacks, batch, logits_mapped, dtype, h->V, d_mask, d_tok, d_lse,
+                                     nullptr, stream)))
             return rc;
-        if ((e = cudaEventRecord(h->ev_t[3], st)) != cudaSuccess) return cuda_status(e);
     } else {
         if ((rc = copy_and_decode_chunks(h, logits_host, dtype, batch, stacks, L, st))) return rc;
     }
     if ((rc = domino_advance(h, d_states, d_stacks, d_tok, batch, d_states, d_stacks, stream))) return rc;
-    cudaError_t e = cudaMemsetAsync(io + L.cnt, 0, sizeof(uint64_t), st);
-    if (e == cudaSuccess)
-        e = launch_mask_vector_count(h->env, d_mask, (long long)batch * h->W, (unsigned long long*)(io + L.cnt), st);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(h->h_io, io, L.in_end, cudaMemcpyDeviceToHost, st);
-    return cuda_status(e);
+    return cuda_status(cudaMemcpyAsync(h->h_io, io, L.in_end, cudaMemcpyDeviceToHost, st));
 }
 
 }  // namespace
@@ -1025,21 +1016,25 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
     const size_t logit_bytes = (size_t)batch * row_bytes;
     const bool stacks = stacks_host != nullptr;
     const IoLayout L = io_layout(batch, stacks);
-    // Pinned (page-locked, mapped) logits are read where they are: the masked
-    // pass pulls only the 16-byte logit vectors that hold an allowed token
-    // across the host link, so masked-out logits never travel, but it starts
-    // after the mask step.  The chunked copy moves every byte while the mask
-    // step runs.  The choice compares the two with the last step's mask
-    // density, mask-step time and link rate:
-    //   in place: t_step + density * bytes / rate;  copy: max(bytes / rate, t_step).
+    // Pinned (page-locked, mapped) bf16 logits can be read where they are: the
+    // mask step folds each tile's allowed logits, so only those cross the host
+    // link, while the walk runs.  Or they are copied in chunks while the mask
+    // step runs and decoded as they land.  Which is faster depends on the
+    // masks' density and on the link's read granularity, so it is measured:
+    // each path's host wall time is taken on settled calls (no buffer growth,
+    // no recording), the faster one is used, and every 64th call takes the
+    // other to keep its time current.
+    const auto t_enter = std::chrono::steady_clock::now();
     cudaPointerAttributes pa{};
     const bool pinned = cudaPointerGetAttributes(&pa, logits_host) == cudaSuccess && pa.type == cudaMemoryTypeHost &&
                         pa.devicePointer != nullptr;
     if (!pinned) cudaGetLastError();
     bool mapped = pinned && dtype == DOMINO_DTYPE_BF16;
-    if (mapped && h->link_gbs > 0.0) {
-        const double t_copy = (double)logit_bytes / (h->link_gbs * 1e6);   // ms
-        mapped = h->t_step_ms + h->vec_density * t_copy < std::max(t_copy, h->t_step_ms);
+    const bool choice = mapped;
+    if (choice) {
+        if (h->t_wall_ms[1] == 0.0) mapped = true;
+        else if (h->t_wall_ms[0] == 0.0) mapped = false;
+        else mapped = (h->t_wall_ms[1] <= h->t_wall_ms[0]) != (h->host_calls % 64 == 63);
     }
     const bool grow = (!mapped && h->s_logits.n < logit_bytes) || h->s_io.n < L.in_end ||
                       h->s_mask.n < (size_t)batch * (size_t)h->W * 4 || h->h_io_n < L.in_end || !h->cp_stream;
@@ -1072,11 +1067,10 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
     }
     std::memcpy((char*)h->h_io + L.st, states_host, (size_t)batch * 4);
     if (stacks) std::memcpy((char*)h->h_io + L.sk, stacks_host, (size_t)batch * 8);
-    // The step's copies and launches, recorded once per set of buffers on a
-    // non-default stream (the default stream cannot be captured) and replayed
-    // afterwards.  The first two calls of a handle run them directly: the
-    // first sets kernel attributes, the second times the mask step and the
-    // link for the path choice warm (replays update the mask density only).
+    // The step's copies and launches, recorded once per set of buffers and
+    // path on a non-default stream (the default stream cannot be captured) and
+    // replayed afterwards.  The first two calls of a handle run them directly
+    // (the first sets kernel attributes).
     const void* key[16] = {logits_host, (const void*)(intptr_t)batch,
                            (const void*)(intptr_t)(dtype * 4 + (mapped ? 1 : 0) + (stacks ? 2 : 0)), h->s_logits.p,
                            h->s_mask.p, h->s_io.p, h->h_io, (const void*)st, nullptr, nullptr, nullptr, nullptr,
@@ -1088,7 +1082,8 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
             hg.used = h->host_calls;
         }
     cudaError_t e = cudaSuccess;
-    if (!exec && st != nullptr && h->host_calls > 1) {
+    const bool record = !exec && st != nullptr && h->host_calls > 1;
+    if (record) {
         cudaGraph_t gr = nullptr;
         e = cudaStreamBeginCapture(st, cudaStreamCaptureModeRelaxed);
         if (e != cudaSuccess) return cuda_status(e);
@@ -1128,17 +1123,9 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
     if (lse_host) std::memcpy(lse_host, io + L.lse, (size_t)batch * 4);
     std::memcpy(states_host, io + L.st, (size_t)batch * 4);
     if (stacks) std::memcpy(stacks_host, io + L.sk, (size_t)batch * 8);
-    uint64_t count = 0;
-    std::memcpy(&count, io + L.cnt, sizeof(count));
-    h->vec_density = (double)count / ((double)batch * h->W * 4.0);
-    float ms = 0.f;
-    if (cudaEventElapsedTime(&ms, h->ev_t[0], h->ev_t[1]) == cudaSuccess) h->t_step_ms = ms;
-    // the link rate: bytes copied over the copy time, or the vectors read in
-    // place over the in-place pass's time (that pass is bound by the link)
-    const double moved = mapped ? h->vec_density * (double)logit_bytes : (double)logit_bytes;
-    if (moved > (double)(1 << 20) && cudaEventElapsedTime(&ms, h->ev_t[2], h->ev_t[3]) == cudaSuccess && ms > 0.f)
-        h->link_gbs = moved / ((double)ms * 1e6);
-    cudaGetLastError();
+    if (choice && !grow && !record && h->host_calls > 1)
+        h->t_wall_ms[mapped ? 1 : 0] =
+            std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t_enter).count();
     return DOMINO_OK;
 }
 

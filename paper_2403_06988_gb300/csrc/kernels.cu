@@ -1440,24 +1440,6 @@ __global__ void __launch_bounds__(kAdvanceThreads)
     if (stacks_out && chain_stacks) stacks_out[b] = chain_stacks[(size_t)b * (s + 1) + k];
 }
 
-// Number of mask bytes that are not zero, i.e. of 16-byte bf16 logit vectors
-// holding an allowed token (the host-buffer step uses it to choose between
-// reading pinned logits in place and copying them).
-__global__ void __launch_bounds__(kLogitThreads)
-    mask_vector_count_kernel(const uint32_t* __restrict__ mask, long long n_words,
-                             unsigned long long* __restrict__ count) {
-    pdl_wait();
-    pdl_trigger();
-    unsigned int c = 0;
-    for (long long i = (long long)blockIdx.x * kLogitThreads + threadIdx.x; i < n_words;
-         i += (long long)gridDim.x * kLogitThreads) {
-        const uint32_t w = __ldg(mask + i);
-        c += ((w & 0xFFu) != 0u) + ((w & 0xFF00u) != 0u) + ((w & 0xFF0000u) != 0u) + ((w & 0xFF000000u) != 0u);
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) c += __shfl_xor_sync(0xffffffffu, c, off);
-    if ((threadIdx.x & 31) == 0 && c) atomicAdd(count, (unsigned long long)c);
-}
 
 // Alg. 1 update from the precomputed state x token table: one read of
 // next[s][t] per sequence (EOS or -1: the start state; a rejected token's
@@ -1803,12 +1785,6 @@ cudaError_t launch_advance_table(const int32_t* table_next, int32_t Q, int32_t V
                       states, tokens, batch, states_out, err);
 }
 
-cudaError_t launch_mask_vector_count(const LaunchEnv& env, const uint32_t* mask, long long n_words,
-                                     unsigned long long* count, cudaStream_t st) {
-    const long long want = (n_words + kLogitThreads - 1) / kLogitThreads;
-    const unsigned grid = (unsigned)std::max<long long>(1, std::min<long long>(want, 4LL * env.num_sms));
-    return launch_pdl(mask_vector_count_kernel, dim3(grid), dim3(kLogitThreads), 0, st, mask, n_words, count);
-}
 
 cudaError_t launch_propose_check(const StepView& v, bool stack, int mode, const int32_t* states,
                                  const uint64_t* stacks, const int32_t* proposals, int32_t batch, int32_t* tokens_out,

@@ -353,6 +353,37 @@ def test_decode_step_host_replayed_steps_match_oracle(config):
     d.close()
 
 
+def test_decode_step_host_path_choice_keeps_results():
+    """Pinned bf16 logits: the handle times the in-place and the copy path on
+    its own calls, uses the faster and retimes the other every 64th call; 70
+    replayed steps cover both paths and the switch, every step equal to the
+    oracle."""
+    import oracle
+    w = workload(2)
+    d = Domino.from_parts(w.automaton, w.vocab, device=0)
+    P = problem(2)
+    states, _ = w.initial_configs()
+    s_host = torch.from_numpy(states.copy()).pin_memory()
+    tok = torch.empty(len(states), dtype=torch.int32).pin_memory()
+    lse_h = torch.empty(len(states), dtype=torch.float32).pin_memory()
+    bufs = [torch.from_numpy(w.logits(60 + i).view(np.int16)).pin_memory() for i in range(2)]
+    s_o = states.copy()
+    st = torch.cuda.Stream()
+    for i in range(70):
+        b = bufs[i % 2]
+        B.domino_decode_step_host(d.h, b.data_ptr(), B.DTYPE_BF16, len(states), s_host.data_ptr(), None,
+                                  tok.data_ptr(), lse_h.data_ptr(), stream=st.cuda_stream)
+        m, _, _ = P.step_mask(s_o, None, n_threads=NT)
+        a_o, l_o, _ = oracle.mask_logits(b.numpy().view(np.uint16), m)
+        s_o, _, _ = P.advance(s_o, None, a_o, w.automaton.start)
+        assert (tok.numpy() == a_o).all(), i
+        fin = np.isfinite(l_o)
+        assert np.abs(lse_h.numpy()[fin] - l_o[fin]).max(initial=0) < TOL, i
+        assert (s_host.numpy() == s_o).all(), i
+    assert d.device_error() == 0
+    d.close()
+
+
 def test_decode_step_host_matches_device_path():
     w = workload(2)
     states, _ = configs(2)
