@@ -1,8 +1,9 @@
 #!/usr/bin/env python
 """Masked decode-step throughput of the DOMINO hot path on GB300.
 
-One step = C.mask() with v' = m (.) v and the greedy decode folded into it
-(step_decode) -> C.update() (advance) over one batch (Alg. 1).  Default workload: random
+One step = one domino_step_decode call over one batch (Alg. 1): C.mask() with
+v' = m (.) v and the greedy decode folded into it, then C.update() in the same
+call's per-row merge.  Default workload: random
 sparse DFA (Q = 5000, 32 byte classes), V = 128256, batch 256, bf16 logits
 N(0, 3), rotating over enough logits buffers to exceed twice the L2.
 
@@ -477,14 +478,15 @@ def run_domino(args, dist: Dist):
     p_mask, p_arg, p_lse = mask.data_ptr(), argmax.data_ptr(), lse.data_ptr()
     p_lp = logprobs.data_ptr() if logprobs is not None else None
     p_logits = [t.data_ptr() for t in logits]
-    # one step = the mask step with the greedy decode folded in (plus the
-    # log-probs pass where the workload asks for them), then the update
-    launches_per_step = 3 + (1 if w.want_logprobs else 0)
+    # one step = one call: the mask step with the greedy decode folded in, the
+    # per-row merge that also advances each row (plus the log-probs pass where
+    # the workload asks for them); fp32 logits run the separate kernels
+    fused = w.logits_dtype == "bf16"
+    launches_per_step = (2 if fused else 3) + (1 if w.want_logprobs else 0)
 
     def step(i, stream_ptr):
         rc = L.domino_step_decode(h, p_states, p_stacks, Bsz, p_logits[i % nbuf], dtype_code, V, p_mask, p_arg, p_lse,
-                                  p_lp, stream_ptr)
-        rc |= L.domino_advance(h, p_states, p_stacks, p_arg, Bsz, p_states, p_stacks, stream_ptr)
+                                  p_lp, p_states, p_stacks, stream_ptr)
         if rc:
             raise RuntimeError(f"domino call failed ({rc})")
 
@@ -558,7 +560,7 @@ def run_domino(args, dist: Dist):
 
     def k_fused(i, sp):
         if L.domino_step_decode(h, p_states, p_stacks, Bsz, p_logits[i % nbuf], dtype_code, V, p_mask, p_arg, p_lse,
-                                p_lp, sp):
+                                p_lp, None, None, sp):
             raise RuntimeError("step_decode failed")
 
     def k_adv(i, sp):

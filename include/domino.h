@@ -181,24 +181,30 @@ int domino_mask_logits(domino_t h, const void* logits_dev, int32_t dtype, int32_
 int domino_advance(domino_t h, const int32_t* states_dev, const uint64_t* stacks_dev, const int32_t* tokens_dev,
                    int32_t batch, int32_t* states_out, uint64_t* stacks_out, void* stream);
 
-/* C.mask() and the greedy decode of Alg. 1 in one pass: domino_step_mask's
- * mask (written to mask_dev as there) and domino_mask_logits' argmax, lse and
- * log-probs, with the masked logits folded by the mask step itself, tile by
- * tile, as soon as a tile's bits are known (then a small per-row merge; the
- * log-probs, when asked for, take one more pass over the logits).
+/* One step of Alg. 1 on the device: C.mask(), the greedy decode and, when
+ * states_out is given, C.update(o).  domino_step_mask's mask (written to
+ * mask_dev as there), domino_mask_logits' argmax, lse and log-probs, with the
+ * masked logits folded by the mask step itself, tile by tile, as soon as a
+ * tile's bits are known (then a small per-row merge, which also advances each
+ * row by its argmax as domino_advance does; the log-probs, when asked for,
+ * take one more pass over the logits).
  *   states_dev, stacks_dev, batch: as domino_step_mask;
  *   logits_dev, dtype, row_stride_elems: as domino_mask_logits; may point to
  *   device memory or to pinned host memory;
  *   mask_dev uint32 [batch][W] (required); argmax_dev int32 [batch]
  *   (required); lse_dev float [batch] or NULL; logprobs_dev float [batch][V]
- *   or NULL (requires lse_dev).
+ *   or NULL (requires lse_dev);
+ *   states_out int32 [batch] or NULL (no update), stacks_out uint64 [batch]
+ *   (required with states_out when stacks_dev is given): the configurations
+ *   after the decoded token; they may alias states_dev / stacks_dev.
  * The fused form needs bf16 rows on 16-byte boundaries; other inputs run the
  * two kernels one after the other.  Results equal domino_step_mask followed
  * by domino_mask_logits.  The first call with a larger batch allocates
  * scratch and synchronises `stream`. */
 int domino_step_decode(domino_t h, const int32_t* states_dev, const uint64_t* stacks_dev, int32_t batch,
                        const void* logits_dev, int32_t dtype, int64_t row_stride_elems, uint32_t* mask_dev,
-                       int32_t* argmax_dev, float* lse_dev, float* logprobs_dev, void* stream);
+                       int32_t* argmax_dev, float* lse_dev, float* logprobs_dev, int32_t* states_out,
+                       uint64_t* stacks_out, void* stream);
 
 /* Alg. 1 with the greedy decode replaced by sampling: tokens_dev[b] is a draw
  * from softmax(logits / temperature) restricted to the allowed tokens of

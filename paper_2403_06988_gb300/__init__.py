@@ -65,8 +65,10 @@ class Domino:
         B.domino_step_mask(self.h, states, stacks, b, mask, nxt, stream)
         return mask, nxt
 
-    def step_decode(self, states, stacks, logits, want_logprobs: bool = False, out_mask=None, stream=None):
-        """Mask step fused with the masked greedy decode: returns (mask, argmax, lse, logprobs or None)."""
+    def step_decode(self, states, stacks, logits, want_logprobs: bool = False, advance: bool = False, out_mask=None,
+                    stream=None):
+        """Mask step fused with the masked greedy decode: returns (mask, argmax, lse, logprobs or None).
+        advance: states (and stacks) are then updated in place by the decoded tokens."""
         import torch
         b = states.shape[0]
         dtype = DTYPE_BF16 if logits.dtype == torch.bfloat16 else DTYPE_F32
@@ -81,7 +83,7 @@ class Domino:
         lp = torch.empty((b, self.info()["n_tokens"]), dtype=torch.float32, device=states.device) if want_logprobs \
             else None
         B.domino_step_decode(self.h, states, stacks, b, logits.data_ptr(), dtype, logits.stride(0), mask, argmax, lse,
-                             lp, stream)
+                             lp, states if advance else None, stacks if advance else None, stream)
         return mask, argmax, lse, lp
 
     def precompute_table(self, want_next: bool = True, want_mask: bool = True, stream=None):

@@ -73,7 +73,7 @@ _SIGS = {
     "domino_spec_update": [P, P, P, P, P, P, P, I32, P],
     "domino_spec_propose": [P, P, P, P, P, I32, I32, I32, P, P, P, P, P],
     "domino_spec_accept": [P, P, P, P, P, P, I32, I32, P, P, P, P, P],
-    "domino_step_decode": [P, P, P, I32, P, I32, I64, P, P, P, P, P],
+    "domino_step_decode": [P, P, P, I32, P, I32, I64, P, P, P, P, P, P, P],
 }
 
 
@@ -213,10 +213,12 @@ def domino_advance(h: int, states_dev, stacks_dev, tokens_dev, batch: int, state
 
 
 def domino_step_decode(h: int, states_dev, stacks_dev, batch: int, logits_dev, dtype: int, row_stride_elems: int,
-                       mask_dev, argmax_dev, lse_dev=None, logprobs_dev=None, stream=None) -> None:
+                       mask_dev, argmax_dev, lse_dev=None, logprobs_dev=None, states_out=None, stacks_out=None,
+                       stream=None) -> None:
     _check("domino_step_decode", lib().domino_step_decode(
         h, _ptr(states_dev), _ptr(stacks_dev), int(batch), _ptr(logits_dev), int(dtype), int(row_stride_elems),
-        _ptr(mask_dev), _ptr(argmax_dev), _ptr(lse_dev), _ptr(logprobs_dev), _stream(stream)))
+        _ptr(mask_dev), _ptr(argmax_dev), _ptr(lse_dev), _ptr(logprobs_dev), _ptr(states_out), _ptr(stacks_out),
+        _stream(stream)))
 
 
 def domino_mask_sample(h: int, logits_dev, dtype: int, batch: int, row_stride_elems: int, mask_dev,

@@ -98,9 +98,11 @@ cudaError_t launch_step_mask(const StepView& v, const LaunchEnv& env, bool stack
 
 // The mask step fused with the masked decode (bf16 logits, rows on 16-byte
 // boundaries): fuse_part [batch][n_windows] receives per-window partials,
-// merged into argmax / lse by launch_fused_combine.
-cudaError_t launch_fused_combine(const float4* part, int32_t batch, int32_t n_windows, int32_t* argmax, float* lse,
-                                 cudaStream_t st);
+// merged into argmax / lse by launch_fused_combine, which also advances each
+// row by its argmax when states_out is given (outputs may alias the inputs).
+cudaError_t launch_fused_combine(const StepView& v, bool stack, int mode, const float4* part, int32_t batch,
+                                 int32_t n_windows, int32_t* argmax, float* lse, const int32_t* states,
+                                 const uint64_t* stacks, int32_t* states_out, uint64_t* stacks_out, cudaStream_t st);
 
 // Log-probabilities only (bf16 logits, rows on 16-byte boundaries), given the
 // rows' lse: logprobs[b][t] = logit - lse[b] for allowed t, -inf else.

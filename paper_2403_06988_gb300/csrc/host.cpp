@@ -724,23 +724,29 @@ int domino_advance(domino_t h, const int32_t* states_dev, const uint64_t* stacks
 
 int domino_step_decode(domino_t h, const int32_t* states_dev, const uint64_t* stacks_dev, int32_t batch,
                        const void* logits_dev, int32_t dtype, int64_t row_stride_elems, uint32_t* mask_dev,
-                       int32_t* argmax_dev, float* lse_dev, float* logprobs_dev, void* stream) {
+                       int32_t* argmax_dev, float* lse_dev, float* logprobs_dev, int32_t* states_out,
+                       uint64_t* stacks_out, void* stream) {
     int rc = ready_for_compute(h);
     if (rc) return rc;
     if (dtype != DOMINO_DTYPE_F32 && dtype != DOMINO_DTYPE_BF16) return DOMINO_E_INVALID_ARG;
     if (batch < 0 || row_stride_elems < h->V) return DOMINO_E_INVALID_ARG;
     if (batch == 0) return DOMINO_OK;
-    if (!states_dev || !logits_dev || !mask_dev || !argmax_dev || (logprobs_dev && !lse_dev))
+    if (!states_dev || !logits_dev || !mask_dev || !argmax_dev || (logprobs_dev && !lse_dev) ||
+        (states_out && stacks_dev && !stacks_out))
         return DOMINO_E_INVALID_ARG;
     DeviceGuard g(h->device);
     cudaStream_t st = (cudaStream_t)stream;
     const bool fusable = dtype == DOMINO_DTYPE_BF16 && reinterpret_cast<uintptr_t>(logits_dev) % 16 == 0 &&
                          ((size_t)row_stride_elems * 2) % 16 == 0 &&
                          (int64_t)batch * h->n_windows < (int64_t)INT32_MAX;   // partial slots are int
-    if (!fusable) {   // the two kernels one after the other
+    if (!fusable) {   // the kernels one after the other
         if ((rc = domino_step_mask(h, states_dev, stacks_dev, batch, mask_dev, nullptr, stream))) return rc;
-        return domino_mask_logits(h, logits_dev, dtype, batch, row_stride_elems, mask_dev, argmax_dev, lse_dev,
-                                  logprobs_dev, stream);
+        if ((rc = domino_mask_logits(h, logits_dev, dtype, batch, row_stride_elems, mask_dev, argmax_dev, lse_dev,
+                                     logprobs_dev, stream)))
+            return rc;
+        if (!states_out) return DOMINO_OK;
+        return domino_advance(h, states_dev, stacks_dev, argmax_dev, batch, states_out, stacks_dev ? stacks_out : nullptr,
+                              stream);
     }
     const size_t part_bytes = (size_t)batch * (size_t)h->n_windows * sizeof(float4);
     if (h->d_fpart.n < part_bytes) {
@@ -758,7 +764,8 @@ int domino_step_decode(domino_t h, const int32_t* states_dev, const uint64_t* st
                                      st, nullptr, nullptr, logits_dev, row_stride_elems, (float4*)h->d_fpart.p,
                                      on_device);
     if (e == cudaSuccess)
-        e = launch_fused_combine((const float4*)h->d_fpart.p, batch, h->n_windows, argmax_dev, lse_dev, st);
+        e = launch_fused_combine(v, h->stack, mode, (const float4*)h->d_fpart.p, batch, h->n_windows, argmax_dev,
+                                 lse_dev, states_dev, stacks_dev, states_out, stacks_dev ? stacks_out : nullptr, st);
     if (e == cudaSuccess && logprobs_dev)
         e = launch_logprobs_bf16(h->env, logits_dev, batch, row_stride_elems, h->V, mask_dev, lse_dev, logprobs_dev,
                                  st);
@@ -989,12 +996,12 @@ int enqueue_host_step(domino_ctx* h, const void* logits_host, void* logits_mappe
             cudaMemcpyAsync(io + L.st, (char*)h->h_io + L.st, L.in_end - L.st, cudaMemcpyHostToDevice, st);
         if (e != cudaSuccess) return cuda_status(e);
         if ((rc = domino_step_decode(h, d_states, d_stacks, batch, logits_mapped, dtype, h->V, d_mask, d_tok, d_lse,
-                                     nullptr, stream)))
+                                     nullptr, d_states, d_stacks, stream)))
             return rc;
     } else {
         if ((rc = copy_and_decode_chunks(h, logits_host, dtype, batch, stacks, L, st))) return rc;
+        if ((rc = domino_advance(h, d_states, d_stacks, d_tok, batch, d_states, d_stacks, stream))) return rc;
     }
-    if ((rc = domino_advance(h, d_states, d_stacks, d_tok, batch, d_states, d_stacks, stream))) return rc;
     return cuda_status(cudaMemcpyAsync(h->h_io, io, L.in_end, cudaMemcpyDeviceToHost, st));
 }
 

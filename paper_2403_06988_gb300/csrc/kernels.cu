@@ -1228,17 +1228,14 @@ __global__ void __launch_bounds__(kLogitThreads)
 // ---------------------------------------------------------------------------
 // advance
 // ---------------------------------------------------------------------------
+// C.update() for one row: row b's configuration walks token t (t < 0 or EOS:
+// the start state; a rejected token: state 0; t >= V: state 0 and the error
+// word).  Reads the configuration before writing, so the outputs may alias it.
 template <bool STACK, int MODE>
-__global__ void __launch_bounds__(kAdvanceThreads)
-    advance_kernel(const StepView v, const int32_t* __restrict__ states, const uint64_t* __restrict__ stacks,
-                   const int32_t* __restrict__ tokens, int32_t batch, int32_t* __restrict__ states_out,
-                   uint64_t* __restrict__ stacks_out) {
+__device__ __forceinline__ void advance_row(const StepView& v, const int32_t* __restrict__ states,
+                                            const uint64_t* __restrict__ stacks, int b, int32_t t,
+                                            int32_t* __restrict__ states_out, uint64_t* __restrict__ stacks_out) {
     using E = typename std::conditional<STACK, uint32_t, uint16_t>::type;
-    pdl_wait();
-    pdl_trigger();
-    const int b = blockIdx.x * kAdvanceThreads + threadIdx.x;
-    if (b >= batch) return;
-    const int32_t t = tokens[b];
     uint32_t s = 0, bits = 0, depth = 0;
     if (t < 0 || t == v.eos_id) {
         s = (uint32_t)v.start;   // the sequence ended; the next one starts from init
@@ -1267,6 +1264,18 @@ __global__ void __launch_bounds__(kAdvanceThreads)
     }
     states_out[b] = (int32_t)s;
     if (stacks_out) stacks_out[b] = ((uint64_t)depth << 32) | bits;
+}
+
+template <bool STACK, int MODE>
+__global__ void __launch_bounds__(kAdvanceThreads)
+    advance_kernel(const StepView v, const int32_t* __restrict__ states, const uint64_t* __restrict__ stacks,
+                   const int32_t* __restrict__ tokens, int32_t batch, int32_t* __restrict__ states_out,
+                   uint64_t* __restrict__ stacks_out) {
+    pdl_wait();
+    pdl_trigger();
+    const int b = blockIdx.x * kAdvanceThreads + threadIdx.x;
+    if (b >= batch) return;
+    advance_row<STACK, MODE>(v, states, stacks, b, tokens[b], states_out, stacks_out);
 }
 
 // Opportunistic masking, the check: is row b's proposal (its unmasked argmax)
@@ -1669,9 +1678,18 @@ cudaError_t launch_step_mask(const StepView& v, const LaunchEnv& env, bool stack
 }
 
 // Merges each row's per-window partials of the fused step: one warp per row.
+// ADV: lane 0 then advances the row by its argmax (C.update of the same step).
+struct AdvanceArgs {
+    const int32_t* states;
+    const uint64_t* stacks;
+    int32_t* states_out;   // nullptr: no update
+    uint64_t* stacks_out;
+};
+
+template <bool ADV, bool STACK, int MODE>
 __global__ void __launch_bounds__(kLogitThreads)
-    fused_combine_kernel(const float4* __restrict__ part, int32_t batch, int32_t n_windows,
-                         int32_t* __restrict__ argmax, float* __restrict__ lse) {
+    fused_combine_kernel(const StepView v, const float4* __restrict__ part, int32_t batch, int32_t n_windows,
+                         int32_t* __restrict__ argmax, float* __restrict__ lse, const AdvanceArgs adv) {
     pdl_wait();
     pdl_trigger();
     const int r = blockIdx.x * (kLogitThreads / 32) + (threadIdx.x >> 5), lane = threadIdx.x & 31;
@@ -1684,15 +1702,39 @@ __global__ void __launch_bounds__(kLogitThreads)
     }
     warp_merge(m, idx, s);
     if (lane == 0) {
-        argmax[r] = m == -INFINITY ? -1 : idx;
+        const int32_t t = m == -INFINITY ? -1 : idx;
+        argmax[r] = t;
         if (lse) lse[r] = m == -INFINITY ? -INFINITY : m + logf(s);
+        if constexpr (ADV) advance_row<STACK, MODE>(v, adv.states, adv.stacks, r, t, adv.states_out, adv.stacks_out);
     }
 }
 
-cudaError_t launch_fused_combine(const float4* part, int32_t batch, int32_t n_windows, int32_t* argmax, float* lse,
-                                 cudaStream_t st) {
-    const unsigned grid = (unsigned)((batch + kLogitThreads / 32 - 1) / (kLogitThreads / 32));
-    return launch_pdl(fused_combine_kernel, dim3(grid), dim3(kLogitThreads), 0, st, part, batch, n_windows, argmax, lse);
+template <bool STACK>
+cudaError_t launch_combine_adv(const StepView& v, int mode, const float4* part, int32_t batch, int32_t n_windows,
+                               int32_t* argmax, float* lse, const AdvanceArgs& adv, dim3 grid, cudaStream_t st) {
+    switch (mode) {
+        case kSparse32Smem:
+            return launch_pdl(fused_combine_kernel<true, STACK, kSparse32Smem>, grid, dim3(kLogitThreads), 0, st, v,
+                              part, batch, n_windows, argmax, lse, adv);
+        case kSparse64Smem:
+            return launch_pdl(fused_combine_kernel<true, STACK, kSparse64Smem>, grid, dim3(kLogitThreads), 0, st, v,
+                              part, batch, n_windows, argmax, lse, adv);
+        default:
+            return launch_pdl(fused_combine_kernel<true, STACK, kDenseGlobal>, grid, dim3(kLogitThreads), 0, st, v,
+                              part, batch, n_windows, argmax, lse, adv);
+    }
+}
+
+cudaError_t launch_fused_combine(const StepView& v, bool stack, int mode, const float4* part, int32_t batch,
+                                 int32_t n_windows, int32_t* argmax, float* lse, const int32_t* states,
+                                 const uint64_t* stacks, int32_t* states_out, uint64_t* stacks_out, cudaStream_t st) {
+    const dim3 grid((unsigned)((batch + kLogitThreads / 32 - 1) / (kLogitThreads / 32)));
+    const AdvanceArgs adv{states, stacks, states_out, stacks_out};
+    if (!states_out)
+        return launch_pdl(fused_combine_kernel<false, false, kDenseGlobal>, grid, dim3(kLogitThreads), 0, st, v, part,
+                          batch, n_windows, argmax, lse, adv);
+    if (stack) return launch_combine_adv<true>(v, mode, part, batch, n_windows, argmax, lse, adv, grid, st);
+    return launch_combine_adv<false>(v, mode, part, batch, n_windows, argmax, lse, adv, grid, st);
 }
 
 cudaError_t launch_logprobs_bf16(const LaunchEnv& env, const void* logits, int32_t batch, int64_t row_stride,

@@ -151,3 +151,36 @@ def test_step_decode_logprobs_need_lse():
     with pytest.raises(B.DominoError):
         B.domino_step_decode(d.h, dev(states), None, 4, lg.data_ptr(), B.DTYPE_BF16, V, mask, arg, None, lp)
     d.close()
+
+
+@pytest.mark.parametrize("config", [1, 2, 3, 5])
+def test_step_decode_with_update_matches_oracle(config):
+    """states_out given: the merge advances each row by its argmax in place
+    (config 1, fp32 logits: the separate kernels, then domino_advance)."""
+    import oracle
+    w = workload(config)
+    P = oracle.Problem.from_workload(w)
+    d = Domino.from_parts(w.automaton, w.vocab, device=0)
+    states, stacks = w.initial_configs()
+    has_stack = w.automaton.rules is not None
+    lg = w.logits(11)
+    t = torch.from_numpy(lg.view(np.int16) if lg.dtype == np.uint16 else lg).cuda()
+    dt = B.DTYPE_BF16 if lg.dtype == np.uint16 else B.DTYPE_F32
+    V, b = w.vocab.n_tokens, len(states)
+    st = dev(states)
+    sk = dev(stacks.view(np.int64)) if has_stack else None
+    mask = torch.empty((b, d.info()["n_words"]), dtype=torch.int32, device="cuda")
+    arg = torch.empty(b, dtype=torch.int32, device="cuda")
+    lse = torch.empty(b, dtype=torch.float32, device="cuda")
+    B.domino_step_decode(d.h, st, sk, b, t.data_ptr(), dt, V, mask, arg, lse, None, st, sk)
+    torch.cuda.synchronize()
+    m_o, _, _ = P.step_mask(states, stacks if has_stack else None, n_threads=NT)
+    a_o, l_o, _ = oracle.mask_logits(lg, m_o, n_threads=NT)
+    s_o, k_o, bad = P.advance(states, stacks if has_stack else None, a_o, w.automaton.start)
+    assert bad == 0
+    assert (arg.cpu().numpy() == a_o).all()
+    assert (st.cpu().numpy() == s_o).all()
+    if has_stack:
+        assert (sk.cpu().numpy().view(np.uint64) == k_o).all()
+    assert d.device_error() == 0
+    d.close()
