@@ -63,6 +63,7 @@ struct domino_ctx {
     // each direction takes one copy through the pinned staging buffer h_io
     DevBuf s_logits, s_mask, s_io;
     void* h_io = nullptr;
+    void* h_io_dev = nullptr;   // h_io as the device addresses it
     size_t h_io_n = 0;
     // opportunistic masking: proposals, the fallback row list and its length
     DevBuf o_prop, o_rows, o_count;
@@ -914,9 +915,10 @@ int domino_advance_table(domino_t h, const int32_t* table_next_dev, const int32_
 namespace {
 
 // The host-buffer step's small inputs and outputs in one buffer (device s_io,
-// pinned host h_io): [count of non-zero mask bytes | tokens | lse | states |
-// stacks], each part on a 16-byte boundary.  States and stacks go up in one
-// copy, everything comes back in one.
+// pinned host h_io): [tokens | lse | states | stacks], each part on a 16-byte
+// boundary.  The copy path moves states and stacks up in one copy and
+// everything back in one; the in-place path's kernels read and write h_io
+// directly.
 struct IoLayout {
     size_t tok, lse, st, sk, in_end;
 };
@@ -991,13 +993,15 @@ int enqueue_host_step(domino_ctx* h, const void* logits_host, void* logits_mappe
     uint32_t* d_mask = (uint32_t*)h->s_mask.p;
     int32_t* d_tok = (int32_t*)(io + L.tok);
     float* d_lse = (float*)(io + L.lse);
-    if (mapped) {   // the mask step folds the pinned logits it allows, read in place
-        cudaError_t e =
-            cudaMemcpyAsync(io + L.st, (char*)h->h_io + L.st, L.in_end - L.st, cudaMemcpyHostToDevice, st);
-        if (e != cudaSuccess) return cuda_status(e);
-        if ((rc = domino_step_decode(h, d_states, d_stacks, batch, logits_mapped, dtype, h->V, d_mask, d_tok, d_lse,
-                                     nullptr, d_states, d_stacks, stream)))
-            return rc;
+    if (mapped) {
+        // the mask step folds the pinned logits it allows, read in place; the
+        // configurations are read from and the results written to the pinned
+        // staging buffer itself (no copies: two kernels)
+        char* hio = (char*)h->h_io_dev;
+        int32_t* m_states = (int32_t*)(hio + L.st);
+        uint64_t* m_stacks = stacks ? (uint64_t*)(hio + L.sk) : nullptr;
+        return domino_step_decode(h, m_states, m_stacks, batch, logits_mapped, dtype, h->V, d_mask,
+                                  (int32_t*)(hio + L.tok), (float*)(hio + L.lse), nullptr, m_states, m_stacks, stream);
     } else {
         if ((rc = copy_and_decode_chunks(h, logits_host, dtype, batch, stacks, L, st))) return rc;
         if ((rc = domino_advance(h, d_states, d_stacks, d_tok, batch, d_states, d_stacks, stream))) return rc;
@@ -1060,6 +1064,12 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
             cudaGetLastError();
             h->h_io = nullptr;
             return DOMINO_E_OOM;
+        }
+        if (cudaHostGetDevicePointer(&h->h_io_dev, h->h_io, 0) != cudaSuccess) {
+            cudaGetLastError();
+            cudaFreeHost(h->h_io);
+            h->h_io = h->h_io_dev = nullptr;
+            return DOMINO_E_CUDA;
         }
         h->h_io_n = L.in_end;
     }
