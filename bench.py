@@ -198,9 +198,10 @@ def ncu_traffic(name: str) -> dict:
             digest = hashlib.sha256(f.read()).hexdigest()[:16]
     except (OSError, ValueError):
         return {}
-    if rec.get("kernels_cu_sha256_16") != digest:
+    ent = rec.get("per_workload", {}).get(name, {})
+    if ent.get("kernels_cu_sha256_16") != digest:
         return {}
-    return {k: v for k, v in rec.get("per_launch_bytes", {}).get(name, {}).items()}
+    return dict(ent.get("per_launch_bytes", {}))
 
 
 def cpu_cores() -> int:
@@ -752,6 +753,7 @@ def run_domino(args, dist: Dist):
                       "dram_bytes_ncu": traffic.get("step_mask")},
         "step_decode": {"us": per_kernel["step_decode"] * 1e3,
                         "separate_us": (per_kernel["step_mask"] + per_kernel["mask_logits"]) * 1e3,
+                        "dram_bytes_ncu": traffic.get("step_decode_fused"),
                         "note": "the timed step's mask + decode: the mask step folds the allowed logits of each "
                                 "tile (then a per-row merge; log-probs in one more pass where asked for)"},
         "advance": {"us": per_kernel["advance"] * 1e3},
