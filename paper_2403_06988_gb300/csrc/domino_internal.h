@@ -20,7 +20,6 @@ constexpr int kStepThreads = 1024;             // step kernel CTA size (one CTA 
 constexpr int kRowsPerTile = 4;                // fewest rows per tile (mask only; small batches)
 constexpr int kMaxRowsPerTile = 32;            // most rows per tile (one warp ballot)
 constexpr int kRowsPerTileNext = 8;            // rows per tile when next states are written
-constexpr int kUnitSlots = 32;                 // slots per work unit (one per lane)
 constexpr int kWalkChains = 4;                 // rows walked together by one lane (independent chains)
 constexpr int kHeadBytes = 16;                 // class ids per 16-byte head block
 constexpr int kInlineBytes = 32;               // class ids stored inline per token (two head blocks)
@@ -54,13 +53,9 @@ struct StepView {
     const int32_t* tail_off;  // [n_slots] offset of bytes 32.. in `tail`
     const uint8_t* tail;      // class ids of bytes 32.. of tokens longer than 32 bytes
     const int32_t* pos_of;    // [V] slot of original id
-    // work units: a unit is <= 32 consecutive slots of one first-class group,
-    // packed as class (bits 0..7) | first slot (bits 8..18) | count-1 (bits 19..23)
-    const uint32_t* units;    // all windows' units, window w at [unit_off[w], unit_off[w+1])
-    const int32_t* unit_off;  // [n_windows + 1]
-    const uint16_t* cls_units; // [n_windows][K + 1]: window-local first unit of each first class
+    // the slots of first class c in window w are [cls_start[w][c], cls_start[w][c + 1])
+    const uint16_t* cls_start; // [n_windows][K + 1]
     const int16_t* eos_slot;  // [n_windows] window-local slot of EOS, -1 if not in the window
-    int32_t max_units;        // max units of one window
     int32_t V, W, n_windows, eos_id;
     // automaton
     const uint16_t* t16;      // [Q][K] (DFA)

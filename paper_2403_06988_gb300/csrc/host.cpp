@@ -52,8 +52,7 @@ struct domino_ctx {
     int64_t dense_ret_off = 0, sp_tgt_off = 0, sp_ret_off = 0;
 
     // ---- device copies
-    DevBuf d_head, d_info, d_tail_off, d_tail, d_pos_of, d_units, d_unit_off, d_cls_units, d_eos_slot;
-    int32_t max_units = 0;
+    DevBuf d_head, d_info, d_tail_off, d_tail, d_pos_of, d_cls_start, d_eos_slot;
     DevBuf d_dense, d_sparse, d_accept, d_self, d_tok_cls;
     DevBuf d_err, d_partials, d_counters, d_lse_tmp, d_fpart;
     bool arena_ready = false;
@@ -111,8 +110,8 @@ void dev_free(DevBuf& b) {
 }
 
 int64_t dev_bytes(const domino_ctx* h) {
-    const DevBuf* all[] = {&h->d_head, &h->d_info, &h->d_tail_off, &h->d_tail, &h->d_pos_of, &h->d_units,
-                           &h->d_unit_off, &h->d_cls_units, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_self, &h->d_tok_cls, &h->d_err, &h->d_fpart, &h->d_partials,
+    const DevBuf* all[] = {&h->d_head, &h->d_info, &h->d_tail_off, &h->d_tail, &h->d_pos_of, &h->d_cls_start,
+                           &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_self, &h->d_tok_cls, &h->d_err, &h->d_fpart, &h->d_partials,
                            &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_mask, &h->s_io,
                            &h->o_prop, &h->o_rows, &h->o_count};
     int64_t n = 0;
@@ -183,10 +182,7 @@ int build_arena(domino_ctx* h) {
     std::vector<uint32_t> info((size_t)n_slots, 0);
     std::vector<int32_t> tail_off((size_t)n_slots, 0), pos_of((size_t)V, 0);
     std::vector<uint16_t> gstart((size_t)(K + 1), 0);
-    std::vector<uint32_t> units;
-    std::vector<int32_t> unit_off((size_t)nw + 1, 0);
-    std::vector<uint16_t> cls_units((size_t)nw * (size_t)(h->K + 1), 0);   // [window][class]: first unit
-    int32_t max_units = 0;
+    std::vector<uint16_t> cls_start((size_t)nw * (size_t)(h->K + 1), 0);   // [window][class]: first slot
     std::vector<int16_t> eos_slot((size_t)nw, -1);
     std::vector<uint8_t> tail;
     std::vector<int32_t> ids;
@@ -217,18 +213,8 @@ int build_arena(domino_ctx* h) {
             }
         }
         while (c_next <= K) gs[c_next++] = (uint16_t)(hi - lo);
-        // work units: <= kUnitSlots consecutive slots of one first-class group;
-        // each class's units are contiguous, from cls_units[w][c] on
-        for (int c = 0; c < K; c++) {
-            cls_units[(size_t)w * (K + 1) + c] = (uint16_t)(units.size() - (size_t)unit_off[(size_t)w]);
-            for (int b = gs[c]; b < gs[c + 1]; b += kUnitSlots) {
-                const int n = std::min(kUnitSlots, gs[c + 1] - b);
-                units.push_back((uint32_t)c | ((uint32_t)b << 8) | ((uint32_t)(n - 1) << 19));
-            }
-        }
-        cls_units[(size_t)w * (K + 1) + K] = (uint16_t)(units.size() - (size_t)unit_off[(size_t)w]);
-        unit_off[(size_t)w + 1] = (int32_t)units.size();
-        max_units = std::max(max_units, unit_off[(size_t)w + 1] - unit_off[(size_t)w]);
+        // the slots of first class c are [gs[c], gs[c + 1]) of the window
+        std::copy(gs, gs + K + 1, cls_start.begin() + (ptrdiff_t)((size_t)w * (K + 1)));
     }
     if (tail.size() > (size_t)INT32_MAX) return DOMINO_E_UNSUPPORTED;
     int rc;
@@ -237,15 +223,12 @@ int build_arena(domino_ctx* h) {
     if ((rc = dev_upload(h->d_tail_off, tail_off.data(), tail_off.size() * 4))) return rc;
     if ((rc = dev_upload(h->d_tail, tail.data(), tail.size()))) return rc;
     if ((rc = dev_upload(h->d_pos_of, pos_of.data(), pos_of.size() * 4))) return rc;
-    if ((rc = dev_upload(h->d_units, units.data(), units.size() * 4))) return rc;
-    if ((rc = dev_upload(h->d_unit_off, unit_off.data(), unit_off.size() * 4))) return rc;
-    if ((rc = dev_upload(h->d_cls_units, cls_units.data(), cls_units.size() * 2))) return rc;
+    if ((rc = dev_upload(h->d_cls_start, cls_start.data(), cls_start.size() * 2))) return rc;
     if (self) {
         if ((rc = dev_upload(h->d_tok_cls, tok_cls.data(), tok_cls.size() * 8))) return rc;
     } else {
         dev_free(h->d_tok_cls);
     }
-    h->max_units = max_units;
     if ((rc = dev_upload(h->d_eos_slot, eos_slot.data(), eos_slot.size() * 2))) return rc;
     h->n_windows = nw;
     h->arena_ready = true;
@@ -259,10 +242,7 @@ StepView make_view(domino_ctx* h) {
     v.tail_off = (const int32_t*)h->d_tail_off.p;
     v.tail = (const uint8_t*)h->d_tail.p;
     v.pos_of = (const int32_t*)h->d_pos_of.p;
-    v.units = (const uint32_t*)h->d_units.p;
-    v.unit_off = (const int32_t*)h->d_unit_off.p;
-    v.cls_units = (const uint16_t*)h->d_cls_units.p;
-    v.max_units = h->max_units;
+    v.cls_start = (const uint16_t*)h->d_cls_start.p;
     v.eos_slot = (const int16_t*)h->d_eos_slot.p;
     v.V = h->V;
     v.W = h->W;
@@ -373,8 +353,8 @@ int domino_destroy(domino_t h) {
     if (h->device >= 0) {
         DeviceGuard g(h->device);
         cudaDeviceSynchronize();
-        DevBuf* all[] = {&h->d_head, &h->d_info, &h->d_tail_off, &h->d_tail, &h->d_pos_of, &h->d_units,
-                         &h->d_unit_off, &h->d_cls_units, &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_self, &h->d_tok_cls, &h->d_err, &h->d_fpart, &h->d_partials,
+        DevBuf* all[] = {&h->d_head, &h->d_info, &h->d_tail_off, &h->d_tail, &h->d_pos_of, &h->d_cls_start,
+                         &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_self, &h->d_tok_cls, &h->d_err, &h->d_fpart, &h->d_partials,
                          &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_mask, &h->s_io,
                          &h->o_prop, &h->o_rows, &h->o_count};
         for (auto* b : all) dev_free(*b);

@@ -204,25 +204,29 @@ struct FuseArgs {
 
 // Shared-memory layout of the step kernel (offsets in bytes).
 struct StepLayout {
-    int head, info, units, cls, tokcls, items, rows, ctrl, rowmask, cfg, mtile, ntile, accept, self, table, total;
+    int head, info, cls, tokcls, pairs, rows, ctrl, cfg, mtile, ntile, accept, self, table, total;
 };
 
-__host__ __device__ inline StepLayout step_layout(int K, int R, bool next, bool stack, int max_units, int Q,
-                                                  int table_bytes, bool self) {
+// Walk pairs: (token slot, group of up to kWalkChains live rows of the token's
+// first class), packed as slot (bits 0..9) | the group's rows (5 bits each,
+// bits 10..29) | rows in the group - 1 (bits 30..31).  A tile lists at most
+// kWin x ceil(R / kWalkChains) of them.
+static_assert(kWalkChains == 4 && kMaxRowsPerTile <= 32 && kWin == 1024, "walk pair packing");
+
+__host__ __device__ inline StepLayout step_layout(int K, int R, bool next, bool stack, int Q, int table_bytes,
+                                                  bool self) {
     StepLayout L{};
     int o = 0;
     L.head = o;    o += kWin * 32;
     L.info = o;    o += kWin * 4;
-    L.units = o;   o += align16(max_units * 4);
     L.cls = o;     o += align16((K + 1) * 2);
     L.tokcls = o;  o += self ? kWin * 8 : 0;
-    L.items = o;   o += align16(max_units * ((R + kWalkChains - 1) / kWalkChains) * 4);
+    L.pairs = o;   o += kWin * ((R + kWalkChains - 1) / kWalkChains) * 4;
     L.rows = o;    o += R * 16;
     L.ctrl = o;    o += 16;
-    L.rowmask = o; o += align16(K * 4);
     L.cfg = o;     o += align16(R * K * (stack ? 16 : 4));
     L.mtile = o;   o += align16(R * 32 * 4);
-    L.ntile = o;   o += next ? R * kWin * 4 : 0;
+    L.ntile = o;   o += next ? R * kWin * 2 : 0;   // next states < Q <= 65535: staged as u16
     L.accept = o;  o += align16(((Q + 31) / 32) * 4);
     L.self = o;    o += self ? align16(Q * 8) : 0;
     L.table = o;   o += align16(table_bytes);
@@ -390,20 +394,17 @@ __global__ void __launch_bounds__(kStepThreads, 1)
     extern __shared__ __align__(16) unsigned char smem[];
     const int K = v.K;
     const bool use_self = v.self_mask != nullptr;
-    const StepLayout L = step_layout(K, R, NEXT, STACK, v.max_units, v.Q, MODE == kDenseGlobal ? 0 : img_bytes,
-                                     use_self);
+    const StepLayout L = step_layout(K, R, NEXT, STACK, v.Q, MODE == kDenseGlobal ? 0 : img_bytes, use_self);
     uint4* s_head = reinterpret_cast<uint4*>(smem + L.head);
     uint32_t* s_info = reinterpret_cast<uint32_t*>(smem + L.info);
-    uint32_t* s_units = reinterpret_cast<uint32_t*>(smem + L.units);
-    uint16_t* s_cls = reinterpret_cast<uint16_t*>(smem + L.cls);      // [K + 1] first unit of each first class
-    uint32_t* s_items = reinterpret_cast<uint32_t*>(smem + L.items);   // unit | chain group << 16
+    uint16_t* s_cls = reinterpret_cast<uint16_t*>(smem + L.cls);      // [K + 1] first slot of each first class
+    uint32_t* s_pairs = reinterpret_cast<uint32_t*>(smem + L.pairs);   // walk pairs of the tile
     uint4* s_rows = reinterpret_cast<uint4*>(smem + L.rows);
-    int* s_ctrl = reinterpret_cast<int*>(smem + L.ctrl);   // -, items listed, EOS slot, unit count
-    uint32_t* s_rowmask = reinterpret_cast<uint32_t*>(smem + L.rowmask);
+    int* s_ctrl = reinterpret_cast<int*>(smem + L.ctrl);   // -, pairs listed, EOS slot, -
     uint32_t* s_cfg = reinterpret_cast<uint32_t*>(smem + L.cfg);   // [R][K] state (DFA)
     uint4* s_cfg4 = reinterpret_cast<uint4*>(smem + L.cfg);        // [R][K] (state, bits, depth) (pushdown)
     uint32_t* s_mtile = reinterpret_cast<uint32_t*>(smem + L.mtile);
-    int32_t* s_ntile = reinterpret_cast<int32_t*>(smem + L.ntile);
+    uint16_t* s_ntile = reinterpret_cast<uint16_t*>(smem + L.ntile);   // [R][kWin] next states
     uint32_t* s_accept = reinterpret_cast<uint32_t*>(smem + L.accept);
     unsigned long long* s_self = reinterpret_cast<unsigned long long*>(smem + L.self);       // [Q]
     unsigned long long* s_tokcls = reinterpret_cast<unsigned long long*>(smem + L.tokcls);   // [kWin]
@@ -475,13 +476,8 @@ __global__ void __launch_bounds__(kStepThreads, 1)
             s_head[2 * tid + 1] = __ldg(v.head + 2 * ((size_t)w * kWin + tid) + 1);
             s_info[tid] = __ldg(v.info + (size_t)w * kWin + tid);
             if (use_self) s_tokcls[tid] = __ldg(v.tok_cls + (size_t)w * kWin + tid);
-            const int u0 = __ldg(v.unit_off + w), nu = __ldg(v.unit_off + w + 1) - u0;
-            for (int i = tid; i < nu; i += kStepThreads) s_units[i] = __ldg(v.units + u0 + i);
-            for (int i = tid; i <= K; i += kStepThreads) s_cls[i] = __ldg(v.cls_units + (size_t)w * (K + 1) + i);
-            if (tid == 0) {
-                s_ctrl[2] = __ldg(v.eos_slot + w);
-                s_ctrl[3] = nu;
-            }
+            for (int i = tid; i <= K; i += kStepThreads) s_cls[i] = __ldg(v.cls_start + (size_t)w * (K + 1) + i);
+            if (tid == 0) s_ctrl[2] = __ldg(v.eos_slot + w);
             cur_w = w;
         }
         if (tid < nr) {
@@ -492,7 +488,7 @@ __global__ void __launch_bounds__(kStepThreads, 1)
                 s_rows[tid] = decode_row(v, pf_s, pf_w, stacks != nullptr, s_accept, w == 0);
             }
         }
-        if (tid == 0) s_ctrl[1] = 0;   // items listed so far
+        if (tid == 0) s_ctrl[1] = 0;   // pairs listed so far
         for (int i = tid; i < nr * 32; i += kStepThreads) s_mtile[i] = 0u;
         if (fuse.prefetch) {
             // the tile's logits head for L2 while the walk runs: one 128-byte
@@ -506,15 +502,16 @@ __global__ void __launch_bounds__(kStepThreads, 1)
             }
         }
         if constexpr (NEXT) {
-            for (int i = tid; i < nr * (kWin / 4); i += kStepThreads)
+            for (int i = tid; i < nr * (kWin / 8); i += kStepThreads)
                 reinterpret_cast<int4*>(s_ntile)[i] = make_int4(0, 0, 0, 0);
         }
         __syncthreads();
 
         // first transition once per (row, first class): lane r of a warp takes
         // row r, the ballot gives the class's live rows; the warp then lists
-        // the work items of the class's units, (unit, group of up to
-        // kWalkChains live rows), for the warps to walk
+        // the class's walk pairs, every (token, group of up to kWalkChains
+        // live rows) with the group's rows packed into the pair, so that the
+        // warps walk 32 pairs at a time whatever the class sizes
         for (int c = warp; c < K; c += kStepThreads / 32) {
             uint32_t s = 0, bits = 0, depth = 0;
             if (lane < nr) {
@@ -536,38 +533,42 @@ __global__ void __launch_bounds__(kStepThreads, 1)
                 }
             }
             const uint32_t live = __ballot_sync(0xffffffffu, s != 0);
-            if (lane == 0) s_rowmask[c] = live;
-            const int ub = s_cls[c], g = (__popc(live) + kWalkChains - 1) / kWalkChains;
-            const int n = (s_cls[c + 1] - ub) * g;
-            if (n > 0) {
+            const int n_live = __popc(live);
+            const int g0 = s_cls[c], nc = s_cls[c + 1] - g0;
+            const int ng = (n_live + kWalkChains - 1) / kWalkChains;
+            if (nc > 0 && ng > 0) {
                 int base = 0;
-                if (lane == 0) base = atomicAdd(&s_ctrl[1], n);
+                if (lane == 0) base = atomicAdd(&s_ctrl[1], nc * ng);
                 base = __shfl_sync(0xffffffffu, base, 0);
-                for (int k = lane; k < n; k += 32)
-                    s_items[base + k] = (uint32_t)(ub + k / g) | ((uint32_t)(k % g) << 16);
+                // this lane's row is live row number `rank` of the class
+                const int rank = __popc(live & ((1u << lane) - 1u));
+                const bool mine = (live >> lane) & 1u;
+                for (int g = 0; g < ng; ++g) {
+                    const uint32_t part = (mine && (rank >> 2) == g) ? ((uint32_t)lane << (5 * (rank & 3))) : 0u;
+                    const uint32_t rows = __reduce_or_sync(0xffffffffu, part) |
+                                          ((uint32_t)(min(kWalkChains, n_live - kWalkChains * g) - 1) << 20);
+                    for (int k = lane; k < nc; k += 32) s_pairs[base + g * nc + k] = (uint32_t)(g0 + k) | (rows << 10);
+                }
             }
         }
         const int eos_local = s_ctrl[2];
         if (tid < nr && eos_local >= 0 && (s_rows[tid].w & 2u)) {
             const int ol = (int)(s_info[eos_local] & 1023u);
             atomicOr(&s_mtile[tid * 32 + (ol >> 5)], 1u << (ol & 31));
-            if constexpr (NEXT) s_ntile[tid * kWin + ol] = (int32_t)s_rows[tid].x;
+            if constexpr (NEXT) s_ntile[tid * kWin + ol] = (uint16_t)s_rows[tid].x;
         }
         __syncthreads();
 
         prefetch(t + 1);
-        const int n_items = s_ctrl[1];
-        for (int it = warp; it < n_items; it += kStepThreads / 32) {
-            const uint32_t item = s_items[it];
-            const uint32_t unit = s_units[item & 0xFFFFu];
-            const int grp = (int)(item >> 16);
-            const int c = (int)(unit & 0xFFu);
-            uint32_t rm = s_rowmask[c];
-            for (int g = 0; g < grp * kWalkChains; ++g) rm &= rm - 1;   // skip earlier groups' rows
-            const int slot = (int)((unit >> 8) & 0x7FFu) + lane;
-            const bool active = lane <= (int)((unit >> 19) & 31u);
+        const int n_pairs = s_ctrl[1];
+        for (int p0 = warp * 32; p0 < n_pairs; p0 += kStepThreads) {
+            const bool active = p0 + lane < n_pairs;
+            const uint32_t pr = active ? s_pairs[p0 + lane] : 0u;
+            const int slot = (int)(pr & 1023u);
             const uint32_t info = active ? s_info[slot] : 0u;
             const uint8_t* hp = reinterpret_cast<const uint8_t*>(s_head + 2 * slot);
+            const int c = hp[0];   // the token's first class
+            const int n_rows = active ? (int)(pr >> 30) + 1 : 0;
             const int len = (int)(info >> 16);
             const int ol = (int)(info & 1023u);
             const uint8_t* tl = len > kInlineBytes ? v.tail + __ldg(v.tail_off + (size_t)w * kWin + slot) : v.tail;
@@ -578,9 +579,8 @@ __global__ void __launch_bounds__(kStepThreads, 1)
                 for (int k = 0; k < kWalkChains; ++k) {
                     rr[k] = -1;
                     sv[k] = bv[k] = dv[k] = 0u;
-                    if (rm) {
-                        rr[k] = __ffs(rm) - 1;
-                        rm &= rm - 1;
+                    if (k < n_rows) {
+                        rr[k] = (int)((pr >> (10 + 5 * k)) & 31u);
                         if constexpr (STACK) {
                             const uint4 cf = s_cfg4[rr[k] * K + c];
                             sv[k] = cf.x;
@@ -606,7 +606,7 @@ __global__ void __launch_bounds__(kStepThreads, 1)
                     for (int k = 0; k < kWalkChains; ++k) {
                         if (rr[k] >= 0 && sv[k]) {
                             atomicOr(&s_mtile[rr[k] * 32 + (ol >> 5)], 1u << (ol & 31));
-                            if constexpr (NEXT) s_ntile[rr[k] * kWin + ol] = (int32_t)sv[k];
+                            if constexpr (NEXT) s_ntile[rr[k] * kWin + ol] = (uint16_t)sv[k];
                         }
                     }
                 }
@@ -791,14 +791,16 @@ __global__ void __launch_bounds__(kStepThreads, 1)
                 const int per_row = in_win / 4;
                 for (int i = tid; i < nr * (kWin / 4); i += kStepThreads) {
                     const int r = i / (kWin / 4), k4 = i % (kWin / 4);
-                    if (k4 < per_row)
+                    if (k4 < per_row) {
+                        const uint2 h = reinterpret_cast<const uint2*>(s_ntile + r * kWin)[k4];
                         __stcs(reinterpret_cast<int4*>(next + (size_t)(r0 + r) * v.V + (size_t)w * kWin) + k4,
-                               reinterpret_cast<const int4*>(s_ntile + r * kWin)[k4]);
+                               make_int4((int)(h.x & 0xFFFFu), (int)(h.x >> 16), (int)(h.y & 0xFFFFu), (int)(h.y >> 16)));
+                    }
                 }
             } else {
                 for (int i = tid; i < nr * kWin; i += kStepThreads) {
                     const int r = i / kWin, k = i % kWin;
-                    if (k < in_win) next[(size_t)(r0 + r) * v.V + (size_t)w * kWin + k] = s_ntile[i];
+                    if (k < in_win) next[(size_t)(r0 + r) * v.V + (size_t)w * kWin + k] = (int32_t)s_ntile[i];
                 }
             }
         }
@@ -1485,7 +1487,7 @@ __global__ void __launch_bounds__(kAdvanceThreads)
 int rows_per_tile(const StepView& v, const LaunchEnv& env, int batch, bool next, bool stack, int img_bytes) {
     if (next) {
         for (int R = kMaxRowsPerTile; R > kRowsPerTileNext; R >>= 1)
-            if (step_layout(v.K, R, true, stack, v.max_units, v.Q, img_bytes, v.self_mask != nullptr).total <=
+            if (step_layout(v.K, R, true, stack, v.Q, img_bytes, v.self_mask != nullptr).total <=
                     env.max_smem_optin &&
                 (long long)((batch + R - 1) / R) * v.n_windows >= 4LL * env.num_sms)
                 return R;
@@ -1512,7 +1514,7 @@ cudaError_t launch_step_t(const StepView& v, const LaunchEnv& env, const int32_t
                           const FuseArgs& fuse, cudaStream_t st) {
     const int img_bytes = MODE == kDenseGlobal ? 0 : (int)table_smem_bytes(v, STACK, MODE);
     const int R = rows_per_tile(v, env, batch, NEXT, STACK, img_bytes);
-    const StepLayout L = step_layout(v.K, R, NEXT, STACK, v.max_units, v.Q, img_bytes, v.self_mask != nullptr);
+    const StepLayout L = step_layout(v.K, R, NEXT, STACK, v.Q, img_bytes, v.self_mask != nullptr);
     auto kern = step_kernel<STACK, MODE, NEXT>;
     // the dynamic shared-memory limit is raised once per device and size, so
     // that launches inside a stream capture make no attribute calls
@@ -1661,7 +1663,7 @@ int64_t table_smem_bytes(const StepView& v, bool stack, int mode) {
 }
 
 int step_fixed_smem_bytes(const StepView& v, bool next) {
-    return step_layout(v.K, next ? kRowsPerTileNext : kMaxRowsPerTile, next, v.t32 != nullptr, v.max_units, v.Q, 0,
+    return step_layout(v.K, next ? kRowsPerTileNext : kMaxRowsPerTile, next, v.t32 != nullptr, v.Q, 0,
                        v.self_mask != nullptr)
         .total;
 }
