@@ -175,8 +175,8 @@ __device__ __forceinline__ void prefetch_l2(const void* p) {
 
 // Folds one row window whose allowed tokens (at most 32) were listed one per
 // lane: t = INT_MAX marks an empty lane, raw the lane's bf16 logit.  Writes
-// (max, lowest index of the max, sum of exp against the max) to part[slot].
-__device__ __forceinline__ void fold_pending(float4* part, int slot, unsigned short raw, int t, int lane) {
+// (max, lowest index of the max, sum of exp against the max) to *out.
+__device__ __forceinline__ void fold_listed(float4* out, unsigned short raw, int t, int lane) {
     const float x = t != INT_MAX ? __uint_as_float((uint32_t)raw << 16) : -INFINITY;
     float m = x;
     int idx = t;
@@ -192,7 +192,167 @@ __device__ __forceinline__ void fold_pending(float4* part, int slot, unsigned sh
     float e = t != INT_MAX ? ex2(fmaf(x, kLog2e, -m * kLog2e)) : 0.0f;
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) e += __shfl_xor_sync(0xffffffffu, e, off);
-    if (lane == 0) part[slot] = make_float4(m, __int_as_float(idx), e, 0.f);
+    if (lane == 0) *out = make_float4(m, __int_as_float(idx), e, 0.f);
+}
+
+// The fused masked decode of one row window: `mrow` holds the row's 32 mask
+// words of window w in shared memory (the warp owns them and uses them as
+// scratch), `lrow` is the row's bf16 logits (device or pinned host memory).
+// Writes (max, lowest index of the max, sum of exp against the max) to *out.
+// By the number n of allowed tokens: n <= 32 lists them one per lane; n <= 128
+// lists them as 16-bit entries and loads up to four per lane at once; denser
+// windows are folded word by word, a word's four 16-byte vectors loaded at once.
+__device__ __forceinline__ void fold_window(uint32_t* mrow, const char* lrow, int w, int V, int W, int lane,
+                                            float4* out) {
+    const int full_words = V / 32;
+    const int j = w * 32 + lane;
+    const uint32_t word = j < W ? mrow[lane] : 0u;
+    const unsigned short* u = reinterpret_cast<const unsigned short*>(lrow);
+    const int c = __popc(word);
+    const int n = __reduce_add_sync(0xffffffffu, c);
+    // exclusive offset of the lane's tokens in the row window's list
+    // (lane order, then bit order)
+    int o = 0;
+    if (n <= 128) {
+        o = c;
+#pragma unroll
+        for (int d = 1; d < 32; d <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, o, d);
+            if (lane >= d) o += y;
+        }
+        o -= c;
+    }
+    if (n <= 32) {
+        // few allowed tokens: listed one per lane, one logit load per lane
+        __syncwarp();
+        uint32_t wd = word;
+        int oo = o;
+        while (wd) {
+            const int e = __ffs(wd) - 1;
+            wd &= wd - 1;
+            mrow[oo++] = (uint32_t)(lane * 32 + e);
+        }
+        __syncwarp();
+        int t = INT_MAX;
+        unsigned short raw = 0;
+        if (lane < n) {
+            t = w * kWin + (int)mrow[lane];
+            raw = __ldcs(u + t);
+        }
+        fold_listed(out, raw, t, lane);
+    } else if (n <= 128) {
+        // up to four tokens per lane: listed (16-bit entries, two
+        // rounds of 64) and loaded together, then a lane-local
+        // maximum, the warp's argmax and the warp's sum
+        unsigned short* lst = reinterpret_cast<unsigned short*>(mrow);
+        int tk[4];
+        unsigned short raw[4];
+        uint32_t wd = word;
+        int oo = o;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            __syncwarp();
+            while (wd && oo < 64 * (h + 1)) {
+                const int e = __ffs(wd) - 1;
+                wd &= wd - 1;
+                lst[oo++ - 64 * h] = (unsigned short)(lane * 32 + e);
+            }
+            __syncwarp();
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+                const int k = 64 * h + 32 * q + lane;
+                tk[2 * h + q] = k < n ? w * kWin + (int)lst[k - 64 * h] : INT_MAX;
+                raw[2 * h + q] = k < n ? __ldcs(u + tk[2 * h + q]) : (unsigned short)0;
+            }
+        }
+        float m = -INFINITY;
+        int idx = INT_MAX;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {   // tokens ascend with q
+            const float x = __uint_as_float((uint32_t)raw[q] << 16);
+            if (tk[q] != INT_MAX && x > m) {
+                m = x;
+                idx = tk[q];
+            }
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+            const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+            const int i2 = __shfl_xor_sync(0xffffffffu, idx, off);
+            if (m2 > m || (m2 == m && i2 < idx)) {
+                m = m2;
+                idx = i2;
+            }
+        }
+        const float mL = m * kLog2e;
+        float sum = 0.0f;
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+            if (tk[q] != INT_MAX) sum += ex2(fmaf(__uint_as_float((uint32_t)raw[q] << 16), kLog2e, -mL));
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+        if (lane == 0)
+            *out = make_float4(m, __int_as_float(idx), sum, 0.f);
+    } else {
+        float m = -INFINITY, mL = -INFINITY, sum = 0.0f;
+        int idx = INT_MAX;
+        uint32_t wd = word;
+        const int t0 = j * 32;
+        if (wd && j < full_words) {
+            // many allowed tokens: each lane folds its own word, the
+            // word's four 16-byte vectors loaded at once; compact
+            // loops, since where masks are sparse this path runs
+            // rarely and its code is fetched cold
+            const uint4* src = reinterpret_cast<const uint4*>(lrow) + (size_t)j * 4;
+            const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+            const uint4 q0 = (wd & 0xFFu) ? __ldcs(src) : z;
+            const uint4 q1 = (wd & 0xFF00u) ? __ldcs(src + 1) : z;
+            const uint4 q2 = (wd & 0xFF0000u) ? __ldcs(src + 2) : z;
+            const uint4 q3 = (wd & 0xFF000000u) ? __ldcs(src + 3) : z;
+            // the word's maximum (lowest index on ties), then the sum of
+            // its terms: no dependence chain through the exponentials
+            int wi = 0;
+#pragma unroll 1
+            for (int k = 0; k < 4; ++k) {
+                const uint32_t bits = (wd >> (8 * k)) & 0xFFu;
+                const uint4 q = k == 0 ? q0 : k == 1 ? q1 : k == 2 ? q2 : q3;
+                const uint32_t qs[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const float x = (e & 1) ? bf16_hi(qs[e >> 1]) : bf16_lo(qs[e >> 1]);
+                    if (((bits >> e) & 1u) && x > m) {
+                        m = x;
+                        wi = 8 * k + e;
+                    }
+                }
+            }
+            mL = m * kLog2e;
+            idx = t0 + wi;
+#pragma unroll 1
+            for (int k = 0; k < 4; ++k) {
+                const uint32_t bits = (wd >> (8 * k)) & 0xFFu;
+                const uint4 q = k == 0 ? q0 : k == 1 ? q1 : k == 2 ? q2 : q3;
+                const uint32_t qs[4] = {q.x, q.y, q.z, q.w};
+                float acc = 0.0f;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const float x = (e & 1) ? bf16_hi(qs[e >> 1]) : bf16_lo(qs[e >> 1]);
+                    acc += ((bits >> e) & 1u) ? ex2(fmaf(x, kLog2e, -mL)) : 0.0f;
+                }
+                sum += acc;
+            }
+        } else {   // the row's partial last word
+            while (wd) {
+                const int e = __ffs(wd) - 1;
+                wd &= wd - 1;
+                if (t0 + e < V)
+                    acc_add(m, mL, idx, sum, __uint_as_float((uint32_t)__ldcs(u + t0 + e) << 16), t0 + e);
+            }
+        }
+        warp_merge(m, idx, sum);
+        if (lane == 0)
+            *out = make_float4(m, __int_as_float(idx), sum, 0.f);
+    }
 }
 
 struct FuseArgs {
@@ -225,7 +385,7 @@ __host__ __device__ inline StepLayout step_layout(int K, int R, bool next, bool 
     L.rows = o;    o += R * 16;
     L.ctrl = o;    o += 16;
     L.cfg = o;     o += align16(R * K * (stack ? 16 : 4));
-    L.mtile = o;   o += align16(R * 32 * 4);
+    L.mtile = o;   o += align16(R * 32 * 4) * (next ? 1 : 2);   // mask only: two tiles, see step_kernel
     L.ntile = o;   o += next ? R * kWin * 2 : 0;   // next states < Q <= 65535: staged as u16
     L.accept = o;  o += align16(((Q + 31) / 32) * 4);
     L.self = o;    o += self ? align16(Q * 8) : 0;
@@ -400,7 +560,7 @@ __global__ void __launch_bounds__(kStepThreads, 1)
     uint16_t* s_cls = reinterpret_cast<uint16_t*>(smem + L.cls);      // [K + 1] first slot of each first class
     uint32_t* s_pairs = reinterpret_cast<uint32_t*>(smem + L.pairs);   // walk pairs of the tile
     uint4* s_rows = reinterpret_cast<uint4*>(smem + L.rows);
-    int* s_ctrl = reinterpret_cast<int*>(smem + L.ctrl);   // -, pairs listed, EOS slot, -
+    int* s_ctrl = reinterpret_cast<int*>(smem + L.ctrl);   // rows drained, pairs listed, EOS slot, last rows drained
     uint32_t* s_cfg = reinterpret_cast<uint32_t*>(smem + L.cfg);   // [R][K] state (DFA)
     uint4* s_cfg4 = reinterpret_cast<uint4*>(smem + L.cfg);        // [R][K] (state, bits, depth) (pushdown)
     uint32_t* s_mtile = reinterpret_cast<uint32_t*>(smem + L.mtile);
@@ -462,15 +622,45 @@ __global__ void __launch_bounds__(kStepThreads, 1)
     };
     prefetch(t0);
     int cur_w = -1;
-    // a sparse fold in flight (fused decode): partial slot (-1: none), the
-    // lane's token (INT_MAX: none) and its raw bf16 logit
-    int p_slot = -1, p_t = INT_MAX;
-    unsigned short p_raw = 0;
+    // Mask only (no next states): the mask tile is double-buffered and a
+    // tile's write-out and masked decode run in the next tile's walk interval,
+    // a row at a time to whichever warp asks next (warps that finish walking
+    // early take them); the last tile's after the loop.  pw / pr0 / pnr: the
+    // previous tile's window, first row and row count.
+    int pw = 0, pr0 = 0, pnr = 0;
+    // the previous tile's rows: each warp that asks takes one, writes its 32
+    // mask words out, folds its allowed logits (fused decode) and clears the
+    // words for the tile after next
+    auto drain = [&](int tp, int* counter) {
+        uint32_t* pm = s_mtile + (tp & 1) * R * 32;
+        for (;;) {
+            int r = 0;
+            if (lane == 0) r = atomicAdd(counter, 1);
+            r = __shfl_sync(0xffffffffu, r, 0);
+            if (r >= pnr) break;
+            const int j = pw * 32 + lane;
+            if (mask && j < v.W) mask[(size_t)(pr0 + r) * v.W + j] = pm[r * 32 + lane];
+            if (fuse.logits)
+                fold_window(pm + r * 32, reinterpret_cast<const char*>(fuse.logits) + (size_t)(pr0 + r) * fuse.stride * 2,
+                            pw, v.V, v.W, lane, fuse.part + (size_t)(pr0 + r) * v.n_windows + pw);
+            __syncwarp();
+            pm[r * 32 + lane] = 0u;
+        }
+    };
+    if constexpr (!NEXT) {
+        for (int i = tid; i < 2 * R * 32; i += kStepThreads) s_mtile[i] = 0u;
+        if (tid == 0) s_ctrl[3] = 0;   // the last tile's row counter
+    }
     for (int t = t0; t < t1; ++t) {
         const int w = t / n_row_tiles;
         const int r0 = (t - w * n_row_tiles) * R;
         const int nr = min(R, batch - r0);
-        __syncthreads();   // the previous tile is fully consumed
+        uint32_t* mt = s_mtile + (NEXT ? 0 : (t & 1) * R * 32);   // this tile's mask words [R][32]
+        __syncthreads();   // the previous tile's walk is done
+        if (tid == 0) {
+            s_ctrl[0] = 0;   // rows of the previous tile handed out
+            s_ctrl[1] = 0;   // pairs listed so far
+        }
         if (w != cur_w) {
             s_head[2 * tid] = __ldg(v.head + 2 * ((size_t)w * kWin + tid));
             s_head[2 * tid + 1] = __ldg(v.head + 2 * ((size_t)w * kWin + tid) + 1);
@@ -488,8 +678,8 @@ __global__ void __launch_bounds__(kStepThreads, 1)
                 s_rows[tid] = decode_row(v, pf_s, pf_w, stacks != nullptr, s_accept, w == 0);
             }
         }
-        if (tid == 0) s_ctrl[1] = 0;   // pairs listed so far
-        for (int i = tid; i < nr * 32; i += kStepThreads) s_mtile[i] = 0u;
+        if constexpr (NEXT)
+            for (int i = tid; i < nr * 32; i += kStepThreads) mt[i] = 0u;
         if (fuse.prefetch) {
             // the tile's logits head for L2 while the walk runs: one 128-byte
             // line per thread, every line start inside the row's window slice
@@ -554,7 +744,7 @@ __global__ void __launch_bounds__(kStepThreads, 1)
         const int eos_local = s_ctrl[2];
         if (tid < nr && eos_local >= 0 && (s_rows[tid].w & 2u)) {
             const int ol = (int)(s_info[eos_local] & 1023u);
-            atomicOr(&s_mtile[tid * 32 + (ol >> 5)], 1u << (ol & 31));
+            atomicOr(&mt[tid * 32 + (ol >> 5)], 1u << (ol & 31));
             if constexpr (NEXT) s_ntile[tid * kWin + ol] = (uint16_t)s_rows[tid].x;
         }
         __syncthreads();
@@ -605,185 +795,27 @@ __global__ void __launch_bounds__(kStepThreads, 1)
 #pragma unroll
                     for (int k = 0; k < kWalkChains; ++k) {
                         if (rr[k] >= 0 && sv[k]) {
-                            atomicOr(&s_mtile[rr[k] * 32 + (ol >> 5)], 1u << (ol & 31));
+                            atomicOr(&mt[rr[k] * 32 + (ol >> 5)], 1u << (ol & 31));
                             if constexpr (NEXT) s_ntile[rr[k] * kWin + ol] = (uint16_t)sv[k];
                         }
                     }
                 }
             }
         }
-        __syncthreads();
-
-        // coalesced write-out in original-id order
-        if (mask) {
-            for (int i = tid; i < nr * 32; i += kStepThreads) {
-                const int r = i >> 5, word = w * 32 + (i & 31);
-                if (word < v.W) mask[(size_t)(r0 + r) * v.W + word] = s_mtile[i];
-            }
-        }
-        if constexpr (!NEXT) {
-            if (fuse.logits) {
-                if (p_slot >= 0) {   // the previous tile's sparse fold, its loads landed
-                    fold_pending(fuse.part, p_slot, p_raw, p_t, lane);
-                    p_slot = -1;
-                }
-                // the masked decode of this tile: warp r folds row r of the window
-                // (the write-out above gave row r's words to warp r alone, so
-                // the warp may reuse that row of the tile as scratch)
-                const int full_words = v.V / 32;
-                for (int r = warp; r < nr; r += kStepThreads / 32) {
-                    const int j = w * 32 + lane;
-                    const uint32_t word = j < v.W ? s_mtile[r * 32 + lane] : 0u;
-                    const int c = __popc(word);
-                    const int n = __reduce_add_sync(0xffffffffu, c);
-                    const char* lrow = reinterpret_cast<const char*>(fuse.logits) + (size_t)(r0 + r) * fuse.stride * 2;
-                    const unsigned short* u = reinterpret_cast<const unsigned short*>(lrow);
-                    // exclusive offset of the lane's tokens in the row window's list
-                    // (lane order, then bit order)
-                    int o = 0;
-                    if (n <= 128) {
-                        o = c;
-#pragma unroll
-                        for (int d = 1; d < 32; d <<= 1) {
-                            const int y = __shfl_up_sync(0xffffffffu, o, d);
-                            if (lane >= d) o += y;
-                        }
-                        o -= c;
-                    }
-                    if (n <= 32) {
-                        // few allowed tokens: listed one per lane, the logit loaded
-                        // now and folded after the next tile's walk (fold_pending),
-                        // which hides the load's latency
-                        __syncwarp();
-                        uint32_t wd = word;
-                        int oo = o;
-                        while (wd) {
-                            const int e = __ffs(wd) - 1;
-                            wd &= wd - 1;
-                            s_mtile[r * 32 + oo++] = (uint32_t)(lane * 32 + e);
-                        }
-                        __syncwarp();
-                        p_t = INT_MAX;
-                        if (lane < n) {
-                            p_t = w * kWin + (int)s_mtile[r * 32 + lane];
-                            p_raw = __ldcs(u + p_t);
-                        }
-                        p_slot = (r0 + r) * v.n_windows + w;
-                    } else if (n <= 128) {
-                        // up to four tokens per lane: listed (16-bit entries, two
-                        // rounds of 64) and loaded together, then a lane-local
-                        // maximum, the warp's argmax and the warp's sum
-                        unsigned short* lst = reinterpret_cast<unsigned short*>(s_mtile + r * 32);
-                        int tk[4];
-                        unsigned short raw[4];
-                        uint32_t wd = word;
-                        int oo = o;
-#pragma unroll
-                        for (int h = 0; h < 2; ++h) {
-                            __syncwarp();
-                            while (wd && oo < 64 * (h + 1)) {
-                                const int e = __ffs(wd) - 1;
-                                wd &= wd - 1;
-                                lst[oo++ - 64 * h] = (unsigned short)(lane * 32 + e);
-                            }
-                            __syncwarp();
-#pragma unroll
-                            for (int q = 0; q < 2; ++q) {
-                                const int k = 64 * h + 32 * q + lane;
-                                tk[2 * h + q] = k < n ? w * kWin + (int)lst[k - 64 * h] : INT_MAX;
-                                raw[2 * h + q] = k < n ? __ldcs(u + tk[2 * h + q]) : (unsigned short)0;
-                            }
-                        }
-                        float m = -INFINITY;
-                        int idx = INT_MAX;
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) {   // tokens ascend with q
-                            const float x = __uint_as_float((uint32_t)raw[q] << 16);
-                            if (tk[q] != INT_MAX && x > m) {
-                                m = x;
-                                idx = tk[q];
-                            }
-                        }
-#pragma unroll
-                        for (int off = 16; off > 0; off >>= 1) {
-                            const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
-                            const int i2 = __shfl_xor_sync(0xffffffffu, idx, off);
-                            if (m2 > m || (m2 == m && i2 < idx)) {
-                                m = m2;
-                                idx = i2;
-                            }
-                        }
-                        const float mL = m * kLog2e;
-                        float sum = 0.0f;
-#pragma unroll
-                        for (int q = 0; q < 4; ++q)
-                            if (tk[q] != INT_MAX) sum += ex2(fmaf(__uint_as_float((uint32_t)raw[q] << 16), kLog2e, -mL));
-#pragma unroll
-                        for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
-                        if (lane == 0)
-                            fuse.part[(size_t)(r0 + r) * v.n_windows + w] = make_float4(m, __int_as_float(idx), sum, 0.f);
-                    } else {
-                        float m = -INFINITY, mL = -INFINITY, sum = 0.0f;
-                        int idx = INT_MAX;
-                        uint32_t wd = word;
-                        const int t0 = j * 32;
-                        if (wd && j < full_words) {
-                            // many allowed tokens: each lane folds its own word, the
-                            // word's four 16-byte vectors loaded at once; compact
-                            // loops, since where masks are sparse this path runs
-                            // rarely and its code is fetched cold
-                            const uint4* src = reinterpret_cast<const uint4*>(lrow) + (size_t)j * 4;
-                            const uint4 z = make_uint4(0u, 0u, 0u, 0u);
-                            const uint4 q0 = (wd & 0xFFu) ? __ldcs(src) : z;
-                            const uint4 q1 = (wd & 0xFF00u) ? __ldcs(src + 1) : z;
-                            const uint4 q2 = (wd & 0xFF0000u) ? __ldcs(src + 2) : z;
-                            const uint4 q3 = (wd & 0xFF000000u) ? __ldcs(src + 3) : z;
-                            // the word's maximum (lowest index on ties), then the sum of
-                            // its terms: no dependence chain through the exponentials
-                            int wi = 0;
-#pragma unroll 1
-                            for (int k = 0; k < 4; ++k) {
-                                const uint32_t bits = (wd >> (8 * k)) & 0xFFu;
-                                const uint4 q = k == 0 ? q0 : k == 1 ? q1 : k == 2 ? q2 : q3;
-                                const uint32_t qs[4] = {q.x, q.y, q.z, q.w};
-#pragma unroll
-                                for (int e = 0; e < 8; ++e) {
-                                    const float x = (e & 1) ? bf16_hi(qs[e >> 1]) : bf16_lo(qs[e >> 1]);
-                                    if (((bits >> e) & 1u) && x > m) {
-                                        m = x;
-                                        wi = 8 * k + e;
-                                    }
-                                }
-                            }
-                            mL = m * kLog2e;
-                            idx = t0 + wi;
-#pragma unroll 1
-                            for (int k = 0; k < 4; ++k) {
-                                const uint32_t bits = (wd >> (8 * k)) & 0xFFu;
-                                const uint4 q = k == 0 ? q0 : k == 1 ? q1 : k == 2 ? q2 : q3;
-                                const uint32_t qs[4] = {q.x, q.y, q.z, q.w};
-                                float acc = 0.0f;
-#pragma unroll
-                                for (int e = 0; e < 8; ++e) {
-                                    const float x = (e & 1) ? bf16_hi(qs[e >> 1]) : bf16_lo(qs[e >> 1]);
-                                    acc += ((bits >> e) & 1u) ? ex2(fmaf(x, kLog2e, -mL)) : 0.0f;
-                                }
-                                sum += acc;
-                            }
-                        } else {   // the row's partial last word
-                            while (wd) {
-                                const int e = __ffs(wd) - 1;
-                                wd &= wd - 1;
-                                if (t0 + e < v.V)
-                                    acc_add(m, mL, idx, sum, __uint_as_float((uint32_t)__ldcs(u + t0 + e) << 16), t0 + e);
-                            }
-                        }
-                        warp_merge(m, idx, sum);
-                        if (lane == 0)
-                            fuse.part[(size_t)(r0 + r) * v.n_windows + w] = make_float4(m, __int_as_float(idx), sum, 0.f);
-                    }
+        if constexpr (NEXT) {
+            __syncthreads();
+            // coalesced write-out in original-id order
+            if (mask) {
+                for (int i = tid; i < nr * 32; i += kStepThreads) {
+                    const int r = i >> 5, word = w * 32 + (i & 31);
+                    if (word < v.W) mask[(size_t)(r0 + r) * v.W + word] = mt[i];
                 }
             }
+        } else {
+            if (t > t0) drain(t - 1, &s_ctrl[0]);
+            pw = w;
+            pr0 = r0;
+            pnr = nr;
         }
         if constexpr (NEXT) {
             const int in_win = min(kWin, v.V - w * kWin);
@@ -806,7 +838,10 @@ __global__ void __launch_bounds__(kStepThreads, 1)
         }
     }
     if constexpr (!NEXT) {
-        if (p_slot >= 0) fold_pending(fuse.part, p_slot, p_raw, p_t, lane);
+        if (t1 > t0) {
+            __syncthreads();   // the last tile's walk is done
+            drain(t1 - 1, &s_ctrl[3]);
+        }
     }
 }
 
