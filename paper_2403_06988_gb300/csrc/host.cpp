@@ -732,6 +732,7 @@ int domino_step_decode(domino_t h, const int32_t* states_dev, const uint64_t* st
     const size_t part_bytes = (size_t)batch * (size_t)h->n_windows * sizeof(float4);
     if (h->d_fpart.n < part_bytes) {
         if (cudaStreamSynchronize(st) != cudaSuccess) return cuda_status(cudaGetLastError());
+        clear_host_graphs(h);   // recorded host-buffer steps name this buffer
         if ((rc = dev_reserve(h->d_fpart, part_bytes))) return rc;
     }
     // logits in device memory are pulled into L2 a tile ahead of their fold;
