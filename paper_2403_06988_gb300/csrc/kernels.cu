@@ -383,7 +383,7 @@ __host__ __device__ inline StepLayout step_layout(int K, int R, bool next, bool 
     L.tokcls = o;  o += self ? kWin * 8 : 0;
     L.pairs = o;   o += kWin * ((R + kWalkChains - 1) / kWalkChains) * 4;
     L.rows = o;    o += R * 16;
-    L.ctrl = o;    o += 16;
+    L.ctrl = o;    o += 32;
     L.cfg = o;     o += align16(R * K * (stack ? 16 : 4));
     L.mtile = o;   o += align16(R * 32 * 4) * (next ? 1 : 2);   // mask only: two tiles, see step_kernel
     L.ntile = o;   o += next ? R * kWin * 2 : 0;   // next states < Q <= 65535: staged as u16
@@ -560,7 +560,8 @@ __global__ void __launch_bounds__(kStepThreads, 1)
     uint16_t* s_cls = reinterpret_cast<uint16_t*>(smem + L.cls);      // [K + 1] first slot of each first class
     uint32_t* s_pairs = reinterpret_cast<uint32_t*>(smem + L.pairs);   // walk pairs of the tile
     uint4* s_rows = reinterpret_cast<uint4*>(smem + L.rows);
-    int* s_ctrl = reinterpret_cast<int*>(smem + L.ctrl);   // rows drained, pairs listed, EOS slot, last rows drained
+    // rows drained, pairs listed, EOS slot, last rows drained, chunks claimed
+    int* s_ctrl = reinterpret_cast<int*>(smem + L.ctrl);
     uint32_t* s_cfg = reinterpret_cast<uint32_t*>(smem + L.cfg);   // [R][K] state (DFA)
     uint4* s_cfg4 = reinterpret_cast<uint4*>(smem + L.cfg);        // [R][K] (state, bits, depth) (pushdown)
     uint32_t* s_mtile = reinterpret_cast<uint32_t*>(smem + L.mtile);
@@ -660,6 +661,7 @@ __global__ void __launch_bounds__(kStepThreads, 1)
         if (tid == 0) {
             s_ctrl[0] = 0;   // rows of the previous tile handed out
             s_ctrl[1] = 0;   // pairs listed so far
+            s_ctrl[4] = 0;   // chunks of 32 pairs claimed
         }
         if (w != cur_w) {
             s_head[2 * tid] = __ldg(v.head + 2 * ((size_t)w * kWin + tid));
@@ -751,7 +753,18 @@ __global__ void __launch_bounds__(kStepThreads, 1)
 
         prefetch(t + 1);
         const int n_pairs = s_ctrl[1];
-        for (int p0 = warp * 32; p0 < n_pairs; p0 += kStepThreads) {
+        // chunks of 32 pairs: round-robin over the warps, or, for a pushdown
+        // automaton (the self-loop skip and the long walks inside strings make
+        // chunk times vary) with many chunks per warp, to whichever warp
+        // claims the next one
+        const bool claim = STACK && n_pairs > 4 * kStepThreads;
+        auto next_chunk = [&](int p) {
+            if (!claim) return p + kStepThreads;
+            int c = 0;
+            if (lane == 0) c = atomicAdd(&s_ctrl[4], 1);
+            return __shfl_sync(0xffffffffu, c, 0) * 32;
+        };
+        for (int p0 = claim ? next_chunk(0) : warp * 32; p0 < n_pairs; p0 = next_chunk(p0)) {
             const bool active = p0 + lane < n_pairs;
             const uint32_t pr = active ? s_pairs[p0 + lane] : 0u;
             const int slot = (int)(pr & 1023u);
