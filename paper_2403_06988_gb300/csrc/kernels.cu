@@ -137,27 +137,6 @@ __device__ __forceinline__ void warp_merge(float& m, int& idx, float& s) {
     }
 }
 
-// CTA-wide (m, idx, s); the result is valid in thread 0.  Uses two barriers.
-__device__ __forceinline__ void block_merge(float& m, int& idx, float& s) {
-    __shared__ float sm_m[kLogitThreads / 32], sm_s[kLogitThreads / 32];
-    __shared__ int sm_i[kLogitThreads / 32];
-    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-    warp_merge(m, idx, s);
-    __syncthreads();   // protect sm_* against the previous call's readers
-    if (lane == 0) {
-        sm_m[wid] = m;
-        sm_i[wid] = idx;
-        sm_s[wid] = s;
-    }
-    __syncthreads();
-    if (wid == 0) {
-        m = lane < kLogitThreads / 32 ? sm_m[lane] : -INFINITY;
-        idx = lane < kLogitThreads / 32 ? sm_i[lane] : INT_MAX;
-        s = lane < kLogitThreads / 32 ? sm_s[lane] : 0.0f;
-        warp_merge(m, idx, s);
-    }
-}
-
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
@@ -392,11 +371,6 @@ __host__ __device__ inline StepLayout step_layout(int K, int R, bool next, bool 
     L.table = o;   o += align16(table_bytes);
     L.total = o;
     return L;
-}
-
-__device__ __forceinline__ uint32_t head_byte(const uint4& h, int i) {
-    uint32_t w = (i < 4) ? h.x : (i < 8) ? h.y : (i < 12) ? h.z : h.w;
-    return (w >> (8 * (i & 3))) & 0xFFu;
 }
 
 // Transition lookup for the four table modes.
