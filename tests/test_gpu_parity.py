@@ -506,7 +506,7 @@ def test_ragged_vocab_long_tokens_eos_in_middle():
     toks = set()
     while len(toks) < 2500:
         L = int(rng.integers(1, 40))
-        toks.add(bytes(rng.choice(list(b"-0123456789x"), L)))
+        toks.add(rng.choice(np.frombuffer(b"-0123456789x", np.uint8), L).tobytes())
     toks = sorted(toks)
     toks.insert(700, b"")          # EOS
     toks.insert(1500, b"")         # an empty token that is not EOS
