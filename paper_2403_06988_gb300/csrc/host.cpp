@@ -13,6 +13,8 @@
 #include <unordered_map>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "domino.h"
 #include "domino_internal.h"
 
@@ -293,6 +295,17 @@ int cuda_status(cudaError_t e) {
     return DOMINO_E_CUDA;
 }
 
+// An NVTX range named after each C ABI call that does work (a no-op unless a
+// profiler is attached), so that a timeline shows the library's calls above
+// the kernels they launch.
+struct ApiRange {
+    explicit ApiRange(const char* name) { nvtxRangePushA(name); }
+    ~ApiRange() { nvtxRangePop(); }
+    ApiRange(const ApiRange&) = delete;
+    ApiRange& operator=(const ApiRange&) = delete;
+};
+#define DOMINO_API_RANGE() const ApiRange api_range_(__func__)
+
 }  // namespace
 
 extern "C" {
@@ -374,6 +387,7 @@ int domino_destroy(domino_t h) {
 
 int domino_load_vocab(domino_t h, const uint8_t* bytes, const int64_t* offsets, int32_t n_tokens,
                       int32_t eos_id) {
+    DOMINO_API_RANGE();
     if (h) clear_host_graphs(h);
     if (!h || !offsets || n_tokens < 1 || n_tokens > (1 << 24)) return DOMINO_E_INVALID_ARG;
     if (eos_id < -1 || eos_id >= n_tokens || offsets[0] != 0) return DOMINO_E_INVALID_ARG;
@@ -404,6 +418,7 @@ int domino_load_vocab(domino_t h, const uint8_t* bytes, const int64_t* offsets, 
 int domino_load_automaton(domino_t h, const int32_t* delta, int32_t n_states, const uint8_t* live,
                           const uint8_t* accepting, int32_t start_state, const domino_stack_rule* rules,
                           int32_t n_rules, int32_t max_depth) {
+    DOMINO_API_RANGE();
     if (!h || !delta || !live || n_states < 1 || n_states > DOMINO_MAX_STATES) return DOMINO_E_INVALID_ARG;
     if (start_state < 0 || start_state >= n_states || max_depth < 0 || max_depth > DOMINO_MAX_DEPTH)
         return DOMINO_E_INVALID_ARG;
@@ -649,6 +664,7 @@ int domino_get_byte_classes(domino_t h, uint8_t* classes_out) {
 
 int domino_step_mask(domino_t h, const int32_t* states_dev, const uint64_t* stacks_dev, int32_t batch,
                      uint32_t* mask_dev, int32_t* next_dev, void* stream) {
+    DOMINO_API_RANGE();
     int rc = ready_for_compute(h);
     if (rc) return rc;
     if (batch < 0 || (batch > 0 && (!states_dev || !mask_dev))) return DOMINO_E_INVALID_ARG;
@@ -661,6 +677,7 @@ int domino_step_mask(domino_t h, const int32_t* states_dev, const uint64_t* stac
 }
 
 int domino_precompute_table(domino_t h, int32_t* next_dev, uint32_t* mask_dev, void* stream) {
+    DOMINO_API_RANGE();
     int rc = ready_for_compute(h);
     if (rc) return rc;
     if (!next_dev && !mask_dev) return DOMINO_E_INVALID_ARG;
@@ -675,6 +692,7 @@ int domino_precompute_table(domino_t h, int32_t* next_dev, uint32_t* mask_dev, v
 int domino_mask_logits(domino_t h, const void* logits_dev, int32_t dtype, int32_t batch,
                        int64_t row_stride_elems, const uint32_t* mask_dev, int32_t* argmax_dev, float* lse_dev,
                        float* logprobs_dev, void* stream) {
+    DOMINO_API_RANGE();
     if (!h) return DOMINO_E_INVALID_ARG;
     if (is_host_only(h)) return DOMINO_E_NO_DEVICE;
     if (!h->vocab_loaded) return DOMINO_E_NOT_LOADED;
@@ -691,6 +709,7 @@ int domino_mask_logits(domino_t h, const void* logits_dev, int32_t dtype, int32_
 
 int domino_advance(domino_t h, const int32_t* states_dev, const uint64_t* stacks_dev, const int32_t* tokens_dev,
                    int32_t batch, int32_t* states_out, uint64_t* stacks_out, void* stream) {
+    DOMINO_API_RANGE();
     int rc = ready_for_compute(h);
     if (rc) return rc;
     if (batch < 0) return DOMINO_E_INVALID_ARG;
@@ -707,6 +726,7 @@ int domino_step_decode(domino_t h, const int32_t* states_dev, const uint64_t* st
                        const void* logits_dev, int32_t dtype, int64_t row_stride_elems, uint32_t* mask_dev,
                        int32_t* argmax_dev, float* lse_dev, float* logprobs_dev, int32_t* states_out,
                        uint64_t* stacks_out, void* stream) {
+    DOMINO_API_RANGE();
     int rc = ready_for_compute(h);
     if (rc) return rc;
     if (dtype != DOMINO_DTYPE_F32 && dtype != DOMINO_DTYPE_BF16) return DOMINO_E_INVALID_ARG;
@@ -757,6 +777,7 @@ int domino_step_decode(domino_t h, const int32_t* states_dev, const uint64_t* st
 int domino_mask_sample(domino_t h, const void* logits_dev, int32_t dtype, int32_t batch, int64_t row_stride_elems,
                        const uint32_t* mask_dev, float temperature, uint64_t seed, uint64_t offset,
                        int32_t* tokens_dev, void* stream) {
+    DOMINO_API_RANGE();
     if (!h) return DOMINO_E_INVALID_ARG;
     if (is_host_only(h)) return DOMINO_E_NO_DEVICE;
     if (!h->vocab_loaded) return DOMINO_E_NOT_LOADED;
@@ -776,6 +797,7 @@ int domino_opportunistic_step(domino_t h, const void* logits_dev, int32_t dtype,
                               int64_t row_stride_elems, const int32_t* states_dev, const uint64_t* stacks_dev,
                               uint32_t* mask_scratch_dev, int32_t* tokens_dev, int32_t* n_fallback_dev,
                               void* stream) {
+    DOMINO_API_RANGE();
     int rc = ready_for_compute(h);
     if (rc) return rc;
     if (dtype != DOMINO_DTYPE_F32 && dtype != DOMINO_DTYPE_BF16) return DOMINO_E_INVALID_ARG;
@@ -817,6 +839,7 @@ int domino_opportunistic_step(domino_t h, const void* logits_dev, int32_t dtype,
 int domino_spec_update(domino_t h, uint32_t* counts_dev, uint64_t* best_dev, uint32_t* reached_dev,
                        const int32_t* states_dev, const uint64_t* stacks_dev, const int32_t* tokens_dev,
                        int32_t batch, void* stream) {
+    DOMINO_API_RANGE();
     int rc = ready_for_compute(h);
     if (rc) return rc;
     if (batch < 0) return DOMINO_E_INVALID_ARG;
@@ -832,6 +855,7 @@ int domino_spec_propose(domino_t h, const uint64_t* best_dev, const uint32_t* re
                         const int32_t* states_dev, const uint64_t* stacks_dev, int32_t batch, int32_t s,
                         int32_t min_permille, int32_t* proposals_dev, int32_t* n_prop_dev,
                         int32_t* chain_states_dev, uint64_t* chain_stacks_dev, void* stream) {
+    DOMINO_API_RANGE();
     int rc = ready_for_compute(h);
     if (rc) return rc;
     if (batch < 0 || s < 1 || min_permille < 0 || min_permille > 1000) return DOMINO_E_INVALID_ARG;
@@ -851,6 +875,7 @@ int domino_spec_accept(domino_t h, const int32_t* proposals_dev, const int32_t* 
                        const int32_t* decoded_dev, const int32_t* chain_states_dev, const uint64_t* chain_stacks_dev,
                        int32_t batch, int32_t s, int32_t* n_accept_dev, int32_t* tokens_out_dev,
                        int32_t* states_out_dev, uint64_t* stacks_out_dev, void* stream) {
+    DOMINO_API_RANGE();
     if (!h) return DOMINO_E_INVALID_ARG;
     if (is_host_only(h)) return DOMINO_E_NO_DEVICE;
     if (batch < 0 || s < 1) return DOMINO_E_INVALID_ARG;
@@ -866,6 +891,7 @@ int domino_spec_accept(domino_t h, const int32_t* proposals_dev, const int32_t* 
 int domino_mask_logits_table(domino_t h, const void* logits_dev, int32_t dtype, int32_t batch,
                              int64_t row_stride_elems, const uint32_t* table_mask_dev, const int32_t* states_dev,
                              int32_t* argmax_dev, float* lse_dev, float* logprobs_dev, void* stream) {
+    DOMINO_API_RANGE();
     int rc = ready_for_compute(h);
     if (rc) return rc;
     if (h->stack) return DOMINO_E_UNSUPPORTED;
@@ -882,6 +908,7 @@ int domino_mask_logits_table(domino_t h, const void* logits_dev, int32_t dtype, 
 
 int domino_advance_table(domino_t h, const int32_t* table_next_dev, const int32_t* states_dev,
                          const int32_t* tokens_dev, int32_t batch, int32_t* states_out, void* stream) {
+    DOMINO_API_RANGE();
     int rc = ready_for_compute(h);
     if (rc) return rc;
     if (h->stack) return DOMINO_E_UNSUPPORTED;
@@ -995,6 +1022,7 @@ int enqueue_host_step(domino_ctx* h, const void* logits_host, void* logits_mappe
 int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, int32_t batch,
                             int32_t* states_host, uint64_t* stacks_host, int32_t* tokens_host, float* lse_host,
                             void* stream) {
+    DOMINO_API_RANGE();
     int rc = ready_for_compute(h);
     if (rc) return rc;
     if (dtype != DOMINO_DTYPE_F32 && dtype != DOMINO_DTYPE_BF16) return DOMINO_E_INVALID_ARG;
