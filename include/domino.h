@@ -200,7 +200,9 @@ int domino_advance(domino_t h, const int32_t* states_dev, const uint64_t* stacks
  * The fused form needs bf16 rows on 16-byte boundaries; other inputs run the
  * two kernels one after the other.  Results equal domino_step_mask followed
  * by domino_mask_logits.  The first call with a larger batch allocates
- * scratch and synchronises `stream`. */
+ * scratch and synchronises `stream`; if `stream` is being captured into a
+ * CUDA graph at that point, the call returns DOMINO_E_INVALID_ARG and
+ * launches nothing (make one uncaptured call at the largest batch first). */
 int domino_step_decode(domino_t h, const int32_t* states_dev, const uint64_t* stacks_dev, int32_t batch,
                        const void* logits_dev, int32_t dtype, int64_t row_stride_elems, uint32_t* mask_dev,
                        int32_t* argmax_dev, float* lse_dev, float* logprobs_dev, int32_t* states_out,

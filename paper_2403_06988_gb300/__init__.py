@@ -16,7 +16,16 @@ from ._binding import DominoError, DTYPE_BF16, DTYPE_F32  # noqa: F401
 
 
 class Domino:
-    """One library handle: a vocabulary plus a scanner (+ bracket rules)."""
+    """One library handle: a vocabulary plus a scanner (+ bracket rules).
+
+    fill_byte: None (default), or a byte value that every output buffer this
+    holder allocates is filled with before the call that writes it.  A word a
+    kernel leaves unwritten then keeps that pattern (0xAB bytes, say) instead
+    of whatever the allocator handed back, so an exact comparison catches it.
+    A debugging aid; it costs one fill per output.
+    """
+
+    fill_byte: Optional[int] = None
 
     def __init__(self, device: int = 0):
         self.device = device
@@ -51,17 +60,23 @@ class Domino:
     def info(self) -> dict:
         return B.domino_get_info(self.h)
 
+    def _empty(self, shape, dtype, device):
+        import torch
+        t = torch.empty(shape, dtype=dtype, device=device)
+        if self.fill_byte is not None and t.numel():
+            t.view(torch.uint8).fill_(self.fill_byte)
+        return t
+
     # -- compute (torch tensors on this handle's device) -----------------------
     def step_mask(self, states, stacks=None, want_next: bool = False, out_mask=None, out_next=None,
                   stream=None):
         import torch
         info = self.info()
         b = states.shape[0]
-        mask = out_mask if out_mask is not None else torch.empty((b, info["n_words"]), dtype=torch.int32,
-                                                                 device=states.device)
+        mask = out_mask if out_mask is not None else self._empty((b, info["n_words"]), torch.int32, states.device)
         nxt = out_next
         if want_next and nxt is None:
-            nxt = torch.empty((b, info["n_tokens"]), dtype=torch.int32, device=states.device)
+            nxt = self._empty((b, info["n_tokens"]), torch.int32, states.device)
         B.domino_step_mask(self.h, states, stacks, b, mask, nxt, stream)
         return mask, nxt
 
@@ -76,12 +91,11 @@ class Domino:
             raise TypeError("logits must be float32 or bfloat16")
         if logits.stride(1) != 1:
             raise ValueError("logits rows must be contiguous")
-        mask = out_mask if out_mask is not None else torch.empty((b, self.info()["n_words"]), dtype=torch.int32,
-                                                                 device=states.device)
-        argmax = torch.empty(b, dtype=torch.int32, device=states.device)
-        lse = torch.empty(b, dtype=torch.float32, device=states.device)
-        lp = torch.empty((b, self.info()["n_tokens"]), dtype=torch.float32, device=states.device) if want_logprobs \
-            else None
+        mask = out_mask if out_mask is not None else self._empty((b, self.info()["n_words"]), torch.int32,
+                                                                 states.device)
+        argmax = self._empty(b, torch.int32, states.device)
+        lse = self._empty(b, torch.float32, states.device)
+        lp = self._empty((b, self.info()["n_tokens"]), torch.float32, states.device) if want_logprobs else None
         B.domino_step_decode(self.h, states, stacks, b, logits.data_ptr(), dtype, logits.stride(0), mask, argmax, lse,
                              lp, states if advance else None, stacks if advance else None, stream)
         return mask, argmax, lse, lp
@@ -90,8 +104,8 @@ class Domino:
         import torch
         info = self.info()
         dev = f"cuda:{self.device}"
-        nxt = torch.empty((info["n_states"], info["n_tokens"]), dtype=torch.int32, device=dev) if want_next else None
-        mask = torch.empty((info["n_states"], info["n_words"]), dtype=torch.int32, device=dev) if want_mask else None
+        nxt = self._empty((info["n_states"], info["n_tokens"]), torch.int32, dev) if want_next else None
+        mask = self._empty((info["n_states"], info["n_words"]), torch.int32, dev) if want_mask else None
         B.domino_precompute_table(self.h, nxt, mask, stream)
         return nxt, mask
 
@@ -107,11 +121,11 @@ class Domino:
             raise ValueError("logits rows must be contiguous")
         argmax, lse, lp = out if out is not None else (None, None, None)
         if argmax is None:
-            argmax = torch.empty(b, dtype=torch.int32, device=logits.device)
+            argmax = self._empty(b, torch.int32, logits.device)
         if want_lse and lse is None:
-            lse = torch.empty(b, dtype=torch.float32, device=logits.device)
+            lse = self._empty(b, torch.float32, logits.device)
         if want_logprobs and lp is None:
-            lp = torch.empty((b, V), dtype=torch.float32, device=logits.device)
+            lp = self._empty((b, V), torch.float32, logits.device)
         B.domino_mask_logits(self.h, logits.data_ptr(), dtype, b, logits.stride(0), mask, argmax,
                              lse if want_lse else None, lp if want_logprobs else None, stream)
         return argmax, (lse if want_lse else None), (lp if want_logprobs else None)
@@ -130,7 +144,7 @@ class Domino:
         dtype = DTYPE_BF16 if logits.dtype == torch.bfloat16 else DTYPE_F32
         if logits.stride(1) != 1:
             raise ValueError("logits rows must be contiguous")
-        tokens = torch.empty(b, dtype=torch.int32, device=logits.device)
+        tokens = self._empty(b, torch.int32, logits.device)
         B.domino_mask_sample(self.h, logits, dtype, b, logits.stride(0), mask, temperature, seed, offset, tokens,
                              stream)
         return tokens
@@ -143,8 +157,8 @@ class Domino:
         if logits.stride(1) != 1:
             raise ValueError("logits rows must be contiguous")
         W = self.info()["n_words"]
-        scratch = torch.empty((b, W), dtype=torch.int32, device=logits.device)
-        tokens = torch.empty(b, dtype=torch.int32, device=logits.device)
+        scratch = self._empty((b, W), torch.int32, logits.device)
+        tokens = self._empty(b, torch.int32, logits.device)
         n_fb = torch.zeros(1, dtype=torch.int32, device=logits.device)
         B.domino_opportunistic_step(self.h, logits, dtype, b, logits.stride(0), states, stacks, scratch, tokens, n_fb,
                                     stream)
@@ -159,9 +173,9 @@ class Domino:
         dtype = DTYPE_BF16 if logits.dtype == torch.bfloat16 else DTYPE_F32
         if logits.stride(1) != 1:
             raise ValueError("logits rows must be contiguous")
-        argmax = torch.empty(b, dtype=torch.int32, device=logits.device)
-        lse = torch.empty(b, dtype=torch.float32, device=logits.device) if want_lse else None
-        lp = torch.empty((b, V), dtype=torch.float32, device=logits.device) if want_logprobs else None
+        argmax = self._empty(b, torch.int32, logits.device)
+        lse = self._empty(b, torch.float32, logits.device) if want_lse else None
+        lp = self._empty((b, V), torch.float32, logits.device) if want_logprobs else None
         B.domino_mask_logits_table(self.h, logits, dtype, b, logits.stride(0), table_mask, states, argmax, lse, lp,
                                    stream)
         return argmax, lse, lp

@@ -751,6 +751,12 @@ int domino_step_decode(domino_t h, const int32_t* states_dev, const uint64_t* st
     }
     const size_t part_bytes = (size_t)batch * (size_t)h->n_windows * sizeof(float4);
     if (h->d_fpart.n < part_bytes) {
+        // growing the partials buffer synchronises the stream and reallocates,
+        // neither of which a stream capture allows: the first call at a larger
+        // batch must run uncaptured
+        cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+        if (cudaStreamIsCapturing(st, &cs) != cudaSuccess) return cuda_status(cudaGetLastError());
+        if (cs != cudaStreamCaptureStatusNone) return DOMINO_E_INVALID_ARG;
         if (cudaStreamSynchronize(st) != cudaSuccess) return cuda_status(cudaGetLastError());
         clear_host_graphs(h);   // recorded host-buffer steps name this buffer
         if ((rc = dev_reserve(h->d_fpart, part_bytes))) return rc;
@@ -1056,13 +1062,18 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
         else if (h->t_wall_ms[0] == 0.0) mapped = false;
         else mapped = (h->t_wall_ms[1] <= h->t_wall_ms[0]) != (h->host_calls % 64 == 63);
     }
+    // the in-place path runs the fused decode, whose per-window partials
+    // buffer is grown here too, before any recording
+    const size_t fpart_bytes = (size_t)batch * (size_t)h->n_windows * sizeof(float4);
     const bool grow = (!mapped && h->s_logits.n < logit_bytes) || h->s_io.n < L.in_end ||
-                      h->s_mask.n < (size_t)batch * (size_t)h->W * 4 || h->h_io_n < L.in_end || !h->cp_stream;
+                      h->s_mask.n < (size_t)batch * (size_t)h->W * 4 || h->h_io_n < L.in_end || !h->cp_stream ||
+                      (mapped && h->d_fpart.n < fpart_bytes);
     if (grow) {   // buffers may move: recorded steps that use them are dropped
         if (cudaStreamSynchronize(st) != cudaSuccess) return cuda_status(cudaGetLastError());
         clear_host_graphs(h);
     }
     if (!mapped && (rc = dev_reserve(h->s_logits, logit_bytes))) return rc;
+    if (mapped && (rc = dev_reserve(h->d_fpart, fpart_bytes))) return rc;
     if ((rc = dev_reserve(h->s_mask, (size_t)batch * (size_t)h->W * 4))) return rc;
     if ((rc = dev_reserve(h->s_io, L.in_end))) return rc;
     if (h->h_io_n < L.in_end) {

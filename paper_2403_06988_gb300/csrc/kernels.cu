@@ -518,6 +518,15 @@ __device__ __forceinline__ uint4 read_row(const StepView& v, const int32_t* __re
     return decode_row(v, sv, w, stacks != nullptr, v.accept_bits, report);
 }
 
+// read_row for configurations that the same kernel overwrites (the update
+// writes its outputs in place): coherent loads, no read-only path.
+__device__ __forceinline__ uint4 read_row_rw(const StepView& v, const int32_t* states, const uint64_t* stacks, int b,
+                                             bool report) {
+    const int32_t sv = __ldcg(states + b);
+    const unsigned long long w = stacks ? __ldcg(reinterpret_cast<const unsigned long long*>(stacks) + b) : 0ull;
+    return decode_row(v, sv, w, stacks != nullptr, v.accept_bits, report);
+}
+
 template <bool STACK, int MODE, bool NEXT>
 __global__ void __launch_bounds__(kStepThreads, 1)
     step_kernel(const StepView v, const uint4* __restrict__ img, int img_bytes, int img_tgt_off, int img_ret_off,
@@ -1256,9 +1265,8 @@ __global__ void __launch_bounds__(kLogitThreads)
 // the start state; a rejected token: state 0; t >= V: state 0 and the error
 // word).  Reads the configuration before writing, so the outputs may alias it.
 template <bool STACK, int MODE>
-__device__ __forceinline__ void advance_row(const StepView& v, const int32_t* __restrict__ states,
-                                            const uint64_t* __restrict__ stacks, int b, int32_t t,
-                                            int32_t* __restrict__ states_out, uint64_t* __restrict__ stacks_out) {
+__device__ __forceinline__ void advance_row(const StepView& v, const int32_t* states, const uint64_t* stacks, int b,
+                                            int32_t t, int32_t* states_out, uint64_t* stacks_out) {
     using E = typename std::conditional<STACK, uint32_t, uint16_t>::type;
     uint32_t s = 0, bits = 0, depth = 0;
     if (t < 0 || t == v.eos_id) {
@@ -1266,7 +1274,7 @@ __device__ __forceinline__ void advance_row(const StepView& v, const int32_t* __
     } else if (t >= v.V) {
         atomicOr(v.err, DOMINO_DEVERR_BAD_TOKEN);
     } else {
-        const uint4 rc = read_row(v, states, stacks, b, true);
+        const uint4 rc = read_row_rw(v, states, stacks, b, true);
         if (rc.w & 1u) {
             // the table image the step kernel staged (L2-resident) read from global memory
             Tab<E, MODE == kDenseSmem ? kDenseGlobal : MODE> tab;
@@ -1292,9 +1300,8 @@ __device__ __forceinline__ void advance_row(const StepView& v, const int32_t* __
 
 template <bool STACK, int MODE>
 __global__ void __launch_bounds__(kAdvanceThreads)
-    advance_kernel(const StepView v, const int32_t* __restrict__ states, const uint64_t* __restrict__ stacks,
-                   const int32_t* __restrict__ tokens, int32_t batch, int32_t* __restrict__ states_out,
-                   uint64_t* __restrict__ stacks_out) {
+    advance_kernel(const StepView v, const int32_t* states, const uint64_t* stacks,
+                   const int32_t* __restrict__ tokens, int32_t batch, int32_t* states_out, uint64_t* stacks_out) {
     pdl_wait();
     pdl_trigger();
     const int b = blockIdx.x * kAdvanceThreads + threadIdx.x;
@@ -1476,11 +1483,12 @@ __global__ void __launch_bounds__(kAdvanceThreads)
 
 // Alg. 1 update from the precomputed state x token table: one read of
 // next[s][t] per sequence (EOS or -1: the start state; a rejected token's
-// entry is 0, the dead state).
+// entry is 0, the dead state).  states_out may alias states: each thread reads
+// its row before writing it.
 __global__ void __launch_bounds__(kAdvanceThreads)
     advance_table_kernel(const int32_t* __restrict__ table_next, int32_t Q, int32_t V, int32_t eos_id, int32_t start,
-                         const int32_t* __restrict__ states, const int32_t* __restrict__ tokens, int32_t batch,
-                         int32_t* __restrict__ states_out, uint32_t* __restrict__ err) {
+                         const int32_t* states, const int32_t* __restrict__ tokens, int32_t batch,
+                         int32_t* states_out, uint32_t* __restrict__ err) {
     pdl_wait();
     pdl_trigger();
     const int b = blockIdx.x * kAdvanceThreads + threadIdx.x;
@@ -1541,12 +1549,16 @@ cudaError_t launch_step_t(const StepView& v, const LaunchEnv& env, const int32_t
     // the dynamic shared-memory limit is raised once per device and size, so
     // that launches inside a stream capture make no attribute calls
     static int configured[kMaxDevices] = {0};
+    static std::mutex mu;   // handles on different host threads share it
     int dev = 0;
     cudaGetDevice(&dev);
-    if (L.total > 48 * 1024 && dev < kMaxDevices && configured[dev] < L.total) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L.total);
-        if (e != cudaSuccess) return e;
-        configured[dev] = L.total;
+    if (L.total > 48 * 1024 && dev < kMaxDevices) {
+        std::lock_guard<std::mutex> lk(mu);
+        if (configured[dev] < L.total) {
+            cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L.total);
+            if (e != cudaSuccess) return e;
+            configured[dev] = L.total;
+        }
     }
     const int n_row_tiles = (batch + R - 1) / R;
     const int n_tiles = n_row_tiles * v.n_windows;
@@ -1602,15 +1614,20 @@ int occupancy(const void* kern, int threads) {
     };
     static Entry cache[64];
     static int used = 0;
+    static std::mutex mu;   // handles on different host threads share the cache
     int dev = 0;
     cudaGetDevice(&dev);
-    for (int i = 0; i < used; i++)
-        if (cache[i].fn == kern && cache[i].dev == dev) return cache[i].n;
+    {
+        std::lock_guard<std::mutex> lk(mu);
+        for (int i = 0; i < used; i++)
+            if (cache[i].fn == kern && cache[i].dev == dev) return cache[i].n;
+    }
     int n = 1;
     if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kern, threads, 0) != cudaSuccess || n < 1) {
         cudaGetLastError();
         n = 1;
     }
+    std::lock_guard<std::mutex> lk(mu);
     if (used < 64) cache[used++] = Entry{kern, dev, n};
     return n;
 }

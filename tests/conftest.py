@@ -18,3 +18,20 @@ def oracle_lib():
     import oracle
     oracle.build()
     return oracle
+
+
+@pytest.fixture(autouse=True)
+def _poison_outputs(request):
+    """GPU tests: every output the Domino holder allocates starts as 0xAB
+    bytes, so that a word a kernel leaves unwritten fails the exact
+    comparison instead of passing on whatever the allocator returned."""
+    if request.node.get_closest_marker("gpu") is None:
+        yield
+        return
+    from paper_2403_06988_gb300 import Domino
+    from poison import POISON_BYTE
+    Domino.fill_byte = POISON_BYTE
+    try:
+        yield
+    finally:
+        Domino.fill_byte = None

@@ -10,7 +10,7 @@ from a counter.  Batch 256 and 38 vocabulary windows make 8 x 38 = 304 tiles,
 two per SM of a GB300, so the kernel takes 32 rows per tile.
 
 Masks, next states, argmax and updated configurations: bit-exact against the
-oracle; lse within 1e-3.
+oracle; lse within 1e-3.  Outputs start as 0xAB bytes (tests/poison.py).
 """
 import os
 
@@ -23,6 +23,8 @@ torch = pytest.importorskip("torch")
 
 from paper_2403_06988_gb300 import Domino, synth  # noqa: E402
 from paper_2403_06988_gb300 import _binding as B  # noqa: E402
+import poison  # noqa: E402
+from poison import assert_exact, assert_no_poison  # noqa: E402
 
 TOL = 1e-3
 NT = os.cpu_count() or 1
@@ -95,22 +97,23 @@ def check_step(a, v, states, stacks, seed):
     mask, nxt = d.step_mask(st, sk, want_next=True)
     m_o, n_o, bad = P.step_mask(states, stacks, want_next=True, n_threads=NT)
     assert bad == 0
-    assert (mask.cpu().numpy().view(np.uint32) == m_o).all()
-    assert (nxt.cpu().numpy() == n_o).all()
+    assert_exact(mask, m_o, "mask")
+    assert_exact(nxt, n_o, "next")
     # the fused step: decode folded into the walk, rows advanced in place
     rng = np.random.default_rng(seed)
     lg = synth.f32_to_bf16_bits(rng.normal(0.0, 3.0, (len(states), V)).astype(np.float32))
     t = dev(lg.view(np.int16)).view(torch.bfloat16)
-    m2 = torch.empty_like(mask)
-    arg = torch.empty(len(states), dtype=torch.int32, device="cuda")
-    lse = torch.empty(len(states), dtype=torch.float32, device="cuda")
+    m2 = poison.empty_like(mask)
+    arg = poison.empty(len(states), torch.int32)
+    lse = poison.empty(len(states), torch.float32)
     B.domino_step_decode(d.h, st, sk, len(states), t.data_ptr(), B.DTYPE_BF16, V, m2, arg, lse, None, st, sk)
     torch.cuda.synchronize()
     a_o, l_o, _ = oracle.mask_logits(lg, m_o, n_threads=NT)
     s_o, k_o, bad = P.advance(states, stacks, a_o, a.start)
     assert bad == 0
-    assert (m2.cpu().numpy().view(np.uint32) == m_o).all()
-    assert (arg.cpu().numpy() == a_o).all()
+    assert_exact(m2, m_o, "mask of the fused step")
+    assert_exact(arg, a_o, "argmax")
+    assert_no_poison(lse, "lse")
     assert np.abs(lse.cpu().numpy().astype(np.float64) - l_o).max() < TOL
     assert (st.cpu().numpy() == s_o).all()
     if has_stack:

@@ -1,6 +1,7 @@
 """Opportunistic masking (Sec. 3.5, further optimisations): the unmasked argmax
 is proposed and checked with one walk; only rejected rows get a mask.  The
-tokens must equal the masked greedy decode of the oracle, bit for bit."""
+tokens must equal the masked greedy decode of the oracle, bit for bit.
+Output buffers start as 0xAB bytes (tests/poison.py)."""
 import functools
 import os
 
@@ -13,6 +14,7 @@ torch = pytest.importorskip("torch")
 
 from paper_2403_06988_gb300 import Domino, synth  # noqa: E402
 from paper_2403_06988_gb300 import _binding as B  # noqa: E402
+from poison import assert_exact  # noqa: E402
 
 NT = os.cpu_count() or 1
 
@@ -81,7 +83,7 @@ def test_opportunistic_matches_masked_greedy(config, obedient):
     d = handle(config)
     sk = dev(stacks.view(np.int64)) if w.automaton.rules is not None else None
     tok, n_fb = d.opportunistic_step(logits_tensor(lg), dev(states), sk)
-    assert (tok.cpu().numpy() == want).all()
+    assert_exact(tok, np.asarray(want, np.int32), "tokens")
     assert int(n_fb.item()) == n_rej
     if obedient:
         assert n_rej == int((want < 0).sum())      # only rows with nothing allowed fall back
@@ -106,7 +108,7 @@ def test_opportunistic_decode_loop_with_advance():
         d.advance(st, None, tok)
         a_o, _, _ = oracle.mask_logits(lg, m_o)
         s_o, _, _ = P.advance(s_o, None, a_o, w.automaton.start)
-        assert (tok.cpu().numpy() == a_o).all(), i
+        assert_exact(tok, np.asarray(a_o, np.int32), f"tokens, step {i}")
         assert (st.cpu().numpy() == s_o).all(), i
 
 
@@ -136,6 +138,6 @@ def test_opportunistic_more_rows_than_one_logits_pass():
     x[:, int(np.argmin(allowed_rows))] += 50.0          # a token almost never allowed wins every proposal
     want, _, _ = oracle.mask_logits(x, m)
     tok, n_fb = d.opportunistic_step(dev(x), dev(states))
-    assert (tok.cpu().numpy() == want).all()
+    assert_exact(tok, np.asarray(want, np.int32), "tokens")
     assert int(n_fb.item()) > 4096
 

@@ -3,6 +3,8 @@
 Masks, next states, argmax, advanced configurations: bit-exact.
 lse and log-probs: within 1e-3 absolute (fp32 accumulation of bf16/fp32
 inputs against the oracle's float64).
+Every output buffer starts filled with 0xAB bytes (tests/poison.py), so a
+word a kernel leaves unwritten fails the comparison.
 """
 import functools
 import os
@@ -16,6 +18,8 @@ torch = pytest.importorskip("torch")
 
 from paper_2403_06988_gb300 import Domino, synth  # noqa: E402
 from paper_2403_06988_gb300 import _binding as B  # noqa: E402
+import poison  # noqa: E402
+from poison import assert_exact, assert_no_poison  # noqa: E402
 
 TOL = 1e-3
 NT = os.cpu_count() or 1
@@ -68,13 +72,15 @@ def logits_tensor(np_logits):
 
 
 def assert_logits_match(arg_g, lse_g, lp_g, arg_o, lse_o, lp_o):
-    assert (arg_g.cpu().numpy() == arg_o).all()
+    assert_exact(arg_g, np.asarray(arg_o, np.int32), "argmax")
     if lse_g is not None:
+        assert_no_poison(lse_g, "lse")
         lg = lse_g.cpu().numpy().astype(np.float64)
         fin = np.isfinite(lse_o)
         assert (np.isfinite(lg) == fin).all()
         assert np.abs(lg[fin] - lse_o[fin]).max(initial=0) < TOL
     if lp_g is not None:
+        assert_no_poison(lp_g, "log-probs")
         pg = lp_g.cpu().numpy().astype(np.float64)
         fin = np.isfinite(lp_o)
         assert (np.isfinite(pg) == fin).all()
@@ -98,9 +104,9 @@ def test_step_mask_parity(config):
     m_o, n_o, bad = problem(config).step_mask(states, stacks if sk is not None else None, want_next=True,
                                               n_threads=NT)
     assert bad == 0
-    assert (u32(mask) == m_o).all()
-    assert (u32(mask2) == m_o).all()
-    assert (nxt.cpu().numpy() == n_o).all()
+    assert_exact(mask, m_o, "mask")
+    assert_exact(mask2, m_o, "mask (no next states)")
+    assert_exact(nxt, n_o, "next")
     assert d.device_error() == 0
 
 
@@ -119,7 +125,9 @@ def test_step_mask_depth32_rows():
     d = handle(5)
     mask, nxt = d.step_mask(dev(st), dev(sk.view(np.int64)), want_next=True)
     m_o, n_o, bad = problem(5).step_mask(st, sk, want_next=True, n_threads=NT)
-    assert bad == 0 and (u32(mask) == m_o).all() and (nxt.cpu().numpy() == n_o).all()
+    assert bad == 0
+    assert_exact(mask, m_o, "mask")
+    assert_exact(nxt, n_o, "next")
     toks = w.vocab.tokens()
     lb = toks.index(b"{")
     push_states = {int(r["state"]) for r in w.automaton.rules if r["kind"] == synth.RULE_PUSH}
@@ -191,9 +199,9 @@ def test_mask_logits_ragged_and_unaligned(V, stride, dtype):
     m = np.packbits(packed, axis=1, bitorder="little").view("<u4")
     arg_o, lse_o, lp_o = oracle.mask_logits(x, m, n_tokens=V, want_logprobs=True)
     xt = logits_tensor(x)
-    argmax = torch.empty(B_, dtype=torch.int32, device=DEV)
-    lse = torch.empty(B_, dtype=torch.float32, device=DEV)
-    lp = torch.empty((B_, V), dtype=torch.float32, device=DEV)
+    argmax = poison.empty(B_, torch.int32, DEV)
+    lse = poison.empty(B_, torch.float32, DEV)
+    lp = poison.empty((B_, V), torch.float32, DEV)
     B.domino_mask_logits(d.h, xt.data_ptr(), B.DTYPE_BF16 if dtype == "bf16" else B.DTYPE_F32, B_, stride,
                          dev(m.view(np.int32)), argmax, lse, lp)
     assert_logits_match(argmax, lse, lp, arg_o, lse_o, lp_o)
@@ -243,15 +251,15 @@ def test_advance_parity(config):
     d = handle(config)
     st = dev(states)
     sk = dev(stacks.view(np.int64)) if has_stack else None
-    so = torch.empty_like(st)
-    wo = torch.empty_like(sk) if has_stack else None
+    so = poison.empty_like(st)
+    wo = poison.empty_like(sk) if has_stack else None
     d.advance(st, sk, dev(tokens), states_out=so, stacks_out=wo)
-    assert (so.cpu().numpy() == so_o).all()
+    assert_exact(so, so_o, "states")
     if has_stack:
-        assert (wo.cpu().numpy().view(np.uint64) == wo_o).all()
+        assert_exact(wo, wo_o, "stacks")
     # in place
     d.advance(st, sk, dev(tokens))
-    assert (st.cpu().numpy() == so_o).all()
+    assert_exact(st, so_o, "states in place")
 
 
 @pytest.mark.parametrize("config,steps", [(1, 64), (2, 40), (5, 12)])
@@ -273,7 +281,7 @@ def test_decode_loop_parity(config, steps):
         m_o, _, _ = problem(config).step_mask(s_o, k_o if has_stack else None, n_threads=NT)
         a_o, l_o, _ = oracle.mask_logits(lg, m_o)
         s_o, k_o, _ = problem(config).advance(s_o, k_o if has_stack else None, a_o, w.automaton.start)
-        assert (u32(mask) == m_o).all(), i
+        assert_exact(mask, m_o, f"mask, step {i}")
         assert_logits_match(arg, lse, None, a_o, l_o, None)
         assert (st.cpu().numpy() == s_o).all(), i
         if has_stack:
@@ -297,15 +305,16 @@ def test_decode_step_host_matches_oracle(config, pinned):
         lg = lg.view(np.uint16) if lg.dtype == np.int16 else lg
     s_host = states.copy()
     k_host = stacks.copy() if has_stack else None
-    tok = np.zeros(len(states), np.int32)
-    lse_h = np.zeros(len(states), np.float32)
+    tok = poison.host(len(states), np.int32)
+    lse_h = poison.host(len(states), np.float32)
     dt = B.DTYPE_BF16 if lg.dtype == np.uint16 else B.DTYPE_F32
     B.domino_decode_step_host(d.h, lg, dt, len(states), s_host, k_host, tok, lse_h, stream=0)
     P = problem(config)
     m, _, _ = P.step_mask(states, stacks if has_stack else None, n_threads=NT)
     a_o, l_o, _ = oracle.mask_logits(lg, m)
     s_o, k_o, _ = P.advance(states, stacks if has_stack else None, a_o, w.automaton.start)
-    assert (tok == a_o).all()
+    assert_exact(tok, a_o, "tokens")
+    assert_no_poison(lse_h, "lse")
     fin = np.isfinite(l_o)
     assert np.abs(lse_h[fin] - l_o[fin]).max(initial=0) < TOL
     assert (s_host == s_o).all()
@@ -327,14 +336,16 @@ def test_decode_step_host_replayed_steps_match_oracle(config):
     states, stacks = w.initial_configs()
     s_host = torch.from_numpy(states.copy()).pin_memory()
     k_host = torch.from_numpy(stacks.view(np.int64).copy()).pin_memory() if has_stack else None
-    tok = torch.empty(len(states), dtype=torch.int32).pin_memory()
-    lse_h = torch.empty(len(states), dtype=torch.float32).pin_memory()
+    tok = poison.empty(len(states), torch.int32, pin=True)
+    lse_h = poison.empty(len(states), torch.float32, pin=True)
     bufs = [torch.from_numpy(w.logits(40 + i).view(np.int16)).pin_memory() for i in range(2)]
     bufs.append(torch.from_numpy(w.logits(42).view(np.int16)))          # pageable: the copy path
     s_o, k_o = states.copy(), stacks.copy()
     st = torch.cuda.Stream()
     for i in range(7):
         b = bufs[i % 3]
+        tok.view(torch.uint8).fill_(poison.POISON_BYTE)
+        lse_h.view(torch.uint8).fill_(poison.POISON_BYTE)
         B.domino_decode_step_host(d.h, b.data_ptr(), B.DTYPE_BF16, len(states), s_host.data_ptr(),
                                   k_host.data_ptr() if has_stack else None, tok.data_ptr(), lse_h.data_ptr(),
                                   stream=st.cuda_stream)
@@ -343,7 +354,8 @@ def test_decode_step_host_replayed_steps_match_oracle(config):
         a_o, l_o, _ = oracle.mask_logits(lg, m)
         s_o, k_o2, _ = P.advance(s_o, k_o if has_stack else None, a_o, w.automaton.start)
         k_o = k_o2 if has_stack else k_o
-        assert (tok.numpy() == a_o).all(), i
+        assert_exact(tok, a_o, f"tokens, step {i}")
+        assert_no_poison(lse_h, f"lse, step {i}")
         fin = np.isfinite(l_o)
         assert np.abs(lse_h.numpy()[fin] - l_o[fin]).max(initial=0) < TOL
         assert (s_host.numpy() == s_o).all(), i
@@ -364,21 +376,66 @@ def test_decode_step_host_path_choice_keeps_results():
     P = problem(2)
     states, _ = w.initial_configs()
     s_host = torch.from_numpy(states.copy()).pin_memory()
-    tok = torch.empty(len(states), dtype=torch.int32).pin_memory()
-    lse_h = torch.empty(len(states), dtype=torch.float32).pin_memory()
+    tok = poison.empty(len(states), torch.int32, pin=True)
+    lse_h = poison.empty(len(states), torch.float32, pin=True)
     bufs = [torch.from_numpy(w.logits(60 + i).view(np.int16)).pin_memory() for i in range(2)]
     s_o = states.copy()
     st = torch.cuda.Stream()
     for i in range(70):
         b = bufs[i % 2]
+        tok.view(torch.uint8).fill_(poison.POISON_BYTE)
+        lse_h.view(torch.uint8).fill_(poison.POISON_BYTE)
         B.domino_decode_step_host(d.h, b.data_ptr(), B.DTYPE_BF16, len(states), s_host.data_ptr(), None,
                                   tok.data_ptr(), lse_h.data_ptr(), stream=st.cuda_stream)
         m, _, _ = P.step_mask(s_o, None, n_threads=NT)
         a_o, l_o, _ = oracle.mask_logits(b.numpy().view(np.uint16), m)
         s_o, _, _ = P.advance(s_o, None, a_o, w.automaton.start)
-        assert (tok.numpy() == a_o).all(), i
+        assert_exact(tok, a_o, f"tokens, step {i}")
+        assert_no_poison(lse_h, f"lse, step {i}")
         fin = np.isfinite(l_o)
         assert np.abs(lse_h.numpy()[fin] - l_o[fin]).max(initial=0) < TOL, i
+        assert (s_host.numpy() == s_o).all(), i
+    assert d.device_error() == 0
+    d.close()
+
+
+def test_decode_step_host_batch_grows_on_a_recording_stream():
+    """Pinned bf16 logits on a non-default stream, with batches growing from
+    call to call.  On a fresh handle the first calls take the in-place path
+    (it has not been timed yet), and from the third call on a step is recorded
+    into a CUDA graph: the fused decode's per-window partials must have grown
+    before that recording starts.  Three calls at one batch, then larger
+    batches, every call equal to the oracle."""
+    import oracle
+    w = workload(2)
+    d = Domino.from_parts(w.automaton, w.vocab, device=0)
+    P = problem(2)
+    st = torch.cuda.Stream()
+    plan = [8, 16, 32, 32, 32, 32, 64, 64, 96]
+    big = max(plan)
+    rng = np.random.default_rng(123)
+    live = np.nonzero(w.automaton.live)[0]
+    s_all = rng.choice(live, size=big).astype(np.int32)
+    lg_all = torch.from_numpy(w.logits(70, batch=big).view(np.int16)).pin_memory()
+    s_host = torch.from_numpy(s_all.copy()).pin_memory()
+    tok = poison.empty(big, torch.int32, pin=True)
+    lse_h = poison.empty(big, torch.float32, pin=True)
+    s_o = s_all.copy()
+    for i, b in enumerate(plan):
+        tok.view(torch.uint8).fill_(poison.POISON_BYTE)
+        lse_h.view(torch.uint8).fill_(poison.POISON_BYTE)
+        before = s_o[:b].copy()
+        B.domino_decode_step_host(d.h, lg_all.data_ptr(), B.DTYPE_BF16, b, s_host.data_ptr(), None, tok.data_ptr(),
+                                  lse_h.data_ptr(), stream=st.cuda_stream)
+        lg = lg_all.numpy().view(np.uint16)[:b]
+        m, _, _ = P.step_mask(before, None, n_threads=NT)
+        a_o, l_o, _ = oracle.mask_logits(lg, m)
+        nxt, _, _ = P.advance(before, None, a_o, w.automaton.start)
+        s_o[:b] = nxt
+        assert_exact(tok[:b], a_o, f"tokens, call {i} (batch {b})")
+        assert_no_poison(lse_h[:b], f"lse, call {i}")
+        fin = np.isfinite(l_o)
+        assert np.abs(lse_h.numpy()[:b][fin] - l_o[fin]).max(initial=0) < TOL, i
         assert (s_host.numpy() == s_o).all(), i
     assert d.device_error() == 0
     d.close()
@@ -394,9 +451,10 @@ def test_decode_step_host_matches_device_path():
     nxt = dev(states)
     d.advance(nxt, None, arg)
     s_host = states.copy()
-    tok = np.zeros(len(states), np.int32)
-    lse_h = np.zeros(len(states), np.float32)
+    tok = poison.host(len(states), np.int32)
+    lse_h = poison.host(len(states), np.float32)
     B.domino_decode_step_host(d.h, lg, B.DTYPE_BF16, len(states), s_host, None, tok, lse_h, stream=0)
+    assert_no_poison(lse_h, "lse")
     assert (tok == arg.cpu().numpy()).all()
     assert (s_host == nxt.cpu().numpy()).all()
     assert np.abs(lse_h - lse.cpu().numpy()).max() < 1e-6
@@ -411,34 +469,42 @@ def test_precompute_table_full_config2():
     nxt, mask = d.precompute_table()
     Q = w.automaton.n_states
     m_o, n_o, _ = problem(2).step_mask(np.arange(Q, dtype=np.int32), want_next=True, n_threads=NT)
-    assert (u32(mask) == m_o).all()
-    assert (nxt.cpu().numpy() == n_o).all()
+    assert_exact(mask, m_o, "table mask")
+    assert_exact(nxt, n_o, "table next")
 
 
-def test_precompute_table_config4_sampled_rows():
-    """Full-size state x token table: sampled rows exactly, invariants everywhere."""
+def test_precompute_table_config4_full():
+    """The full-size state x token table (Q = 20000, V = 128256, Alg. 2's
+    traversal for every state): every row of mask and next states equal to the
+    all-core oracle, compared in blocks of 2000 states; the table's invariants
+    on the device; table row q == step_mask from q on sampled rows."""
     w = workload(4)
     d = Domino.from_parts(w.automaton, w.vocab, device=0)
     nxt, mask = d.precompute_table()
+    torch.cuda.synchronize()
     Q, V = w.automaton.n_states, w.vocab.n_tokens
     assert nxt.shape == (Q, V)
-    rng = np.random.default_rng(44)
-    rows = np.unique(np.concatenate([[0, 1, 2, Q - 1, 1999, 2000, 2001], rng.integers(0, Q, 57)])).astype(np.int32)
-    m_o, n_o, _ = problem_c4().step_mask(rows, want_next=True, n_threads=NT)
-    assert (u32(mask[rows.tolist()]) == m_o).all()
-    assert (nxt[rows.tolist()].cpu().numpy() == n_o).all()
+    P = problem_c4()
+    blk = 2000
+    for q0 in range(0, Q, blk):
+        q1 = min(Q, q0 + blk)
+        m_o, n_o, bad = P.step_mask(np.arange(q0, q1, dtype=np.int32), want_next=True, n_threads=NT)
+        assert bad == 0
+        assert_exact(mask[q0:q1], m_o, f"table mask, states {q0}..{q1 - 1}")
+        assert_exact(nxt[q0:q1], n_o, f"table next, states {q0}..{q1 - 1}")
+        del m_o, n_o
     # invariants on the whole table, computed on the device
-    W = (V + 31) // 32
     tok = torch.arange(V, device=DEV)
-    for q0 in range(0, Q, 2000):
-        blk_n = nxt[q0:q0 + 2000]
-        blk_m = mask[q0:q0 + 2000]
+    for q0 in range(0, Q, blk):
+        blk_n = nxt[q0:q0 + blk]
+        blk_m = mask[q0:q0 + blk]
         bit = (blk_m[:, tok >> 5] >> (tok & 31).to(torch.int32)) & 1
         assert torch.equal(bit == 1, blk_n != 0)
     assert int(mask[0].abs().sum()) == 0 and int(nxt[0].abs().sum()) == 0
     # table row q == step_mask from q
-    qs = dev(rows)
-    sm, sn = d.step_mask(qs, None, want_next=True)
+    rng = np.random.default_rng(44)
+    rows = np.unique(np.concatenate([[0, 1, 2, Q - 1, 1999, 2000, 2001], rng.integers(0, Q, 57)])).astype(np.int32)
+    sm, sn = d.step_mask(dev(rows), None, want_next=True)
     assert torch.equal(sm, mask[rows.tolist()]) and torch.equal(sn, nxt[rows.tolist()])
     del nxt, mask
     d.close()
@@ -469,9 +535,11 @@ def test_fig3_worked_example_on_gpu():
                             want_next=True)
     allowed = [b"0", b"1", b"2", b"12", b")", b"+", b"+1", b"1 +"]
     toks = v.tokens()
-    bits = u32(mask)[0]
+    want = np.zeros((1, (len(toks) + 31) // 32), np.uint32)
     for t, tok in enumerate(toks):
-        assert bool((bits[t >> 5] >> (t & 31)) & 1) == (tok in allowed), tok
+        if tok in allowed:
+            want[0, t >> 5] |= np.uint32(1 << (t & 31))
+    assert_exact(mask, want, "Fig. 3 mask after (12")
 
 
 @pytest.mark.parametrize("name", ["dyck2", "int_regex", "dyck_ctx"])
@@ -494,7 +562,9 @@ def test_tiny_grammar_parity(name):
     stacks = np.array(stacks, np.uint64)
     mask, nxt = d.step_mask(dev(states), dev(stacks.view(np.int64)), want_next=True)
     m_o, n_o, bad = P.step_mask(states, stacks, want_next=True)
-    assert bad == 0 and (u32(mask) == m_o).all() and (nxt.cpu().numpy() == n_o).all()
+    assert bad == 0
+    assert_exact(mask, m_o, "mask")
+    assert_exact(nxt, n_o, "next")
 
 
 def test_ragged_vocab_long_tokens_eos_in_middle():
@@ -517,7 +587,8 @@ def test_ragged_vocab_long_tokens_eos_in_middle():
     states = np.array([1, 2, 3, 4, 0, 1, 3], np.int32)
     mask, nxt = d.step_mask(dev(states), None, want_next=True)
     m_o, n_o, _ = P.step_mask(states, want_next=True)
-    assert (u32(mask) == m_o).all() and (nxt.cpu().numpy() == n_o).all()
+    assert_exact(mask, m_o, "mask")
+    assert_exact(nxt, n_o, "next")
     assert (u32(mask)[:, -1] >> (v.n_tokens % 32) == 0).all()
 
 
@@ -531,6 +602,10 @@ def test_invalid_inputs_set_error_word():
     m = u32(mask)
     assert (m[1:] == 0).all() and (nxt[1:] == 0).all()
     assert m[0].any()
+    m_o, n_o, bad = problem(5).step_mask(states, stacks, want_next=True)
+    assert bad == 5
+    assert_exact(mask, m_o, "mask")
+    assert_exact(nxt, n_o, "next")
     code = d.device_error()
     assert code == (B.DEVERR_BAD_STATE | B.DEVERR_BAD_STACK)
     assert d.device_error() == 0                      # cleared on read

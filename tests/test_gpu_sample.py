@@ -1,6 +1,7 @@
 """Sampling decode (Gumbel-max, Philox4x32-10 uniforms) through the C ABI
 against the oracle's draw: tokens bit-exact on the same logits, masks, seed and
-offset.  Masks fed to both sides come from the oracle."""
+offset.  Masks fed to both sides come from the oracle.  Output buffers start
+as 0xAB bytes (tests/poison.py)."""
 import functools
 import os
 
@@ -13,6 +14,8 @@ torch = pytest.importorskip("torch")
 
 from paper_2403_06988_gb300 import Domino, synth  # noqa: E402
 from paper_2403_06988_gb300 import _binding as B  # noqa: E402
+import poison  # noqa: E402
+from poison import assert_exact  # noqa: E402
 
 NT = os.cpu_count() or 1
 
@@ -64,7 +67,7 @@ def test_sample_matches_oracle_on_workloads(config, temperature, seed, offset):
     want = oracle.mask_sample(lg, m, temperature, seed, offset, n_threads=NT)
     d = Domino.from_parts(w.automaton, w.vocab, device=0)
     got = d.mask_sample(logits_tensor(lg), dev(m.view(np.int32)), temperature, seed, offset)
-    assert (got.cpu().numpy() == want).all()
+    assert_exact(got, np.asarray(want, np.int32), "draws")
     greedy, _, _ = oracle.mask_logits(lg, m)
     assert ((want >= 0) == (greedy >= 0)).all()
     d.close()
@@ -84,12 +87,12 @@ def test_sample_ragged_and_unaligned(V, stride, dtype):
     bits[0] = False
     m = packed(bits)
     want = oracle.mask_sample(x, m, 0.9, 99, 3, n_tokens=V)
-    tok = torch.empty(B_, dtype=torch.int32, device="cuda")
+    tok = poison.empty(B_, torch.int32)
     lg = logits_tensor(x)   # held across the call: nothing else may reuse its memory
     B.domino_mask_sample(d.h, lg.data_ptr(), B.DTYPE_BF16 if dtype == "bf16" else B.DTYPE_F32, B_,
                          stride, dev(m.view(np.int32)), 0.9, 99, 3, tok)
-    got = tok.cpu().numpy()
-    assert (got == want).all() and got[0] == -1
+    assert_exact(tok, np.asarray(want, np.int32), "draws")
+    assert int(tok[0]) == -1
     d.close()
 
 
@@ -100,8 +103,8 @@ def test_sample_rows_beyond_one_pass_use_their_own_counter():
     x = np.zeros((B_, V), np.float32)                 # uniform: the draw is decided by the counter alone
     m = packed(np.ones((B_, V), bool))
     want = oracle.mask_sample(x, m, 1.0, 5, 6, n_threads=NT)
-    got = d.mask_sample(dev(x), dev(m.view(np.int32)), 1.0, 5, 6).cpu().numpy()
-    assert (got == want).all()
+    got = d.mask_sample(dev(x), dev(m.view(np.int32)), 1.0, 5, 6)
+    assert_exact(got, np.asarray(want, np.int32), "draws")
     d.close()
 
 

@@ -1,6 +1,7 @@
 """Count-based speculation (Sec. 3.6) through the C ABI against the oracle:
 after the same sequence of count updates, the proposals, their number and the
-configuration chains are identical; acceptance of a verification pass agrees."""
+configuration chains are identical; acceptance of a verification pass agrees.
+Output buffers start as 0xAB bytes (tests/poison.py)."""
 import functools
 import os
 
@@ -13,6 +14,8 @@ torch = pytest.importorskip("torch")
 
 from paper_2403_06988_gb300 import Domino, synth  # noqa: E402
 from paper_2403_06988_gb300 import _binding as B  # noqa: E402
+import poison  # noqa: E402
+from poison import assert_exact  # noqa: E402
 
 NT = os.cpu_count() or 1
 
@@ -54,10 +57,10 @@ class GpuSpec:
 
     def propose(self, states, stacks, s, permille):
         b = len(states)
-        prop = torch.empty((b, s), dtype=torch.int32, device="cuda")
-        n = torch.empty(b, dtype=torch.int32, device="cuda")
-        cs = torch.empty((b, s + 1), dtype=torch.int32, device="cuda")
-        ck = torch.empty((b, s + 1), dtype=torch.int64, device="cuda") if stacks is not None else None
+        prop = poison.empty((b, s), torch.int32)
+        n = poison.empty(b, torch.int32)
+        cs = poison.empty((b, s + 1), torch.int32)
+        ck = poison.empty((b, s + 1), torch.int64) if stacks is not None else None
         B.domino_spec_propose(self.d.h, self.best, self.reached, dev(states),
                               dev(stacks.view(np.int64)) if stacks is not None else None, b, s, permille, prop, n, cs,
                               ck)
@@ -97,11 +100,11 @@ def test_proposals_match_oracle_after_the_same_updates(config):
         for s, permille in ((4, 0), (6, 400), (3, 900)):
             po, no, co, ko = osp.propose(states, stacks, s, permille)
             pg, ng, cg, kg = gsp.propose(states, stacks, s, permille)
-            assert (host(pg, np.int32) == po).all()
-            assert (host(ng, np.int32) == no).all()
-            assert (host(cg, np.int32) == co).all()
+            assert_exact(pg, po, "proposals")
+            assert_exact(ng, no, "number of proposals")
+            assert_exact(cg, co, "chain states")
             if ko is not None:
-                assert (host(kg, np.uint64) == ko).all()
+                assert_exact(kg, ko, "chain stacks")
     assert int(no.max()) >= 0
     d.close()
 
@@ -127,17 +130,17 @@ def test_accept_matches_oracle(config):
     dec, _, _ = oracle.mask_logits(lg, m)
     dec = dec.reshape(batch, s + 1)
     want = oracle.spec_accept(prop, n, dec)
-    na = torch.empty(batch, dtype=torch.int32, device="cuda")
-    tk = torch.empty(batch, dtype=torch.int32, device="cuda")
-    so = torch.empty(batch, dtype=torch.int32, device="cuda")
-    ko = torch.empty(batch, dtype=torch.int64, device="cuda") if ck is not None else None
+    na = poison.empty(batch, torch.int32)
+    tk = poison.empty(batch, torch.int32)
+    so = poison.empty(batch, torch.int32)
+    ko = poison.empty(batch, torch.int64) if ck is not None else None
     B.domino_spec_accept(d.h, dev(prop), dev(n), dev(dec), dev(cs), dev(ck.view(np.int64)) if ck is not None else None,
                          batch, s, na, tk, so, ko)
+    assert_exact(na, np.asarray(want, np.int32), "accepted")
     k = host(na, np.int32)
-    assert (k == want).all()
     rows = np.arange(batch)
-    assert (host(tk, np.int32) == dec[rows, k]).all()
-    assert (host(so, np.int32) == cs[rows, k]).all()
+    assert_exact(tk, np.ascontiguousarray(dec[rows, k], np.int32), "next tokens")
+    assert_exact(so, np.ascontiguousarray(cs[rows, k]), "chain states")
     if ck is not None:
-        assert (host(ko, np.uint64) == ck[rows, k]).all()
+        assert_exact(ko, np.ascontiguousarray(ck[rows, k]), "chain stacks")
     d.close()

@@ -1,6 +1,7 @@
 """domino_step_decode: the mask step with the masked greedy decode folded into
 it, against the oracle (mask and argmax bit-exact, lse within 1e-3), with
-device and pinned host logits, a ragged vocabulary and invalid rows."""
+device and pinned host logits, a ragged vocabulary and invalid rows.  Output
+buffers start as 0xAB bytes (tests/poison.py)."""
 import functools
 import os
 
@@ -13,6 +14,8 @@ torch = pytest.importorskip("torch")
 
 from paper_2403_06988_gb300 import Domino, synth  # noqa: E402
 from paper_2403_06988_gb300 import _binding as B  # noqa: E402
+import poison  # noqa: E402
+from poison import assert_exact, assert_no_poison  # noqa: E402
 
 TOL = 1e-3
 NT = os.cpu_count() or 1
@@ -36,10 +39,10 @@ def dev(a):
 
 
 def run(d, states, stacks, logits, dtype, stride, batch, W, V=None):
-    mask = torch.empty((batch, W), dtype=torch.int32, device="cuda")
-    arg = torch.empty(batch, dtype=torch.int32, device="cuda")
-    lse = torch.empty(batch, dtype=torch.float32, device="cuda")
-    lp = torch.empty((batch, V), dtype=torch.float32, device="cuda") if V else None
+    mask = poison.empty((batch, W), torch.int32)
+    arg = poison.empty(batch, torch.int32)
+    lse = poison.empty(batch, torch.float32)
+    lp = poison.empty((batch, V), torch.float32) if V else None
     B.domino_step_decode(d.h, states, stacks, batch, logits, dtype, stride, mask, arg, lse, lp)
     torch.cuda.synchronize()
     out = (mask.cpu().numpy().view(np.uint32), arg.cpu().numpy(), lse.cpu().numpy())
@@ -50,12 +53,14 @@ def check(P, states, stacks, lg, V, m, a, l, lp=None):
     import oracle
     m_o, _, _ = P.step_mask(states, stacks, n_threads=NT)
     a_o, l_o, lp_o = oracle.mask_logits(lg, m_o, n_tokens=V, want_logprobs=lp is not None, n_threads=NT)
-    assert (m == m_o).all()
-    assert (a == a_o).all()
+    assert_exact(m, m_o, "mask")
+    assert_exact(a, np.asarray(a_o, np.int32), "argmax")
+    assert_no_poison(l, "lse")
     fin = np.isfinite(l_o)
     assert (np.isfinite(l) == fin).all()
     assert np.abs(l[fin] - l_o[fin]).max(initial=0) < TOL
     if lp is not None:
+        assert_no_poison(lp, "log-probs")
         fin = np.isfinite(lp_o)
         assert (np.isfinite(lp) == fin).all()
         assert np.abs(lp[fin] - lp_o[fin]).max(initial=0) < TOL
@@ -169,18 +174,22 @@ def test_step_decode_with_update_matches_oracle(config):
     V, b = w.vocab.n_tokens, len(states)
     st = dev(states)
     sk = dev(stacks.view(np.int64)) if has_stack else None
-    mask = torch.empty((b, d.info()["n_words"]), dtype=torch.int32, device="cuda")
-    arg = torch.empty(b, dtype=torch.int32, device="cuda")
-    lse = torch.empty(b, dtype=torch.float32, device="cuda")
+    mask = poison.empty((b, d.info()["n_words"]), torch.int32)
+    arg = poison.empty(b, torch.int32)
+    lse = poison.empty(b, torch.float32)
     B.domino_step_decode(d.h, st, sk, b, t.data_ptr(), dt, V, mask, arg, lse, None, st, sk)
     torch.cuda.synchronize()
     m_o, _, _ = P.step_mask(states, stacks if has_stack else None, n_threads=NT)
     a_o, l_o, _ = oracle.mask_logits(lg, m_o, n_threads=NT)
     s_o, k_o, bad = P.advance(states, stacks if has_stack else None, a_o, w.automaton.start)
     assert bad == 0
-    assert (arg.cpu().numpy() == a_o).all()
-    assert (st.cpu().numpy() == s_o).all()
+    assert_exact(mask, m_o, "mask")
+    assert_exact(arg, np.asarray(a_o, np.int32), "argmax")
+    assert_no_poison(lse, "lse")
+    fin = np.isfinite(l_o)
+    assert np.abs(lse.cpu().numpy()[fin] - l_o[fin]).max(initial=0) < TOL
+    assert_exact(st, s_o, "states")
     if has_stack:
-        assert (sk.cpu().numpy().view(np.uint64) == k_o).all()
+        assert_exact(sk, k_o, "stacks")
     assert d.device_error() == 0
     d.close()

@@ -1,6 +1,7 @@
 """Table-driven decode step (Sec. 3.5: masks computed before inference, looked
 up while decoding) against the oracle's walk-based decode loop: argmax and
-states bit-exact, lse and log-probs within 1e-3."""
+states bit-exact, lse and log-probs within 1e-3.  Output buffers start as 0xAB
+bytes (tests/poison.py)."""
 import functools
 import os
 
@@ -13,6 +14,8 @@ torch = pytest.importorskip("torch")
 
 from paper_2403_06988_gb300 import Domino, synth  # noqa: E402
 from paper_2403_06988_gb300 import _binding as B  # noqa: E402
+import poison  # noqa: E402
+from poison import assert_exact, assert_no_poison  # noqa: E402
 
 TOL = 1e-3
 NT = os.cpu_count() or 1
@@ -56,12 +59,14 @@ def test_table_driven_decode_loop_matches_oracle(config, steps, logprobs):
         m_o, _, _ = P.step_mask(s_o, None, n_threads=NT)
         a_o, l_o, lp_o = oracle.mask_logits(lg, m_o, want_logprobs=logprobs)
         s_o, _, _ = P.advance(s_o, None, a_o, w.automaton.start)
-        assert (arg.cpu().numpy() == a_o).all(), i
+        assert_exact(arg, np.asarray(a_o, np.int32), f"argmax, step {i}")
+        assert_no_poison(lse, f"lse, step {i}")
         lg_ = lse.cpu().numpy().astype(np.float64)
         fin = np.isfinite(l_o)
         assert (np.isfinite(lg_) == fin).all()
         assert np.abs(lg_[fin] - l_o[fin]).max(initial=0) < TOL
         if logprobs:
+            assert_no_poison(lp, f"log-probs, step {i}")
             pg = lp.cpu().numpy().astype(np.float64)
             f2 = np.isfinite(lp_o)
             assert (np.isfinite(pg) == f2).all()
@@ -82,7 +87,7 @@ def test_table_driven_invalid_states_and_tokens():
     assert a[0] == -1 and a[1] == -1 and a[2] == -1     # out of range, out of range, dead state
     assert d.device_error() == B.DEVERR_BAD_STATE
     toks = dev(np.array([-1, V, w.vocab.eos_id, 5], np.int32))
-    out = torch.empty(4, dtype=torch.int32, device="cuda")
+    out = poison.empty(4, torch.int32)
     d.advance_table(nxt, dev(np.array([1, 1, 1, Q], np.int32)), toks, states_out=out)
     o = out.cpu().numpy()
     assert o[0] == w.automaton.start and o[1] == 0 and o[2] == w.automaton.start and o[3] == 0
