@@ -52,6 +52,7 @@ extern "C" {
 #define DOMINO_DEVERR_BAD_STATE 1u
 #define DOMINO_DEVERR_BAD_STACK 2u
 #define DOMINO_DEVERR_BAD_TOKEN 4u
+#define DOMINO_DEVERR_INTERNAL 8u   /* a kernel's own consistency check failed (a library bug) */
 
 #define DOMINO_RULE_PUSH 1
 #define DOMINO_RULE_POP 2
@@ -96,6 +97,9 @@ typedef struct {
     int32_t table_in_smem; /* 1 when the transition table is staged in shared memory */
     int32_t device;        /* CUDA ordinal, -1 for a host-only handle */
     int64_t device_bytes;  /* device memory the handle owns */
+    int32_t walk_tree;     /* 1: the mask step walks the vocabulary's prefix tree (domino_get_prefix_tree);
+                              0: it walks every token on its own */
+    int32_t tree_units;    /* subtrees the tree walk deals out (0 without a tree) */
 } domino_info;
 
 /* Creates a handle on CUDA device `cuda_device` (it becomes the current device
@@ -136,6 +140,31 @@ int domino_get_info(domino_t h, domino_info* out);
 
 /* Byte -> class id map of the loaded automaton (256 bytes, host). */
 int domino_get_byte_classes(domino_t h, uint8_t* classes_out);
+
+/* The prefix tree that the mask step walks (host copies, for inspection):
+ * Alg. 2's subterminal tree (Sec. 3.3) over the byte-class strings of every
+ * token except EOS and empty tokens.  Nodes are numbered in preorder, children
+ * by class; node n is 8 uint32 words:
+ *   [0] skip | cls << 24  (n's subtree is nodes [n, skip); cls: the class on
+ *                          the edge into n, 0 for the root, node 0)
+ *   [1] tok_lo  [2] n_end [3] tok_hi   (tokens_out[tok_lo, tok_lo + n_end) end
+ *                          at n; tokens_out[tok_lo, tok_hi) are n's subtree's)
+ *   [4] [5] the classes on the edges below n, a 64-bit set (when K <= 64)
+ *   [6] [7] 0
+ * tokens_out: original token ids in preorder.
+ * upper_out [n_upper][2] = {node, depth}: the root and every node whose
+ *   subtree has more than 64 nodes or more than 8 branching levels, in
+ *   preorder; a row's configuration at each of them is computed first.
+ * units_out [n_units][2] = {root node, index of its parent in upper_out}: the
+ *   subtrees hanging off upper nodes, in preorder; each live (row, unit) pair
+ *   is walked on its own.
+ * sizes_out[4] (required) = {nodes, tokens, upper nodes, units}.  Each array
+ * is copied up to its capacity (in entries) and may be NULL.  Available on
+ * host-only handles too.  DOMINO_E_UNSUPPORTED: the tree exceeds 2^24 - 1
+ * nodes (the mask step then walks every token on its own). */
+int domino_get_prefix_tree(domino_t h, uint32_t* nodes_out, int64_t nodes_cap, int32_t* tokens_out,
+                           int64_t tokens_cap, uint32_t* upper_out, int64_t upper_cap, uint32_t* units_out,
+                           int64_t units_cap, int64_t* sizes_out);
 
 /* Offline precompute (Alg. 2's "for every state q, for every token l,
  * traverse"; Sec. 3.5 "computed before inference starts"): for every state

@@ -25,6 +25,7 @@ DTYPE_BF16 = 1
 DEVERR_BAD_STATE = 1
 DEVERR_BAD_STACK = 2
 DEVERR_BAD_TOKEN = 4
+DEVERR_INTERNAL = 8
 STATUS = {0: "OK", -1: "E_INVALID_ARG", -2: "E_NOT_LOADED", -3: "E_UNSUPPORTED", -4: "E_OOM", -5: "E_CUDA",
           -6: "E_NO_DEVICE"}
 
@@ -44,7 +45,8 @@ class StackRule(ctypes.Structure):
 class Info(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "n_tokens", "n_words", "eos_id", "max_token_len", "n_states", "n_classes", "start_state", "max_depth",
-        "n_rules", "has_stack", "table_in_smem", "device")] + [("device_bytes", ctypes.c_int64)]
+        "n_rules", "has_stack", "table_in_smem", "device")] + [("device_bytes", ctypes.c_int64), ("walk_tree", ctypes.c_int32),
+                                                              ("tree_units", ctypes.c_int32)]
 
 
 _lib = None
@@ -59,6 +61,7 @@ _SIGS = {
     "domino_load_automaton": [P, P, I32, P, P, I32, P, I32, I32],
     "domino_get_info": [P, P],
     "domino_get_byte_classes": [P, P],
+    "domino_get_prefix_tree": [P, P, I64, P, I64, P, I64, P, I64, P],
     "domino_precompute_table": [P, P, P, P],
     "domino_step_mask": [P, P, P, I32, P, P, P],
     "domino_mask_logits": [P, P, I32, I32, I64, P, P, P, P, P],
@@ -187,6 +190,20 @@ def domino_get_byte_classes(h: int) -> np.ndarray:
     out = np.zeros(256, dtype=np.uint8)
     _check("domino_get_byte_classes", lib().domino_get_byte_classes(h, _ptr(out)))
     return out
+
+
+def domino_get_prefix_tree(h: int):
+    """(nodes uint32 [n][8], tokens int32, upper uint32 [u][2], units uint32 [k][2]) of the handle's prefix tree."""
+    sizes = np.zeros(4, dtype=np.int64)
+    _check("domino_get_prefix_tree", lib().domino_get_prefix_tree(h, None, 0, None, 0, None, 0, None, 0, _ptr(sizes)))
+    nodes = np.zeros((int(sizes[0]), 8), dtype=np.uint32)
+    toks = np.zeros(int(sizes[1]), dtype=np.int32)
+    upper = np.zeros((int(sizes[2]), 2), dtype=np.uint32)
+    units = np.zeros((int(sizes[3]), 2), dtype=np.uint32)
+    _check("domino_get_prefix_tree", lib().domino_get_prefix_tree(h, _ptr(nodes), nodes.shape[0], _ptr(toks),
+                                                                   toks.shape[0], _ptr(upper), upper.shape[0],
+                                                                   _ptr(units), units.shape[0], _ptr(sizes)))
+    return nodes, toks, upper, units
 
 
 def domino_precompute_table(h: int, next_dev, mask_dev, stream=None) -> None:

@@ -1,7 +1,7 @@
 """Builds libdomino.so in-tree with nvcc for sm_103a (GB300).
 
-Two translation units (host.cpp: C ABI and loaders; kernels.cu: kernels) are
-compiled in parallel and linked into paper_2403_06988_gb300/libdomino.so.
+Three translation units (host.cpp: C ABI and loaders; kernels.cu and trie.cu:
+kernels) are compiled in parallel and linked into paper_2403_06988_gb300/libdomino.so.
 Objects go to paper_2403_06988_gb300/_build/.
 """
 from __future__ import annotations
@@ -17,7 +17,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libdomino.so")
-SOURCES = ["host.cpp", "kernels.cu"]
+SOURCES = ["host.cpp", "kernels.cu", "trie.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -30,7 +30,8 @@ def nvcc() -> str:
 
 def _inputs():
     files = [os.path.join(CSRC, f) for f in SOURCES]
-    files += [os.path.join(CSRC, "domino_internal.h"), os.path.join(INCLUDE, "domino.h")]
+    files += [os.path.join(CSRC, "domino_internal.h"), os.path.join(CSRC, "walk_common.cuh"),
+              os.path.join(INCLUDE, "domino.h")]
     return files
 
 

@@ -72,6 +72,46 @@ struct StepView {
     uint32_t* err;            // sticky device error word
 };
 
+// Prefix tree of the vocabulary's byte-class strings (the subterminal tree of
+// Sec. 3.3, Alg. 2, over byte classes): a prefix shared by many tokens takes
+// its transitions once per row, and a subtree whose prefix dies is never
+// entered.  Nodes are numbered in preorder (children by class), so a subtree
+// is the contiguous range [n, skip) and the tokens of a subtree are a
+// contiguous range of `dtok`: the tokens that end at n first, then those of
+// its children's subtrees.
+//   node[2n]     = {skip | cls << 24, tok_lo, n_end, tok_hi}
+//   node[2n + 1] = {sub_lo, sub_hi, 0, 0}
+// cls: the class on the edge into n; [tok_lo, tok_lo + n_end): tokens ending
+// at n; [tok_lo, tok_hi): tokens of the subtree; sub: the classes on the edges
+// below n (K <= 64, for the self-loop skip).
+// Upper nodes: the root and every node whose subtree has more than kTrieTile
+// nodes or more than kTrieBranch branching levels (an ancestor of an upper
+// node is upper).  Units: the subtrees hanging off upper nodes.  The units are
+// cut into per-CTA batches that fit in shared memory; for a block of rows a
+// CTA computes each row's configuration at the upper nodes its units hang
+// off ("slots"), then a warp walks a unit for up to 32 rows live at its slot
+// at once, in lockstep over the unit's nodes, with a stack of at most
+// kTrieBranch levels (tree_tile_kernel).  The tokens that end at an upper
+// node are set by the one batch that lists that node as an emitting slot.
+constexpr int kTrieTile = 64;
+constexpr int kTrieBranch = 8;
+constexpr int kTrieMaxSlots = 48;             // slots per batch
+constexpr int32_t kTrieMaxNodes = (1 << 24) - 1;
+
+struct TrieView {
+    const uint4* node;        // [n_nodes][2]
+    const int32_t* dtok;      // original ids in preorder
+    const uint4* upper;       // [n_upper]: {node, path offset, path length, 0}
+    const uint8_t* upath;     // classes of the upper nodes' paths from the root
+    const uint4* batch;       // [n_batches][2]: {first unit, end unit, first node, end node},
+                              //                 {first token, end token, first slot, end slot}
+    const uint4* slot;        // {upper index, first token ending at its node, tokens it sets (0: none), 0}
+    const uint2* unit;        // {root node, slot index within the batch}
+    const int32_t* cta_batch; // [grid + 1]: CTA c takes batches [cta_batch[c], cta_batch[c + 1])
+    int32_t n_nodes, n_upper, grid;
+    int32_t max_nodes, max_toks, max_units, max_slots, max_path;   // the largest batch
+};
+
 struct LaunchEnv {
     int num_sms;
     int max_smem_optin;
@@ -98,6 +138,17 @@ cudaError_t launch_step_mask(const StepView& v, const LaunchEnv& env, bool stack
 cudaError_t launch_fused_combine(const StepView& v, bool stack, int mode, const float4* part, int32_t batch,
                                  int32_t n_windows, int32_t* argmax, float* lse, const int32_t* states,
                                  const uint64_t* stacks, int32_t* states_out, uint64_t* stacks_out, cudaStream_t st);
+
+// The mask step over the prefix tree: tree_clear_kernel (one warp per row:
+// clears the row's mask and next states, sets EOS), then tree_tile_kernel
+// (the units, from shared memory).  states / stacks / batch / row_is_state /
+// mask / next / row_ids / row_count as launch_step_mask.  mode: where the tile
+// kernel reads transitions.
+int trie_tile_smem_bytes(const StepView& v, const TrieView& tv, bool stack, int table_bytes);
+cudaError_t launch_trie_step(const StepView& v, const TrieView& tv, const LaunchEnv& env, bool stack, int mode,
+                             const int32_t* states, const uint64_t* stacks, int32_t batch, bool row_is_state,
+                             uint32_t* mask, int32_t* next, cudaStream_t st, const int32_t* row_ids = nullptr,
+                             const int32_t* row_count = nullptr);
 
 // Log-probabilities only (bf16 logits, rows on 16-byte boundaries), given the
 // rows' lse: logprobs[b][t] = logit - lse[b] for allowed t, -inf else.

@@ -7,6 +7,7 @@
 #include <chrono>
 #include <cmath>
 #include <cstdint>
+#include <cstdlib>
 #include <cstring>
 #include <new>
 #include <numeric>
@@ -58,6 +59,27 @@ struct domino_ctx {
     DevBuf d_dense, d_sparse, d_accept, d_self, d_tok_cls;
     DevBuf d_err, d_partials, d_counters, d_lse_tmp, d_fpart;
     bool arena_ready = false;
+    // prefix tree of the class strings and its per-CTA batches (see TrieView)
+    DevBuf d_tnode, d_tdtok, d_tupper, d_tupath, d_tbatch, d_tslot, d_tunit, d_tcta;
+    std::vector<uint4> t_node;       // host copies (domino_get_prefix_tree)
+    std::vector<int32_t> t_dtok;
+    std::vector<uint4> t_upper;      // {node, path offset, path length, 0}
+    std::vector<uint8_t> t_upath;
+    std::vector<uint2> t_unit;       // {root node, parent upper index}
+    // per-CTA batches (see TrieView)
+    std::vector<uint4> t_batch;      // two per batch
+    std::vector<uint4> t_slot;
+    std::vector<uint2> t_bunit;      // {root node, slot within the batch}
+    std::vector<int32_t> t_cta;      // [grid + 1] first batch of each CTA
+    int32_t t_nodes = 0, t_grid = 0;
+    int32_t t_max_nodes = 0, t_max_toks = 0, t_max_units = 0, t_max_slots = 0, t_max_path = 0;
+    int t_mode = kDenseGlobal;       // where the tile kernel reads transitions
+    bool trie_built = false;         // host arrays valid
+    bool trie_ready = false;         // device copies valid
+    // which walk the mask step takes: -1 chosen from the automaton (see
+    // use_tree), 1 the prefix tree, 0 every token on its own (DOMINO_WALK=tree
+    // or =token in the environment when the handle is created)
+    int walk_pref = -1;
     int32_t n_windows = 0;
     // staging for domino_decode_step_host
     // s_io packs the step's small inputs and outputs (see io_layout) so that
@@ -90,6 +112,9 @@ struct domino_ctx {
 };
 
 namespace {
+
+StepView make_view(domino_ctx* h);
+int cuda_status(cudaError_t e);
 
 struct DeviceGuard {
     int prev = -1;
@@ -148,6 +173,288 @@ void clear_host_graphs(domino_ctx* h) {
     for (auto& g : h->host_graphs) cudaGraphExecDestroy(g.exec);
     h->host_graphs.clear();
     h->t_wall_ms[0] = h->t_wall_ms[1] = 0.0;   // the paths are timed afresh
+}
+
+// The prefix tree of the tokens' class strings (TrieView), built from the
+// tokens sorted by class string: a token shares with its predecessor the
+// nodes of their longest common prefix and opens new nodes for the rest, so
+// nodes come out in preorder.  EOS and empty tokens are not in the tree (the
+// kernel sets EOS from the row's acceptance; other empty tokens are never
+// allowed).  Host arrays only; build_trie uploads them.
+void build_trie_host(domino_ctx* h) {
+    h->trie_built = h->trie_ready = false;
+    h->t_node.clear();
+    h->t_dtok.clear();
+    h->t_upper.clear();
+    h->t_upath.clear();
+    h->t_unit.clear();
+    if (!h->vocab_loaded || !h->auto_loaded) return;
+    std::vector<uint8_t> cls(h->tok_bytes.size());
+    for (size_t i = 0; i < cls.size(); i++) cls[i] = h->byte_class[h->tok_bytes[i]];
+    std::vector<int32_t> order;
+    order.reserve((size_t)h->V);
+    for (int32_t t = 0; t < h->V; t++)
+        if (t != h->eos_id && h->tok_off[t + 1] > h->tok_off[t]) order.push_back(t);
+    auto str = [&](int32_t t) { return cls.data() + h->tok_off[t]; };
+    auto len = [&](int32_t t) { return (size_t)(h->tok_off[t + 1] - h->tok_off[t]); };
+    std::sort(order.begin(), order.end(), [&](int32_t a, int32_t b) {
+        const size_t la = len(a), lb = len(b);
+        const int c = std::memcmp(str(a), str(b), std::min(la, lb));
+        if (c != 0) return c < 0;
+        if (la != lb) return la < lb;
+        return a < b;
+    });
+    std::vector<uint32_t> skip, tok_lo, n_end, tok_hi;
+    std::vector<uint8_t> ncls;
+    std::vector<int32_t> dtok;
+    dtok.reserve(order.size());
+    std::vector<uint32_t> path;   // open nodes, root first
+    auto open_node = [&](uint8_t c) {
+        path.push_back((uint32_t)skip.size());
+        skip.push_back(0);
+        tok_lo.push_back((uint32_t)dtok.size());
+        n_end.push_back(0);
+        tok_hi.push_back(0);
+        ncls.push_back(c);
+    };
+    auto close_node = [&]() {
+        const uint32_t n = path.back();
+        path.pop_back();
+        skip[n] = (uint32_t)skip.size();
+        tok_hi[n] = (uint32_t)dtok.size();
+    };
+    open_node(0);   // root
+    const uint8_t* prev = nullptr;
+    size_t prev_len = 0;
+    for (int32_t t : order) {
+        const uint8_t* s = str(t);
+        const size_t L = len(t);
+        size_t l = 0;
+        while (prev && l < std::min(L, prev_len) && prev[l] == s[l]) l++;
+        while (path.size() > l + 1) close_node();
+        for (size_t d = l; d < L; d++) open_node(s[d]);
+        if (skip.size() > (size_t)kTrieMaxNodes) return;   // too large: the per-token walk is used
+        n_end[path.back()]++;
+        dtok.push_back(t);
+        prev = s;
+        prev_len = L;
+    }
+    while (!path.empty()) close_node();
+    const uint32_t N = (uint32_t)skip.size();
+    // parents, branching heights and the classes below each node (children
+    // have larger ids than their parent: one reverse pass)
+    std::vector<uint32_t> parent(N, 0), bh(N, 0);
+    std::vector<uint64_t> sub(N, 0);
+    const bool subs = h->K <= 64;
+    for (uint32_t n = N; n-- > 0;) {
+        uint32_t m = 0, k = 0;
+        for (uint32_t c = n + 1; c < skip[n]; c = skip[c]) {
+            k++;
+            parent[c] = n;
+            m = std::max(m, bh[c]);
+            if (subs) sub[n] |= (1ull << ncls[c]) | sub[c];
+        }
+        bh[n] = m + (k >= 2 ? 1u : 0u);
+    }
+    // upper nodes (an ancestor of an upper node is upper: subtree size and
+    // branching height only grow towards the root), their paths, and the
+    // units: the subtrees hanging off upper nodes
+    std::vector<int32_t> uidx(N, -1);
+    std::vector<uint4> upper;
+    std::vector<uint8_t> upath;
+    std::vector<uint2> unit;
+    for (uint32_t n = 0; n < N;) {
+        const bool up = n == 0 || skip[n] - n > (uint32_t)kTrieTile || bh[n] > (uint32_t)kTrieBranch;
+        if (up) {
+            uidx[n] = (int32_t)upper.size();
+            const uint32_t off = (uint32_t)upath.size();
+            uint32_t plen = 0;
+            if (n != 0) {
+                const uint4 pu = upper[(size_t)uidx[parent[n]]];
+                upath.insert(upath.end(), upath.begin() + pu.y, upath.begin() + pu.y + pu.z);
+                upath.push_back(ncls[n]);
+                plen = pu.z + 1;
+            }
+            upper.push_back(make_uint4(n, off, plen, 0u));
+            n++;
+        } else {
+            unit.push_back(make_uint2(n, (uint32_t)uidx[parent[n]]));
+            n = skip[n];
+        }
+    }
+    std::vector<uint4> node((size_t)N * 2);
+    for (uint32_t n = 0; n < N; n++) {
+        node[2 * (size_t)n] = make_uint4(skip[n] | ((uint32_t)ncls[n] << 24), tok_lo[n], n_end[n], tok_hi[n]);
+        node[2 * (size_t)n + 1] = make_uint4((uint32_t)sub[n], (uint32_t)(sub[n] >> 32), 0u, 0u);
+    }
+    h->t_node.swap(node);
+    h->t_dtok.swap(dtok);
+    h->t_upper.swap(upper);
+    h->t_upath.swap(upath);
+    h->t_unit.swap(unit);
+    h->t_nodes = (int32_t)N;
+    h->trie_built = true;
+}
+
+// Cuts the units into per-CTA batches that fit in the tile kernel's shared
+// memory next to the transition table, for a grid of one CTA per SM.  Units
+// are dealt out in preorder, about the same number of nodes per CTA; a batch
+// holds a run of one CTA's units, the upper nodes they hang off (slots), and
+// the upper nodes in front of them whose tokens it sets (emitting slots: each
+// upper node with tokens is set by exactly one batch).  Chooses the table
+// placement: in shared memory when that leaves room for batches, else through
+// L1/L2.  false: some unit alone does not fit (the per-token walk is used).
+bool cut_batches(domino_ctx* h) {
+    const int smem = h->env.max_smem_optin > 0 ? h->env.max_smem_optin : 232448;
+    const int grid = h->env.num_sms > 0 ? h->env.num_sms : 1;
+    StepView v = make_view(h);
+    const bool self = !h->self_mask.empty();
+    const std::vector<uint2>& unit = h->t_unit;
+    const std::vector<uint4>& node = h->t_node;
+    const std::vector<uint4>& upper = h->t_upper;
+    auto skip_of = [&](uint32_t n) { return node[2 * (size_t)n].x & 0xFFFFFFu; };
+    // fixed shared memory with an empty batch, per table placement
+    TrieView tv0{};
+    const int fixed = trie_tile_smem_bytes(v, tv0, h->stack, 0) + 1024;
+    constexpr int kMinBatch = 24 * 1024;
+    int mode = kDenseGlobal;
+    int64_t table = 0;
+    const int modes[2] = {kDenseSmem, h->sp_words == 2 ? kSparse32Smem : kSparse64Smem};
+    for (int m : modes) {
+        if (m != kDenseSmem && h->sp_nnz == 0) continue;
+        const int64_t t = table_smem_bytes(v, h->stack, m);
+        if ((int64_t)smem - fixed - t >= kMinBatch) {
+            mode = m;
+            table = t;
+            break;
+        }
+    }
+    std::vector<int64_t> unit_nodes(unit.size());
+    int64_t total = 0;
+    for (size_t u = 0; u < unit.size(); u++) total += unit_nodes[u] = skip_of(unit[u].x) - unit[u].x;
+    const int per_node = 8 + (self ? 8 : 0);
+    for (int64_t budget = (int64_t)smem - fixed - table; budget >= 4096; budget = budget * 9 / 10) {
+        std::vector<uint4> batch, slot;
+        std::vector<uint2> bunit;
+        std::vector<int32_t> cta((size_t)grid + 1, 0);
+        int32_t mx_nodes = 0, mx_toks = 0, mx_units = 0, mx_slots = 0, mx_path = 0;
+        size_t u = 0, up = 0;   // next unit, next upper node whose tokens are unassigned
+        int64_t done = 0;
+        bool ok = true;
+        for (int c = 0; c < grid && ok; c++) {
+            cta[(size_t)c] = (int32_t)(batch.size() / 2);
+            const int64_t goal = total * (c + 1) / grid;
+            size_t ue = u;
+            while (ue < unit.size() && (done < goal || c == grid - 1)) done += unit_nodes[ue++];
+            while (u < ue && ok) {
+                // one batch: units [u, b1) of this CTA
+                const uint32_t n0 = unit[u].x, t0 = node[2 * (size_t)n0].y;
+                const size_t slot0 = slot.size(), unit0 = bunit.size();
+                std::vector<std::pair<uint32_t, uint32_t>> slots;   // (upper index, slot)
+                auto slot_of = [&](uint32_t ui, bool emit) -> int {
+                    for (auto& p : slots)
+                        if (p.first == ui) return (int)p.second;
+                    if ((int)slots.size() >= kTrieMaxSlots) return -1;
+                    const uint32_t n = upper[ui].x;
+                    slot.push_back(make_uint4(ui, node[2 * (size_t)n].y, emit ? node[2 * (size_t)n].z : 0u, 0u));
+                    slots.emplace_back(ui, (uint32_t)slots.size());
+                    mx_path = std::max<int32_t>(mx_path, (int32_t)upper[ui].z);
+                    return (int)slots.size() - 1;
+                };
+                auto bytes_now = [&](uint32_t n1, uint32_t t1) {
+                    return (int64_t)(n1 - n0) * per_node + (int64_t)(t1 - t0) * 4 +
+                           (int64_t)(bunit.size() - unit0) * 4 + (int64_t)slots.size() * (16 + 64);
+                };
+                size_t b1 = u;
+                while (b1 < ue) {
+                    // the upper nodes in front of unit b1 set their tokens here
+                    const size_t keep_slots = slot.size(), keep_units = bunit.size();
+                    const size_t keep_up = up;
+                    const auto keep_list = slots;
+                    bool fit = true;
+                    while (fit && up < upper.size() && upper[up].x < unit[b1].x) {
+                        if (node[2 * (size_t)upper[up].x].z > 0) fit = slot_of((uint32_t)up, true) >= 0;
+                        up++;
+                    }
+                    int sl = fit ? slot_of(unit[b1].y, false) : -1;
+                    fit = sl >= 0;
+                    const uint32_t n1 = skip_of(unit[b1].x), t1 = node[2 * (size_t)unit[b1].x].w;
+                    if (fit) {
+                        bunit.push_back(make_uint2(unit[b1].x, (uint32_t)sl));
+                        fit = n1 - n0 <= 0xFFFFu && t1 - t0 <= 0xFFFFu && bytes_now(n1, t1) <= budget;
+                    }
+                    if (!fit) {   // undo the additions of this unit
+                        slot.resize(keep_slots);
+                        bunit.resize(keep_units);
+                        up = keep_up;
+                        slots = keep_list;
+                        if (b1 == u) ok = false;   // a unit alone does not fit
+                        break;
+                    }
+                    b1++;
+                }
+                if (!ok) break;
+                if (c == grid - 1 && b1 == ue) {   // the last CTA sets the tokens of the trailing upper nodes
+                    while (up < upper.size()) {
+                        if (node[2 * (size_t)upper[up].x].z > 0 && slot_of((uint32_t)up, true) < 0) {
+                            ok = false;
+                            break;
+                        }
+                        up++;
+                    }
+                }
+                const uint32_t n1 = skip_of(unit[b1 - 1].x), t1 = node[2 * (size_t)unit[b1 - 1].x].w;
+                batch.push_back(make_uint4((uint32_t)unit0, (uint32_t)bunit.size(), n0, n1));
+                batch.push_back(make_uint4(t0, t1, (uint32_t)slot0, (uint32_t)slot.size()));
+                mx_nodes = std::max<int32_t>(mx_nodes, (int32_t)(n1 - n0));
+                mx_toks = std::max<int32_t>(mx_toks, (int32_t)(t1 - t0));
+                mx_units = std::max<int32_t>(mx_units, (int32_t)(bunit.size() - unit0));
+                mx_slots = std::max<int32_t>(mx_slots, (int32_t)(slot.size() - slot0));
+                u = b1;
+            }
+        }
+        if (!ok) continue;
+        if (unit.empty()) return false;
+        cta[(size_t)grid] = (int32_t)(batch.size() / 2);
+        TrieView tv{};
+        tv.max_nodes = mx_nodes;
+        tv.max_toks = mx_toks;
+        tv.max_units = mx_units;
+        tv.max_slots = mx_slots;
+        tv.max_path = mx_path;
+        if (trie_tile_smem_bytes(v, tv, h->stack, (int)table) > smem) continue;   // the maxima together: cut tighter
+        h->t_batch.swap(batch);
+        h->t_slot.swap(slot);
+        h->t_bunit.swap(bunit);
+        h->t_cta.swap(cta);
+        h->t_grid = grid;
+        h->t_max_nodes = mx_nodes;
+        h->t_max_toks = mx_toks;
+        h->t_max_units = mx_units;
+        h->t_max_slots = mx_slots;
+        h->t_max_path = mx_path;
+        h->t_mode = mode;
+        return true;
+    }
+    return false;
+}
+
+// The prefix tree and its batches on the device.
+int build_trie(domino_ctx* h) {
+    build_trie_host(h);
+    if (!h->trie_built || !cut_batches(h)) return DOMINO_OK;
+    int rc;
+    auto up = [&](DevBuf& b, const void* p, size_t n) { return dev_upload(b, p, std::max<size_t>(16, n)); };
+    if ((rc = up(h->d_tnode, h->t_node.data(), h->t_node.size() * sizeof(uint4)))) return rc;
+    if ((rc = up(h->d_tdtok, h->t_dtok.data(), h->t_dtok.size() * 4))) return rc;
+    if ((rc = up(h->d_tupper, h->t_upper.data(), h->t_upper.size() * sizeof(uint4)))) return rc;
+    if ((rc = up(h->d_tupath, h->t_upath.data(), h->t_upath.size()))) return rc;
+    if ((rc = up(h->d_tbatch, h->t_batch.data(), h->t_batch.size() * sizeof(uint4)))) return rc;
+    if ((rc = up(h->d_tslot, h->t_slot.data(), h->t_slot.size() * sizeof(uint4)))) return rc;
+    if ((rc = up(h->d_tunit, h->t_bunit.data(), h->t_bunit.size() * sizeof(uint2)))) return rc;
+    if ((rc = up(h->d_tcta, h->t_cta.data(), h->t_cta.size() * 4))) return rc;
+    h->trie_ready = true;
+    return DOMINO_OK;
 }
 
 // Byte-class strings of every token, the window sort and the slot arrays.
@@ -233,6 +540,7 @@ int build_arena(domino_ctx* h) {
     }
     if ((rc = dev_upload(h->d_eos_slot, eos_slot.data(), eos_slot.size() * 2))) return rc;
     h->n_windows = nw;
+    if ((rc = build_trie(h))) return rc;
     h->arena_ready = true;
     return DOMINO_OK;
 }
@@ -282,6 +590,38 @@ int choose_mode(const domino_ctx* h, const StepView& v, bool next) {
     return kDenseGlobal;
 }
 
+TrieView make_trie_view(const domino_ctx* h) {
+    TrieView tv{};
+    tv.node = (const uint4*)h->d_tnode.p;
+    tv.dtok = (const int32_t*)h->d_tdtok.p;
+    tv.upper = (const uint4*)h->d_tupper.p;
+    tv.upath = (const uint8_t*)h->d_tupath.p;
+    tv.batch = (const uint4*)h->d_tbatch.p;
+    tv.slot = (const uint4*)h->d_tslot.p;
+    tv.unit = (const uint2*)h->d_tunit.p;
+    tv.cta_batch = (const int32_t*)h->d_tcta.p;
+    tv.n_nodes = h->t_nodes;
+    tv.n_upper = (int32_t)h->t_upper.size();
+    tv.grid = h->t_grid;
+    tv.max_nodes = h->t_max_nodes;
+    tv.max_toks = h->t_max_toks;
+    tv.max_units = h->t_max_units;
+    tv.max_slots = h->t_max_slots;
+    tv.max_path = h->t_max_path;
+    return tv;
+}
+
+// The tree shares each prefix's transitions among the tokens below it and
+// drops a subtree as soon as its prefix dies, so it wins when most prefixes
+// die early (sparse masks).  States that loop on many classes (strings,
+// numbers, whitespace: the self-loop mask) keep long prefixes alive and make
+// rows dense; there the per-token walk, which skips a whole token whose later
+// classes all loop on the state, is faster.
+bool use_tree(const domino_ctx* h) {
+    if (!h->trie_ready || h->walk_pref == 0) return false;
+    return h->walk_pref == 1 || h->self_mask.empty();
+}
+
 int ready_for_compute(domino_ctx* h) {
     if (!h) return DOMINO_E_INVALID_ARG;
     if (is_host_only(h)) return DOMINO_E_NO_DEVICE;
@@ -329,6 +669,10 @@ int domino_create(domino_t* out, int32_t cuda_device) {
     domino_ctx* h = new (std::nothrow) domino_ctx();
     if (!h) return DOMINO_E_OOM;
     h->device = cuda_device < 0 ? -1 : cuda_device;
+    if (const char* w = std::getenv("DOMINO_WALK")) {
+        if (std::strcmp(w, "token") == 0) h->walk_pref = 0;
+        if (std::strcmp(w, "tree") == 0) h->walk_pref = 1;
+    }
     if (h->device >= 0) {
         int n = 0;
         if (cudaGetDeviceCount(&n) != cudaSuccess || cuda_device >= n) {
@@ -369,7 +713,8 @@ int domino_destroy(domino_t h) {
         DevBuf* all[] = {&h->d_head, &h->d_info, &h->d_tail_off, &h->d_tail, &h->d_pos_of, &h->d_cls_start,
                          &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_self, &h->d_tok_cls, &h->d_err, &h->d_fpart, &h->d_partials,
                          &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_mask, &h->s_io,
-                         &h->o_prop, &h->o_rows, &h->o_count};
+                         &h->o_prop, &h->o_rows, &h->o_count, &h->d_tnode, &h->d_tdtok, &h->d_tupper, &h->d_tupath, &h->d_tbatch, &h->d_tslot,
+                         &h->d_tunit, &h->d_tcta};
         for (auto* b : all) dev_free(*b);
         for (cudaEvent_t& e : h->ev_chunk)
             if (e) cudaEventDestroy(e);
@@ -411,7 +756,10 @@ int domino_load_vocab(domino_t h, const uint8_t* bytes, const int64_t* offsets, 
     h->eos_id = eos_id;
     h->max_len = max_len;
     h->vocab_loaded = true;
-    if (is_host_only(h)) return DOMINO_OK;
+    if (is_host_only(h)) {
+        build_trie_host(h);
+        return DOMINO_OK;
+    }
     return build_arena(h);
 }
 
@@ -616,7 +964,10 @@ int domino_load_automaton(domino_t h, const int32_t* delta, int32_t n_states, co
             if (!h->ret.empty()) std::memcpy(sparse_img.data() + h->sp_ret_off, h->ret.data(), h->ret.size() * 2);
         }
     }
-    if (is_host_only(h)) return DOMINO_OK;
+    if (is_host_only(h)) {
+        build_trie_host(h);
+        return DOMINO_OK;
+    }
     int rc;
     if ((rc = dev_upload(h->d_dense, dense_img.data(), dense_img.size()))) return rc;
     if (!sparse_img.empty()) {
@@ -652,6 +1003,8 @@ int domino_get_info(domino_t h, domino_info* out) {
         out->table_in_smem = choose_mode(h, v, false) != kDenseGlobal ? 1 : 0;
     }
     out->device_bytes = dev_bytes(h);
+    out->walk_tree = use_tree(h) ? 1 : 0;
+    out->tree_units = h->trie_ready ? (int32_t)h->t_bunit.size() : 0;
     return DOMINO_OK;
 }
 
@@ -659,6 +1012,33 @@ int domino_get_byte_classes(domino_t h, uint8_t* classes_out) {
     if (!h || !classes_out) return DOMINO_E_INVALID_ARG;
     if (!h->auto_loaded) return DOMINO_E_NOT_LOADED;
     std::memcpy(classes_out, h->byte_class, 256);
+    return DOMINO_OK;
+}
+
+int domino_get_prefix_tree(domino_t h, uint32_t* nodes_out, int64_t nodes_cap, int32_t* tokens_out,
+                           int64_t tokens_cap, uint32_t* upper_out, int64_t upper_cap, uint32_t* units_out,
+                           int64_t units_cap, int64_t* sizes_out) {
+    if (!h || !sizes_out || nodes_cap < 0 || tokens_cap < 0 || upper_cap < 0 || units_cap < 0)
+        return DOMINO_E_INVALID_ARG;
+    if (!h->vocab_loaded || !h->auto_loaded) return DOMINO_E_NOT_LOADED;
+    if (!h->trie_built) return DOMINO_E_UNSUPPORTED;
+    const int64_t nu = (int64_t)h->t_upper.size(), nn = (int64_t)h->t_unit.size();
+    sizes_out[0] = h->t_nodes;
+    sizes_out[1] = (int64_t)h->t_dtok.size();
+    sizes_out[2] = nu;
+    sizes_out[3] = nn;
+    if (nodes_out)
+        std::memcpy(nodes_out, h->t_node.data(), (size_t)std::min<int64_t>(nodes_cap, h->t_nodes) * 2 * sizeof(uint4));
+    if (tokens_out)
+        std::memcpy(tokens_out, h->t_dtok.data(), (size_t)std::min<int64_t>(tokens_cap, (int64_t)h->t_dtok.size()) * 4);
+    for (int64_t i = 0; upper_out && i < std::min(upper_cap, nu); i++) {
+        upper_out[2 * i] = h->t_upper[(size_t)i].x;
+        upper_out[2 * i + 1] = h->t_upper[(size_t)i].z;
+    }
+    for (int64_t i = 0; units_out && i < std::min(units_cap, nn); i++) {
+        units_out[2 * i] = h->t_unit[(size_t)i].x;
+        units_out[2 * i + 1] = h->t_unit[(size_t)i].y;
+    }
     return DOMINO_OK;
 }
 
@@ -671,6 +1051,10 @@ int domino_step_mask(domino_t h, const int32_t* states_dev, const uint64_t* stac
     if (batch == 0) return DOMINO_OK;
     DeviceGuard g(h->device);
     StepView v = make_view(h);
+    if (use_tree(h)) {
+        return cuda_status(launch_trie_step(v, make_trie_view(h), h->env, h->stack, h->t_mode, states_dev, stacks_dev,
+                                            batch, false, mask_dev, next_dev, (cudaStream_t)stream));
+    }
     const int mode = choose_mode(h, v, next_dev != nullptr);
     return cuda_status(launch_step_mask(v, h->env, h->stack, mode, states_dev, stacks_dev, batch, false, mask_dev,
                                         next_dev, (cudaStream_t)stream));
@@ -684,6 +1068,10 @@ int domino_precompute_table(domino_t h, int32_t* next_dev, uint32_t* mask_dev, v
     if (h->stack) return DOMINO_E_UNSUPPORTED;
     DeviceGuard g(h->device);
     StepView v = make_view(h);
+    if (use_tree(h)) {
+        return cuda_status(launch_trie_step(v, make_trie_view(h), h->env, false, h->t_mode, nullptr, nullptr, h->Q,
+                                            true, mask_dev, next_dev, (cudaStream_t)stream));
+    }
     const int mode = choose_mode(h, v, next_dev != nullptr);
     return cuda_status(launch_step_mask(v, h->env, false, mode, nullptr, nullptr, h->Q, true, mask_dev, next_dev,
                                         (cudaStream_t)stream));
@@ -749,6 +1137,7 @@ int domino_step_decode(domino_t h, const int32_t* states_dev, const uint64_t* st
         return domino_advance(h, states_dev, stacks_dev, argmax_dev, batch, states_out, stacks_dev ? stacks_out : nullptr,
                               stream);
     }
+    StepView v = make_view(h);
     const size_t part_bytes = (size_t)batch * (size_t)h->n_windows * sizeof(float4);
     if (h->d_fpart.n < part_bytes) {
         // growing the partials buffer synchronises the stream and reallocates,
@@ -766,7 +1155,6 @@ int domino_step_decode(domino_t h, const int32_t* states_dev, const uint64_t* st
     cudaPointerAttributes pa{};
     const bool on_device = cudaPointerGetAttributes(&pa, logits_dev) == cudaSuccess && pa.type == cudaMemoryTypeDevice;
     if (!on_device) cudaGetLastError();
-    StepView v = make_view(h);
     const int mode = choose_mode(h, v, false);
     cudaError_t e = launch_step_mask(v, h->env, h->stack, mode, states_dev, stacks_dev, batch, false, mask_dev, nullptr,
                                      st, nullptr, nullptr, logits_dev, row_stride_elems, (float4*)h->d_fpart.p,

@@ -1,0 +1,541 @@
+// trie.cu -- C.mask() over the prefix tree of the vocabulary (sm_103a).
+//
+// The mask of a row is the set of tokens whose class string can be walked
+// from the row's configuration without reaching the dead state (Alg. 1's
+// mask at lookahead k = infinity, Sec. 3.5; EOS iff the state accepts with an
+// empty stack).  Walking the prefix tree of all class strings (the
+// subterminal tree of Sec. 3.3 / Alg. 2, over byte classes) takes each shared
+// prefix's transitions once per row and never enters a subtree whose prefix
+// died; it reorders and shares the per-token walks of the plain definition
+// without changing their result.
+//
+// Two kernels (see TrieView for the tree's layout and its batches):
+//  tree_clear_kernel  one warp per row: clears the row's mask (and next
+//                     states) and sets EOS when the state accepts with an
+//                     empty stack.
+//  tree_tile_kernel   persistent CTAs, one per SM.  For each of its batches a
+//                     CTA stages the batch's units (compact node records, the
+//                     units' tokens) in shared memory next to the transition
+//                     table; then, a block of rows at a time:
+//                       1. each row's configuration at every slot (the upper
+//                          nodes the units hang off), by walking the slot's
+//                          path from the row's configuration;
+//                       2. per slot, the list of rows live there; emitting
+//                          slots set the bits of the tokens ending at them;
+//                       3. warps claim units: a warp walks its unit for up to
+//                          32 of the slot's live rows at once, one row per
+//                          lane, in lockstep over the unit's nodes in
+//                          preorder; a subtree is entered while it is live for
+//                          some lane and skipped when it is dead for all; the
+//                          siblings still to visit are kept on a per-warp
+//                          stack (one level per branching node, at most
+//                          kTrieBranch).  A node's tokens set their bits with
+//                          global reductions (and store their next state): a
+//                          few at a time for all the lanes a node is live in,
+//                          or, for long token ranges -- and whole subtrees
+//                          whose classes all loop on a lane's state (the
+//                          self-loop skip) -- spread over the warp's lanes.
+#include <cuda_runtime.h>
+
+#include <climits>
+#include <cstdint>
+#include <mutex>
+
+#include "domino_internal.h"
+#include "walk_common.cuh"
+
+namespace domino {
+namespace {
+
+constexpr int kTileThreads = 1024;
+constexpr int kTileWarps = kTileThreads / 32;
+constexpr int kClearThreads = 256;          // 8 rows per CTA, one warp each
+constexpr int kTrieCfg = 4096;              // (slot, row) configurations per row block
+constexpr int kTrieRowBlock = 512;          // most rows per block
+constexpr int kTrieEmitWarp = 32;           // longer token ranges are spread over the warp's lanes
+constexpr int kTrieMaxDevices = 64;
+
+enum TileCtl : int {
+    kCtlUnit = 0,     // units claimed in this row block
+    kCtlBad = 1,      // a staged record failed its check
+    kCtlWords = 4,
+};
+
+// Shared-memory layout of the tile kernel (byte offsets).
+struct TileLayout {
+    int accept, self, table, nodes, sub, toks, units, slots, paths, rowcfg, cfg, lrows, lcount, stk, ustk, ctl, total;
+};
+
+__host__ __device__ inline TileLayout tile_layout(int Q, bool self, bool stack, int table_bytes, const TrieView& tv) {
+    TileLayout L{};
+    int o = 0;
+    L.accept = o;  o += align16(((Q + 31) / 32) * 4);
+    L.self = o;    o += self ? align16(Q * 8) : 0;
+    L.table = o;   o += align16(table_bytes);
+    L.nodes = o;   o += align16(tv.max_nodes * 8);
+    L.sub = o;     o += self ? align16(tv.max_nodes * 8) : 0;
+    L.toks = o;    o += align16(tv.max_toks * 4);
+    L.units = o;   o += align16(tv.max_units * 4);
+    L.slots = o;   o += align16(tv.max_slots * 16);
+    L.paths = o;   o += align16(tv.max_slots * tv.max_path);
+    L.rowcfg = o;  o += kTrieRowBlock * 16;
+    L.cfg = o;     o += kTrieCfg * (stack ? 8 : 4);
+    L.lrows = o;   o += kTrieCfg * 2;
+    L.lcount = o;  o += align16(kTrieMaxSlots * 4);
+    L.stk = o;     o += kTileWarps * kTrieBranch * 32 * (stack ? 8 : 4);
+    L.ustk = o;    o += kTileWarps * kTrieBranch * 8;
+    L.ctl = o;     o += kCtlWords * 4;
+    L.total = align16(o);
+    return L;
+}
+
+struct TreeArgs {
+    const int32_t* states;
+    const uint64_t* stacks;
+    int32_t batch;          // rows (the cap of a row list)
+    int32_t row_is_state;
+    uint32_t* mask;
+    int32_t* next;
+    int32_t img_bytes, img_tgt_off, img_ret_off;
+};
+
+// Sets a mask bit without waiting for the result (a reduction, not an atomic
+// that returns the old word).
+__device__ __forceinline__ void set_bit(uint32_t* word, uint32_t bit) {
+    asm volatile("red.global.or.b32 [%0], %1;" ::"l"(word), "r"(bit) : "memory");
+}
+
+// ---------------------------------------------------------------------------
+// tree_clear_kernel
+// ---------------------------------------------------------------------------
+template <bool NEXT>
+__global__ void __launch_bounds__(kClearThreads)
+    tree_clear_kernel(const __grid_constant__ StepView v, const __grid_constant__ TreeArgs a, const RowList list) {
+    pdl_wait();
+    pdl_trigger();
+    const int lane = threadIdx.x & 31;
+    const int i = blockIdx.x * (kClearThreads / 32) + (threadIdx.x >> 5);
+    if (i >= list.rows(a.batch)) return;
+    const int W = v.W, V = v.V;
+    uint32_t* mrow = a.mask ? a.mask + (size_t)i * W : nullptr;
+    int32_t* nrow = NEXT && a.next ? a.next + (size_t)i * V : nullptr;
+    if (mrow) {
+        if ((W & 3) == 0 && (reinterpret_cast<uintptr_t>(mrow) & 15) == 0) {
+            for (int j = lane; j < W / 4; j += 32) reinterpret_cast<uint4*>(mrow)[j] = make_uint4(0u, 0u, 0u, 0u);
+        } else {
+            for (int j = lane; j < W; j += 32) mrow[j] = 0u;
+        }
+    }
+    if (nrow) {
+        if ((V & 3) == 0 && (reinterpret_cast<uintptr_t>(nrow) & 15) == 0) {
+            for (int j = lane; j < V / 4; j += 32) __stcs(reinterpret_cast<int4*>(nrow) + j, make_int4(0, 0, 0, 0));
+        } else {
+            for (int j = lane; j < V; j += 32) nrow[j] = 0;
+        }
+    }
+    __syncwarp();   // the row is clear before its EOS bit is set
+    if (lane == 0) {   // the row's configuration: invalid ones set the error word; EOS
+        const int b = list.row(i);
+        uint4 rc;
+        if (a.row_is_state) {
+            const uint32_t q = (uint32_t)b;
+            rc = make_uint4(q, 0u, 0u, 1u | (((__ldg(v.accept_bits + (q >> 5)) >> (q & 31u)) & 1u) ? 2u : 0u));
+        } else {
+            const int32_t sv = __ldg(a.states + b);
+            const unsigned long long w =
+                a.stacks ? __ldg(reinterpret_cast<const unsigned long long*>(a.stacks) + b) : 0ull;
+            rc = decode_row(v, sv, w, a.stacks != nullptr, v.accept_bits, true);
+        }
+        // EOS: allowed iff the state accepts and the stack is empty; the state stays
+        if ((rc.w & 2u) && v.eos_id >= 0) {
+            if (mrow) set_bit(mrow + (v.eos_id >> 5), 1u << (v.eos_id & 31));
+            if (nrow) nrow[v.eos_id] = (int32_t)rc.x;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// tree_tile_kernel
+// ---------------------------------------------------------------------------
+// per-lane configuration packed for shared memory: state | depth << 16 (the
+// stack bits apart)
+__device__ __forceinline__ uint32_t pack_sd(uint32_t s, uint32_t depth) { return s | (depth << 16); }
+
+template <bool STACK, int MODE, bool NEXT>
+struct TileCtx {
+    using E = typename std::conditional<STACK, uint32_t, uint16_t>::type;
+    const StepView& v;
+    const TreeArgs& a;
+    const Tab<E, MODE>& tab;
+    const uint16_t* ret;
+    uint32_t maxd;
+    const unsigned long long* s_self;   // nullptr: no self-loop skip
+    const uint2* snode;                 // {skip - nb | cls << 16, tok - tb | n_end << 16}
+    const unsigned long long* ssub;
+    const int32_t* stok;
+    int nn, nt;                         // staged nodes and tokens
+
+    __device__ __forceinline__ void fail() const { atomicOr(v.err, DOMINO_DEVERR_INTERNAL); }
+
+    __device__ __forceinline__ void emit_one(int row, int t, uint32_t s) const {
+        if ((uint32_t)t >= (uint32_t)v.V) {   // the tree holds token ids only
+            fail();
+            return;
+        }
+        if (a.mask) set_bit(a.mask + (size_t)row * v.W + (t >> 5), 1u << (t & 31));
+        if constexpr (NEXT) {
+            if (a.next) a.next[(size_t)row * v.V + t] = (int32_t)s;
+        }
+    }
+    // Staged tokens [lo, hi) (the same for all lanes) allowed with state s in
+    // the lanes where `on`, each in its lane's row.  Few tokens: a loop over
+    // them, every lane setting its own row's bit.  Many: for each lane that is
+    // on, the warp's lanes split the range.  Warp-uniform control flow.
+    __device__ __forceinline__ void emit(int lane, bool on, int row, int lo, int hi, uint32_t s) const {
+        if (hi - lo <= kTrieEmitWarp) {
+            for (int j = lo; j < hi; ++j) {
+                const int t = stok[j];
+                if (on) emit_one(row, t, s);
+            }
+            return;
+        }
+        for (unsigned m = __ballot_sync(0xffffffffu, on); m; m &= m - 1) {
+            const int src = __ffs(m) - 1;
+            const int r = __shfl_sync(0xffffffffu, row, src);
+            const uint32_t ss = __shfl_sync(0xffffffffu, s, src);
+            for (int j = lo + lane; j < hi; j += 32) emit_one(r, stok[j], ss);
+        }
+    }
+
+    // One warp walks unit root x0 (staged index) for its lanes' rows, in
+    // lockstep: (s, bits, depth) is the lane's configuration at the unit's
+    // parent (s = 0: no row).  stk / ustk: the warp's stack.
+    __device__ __forceinline__ void walk(int lane, int row, int x0, uint32_t s, uint32_t bits, uint32_t depth,
+                                         uint32_t* stk, uint32_t* stkb, uint2* ustk) const {
+        int x = x0, end = x0 + 1, sp = 0;
+        for (;;) {
+            while (x < end) {
+                const uint2 rec = snode[x];   // checked when staged
+                const int xs = (int)(rec.x & 0xFFFFu);
+                uint32_t b2 = bits, d2 = depth;
+                const uint32_t s2 = step_once<STACK>(tab, ret, maxd, s, (rec.x >> 16) & 0xFFu, b2, d2);
+                const bool on = s2 != 0;
+                if (__ballot_sync(0xffffffffu, on)) {
+                    const int tl = (int)(rec.y & 0xFFFFu), ne = (int)(rec.y >> 16);
+                    if (ne) emit(lane, on, row, tl, tl + ne, s2);
+                    if (xs > x + 1) {   // x has children
+                        bool desc = on;
+                        if (s_self) {
+                            // every class below keeps the state: the whole
+                            // subtree is allowed with it
+                            const bool keep = on && (ssub[x] & ~s_self[s2]) == 0ull;
+                            if (__ballot_sync(0xffffffffu, keep)) {
+                                const int th = xs < nn ? (int)(snode[xs].y & 0xFFFFu) : nt;
+                                emit(lane, keep, row, tl + ne, th, s2);
+                            }
+                            desc = desc && !keep;
+                        }
+                        if (__ballot_sync(0xffffffffu, desc)) {
+                            if (xs < end) {
+                                if (sp == kTrieBranch) {   // the tree bounds the stack by kTrieBranch
+                                    if (lane == 0) fail();
+                                    return;
+                                }
+                                stk[sp * 32 + lane] = pack_sd(s, depth);
+                                if constexpr (STACK) stkb[sp * 32 + lane] = bits;
+                                if (lane == 0) ustk[sp] = make_uint2((uint32_t)xs, (uint32_t)end);
+                                ++sp;
+                            }
+                            end = xs;
+                            s = desc ? s2 : 0u;
+                            bits = b2;
+                            depth = d2;
+                            x = x + 1;
+                            continue;
+                        }
+                    }
+                }
+                x = xs;
+            }
+            if (sp == 0) return;
+            --sp;
+            __syncwarp();
+            const uint2 u = ustk[sp];
+            x = (int)u.x;
+            end = (int)u.y;
+            const uint32_t sd = stk[sp * 32 + lane];
+            s = sd & 0xFFFFu;
+            depth = sd >> 16;
+            if constexpr (STACK) bits = stkb[sp * 32 + lane];
+        }
+    }
+};
+
+template <bool STACK, int MODE, bool NEXT>
+__global__ void __launch_bounds__(kTileThreads, 1)
+    tree_tile_kernel(const __grid_constant__ StepView v, const __grid_constant__ TrieView tv,
+                     const uint4* __restrict__ img, const __grid_constant__ TreeArgs a, const RowList list) {
+    using E = typename std::conditional<STACK, uint32_t, uint16_t>::type;
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const bool use_self = v.self_mask != nullptr;
+    const TileLayout L = tile_layout(v.Q, use_self, STACK, MODE == kDenseGlobal ? 0 : a.img_bytes, tv);
+    uint32_t* s_accept = reinterpret_cast<uint32_t*>(smem + L.accept);
+    unsigned long long* s_self = reinterpret_cast<unsigned long long*>(smem + L.self);
+    uint2* snode = reinterpret_cast<uint2*>(smem + L.nodes);
+    unsigned long long* ssub = reinterpret_cast<unsigned long long*>(smem + L.sub);
+    int32_t* stok = reinterpret_cast<int32_t*>(smem + L.toks);
+    uint32_t* sunit = reinterpret_cast<uint32_t*>(smem + L.units);   // root - nb | slot << 16
+    uint4* sslot = reinterpret_cast<uint4*>(smem + L.slots);         // {path length, 0, first token, tokens set}
+    uint8_t* spath = reinterpret_cast<uint8_t*>(smem + L.paths);
+    uint4* rowcfg = reinterpret_cast<uint4*>(smem + L.rowcfg);
+    uint32_t* cfg = reinterpret_cast<uint32_t*>(smem + L.cfg);       // [slot][row] state | depth << 16 (+ bits)
+    uint16_t* lrows = reinterpret_cast<uint16_t*>(smem + L.lrows);   // [slot][k] live rows of the block
+    int* lcount = reinterpret_cast<int*>(smem + L.lcount);
+    uint32_t* stk = reinterpret_cast<uint32_t*>(smem + L.stk);
+    uint2* ustk = reinterpret_cast<uint2*>(smem + L.ustk);
+    int* ctl = reinterpret_cast<int*>(smem + L.ctl);
+    const int b0 = __ldg(tv.cta_batch + blockIdx.x), b1 = __ldg(tv.cta_batch + blockIdx.x + 1);
+    if (b0 >= b1) {   // no units for this CTA
+        pdl_wait();
+        pdl_trigger();
+        return;
+    }
+    for (int i = tid; i < (v.Q + 31) / 32; i += kTileThreads) s_accept[i] = __ldg(v.accept_bits + i);
+    if (use_self)
+        for (int i = tid; i < v.Q; i += kTileThreads) s_self[i] = __ldg(v.self_mask + i);
+    Tab<E, MODE> tab;
+    tab.K = (uint32_t)v.K;
+    const uint16_t* ret;
+    if constexpr (MODE == kDenseGlobal) {
+        tab.dense = reinterpret_cast<const E*>(STACK ? (const void*)v.t32 : (const void*)v.t16);
+        ret = v.ret;
+    } else {
+        uint4* dst = reinterpret_cast<uint4*>(smem + L.table);
+        for (int i = tid; i < a.img_bytes / 16; i += kTileThreads) dst[i] = __ldg(img + i);
+        const unsigned char* t = smem + L.table;
+        tab.dense = reinterpret_cast<const E*>(t);
+        tab.sp = reinterpret_cast<const uint32_t*>(t);
+        tab.tgt = reinterpret_cast<const E*>(t + a.img_tgt_off);
+        ret = reinterpret_cast<const uint16_t*>(t + a.img_ret_off);
+    }
+    const uint32_t maxd = (uint32_t)v.max_depth;
+    uint32_t* wstk = stk + warp * kTrieBranch * 32 * (STACK ? 2 : 1);
+    uint32_t* wstkb = wstk + kTrieBranch * 32;
+    uint2* wustk = ustk + warp * kTrieBranch;
+    bool waited = false;
+    for (int bj = b0; bj < b1; ++bj) {
+        const uint4 bA = __ldg(tv.batch + 2 * bj);       // units [x, y), nodes [z, w)
+        const uint4 bB = __ldg(tv.batch + 2 * bj + 1);   // tokens [x, y), slots [z, w)
+        const int nk = (int)(bA.y - bA.x), nn = (int)(bA.w - bA.z), nt = (int)(bB.y - bB.x);
+        const int ns = (int)(bB.w - bB.z);
+        __syncthreads();   // the previous batch is done with shared memory
+        if (tid == 0) ctl[kCtlBad] = 0;
+        __syncthreads();
+        for (int n = tid; n < nn; n += kTileThreads) {
+            const uint4 r0 = __ldg(tv.node + 2 * ((size_t)bA.z + n));
+            // preorder (a subtree ends after its root) and the node's tokens
+            // inside the batch's: the walk relies on both.  The upper nodes
+            // between a batch's units are staged too (never walked); their
+            // subtrees end past the batch, so skips are clamped to its end.
+            const uint32_t xs = min((r0.x & 0xFFFFFFu) - bA.z, (uint32_t)nn), tl = r0.y - bB.x;
+            if (xs <= (uint32_t)n || tl > (uint32_t)nt || r0.z > (uint32_t)nt - tl) ctl[kCtlBad] = 1;
+            snode[n] = make_uint2(xs | ((r0.x >> 24) << 16), tl | (r0.z << 16));
+            if (use_self) {
+                const uint4 r1 = __ldg(tv.node + 2 * ((size_t)bA.z + n) + 1);
+                ssub[n] = ((unsigned long long)r1.y << 32) | r1.x;
+            }
+        }
+        for (int j = tid; j < nt; j += kTileThreads) stok[j] = __ldg(tv.dtok + bB.x + j);
+        for (int k = tid; k < nk; k += kTileThreads) {
+            const uint2 un = __ldg(tv.unit + bA.x + k);
+            if (un.x < bA.z || un.x >= bA.w || un.y >= (uint32_t)ns) ctl[kCtlBad] = 1;
+            sunit[k] = (un.x - bA.z) | (un.y << 16);
+        }
+        for (int k = tid; k < ns; k += kTileThreads) {
+            const uint4 sl = __ldg(tv.slot + bB.z + k);   // {upper index, first token, tokens set, 0}
+            const uint4 up = __ldg(tv.upper + sl.x);      // {node, path offset, path length, 0}
+            if (up.z > (uint32_t)tv.max_path) ctl[kCtlBad] = 1;
+            sslot[k] = make_uint4(min(up.z, (uint32_t)tv.max_path), 0u, sl.y, sl.z);
+            for (uint32_t d = 0; d < up.z && d < (uint32_t)tv.max_path; ++d)
+                spath[k * tv.max_path + d] = __ldg(tv.upath + up.y + d);
+        }
+        if (!waited) {   // everything above is the static tree; the masks come from tree_clear_kernel
+            pdl_wait();
+            pdl_trigger();
+            waited = true;
+        }
+        __syncthreads();
+        if (ctl[kCtlBad]) {   // a record the walk cannot trust: report and skip the batch
+            if (tid == 0) atomicOr(v.err, DOMINO_DEVERR_INTERNAL);
+            continue;
+        }
+        const TileCtx<STACK, MODE, NEXT> cx{v, a, tab, ret, maxd, use_self ? s_self : nullptr, snode, ssub, stok, nn, nt};
+        const int nrows = list.rows(a.batch);
+        const int rb = max(1, min(kTrieRowBlock, kTrieCfg / max(ns, 1)));
+        for (int r0 = 0; r0 < nrows; r0 += rb) {
+            const int nr = min(rb, nrows - r0);
+            if (tid < ns) lcount[tid] = 0;
+            if (tid == 0) ctl[kCtlUnit] = 0;
+            // 1. the rows' configurations
+            for (int r = tid; r < nr; r += kTileThreads) {
+                const int b = list.row(r0 + r);
+                if (a.row_is_state) {
+                    rowcfg[r] = make_uint4((uint32_t)b, 0u, 0u, 1u);
+                } else {
+                    const int32_t sv = __ldg(a.states + b);
+                    const unsigned long long w =
+                        a.stacks ? __ldg(reinterpret_cast<const unsigned long long*>(a.stacks) + b) : 0ull;
+                    rowcfg[r] = decode_row(v, sv, w, a.stacks != nullptr, s_accept, false);
+                }
+            }
+            __syncthreads();
+            // ... at every slot: the slot's path from the row's configuration
+            for (int f = tid; f < ns * nr; f += kTileThreads) {
+                const int k = f / nr, r = f - k * nr;
+                const uint4 rc = rowcfg[r];
+                uint32_t s = (rc.w & 1u) ? rc.x : 0u, bits = rc.y, depth = rc.z;
+                const int plen = (int)sslot[k].x;
+                for (int d = 0; d < plen && s != 0; ++d)
+                    s = step_once<STACK>(tab, ret, maxd, s, spath[k * tv.max_path + d], bits, depth);
+                cfg[f] = pack_sd(s, depth);
+                if constexpr (STACK) cfg[kTrieCfg + f] = bits;
+            }
+            __syncthreads();
+            // 2. per slot, the rows live there (a warp's lanes take consecutive
+            // rows of one slot: one counter update per warp and slot)
+            for (int f0 = warp * 32; f0 < ns * nr; f0 += kTileThreads) {
+                const int f = f0 + lane;
+                const bool in = f < ns * nr;
+                const int k = in ? f / nr : 0, r = in ? f - k * nr : 0;
+                const uint32_t sd = in ? cfg[f] : 0u;
+                const bool live = in && (sd & 0xFFFFu) != 0u;
+                // lanes of the same slot form runs: one atomic per run
+                const int k0 = __shfl_sync(0xffffffffu, k, 0);
+                const unsigned same = __ballot_sync(0xffffffffu, in && k == k0);
+                const unsigned lv = __ballot_sync(0xffffffffu, live);
+                int base = 0;
+                if (lane == 0 && (lv & same)) base = atomicAdd(&lcount[k0], __popc(lv & same));
+                base = __shfl_sync(0xffffffffu, base, 0);
+                if (live) {
+                    if ((same >> lane) & 1u) {
+                        lrows[k0 * rb + base + __popc(lv & same & ((1u << lane) - 1u))] = (uint16_t)r;
+                    } else {
+                        lrows[k * rb + atomicAdd(&lcount[k], 1)] = (uint16_t)r;
+                    }
+                }
+            }
+            __syncthreads();
+            // emitting slots: the tokens that end at their nodes, for every row
+            // live there, spread over the CTA (read from the preorder list)
+            for (int k = 0; k < ns; ++k) {
+                const uint4 sl = sslot[k];
+                const int nl = lcount[k], nt_k = (int)sl.w;
+                for (int f = tid; f < nl * nt_k; f += kTileThreads) {
+                    const int li = f / nt_k, j = f - li * nt_k;
+                    const int r = lrows[k * rb + li];
+                    cx.emit_one(r0 + r, __ldg(tv.dtok + sl.z + j), cfg[k * nr + r] & 0xFFFFu);
+                }
+            }
+            // 3. warps claim units; a unit is walked for its slot's live rows,
+            // 32 at a time
+            for (;;) {
+                int k = 0;
+                if (lane == 0) k = atomicAdd(&ctl[kCtlUnit], 1);
+                k = __shfl_sync(0xffffffffu, k, 0);
+                if (k >= nk) break;
+                const uint32_t un = sunit[k];
+                const int x0 = (int)(un & 0xFFFFu), sl = (int)(un >> 16);
+                const int n = lcount[sl];
+                for (int c = 0; c < n; c += 32) {
+                    const bool on = c + lane < n;
+                    const int r = on ? lrows[sl * rb + c + lane] : 0;
+                    const uint32_t sd = on ? cfg[sl * nr + r] : 0u;
+                    const uint32_t bits = STACK && on ? cfg[kTrieCfg + sl * nr + r] : 0u;
+                    cx.walk(lane, r0 + r, x0, sd & 0xFFFFu, bits, sd >> 16, wstk, wstkb, wustk);
+                }
+            }
+            __syncthreads();
+        }
+    }
+}
+
+template <bool STACK, int MODE, bool NEXT>
+cudaError_t launch_tree_t(const StepView& v, const TrieView& tv, const LaunchEnv& env, TreeArgs a,
+                          const RowList& list, cudaStream_t st) {
+    const int img_bytes = MODE == kDenseGlobal ? 0 : (int)table_smem_bytes(v, STACK, MODE);
+    a.img_bytes = img_bytes;
+    const uint4* img = nullptr;
+    a.img_tgt_off = a.img_ret_off = 0;
+    if constexpr (MODE != kDenseGlobal) {
+        const size_t esz = STACK ? 4 : 2;
+        if (MODE == kDenseSmem) {
+            img = reinterpret_cast<const uint4*>(STACK ? (const void*)v.t32 : (const void*)v.t16);
+            a.img_ret_off = align16((int)((size_t)v.Q * v.K * esz));
+        } else {
+            img = reinterpret_cast<const uint4*>(v.sp_info);
+            a.img_tgt_off = align16(v.Q * (MODE == kSparse32Smem ? 8 : 16));
+            a.img_ret_off = a.img_tgt_off + align16((int)((size_t)v.sp_nnz * esz));
+        }
+    }
+    const TileLayout L = tile_layout(v.Q, v.self_mask != nullptr, STACK, img_bytes, tv);
+    if (L.total > env.max_smem_optin || tv.max_slots > kTrieMaxSlots || tv.grid > env.num_sms)
+        return cudaErrorInvalidConfiguration;
+    auto tile = tree_tile_kernel<STACK, MODE, NEXT>;
+    static int configured[kTrieMaxDevices] = {0};
+    static std::mutex mu;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (L.total > 48 * 1024 && dev < kTrieMaxDevices) {
+        std::lock_guard<std::mutex> lk(mu);
+        if (configured[dev] < L.total) {
+            cudaError_t e = cudaFuncSetAttribute(tile, cudaFuncAttributeMaxDynamicSharedMemorySize, L.total);
+            if (e != cudaSuccess) return e;
+            configured[dev] = L.total;
+        }
+    }
+    const int clear_grid = (a.batch + kClearThreads / 32 - 1) / (kClearThreads / 32);
+    cudaError_t e = launch_pdl(tree_clear_kernel<NEXT>, dim3(clear_grid), dim3(kClearThreads), 0, st, v, a, list);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(tile, dim3(tv.grid), dim3(kTileThreads), (size_t)L.total, st, v, tv, img, a, list);
+}
+
+template <bool STACK, bool NEXT>
+cudaError_t launch_tree_m(const StepView& v, const TrieView& tv, const LaunchEnv& env, int mode, const TreeArgs& a,
+                          const RowList& list, cudaStream_t st) {
+    switch (mode) {
+        case kDenseSmem: return launch_tree_t<STACK, kDenseSmem, NEXT>(v, tv, env, a, list, st);
+        case kSparse32Smem: return launch_tree_t<STACK, kSparse32Smem, NEXT>(v, tv, env, a, list, st);
+        case kSparse64Smem: return launch_tree_t<STACK, kSparse64Smem, NEXT>(v, tv, env, a, list, st);
+        default: return launch_tree_t<STACK, kDenseGlobal, NEXT>(v, tv, env, a, list, st);
+    }
+}
+
+}  // namespace
+
+int trie_tile_smem_bytes(const StepView& v, const TrieView& tv, bool stack, int table_bytes) {
+    return tile_layout(v.Q, v.self_mask != nullptr, stack, table_bytes, tv).total;
+}
+
+cudaError_t launch_trie_step(const StepView& v, const TrieView& tv, const LaunchEnv& env, bool stack, int mode,
+                             const int32_t* states, const uint64_t* stacks, int32_t batch, bool row_is_state,
+                             uint32_t* mask, int32_t* next, cudaStream_t st, const int32_t* row_ids,
+                             const int32_t* row_count) {
+    if (batch <= 0) return cudaSuccess;
+    TreeArgs a{};
+    a.states = states;
+    a.stacks = stacks;
+    a.batch = batch;
+    a.row_is_state = row_is_state ? 1 : 0;
+    a.mask = mask;
+    a.next = next;
+    const RowList list{row_ids, row_count, 0};
+    if (stack) {
+        return next ? launch_tree_m<true, true>(v, tv, env, mode, a, list, st)
+                    : launch_tree_m<true, false>(v, tv, env, mode, a, list, st);
+    }
+    return next ? launch_tree_m<false, true>(v, tv, env, mode, a, list, st)
+                : launch_tree_m<false, false>(v, tv, env, mode, a, list, st);
+}
+
+}  // namespace domino

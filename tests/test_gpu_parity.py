@@ -96,6 +96,11 @@ def test_step_mask_parity(config):
     w = workload(config)
     states, stacks = configs(config)
     d = handle(config)
+    # the walk chosen from the automaton: the prefix tree unless states loop
+    # on many classes (configs 2 and 5: strings); tests/test_gpu_tree_walk.py
+    # and tests/test_gpu_token_walk.py force each walk
+    if config in (3, 5):
+        assert d.info()["walk_tree"] == (1 if config == 3 else 0)
     st = dev(states)
     sk = dev(stacks.view(np.int64)) if w.automaton.rules is not None else None
     mask, nxt = d.step_mask(st, sk, want_next=True)
@@ -480,6 +485,7 @@ def test_precompute_table_config4_full():
     on the device; table row q == step_mask from q on sampled rows."""
     w = workload(4)
     d = Domino.from_parts(w.automaton, w.vocab, device=0)
+    assert d.info()["walk_tree"] == 1
     nxt, mask = d.precompute_table()
     torch.cuda.synchronize()
     Q, V = w.automaton.n_states, w.vocab.n_tokens
