@@ -271,8 +271,11 @@ struct TileCtx {
     }
 };
 
+// At most 56 registers: a 1024-thread CTA then leaves room on its SM for the
+// next step's tree_clear_kernel CTAs, which start (and wait on this kernel)
+// while it drains instead of after it.
 template <bool STACK, int MODE, bool NEXT>
-__global__ void __launch_bounds__(kTileThreads, 1)
+__global__ void __maxnreg__(56)
     tree_tile_kernel(const __grid_constant__ StepView v, const __grid_constant__ TrieView tv,
                      const uint4* __restrict__ img, const __grid_constant__ TreeArgs a, const RowList list) {
     using E = typename std::conditional<STACK, uint32_t, uint16_t>::type;
