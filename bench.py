@@ -100,7 +100,7 @@ REASONS = {0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_c
 
 
 class ClockSampler:
-    def __init__(self, torch_dev: int, period_s: float = 0.002):
+    def __init__(self, torch_dev: int, period_s: float = 0.001):
         self.period = period_s
         self.samples = []
         self.reasons = 0
@@ -145,7 +145,9 @@ class ClockSampler:
             time.sleep(self.period)
 
     def start(self):
+        """Samples until stop(); may be started again (the samples accumulate)."""
         if self.ok:
+            self._stop = threading.Event()
             self._t = threading.Thread(target=self._run, daemon=True)
             self._t.start()
 
@@ -154,12 +156,19 @@ class ClockSampler:
             self._stop.set()
             self._t.join()
 
-    def summary(self):
+    def summary(self, first: int = 0):
+        """Median SM clock and the throttle reasons seen; `first`: the samples
+        of the headline timed region (the region sampled first)."""
         if not self.ok or not self.samples:
             return {"sm_mhz": None, "sm_max_mhz": self.max_mhz, "reasons": ["unavailable"]}
         names = [n for bit, n in REASONS.items() if self.reasons & bit]
-        return {"sm_mhz": statistics.median(self.samples), "sm_max_mhz": self.max_mhz, "reasons": names,
-                "samples": len(self.samples)}
+        out = {"sm_mhz": statistics.median(self.samples), "sm_max_mhz": self.max_mhz, "reasons": names,
+               "samples": len(self.samples)}
+        if first:
+            out["timed_region_samples"] = first
+            out["note"] = ("sampled every 1 ms during the timed steps and during every per-kernel timing "
+                           "graph of this run")
+        return out
 
 
 def measured_peaks():
@@ -184,22 +193,32 @@ def walk_stats(name: str):
         return None
 
 
+def csrc_digest() -> str:
+    """sha256 (first 16 hex digits) over the device sources, in name order."""
+    import hashlib
+    d = os.path.join(ROOT, "paper_2403_06988_gb300", "csrc")
+    hs = hashlib.sha256()
+    for fn in sorted(os.listdir(d)):
+        if fn.endswith((".cu", ".cuh", ".h")):
+            hs.update(fn.encode())
+            with open(os.path.join(d, fn), "rb") as f:
+                hs.update(f.read())
+    return hs.hexdigest()[:16]
+
+
 def ncu_traffic(name: str) -> dict:
     """DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from
     the committed ncu summary, per kernel; a kernel whose source changed since
     the capture maps to None."""
-    import hashlib
     p = os.path.join(ROOT, "profiles", "traffic.json")
-    src = os.path.join(ROOT, "paper_2403_06988_gb300", "csrc", "kernels.cu")
     try:
         with open(p) as f:
             rec = json.load(f)
-        with open(src, "rb") as f:
-            digest = hashlib.sha256(f.read()).hexdigest()[:16]
+        digest = csrc_digest()
     except (OSError, ValueError):
         return {}
     ent = rec.get("per_workload", {}).get(name, {})
-    if ent.get("kernels_cu_sha256_16") != digest:
+    if ent.get("csrc_sha256_16") != digest:
         return {}
     return dict(ent.get("per_launch_bytes", {}))
 
@@ -244,10 +263,24 @@ def cpu_baseline(w, target_s: float):
         arg, _, _ = oracle.mask_logits(lg, m, want_logprobs=w.want_logprobs, n_threads=cores)
         P.advance(st, sk, arg, w.automaton.start)
     dt = time.perf_counter() - t0
+    # the same step on one core: a quarter of the time budget
+    lg1 = w.logits(0, batch=1)
+    sk1 = stacks[:1] if w.automaton.rules is not None else None
+    reps1, t0 = 0, time.perf_counter()
+    while True:
+        m, _, _ = P.step_mask(states[:1], sk1, n_threads=1)
+        arg, _, _ = oracle.mask_logits(lg1, m, want_logprobs=w.want_logprobs, n_threads=1)
+        P.advance(states[:1], sk1, arg, w.automaton.start)
+        reps1 += 1
+        dt1 = time.perf_counter() - t0
+        if dt1 > target_s / 4:
+            break
     return {"value": rows * V * reps / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
             "sample": f"{reps} decode steps of {rows} of the {w.batch} rows (full vocabulary V={V}); "
                       f"step_mask + mask_logits + advance, OpenMP over rows",
-            "steps_per_s_equiv": reps * rows / w.batch / dt}
+            "steps_per_s_equiv": reps * rows / w.batch / dt,
+            "single_thread": {"value": V * reps1 / dt1, "unit": UNIT, "cores": 1,
+                              "sample": f"{reps1} decode steps of one row"}}
 
 
 # ----------------------------------------------------------------------------
@@ -474,16 +507,19 @@ def run_domino(args, dist: Dist):
     dtype_code = B.DTYPE_BF16 if w.logits_dtype == "bf16" else B.DTYPE_F32
     L = B.lib()
     h = d.h
-    # raw pointers once: per-step host work is three C calls
+    # raw pointers once
     p_states, p_stacks = states.data_ptr(), (stacks.data_ptr() if stack else None)
     p_mask, p_arg, p_lse = mask.data_ptr(), argmax.data_ptr(), lse.data_ptr()
     p_lp = logprobs.data_ptr() if logprobs is not None else None
     p_logits = [t.data_ptr() for t in logits]
-    # one step = one call: the mask step with the greedy decode folded in, the
-    # per-row merge that also advances each row (plus the log-probs pass where
-    # the workload asks for them); fp32 logits run the separate kernels
-    fused = w.logits_dtype == "bf16"
-    launches_per_step = (2 if fused else 3) + (1 if w.want_logprobs else 0)
+    # one step = one call. With the per-token walk and bf16 logits: the mask
+    # step with the greedy decode folded in, then the per-row merge that also
+    # advances each row. With the prefix-tree walk (two launches: clear, tree
+    # tiles) or fp32 logits: mask step, logits pass, update. Plus the
+    # log-probs pass where the workload asks for them.
+    walk_launches = 2 if info.get("walk_tree") else 1
+    fused = w.logits_dtype == "bf16" and not info.get("walk_tree")
+    launches_per_step = (2 if fused else walk_launches + 2) + (1 if w.want_logprobs else 0)
 
     def step(i, stream_ptr):
         rc = L.domino_step_decode(h, p_states, p_stacks, Bsz, p_logits[i % nbuf], dtype_code, V, p_mask, p_arg, p_lse,
@@ -513,8 +549,9 @@ def run_domino(args, dist: Dist):
         torch.cuda.synchronize()
         return g
 
-    def timed(n, body, g, sampler=None):
-        """Device time (ms) of n calls, events on the launching stream, synchronized on both sides."""
+    def timed(n, body, g, sampler=None, reps=1):
+        """Device time (ms) of n calls (`reps` passes of them, averaged), events
+        on the launching stream, synchronized on both sides."""
         t0 = torch.cuda.Event(enable_timing=True)
         t1 = torch.cuda.Event(enable_timing=True)
         dist.barrier()
@@ -523,23 +560,32 @@ def run_domino(args, dist: Dist):
             sampler.start()
         with torch.cuda.stream(s):
             t0.record()
-            if g is not None:
-                g.replay()
-            else:
-                for i in range(n):
-                    body(i, s.cuda_stream)
+            for _ in range(reps):
+                if g is not None:
+                    g.replay()
+                else:
+                    for i in range(n):
+                        body(i, s.cuda_stream)
             t1.record()
         torch.cuda.synchronize()
         if sampler is not None:
             sampler.stop()
         dist.barrier()
-        return t0.elapsed_time(t1)
+        return t0.elapsed_time(t1) / reps
+
+    def timed_long(n, body, g, sampler, min_ms=4.0):
+        """timed() over enough passes of the graph to fill about min_ms of
+        device time: steadier per-launch figures, and clock samples under load
+        even when n is small."""
+        est = timed(n, body, g)
+        return timed(n, body, g, sampler, reps=max(1, min(200, math.ceil(min_ms / max(est, 1e-3)))))
 
     # ---- the timed region: K whole decode steps, nothing else in the graph ----
     graph = capture(K, step)
-    sampler = ClockSampler(dev_id)
+    sampler = ClockSampler(dev_id)   # also runs during the per-kernel graphs below
     ms = timed(K, step, graph, sampler)
     ms_max = dist.max(ms)
+    first_samples = len(sampler.samples)
     err = d.device_error()
     if err:
         raise RuntimeError(f"device error word {err}")
@@ -571,12 +617,27 @@ def run_domino(args, dist: Dist):
         if L.domino_mask_sample(h, p_logits[i % nbuf], dtype_code, Bsz, V, p_mask, ctypes.c_float(1.0),
                                 ctypes.c_uint64(0x5EED), ctypes.c_uint64(i), p_arg, sp):
             raise RuntimeError("mask_sample failed")
+    # the other mask walk, on a second handle: the prefix tree (Alg. 2's
+    # subterminal tree over byte classes) and the per-token walk each timed alone
+    walk_kind = "prefix tree" if info.get("walk_tree") else "per token"
+    os.environ["DOMINO_WALK"] = "token" if info.get("walk_tree") else "tree"
+    d_other = Domino.from_parts(a, v, device=dev_id)
+    del os.environ["DOMINO_WALK"]
+    other_kind = "prefix tree" if d_other.info().get("walk_tree") else "per token"
+    h_other = d_other.h
+
+    def k_step_other(i, sp):
+        if L.domino_step_mask(h_other, p_states, p_stacks, Bsz, p_mask, None, sp):
+            raise RuntimeError("step_mask (other walk) failed")
     per_kernel = {}
-    for name, body in (("step_mask", k_step), ("mask_logits", k_logits), ("step_decode", k_fused),
-                       ("advance", k_adv), ("mask_sample", k_sample)):
+    for name, body in (("step_mask", k_step), ("step_mask_other", k_step_other), ("mask_logits", k_logits),
+                       ("step_decode", k_fused), ("advance", k_adv), ("mask_sample", k_sample)):
         g = capture(Kk, body)
-        per_kernel[name] = dist.max(timed(Kk, body, g)) / Kk      # ms per launch
+        per_kernel[name] = dist.max(timed_long(Kk, body, g, sampler)) / Kk      # ms per launch
         del g
+    if d_other.device_error():
+        raise RuntimeError("device error in the other walk")
+    d_other.close()
     if d.device_error():
         raise RuntimeError("device error after the per-kernel graphs")
 
@@ -607,7 +668,7 @@ def run_domino(args, dist: Dist):
             body(0, s.cuda_stream)
         torch.cuda.synchronize()
         g = capture(Kk, body)
-        ms_o = dist.max(timed(Kk, body, g))
+        ms_o = dist.max(timed_long(Kk, body, g, sampler))
         del g
         opportunistic[name] = {"us": ms_o / Kk * 1e3, "fallback_rows": int(n_fb.item()), "rows": Bsz}
     opportunistic["masked_greedy_us"] = per_kernel["step_decode"] * 1e3
@@ -653,7 +714,7 @@ def run_domino(args, dist: Dist):
             body(0, s.cuda_stream)
         torch.cuda.synchronize()
         g = capture(Kk, body)
-        spec[name + "_us"] = dist.max(timed(Kk, body, g)) / Kk * 1e3
+        spec[name + "_us"] = dist.max(timed_long(Kk, body, g, sampler)) / Kk * 1e3
         del g
     spec["proposals_per_row"] = float(n_prop.float().mean().item())
     spec["count_table_bytes"] = n_keys * V * 4
@@ -693,7 +754,7 @@ def run_domino(args, dist: Dist):
                 t_step(i, s.cuda_stream)
         torch.cuda.synchronize()
         g = capture(K, t_step)
-        ms_t = dist.max(timed(K, t_step, g))
+        ms_t = dist.max(timed_long(K, t_step, g, sampler))
         del g
         if d.device_error():
             raise RuntimeError("device error in the table-driven step")
@@ -735,6 +796,30 @@ def run_domino(args, dist: Dist):
     h2d = logit_bytes + Bsz * 4 + (Bsz * 8 if stack else 0)
     d2h = Bsz * 4 * 3 + (Bsz * 8 if stack else 0)
 
+    # ---- structure of the workload's masks: an untimed decode loop from the
+    # same starting rows, counting allowed tokens and the rows that end (EOS
+    # chosen, or nothing allowed) and so restart from the start state
+    S = 32
+    states.copy_(torch.from_numpy(states0).to(dev))
+    if stack:
+        stacks.copy_(torch.from_numpy(stacks0.view(np.int64)).to(dev))
+    allowed = ends_eos = ends_dead = 0
+    with torch.cuda.stream(s):
+        for i in range(S):
+            step(i, s.cuda_stream)
+            s.synchronize()
+            allowed += int(np.unpackbits(mask.cpu().numpy().view(np.uint8)).sum())
+            am = argmax.cpu().numpy()
+            ends_eos += int((am == v.eos_id).sum()) if v.eos_id >= 0 else 0
+            ends_dead += int((am < 0).sum())
+    torch.cuda.synchronize()
+    structure = {"decode_steps": S, "allowed_fraction": allowed / (S * Bsz * V),
+                 "allowed_per_row": allowed / (S * Bsz),
+                 "resets_per_step": (ends_eos + ends_dead) / S, "eos_per_step": ends_eos / S,
+                 "all_masked_per_step": ends_dead / S, "byte_classes": info["n_classes"],
+                 "walk": walk_kind,
+                 "note": "greedy decode from the bench's starting rows, counted from the mask and argmax outputs"}
+
     # ---- report ---------------------------------------------------------------
     n = dist.world
     value = n * Bsz * V * K / (ms_max / 1e3)
@@ -746,27 +831,38 @@ def run_domino(args, dist: Dist):
     t_ml = per_kernel["mask_logits"] * 1e-3
     t_sm = per_kernel["step_mask"] * 1e-3
     gbs = lg_bytes / t_ml / 1e9
+    ml_dram = traffic.get("mask_logits")
     kernels = {
         "mask_logits": {"us": t_ml * 1e6, "algorithmic_bytes": lg_bytes, "gbs": gbs, "frac_hbm": gbs / hbm_peak,
-                        "dram_bytes_ncu": traffic.get("mask_logits")},
+                        "dram_bytes_ncu": ml_dram,
+                        "dram_gbs": ml_dram / t_ml / 1e9 if ml_dram else None,
+                        "frac_hbm_dram": ml_dram / t_ml / 1e9 / hbm_peak if ml_dram else None},
         "step_mask": {"us": t_sm * 1e6, "checks_per_s": Bsz * V / t_sm, "mask_bytes": Bsz * Wd * 4,
                       "dram_bytes_ncu": traffic.get("step_mask")},
         "step_decode": {"us": per_kernel["step_decode"] * 1e3,
                         "separate_us": (per_kernel["step_mask"] + per_kernel["mask_logits"]) * 1e3,
-                        "dram_bytes_ncu": traffic.get("step_decode_fused"),
-                        "note": "the timed step's mask + decode: the mask step folds the allowed logits of each "
-                                "tile (then a per-row merge; log-probs in one more pass where asked for)"},
+                        "dram_bytes_ncu": traffic.get("step_decode_fused") if fused else None,
+                        "note": ("the timed step's mask + decode: the mask step folds the allowed logits of each "
+                                 "tile (then a per-row merge; log-probs in one more pass where asked for)") if fused
+                        else ("the timed step's mask + decode + update: the mask step, the logits pass, "
+                              "then the update, back to back")},
         "advance": {"us": per_kernel["advance"] * 1e3},
         "mask_sample": {"us": per_kernel["mask_sample"] * 1e3,
                         "gbs": (lg_bytes - Bsz * V * 4 * w.want_logprobs - Bsz * 4) / (per_kernel["mask_sample"] * 1e-3)
                         / 1e9, "note": "Gumbel-max draw at T = 1 over the same masks (Philox per 4 allowed tokens)"},
-        "timing": f"each kernel alone, {Kk} launches back to back in one CUDA graph, events on its stream",
+        "timing": f"each kernel alone, {Kk} launches back to back in one CUDA graph replayed over about 4 ms, "
+                  "events on its stream",
     }
     # transition-lookup peak: one conflict-free 32-lane shared-memory gather per
     # SM clock; every byte the definition walks is one table lookup
     sm_clk = float(peaks.get("sm_max_mhz", 2070.0)) * 1e6
     lookup_peak = torch.cuda.get_device_properties(dev_id).multi_processor_count * 32 * sm_clk / 1e9
+    kernels["step_mask"]["walk"] = walk_kind
+    kernels["step_mask_" + ("token" if info.get("walk_tree") else "tree")] = {
+        "us": per_kernel["step_mask_other"] * 1e3, "walk": other_kind,
+        "checks_per_s": Bsz * V / (per_kernel["step_mask_other"] * 1e-3)}
     if walk is not None:
+        structure["walk_steps_per_check"] = walk
         trans = walk * Bsz * V
         kernels["step_mask"].update({"walk_steps_per_check": walk, "gtransitions_per_s": trans / t_sm / 1e9,
                                      "frac_lookup_peak": trans / t_sm / 1e9 / lookup_peak})
@@ -775,8 +871,12 @@ def run_domino(args, dist: Dist):
                     "unit": "Gtransitions/s", "frac": trans / t_sm / 1e9 / lookup_peak,
                     "traffic": traffic.get("step_mask"), "algorithmic_units_per_launch": trans,
                     "peak_source": f"{lookup_peak:.0f} G lookups/s = SMs x 32 lanes x {sm_clk / 1e6:.0f} MHz",
-                    "note": "walk bound by shared-memory gathers and issue, not HBM; the mask step timed alone "
-                            "(in the timed step the same kernel also folds the logits: kernels.step_decode)"}
+                    "note": ("walk bound by shared-memory gathers and issue, not HBM; the mask step timed alone "
+                             "(in the timed step the same kernel also folds the logits: kernels.step_decode)")
+                    if fused else
+                            ("the prefix-tree mask step (clear + tree-tile kernels, one call) timed alone as it runs "
+                             "in the step; units are the lookups the plain per-token definition makes, of which "
+                             "the tree walk makes fewer (shared prefixes walked once)")}
     else:
         roofline = {"kernel": "mask_logits", "bound": "hbm", "achieved": gbs, "peak": hbm_peak, "unit": "GB/s",
                     "frac": gbs / hbm_peak, "traffic": traffic.get("mask_logits"),
@@ -791,7 +891,7 @@ def run_domino(args, dist: Dist):
                    "l2": f"logits rotate over {nbuf} buffers ({nbuf * logit_bytes / 2**20:.0f} MiB > 2x L2)",
                    "parallelism": f"replicas x{n}", "graph": graph is not None},
         "masked_decode_steps_per_s": n * K / (ms_max / 1e3),
-        "kernels": kernels, "roofline": roofline, "table_driven_step": table_step,
+        "structure": structure, "kernels": kernels, "roofline": roofline, "table_driven_step": table_step,
         "opportunistic": opportunistic, "speculation": spec,
         "e2e": {"value": n * Bsz * V * Ke / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "steps": Ke, "api": "domino_decode_step_host with pinned host buffers",
@@ -799,7 +899,7 @@ def run_domino(args, dist: Dist):
                             "allowed logits cross the link (the handle times both paths and uses the faster)"},
         "gpu_launches": K * launches_per_step,
         "gpu_launches_note": "timed region only; per-kernel graphs and e2e are timed separately",
-        "clocks": sampler.summary(),
+        "clocks": sampler.summary(first_samples),
     }
     if dist.rank == 0 and n == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds)

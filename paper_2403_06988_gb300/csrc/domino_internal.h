@@ -169,6 +169,9 @@ struct SampleArgs {
 // token allowed.  row_ids / row_count (device): only rows row_ids[i] for
 // i < *row_count are processed, their masks being the compact rows i of
 // `mask`; argmax and lse are indexed by batch row; no logprobs.
+// raises the logits kernels' shared-memory limit on the current device; called
+// once per handle and device, outside any stream capture
+cudaError_t prepare_logits_kernels();
 cudaError_t launch_mask_logits(const LaunchEnv& env, const void* logits, int dtype, int32_t batch,
                                int64_t row_stride, int32_t V, const uint32_t* mask, int32_t* argmax, float* lse,
                                float* logprobs, float4* partials, uint32_t* counters, float* lse_tmp,

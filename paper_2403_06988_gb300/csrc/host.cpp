@@ -687,7 +687,8 @@ int domino_create(domino_t* out, int32_t cuda_device) {
         }
         cudaDeviceGetAttribute(&h->env.num_sms, cudaDevAttrMultiProcessorCount, h->device);
         cudaDeviceGetAttribute(&h->env.max_smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device);
-        int rc = dev_reserve(h->d_err, 16);
+        int rc = prepare_logits_kernels() == cudaSuccess ? DOMINO_OK : DOMINO_E_CUDA;
+        if (!rc) rc = dev_reserve(h->d_err, 16);
         if (!rc) rc = dev_reserve(h->d_partials, sizeof(float4) * (size_t)kMaxLogitRows * kMaxSegments);
         if (!rc) rc = dev_reserve(h->d_counters, sizeof(uint32_t) * (size_t)kMaxLogitRows);
         if (!rc) rc = dev_reserve(h->d_lse_tmp, sizeof(float) * (size_t)kMaxLogitRows);
@@ -1125,9 +1126,18 @@ int domino_step_decode(domino_t h, const int32_t* states_dev, const uint64_t* st
         return DOMINO_E_INVALID_ARG;
     DeviceGuard g(h->device);
     cudaStream_t st = (cudaStream_t)stream;
+    // logits in device memory are pulled into L2 a tile ahead of their fold;
+    // host-resident logits are read only where the mask allows a token
+    cudaPointerAttributes pa{};
+    const bool on_device = cudaPointerGetAttributes(&pa, logits_dev) == cudaSuccess && pa.type == cudaMemoryTypeDevice;
+    if (!on_device) cudaGetLastError();
+    // the fold rides on the per-token walk; where the prefix-tree walk is the
+    // faster mask step and the logits sit in device memory, the tree walk, the
+    // logits pass and the update run one after the other instead
     const bool fusable = dtype == DOMINO_DTYPE_BF16 && reinterpret_cast<uintptr_t>(logits_dev) % 16 == 0 &&
                          ((size_t)row_stride_elems * 2) % 16 == 0 &&
-                         (int64_t)batch * h->n_windows < (int64_t)INT32_MAX;   // partial slots are int
+                         (int64_t)batch * h->n_windows < (int64_t)INT32_MAX &&   // partial slots are int
+                         !(on_device && use_tree(h));
     if (!fusable) {   // the kernels one after the other
         if ((rc = domino_step_mask(h, states_dev, stacks_dev, batch, mask_dev, nullptr, stream))) return rc;
         if ((rc = domino_mask_logits(h, logits_dev, dtype, batch, row_stride_elems, mask_dev, argmax_dev, lse_dev,
@@ -1150,11 +1160,6 @@ int domino_step_decode(domino_t h, const int32_t* states_dev, const uint64_t* st
         clear_host_graphs(h);   // recorded host-buffer steps name this buffer
         if ((rc = dev_reserve(h->d_fpart, part_bytes))) return rc;
     }
-    // logits in device memory are pulled into L2 a tile ahead of their fold;
-    // host-resident logits are read only where the mask allows a token
-    cudaPointerAttributes pa{};
-    const bool on_device = cudaPointerGetAttributes(&pa, logits_dev) == cudaSuccess && pa.type == cudaMemoryTypeDevice;
-    if (!on_device) cudaGetLastError();
     const int mode = choose_mode(h, v, false);
     cudaError_t e = launch_step_mask(v, h->env, h->stack, mode, states_dev, stacks_dev, batch, false, mask_dev, nullptr,
                                      st, nullptr, nullptr, logits_dev, row_stride_elems, (float4*)h->d_fpart.p,

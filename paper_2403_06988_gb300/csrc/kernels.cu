@@ -923,6 +923,244 @@ __global__ void __launch_bounds__(kReduceThreads)
     }
 }
 
+// ---- the greedy / log-sum-exp pass over bf16 rows: a compacted gather -----
+// One CTA per row, its warps (up to 16) on consecutive segments of the row's
+// mask words, each segment cut into spans of 32 x kGatherSpan words (lane l
+// holds words l*kGatherSpan ... +kGatherSpan-1 of the span).  Each lane finds
+// its words' 16-byte logit vectors that hold an allowed token (a 32-bit map,
+// one bit per vector), a warp scan places the lanes' lists one after the
+// other in token order, and the warp then loads the listed vectors
+// kGatherRound per lane at once (entry k goes to lane k % 32, so each lane
+// still sees its tokens in increasing order) and folds them.  Zero words cost
+// a few instructions, every load of a span is independent, and a span costs
+// one memory latency whatever its density.  The warps' partials are merged in
+// shared memory.  Logit lines are not kept in L1, and in L2 only when a
+// log-prob pass reads them again (evict-last; otherwise evict-first).
+constexpr int kGatherMaxWarps = 16;   // warps per CTA (one row); two CTAs per SM
+constexpr int kGatherSpan = 8;     // mask words per lane per span (8192 tokens)
+constexpr int kGatherWarpSmem = 32 * kGatherSpan * (4 + 4 * 2);   // a span's words and its list
+constexpr int kGatherRound = 4;    // vectors per lane loaded together
+
+__device__ __forceinline__ uint64_t l2_policy(bool keep) {
+    uint64_t p;
+    if (keep)
+        asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;\n" : "=l"(p));
+    else
+        asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;\n" : "=l"(p));
+    return p;
+}
+
+__device__ __forceinline__ uint4 ld_once16(const void* p, uint64_t pol) {
+    uint4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.L2::cache_hint.v4.u32 {%0, %1, %2, %3}, [%4], %5;\n"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p), "l"(pol));
+    return v;
+}
+
+// bit b of the result: byte b of x is not zero
+__device__ __forceinline__ uint32_t nonzero_bytes(uint32_t x) {
+    x |= x >> 4;
+    x |= x >> 2;
+    x |= x >> 1;
+    return ((x & 0x01010101u) * 0x10204080u) >> 28;
+}
+
+// element e (0..7) of eight bf16 values
+__device__ __forceinline__ float bf16_of(const uint4& q, int e) {
+    const uint32_t h = (e & 4) ? ((e & 2) ? q.w : q.z) : ((e & 2) ? q.y : q.x);
+    return (e & 1) ? bf16_hi(h) : bf16_lo(h);
+}
+
+// chunk: words per warp, a multiple of kGatherSpan.  A sampling pass draws
+// row r with counter row row0 + (batch row of r).
+template <int FOLD>
+__global__ void __launch_bounds__(kGatherMaxWarps * 32, 2)
+    logits_gather_kernel(const void* __restrict__ logits, int64_t stride, const MaskRows mask, int V, int W, int B,
+                         int chunk, int32_t* __restrict__ argmax, float* __restrict__ lse, const SampleArgs sa,
+                         int row0, int keep_l2, const RowList list) {
+    constexpr int kSpanWords = 32 * kGatherSpan;
+    extern __shared__ __align__(16) unsigned char g_smem[];   // per warp: words, then list
+    __shared__ float4 s_part[kGatherMaxWarps];
+    pdl_wait();
+    pdl_trigger();
+    const int r = blockIdx.x;
+    if (r >= list.rows(B)) return;   // the whole CTA
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+    uint32_t* sw = reinterpret_cast<uint32_t*>(g_smem + wid * kGatherWarpSmem);   // a span's mask words
+    uint16_t* lst = reinterpret_cast<uint16_t*>(sw + kSpanWords);                // its vectors, in token order
+    const uint64_t pol = l2_policy(keep_l2 != 0);
+    const int full_vec = V / 8;   // vectors that lie wholly inside the row
+    const int j0 = wid * chunk, j1 = min(W, j0 + chunk);
+    const uint32_t* mrow = mask.row(r, W, threadIdx.x == 0);
+    const int orow = list.row(r);
+    const char* lrow = reinterpret_cast<const char*>(logits) + (size_t)orow * stride * 2;
+    float m = -INFINITY, mL = -INFINITY, s = 0.0f;
+    int idx = INT_MAX;
+    int blk = -1;   // Philox block cached by gumbel()
+    uint4 rnd = make_uint4(0u, 0u, 0u, 0u);
+    // one allowed logit x of token t (t increasing within a lane)
+    auto fold1 = [&](float x, int t) {
+        if constexpr (FOLD == kFoldSample) {
+            const float sx = __fmul_rn(x, sa.inv_t);
+            if (__fadd_rn(sx, kGumbelMax) < m) return;
+            const float sc = __fadd_rn(sx, gumbel(sa, row0 + orow, t, blk, rnd));
+            if (sc > m) {
+                m = sc;
+                idx = t;
+            }
+        } else if constexpr (FOLD == kFoldMax) {
+            if (x > m) {
+                m = x;
+                idx = t;
+            }
+        } else {
+            acc_add(m, mL, idx, s, x, t);
+        }
+    };
+    for (int js = j0; js < j1; js += kSpanWords) {
+        uint32_t w[kGatherSpan];
+        const int jl = js + lane * kGatherSpan;
+        if (mrow && jl + kGatherSpan <= j1 && (reinterpret_cast<uintptr_t>(mrow + jl) & 15) == 0) {
+            const uint4 a = __ldg(reinterpret_cast<const uint4*>(mrow + jl));
+            const uint4 b = __ldg(reinterpret_cast<const uint4*>(mrow + jl) + 1);
+            w[0] = a.x, w[1] = a.y, w[2] = a.z, w[3] = a.w, w[4] = b.x, w[5] = b.y, w[6] = b.z, w[7] = b.w;
+        } else {
+#pragma unroll
+            for (int g = 0; g < kGatherSpan; ++g) w[g] = jl + g < j1 ? mask.word(mrow, jl + g) : 0u;
+        }
+        uint32_t nb = 0;   // bit 4g + b: byte b of word g holds an allowed token
+#pragma unroll
+        for (int g = 0; g < kGatherSpan; ++g) nb |= nonzero_bytes(w[g]) << (4 * g);
+        reinterpret_cast<uint4*>(sw)[2 * lane] = make_uint4(w[0], w[1], w[2], w[3]);
+        reinterpret_cast<uint4*>(sw)[2 * lane + 1] = make_uint4(w[4], w[5], w[6], w[7]);
+        const int c = __popc(nb);
+        int incl = c;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, incl, off);
+            if (lane >= off) incl += y;
+        }
+        const int T = __shfl_sync(0xffffffffu, incl, 31);
+        if (T == 0) continue;   // warp-uniform
+        int pos = incl - c;
+        while (nb) {
+            const int bit = __ffs(nb) - 1;
+            nb &= nb - 1;
+            lst[pos++] = (uint16_t)(lane * 4 * kGatherSpan + bit);
+        }
+        __syncwarp();
+        const int vbase = js * 4;   // the span's first vector in the row
+        // rounds of kGatherRound vectors per lane; the next round's loads are
+        // issued before this round is folded
+        int ent[kGatherRound];
+        uint4 q[kGatherRound];
+        auto load_round = [&](int k0, int(&en)[kGatherRound], uint4(&qq)[kGatherRound]) {
+#pragma unroll
+            for (int i = 0; i < kGatherRound; ++i) {
+                const int k = k0 + i * 32 + lane;
+                en[i] = k < T ? (int)lst[k] : -1;
+                const int vi = vbase + en[i];
+                qq[i] = (en[i] >= 0 && vi < full_vec) ? ld_once16(lrow + (size_t)vi * 16, pol)
+                                                     : make_uint4(0u, 0u, 0u, 0u);
+            }
+        };
+        load_round(0, ent, q);
+        for (int k0 = 0; k0 < T; k0 += 32 * kGatherRound) {
+            int ent_n[kGatherRound];
+            uint4 q_n[kGatherRound];
+            const bool more = k0 + 32 * kGatherRound < T;   // warp-uniform
+            if (more) load_round(k0 + 32 * kGatherRound, ent_n, q_n);
+#pragma unroll
+            for (int i = 0; i < kGatherRound; ++i) {
+                if (ent[i] < 0) continue;
+                const int vi = vbase + ent[i], t0 = vi * 8;
+                uint32_t bm = (sw[ent[i] >> 2] >> (8 * (ent[i] & 3))) & 0xFFu;
+                if (vi >= full_vec) {   // the row's last, partial vector: token by token
+                    while (bm) {
+                        const int e = __ffs(bm) - 1;
+                        bm &= bm - 1;
+                        if (t0 + e >= V) break;
+                        fold1(logit_at<true>(lrow, t0 + e), t0 + e);
+                    }
+                } else if (FOLD == kFoldSample) {
+                    while (bm) {
+                        const int e = __ffs(bm) - 1;
+                        bm &= bm - 1;
+                        fold1(bf16_of(q[i], e), t0 + e);
+                    }
+                } else if (__popc(bm) > 2) {
+                    // a dense vector: its allowed maximum (first on ties), one
+                    // rescale, then its sum, all eight lanes of it predicated;
+                    // earlier vectors hold lower ids, so an equal maximum keeps idx
+                    float xs[8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) xs[e] = ((bm >> e) & 1u) ? bf16_of(q[i], e) : -INFINITY;
+                    float vm = xs[0];
+                    int ve = 0;
+#pragma unroll
+                    for (int e = 1; e < 8; ++e)
+                        if (xs[e] > vm) {
+                            vm = xs[e];
+                            ve = e;
+                        }
+                    if constexpr (FOLD == kFoldMax) {
+                        if (vm > m) {
+                            m = vm;
+                            idx = t0 + ve;
+                        }
+                    } else {
+                        if (vm > m) {
+                            const float vL = vm * kLog2e;
+                            s = s == 0.0f ? 0.0f : s * ex2(mL - vL);
+                            m = vm;
+                            mL = vL;
+                            idx = t0 + ve;
+                        }
+                        float acc = 0.0f;
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) acc += ((bm >> e) & 1u) ? ex2(fmaf(xs[e], kLog2e, -mL)) : 0.0f;
+                        s += acc;
+                    }
+                } else {
+                    while (bm) {
+                        const int e = __ffs(bm) - 1;
+                        bm &= bm - 1;
+                        fold1(bf16_of(q[i], e), t0 + e);
+                    }
+                }
+            }
+            if (more) {
+#pragma unroll
+                for (int i = 0; i < kGatherRound; ++i) {
+                    ent[i] = ent_n[i];
+                    q[i] = q_n[i];
+                }
+            }
+        }
+        __syncwarp();   // the span buffers are rewritten by the next span
+    }
+    warp_merge(m, idx, s);
+    if (lane == 0) s_part[wid] = make_float4(m, __int_as_float(idx), s, 0.f);
+    __syncthreads();
+    if (wid == 0) {
+        m = -INFINITY;
+        s = 0.0f;
+        idx = INT_MAX;
+        if (lane < nwarps) {
+            const float4 p = s_part[lane];
+            m = p.x;
+            idx = __float_as_int(p.y);
+            s = p.z;
+        }
+        warp_merge(m, idx, s);
+        if (lane == 0) {
+            argmax[orow] = m == -INFINITY ? -1 : idx;
+            if (lse) lse[orow] = m == -INFINITY ? -INFINITY : m + logf(s);
+        }
+    }
+}
+
 // logprob[t] = logit[t] - lse for allowed t, -inf otherwise.  VEC (bf16 rows on
 // 16-byte boundaries, V % 4 == 0): a thread takes 16 consecutive tokens when
 // V % 16 == 0 (32 bytes of logits read unconditionally, four float4 stores),
@@ -1352,6 +1590,36 @@ int occupancy(const void* kern, int threads) {
     return n;
 }
 
+// the gather kernels' dynamic shared memory passes the default 48 KB at 16
+// warps: the limit is raised once per device and fold
+template <int FOLD>
+cudaError_t gather_smem_ready() {
+    static bool configured[kMaxDevices] = {false};   // one array per fold
+    static std::mutex mu;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return cudaGetLastError();
+    if (dev >= kMaxDevices) dev = kMaxDevices - 1;
+    std::lock_guard<std::mutex> lk(mu);
+    if (!configured[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(logits_gather_kernel<FOLD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             kGatherMaxWarps * kGatherWarpSmem);
+        if (e != cudaSuccess) return e;
+        configured[dev] = true;
+    }
+    return cudaSuccess;
+}
+
+}  // namespace
+
+cudaError_t prepare_logits_kernels() {
+    cudaError_t e = gather_smem_ready<kFoldLse>();
+    if (e == cudaSuccess) e = gather_smem_ready<kFoldMax>();
+    if (e == cudaSuccess) e = gather_smem_ready<kFoldSample>();
+    return e;
+}
+
+namespace {
+
 template <bool BF16, bool STAGE>
 cudaError_t launch_logits_t(const LaunchEnv& env, const void* logits, int32_t batch, int64_t stride, int32_t V,
                             const MaskRows& mask, int32_t* argmax, float* lse, float* logprobs, float4* partials,
@@ -1384,9 +1652,31 @@ cudaError_t launch_logits_t(const LaunchEnv& env, const void* logits, int32_t ba
         long long per_cta = (N + grid - 1) / grid;
         per_cta = std::max<long long>(per_cta, ((long long)W + kMaxSegments - 3) / (kMaxSegments - 2));
         grid = (int)((N + per_cta - 1) / per_cta);
-        // a sampling pass draws row r of this chunk with counter row r0 + r
-        cudaError_t e0 = launch_pdl(reduce, dim3(grid), dim3(kReduceThreads), 0, st, lg, stride, mk, V, W, rows,
-                                    per_cta, partials, counters, argmax + shift, lse_rows, sa, (int)shift, lst);
+        cudaError_t e0;
+        // the gather takes one CTA per row: used when the rows alone fill the
+        // SMs (with fewer rows the flat split over rows x words keeps more
+        // warps busy)
+        if (BF16 && STAGE && rows > env.num_sms) {
+            auto gather = sample ? logits_gather_kernel<kFoldSample>
+                                 : (lse || logprobs) ? logits_gather_kernel<kFoldLse> : logits_gather_kernel<kFoldMax>;
+            // a warp per span of the row, at most kGatherMaxWarps (two CTAs per
+            // SM); a warp's words rounded up to whole lanes
+            const int nwarps =
+                std::max(1, std::min(kGatherMaxWarps, (W + 32 * kGatherSpan - 1) / (32 * kGatherSpan)));
+            int chunk = (W + nwarps - 1) / nwarps;
+            chunk = (chunk + kGatherSpan - 1) / kGatherSpan * kGatherSpan;
+            const int smem = nwarps * kGatherWarpSmem;
+            if (cudaError_t e = sample ? gather_smem_ready<kFoldSample>()
+                                       : (lse || logprobs) ? gather_smem_ready<kFoldLse>() : gather_smem_ready<kFoldMax>();
+                e != cudaSuccess)
+                return e;
+            e0 = launch_pdl(gather, dim3((unsigned)rows), dim3(nwarps * 32), (size_t)smem, st, lg, stride, mk, V, W,
+                            rows, chunk, argmax + shift, lse_rows, sa, (int)shift, logprobs ? 1 : 0, lst);
+        } else {
+            // a sampling pass draws row r of this chunk with counter row r0 + r
+            e0 = launch_pdl(reduce, dim3(grid), dim3(kReduceThreads), 0, st, lg, stride, mk, V, W, rows, per_cta,
+                            partials, counters, argmax + shift, lse_rows, sa, (int)shift, lst);
+        }
         if (e0 != cudaSuccess) return e0;
         if (logprobs) {
             const long long n_items = (out_vec && STAGE) ? (long long)rows * (V % 16 == 0 ? V / 16 : V / 4) : N;
@@ -1684,6 +1974,10 @@ int noalloc_setup(int dev, NoAllocDevice* out) {
         }
         int sms = 0;
         if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1) {
+            cudaGetLastError();
+            return DOMINO_E_CUDA;
+        }
+        if (domino::prepare_logits_kernels() != cudaSuccess) {
             cudaGetLastError();
             return DOMINO_E_CUDA;
         }

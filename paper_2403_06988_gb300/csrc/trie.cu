@@ -301,7 +301,6 @@ __global__ void __maxnreg__(56)
     const int b0 = __ldg(tv.cta_batch + blockIdx.x), b1 = __ldg(tv.cta_batch + blockIdx.x + 1);
     if (b0 >= b1) {   // no units for this CTA
         pdl_wait();
-        pdl_trigger();
         return;
     }
     for (int i = tid; i < (v.Q + 31) / 32; i += kTileThreads) s_accept[i] = __ldg(v.accept_bits + i);
@@ -364,8 +363,11 @@ __global__ void __maxnreg__(56)
                 spath[k * tv.max_path + d] = __ldg(tv.upath + up.y + d);
         }
         if (!waited) {   // everything above is the static tree; the masks come from tree_clear_kernel
+            // no early launch of the next kernel: one launched early parks its
+            // CTAs beside these, and a logits pass queued that way took about
+            // 10 us longer than one launched when this grid ends (GB300, batch
+            // 256, V = 128256)
             pdl_wait();
-            pdl_trigger();
             waited = true;
         }
         __syncthreads();
