@@ -329,9 +329,51 @@ bool cut_batches(domino_ctx* h) {
             break;
         }
     }
+    // A unit costs about the transitions its walk takes, which depend on the
+    // rows.  For a DFA they are counted here by walking the tree from up to
+    // 1024 states spread evenly over the automaton (the visits inside each
+    // unit); the CTAs' shares are balanced on those counts plus the units'
+    // node counts.  Pushdown automata are balanced on node counts.
     std::vector<int64_t> unit_nodes(unit.size());
+    for (size_t u = 0; u < unit.size(); u++) unit_nodes[u] = skip_of(unit[u].x) - unit[u].x;
+    if (!h->stack && !h->t16.empty() && h->Q > 1 && !unit.empty()) {
+        const int32_t Q = h->Q, K = h->K;
+        const uint32_t N = skip_of(0);
+        std::vector<int32_t> unit_of(N, -1);
+        for (size_t u = 0; u < unit.size(); u++)
+            for (uint32_t n = unit[u].x; n < skip_of(unit[u].x); n++) unit_of[n] = (int32_t)u;
+        std::vector<int64_t> visits(unit.size(), 0);
+        struct Frame {
+            uint32_t next, end, s;
+        };
+        std::vector<Frame> stk;
+        const int32_t stride = std::max<int32_t>(1, (Q - 1) / 1024);
+        for (int32_t q = 1; q < Q; q += stride) {
+            uint32_t n = 1, end = N, s = (uint32_t)q;
+            stk.clear();
+            for (;;) {
+                if (n >= end) {
+                    if (stk.empty()) break;
+                    const Frame f = stk.back();
+                    stk.pop_back();
+                    n = f.next, end = f.end, s = f.s;
+                    continue;
+                }
+                const uint32_t x = node[2 * (size_t)n].x, sk = x & 0xFFFFFFu;
+                const uint32_t s2 = h->t16[(size_t)s * K + (x >> 24)];
+                if (unit_of[n] >= 0) visits[(size_t)unit_of[n]]++;
+                if (s2 != 0 && sk > n + 1) {
+                    stk.push_back({sk, end, s});
+                    n = n + 1, end = sk, s = s2;
+                } else {
+                    n = sk;
+                }
+            }
+        }
+        for (size_t u = 0; u < unit.size(); u++) unit_nodes[u] += visits[u];
+    }
     int64_t total = 0;
-    for (size_t u = 0; u < unit.size(); u++) total += unit_nodes[u] = skip_of(unit[u].x) - unit[u].x;
+    for (size_t u = 0; u < unit.size(); u++) total += unit_nodes[u];
     const int per_node = 8 + (self ? 8 : 0);
     for (int64_t budget = (int64_t)smem - fixed - table; budget >= 4096; budget = budget * 9 / 10) {
         std::vector<uint4> batch, slot;
