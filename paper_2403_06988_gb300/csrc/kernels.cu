@@ -1258,13 +1258,33 @@ __global__ void __launch_bounds__(kLogitThreads)
 // ---------------------------------------------------------------------------
 template <bool STACK, int MODE>
 __global__ void __launch_bounds__(kAdvanceThreads)
-    advance_kernel(const StepView v, const int32_t* states, const uint64_t* stacks,
-                   const int32_t* __restrict__ tokens, int32_t batch, int32_t* states_out, uint64_t* stacks_out) {
+    advance_kernel(const StepView v, const uint4* __restrict__ img, int img_words, int tgt_off, int ret_off,
+                   const int32_t* states, const uint64_t* stacks, const int32_t* __restrict__ tokens, int32_t batch,
+                   int32_t* states_out, uint64_t* stacks_out) {
+    using E = typename std::conditional<STACK, uint32_t, uint16_t>::type;
+    extern __shared__ __align__(16) unsigned char adv_smem[];
+    if constexpr (MODE != kDenseGlobal) {
+        // the table image (written at load time, by no kernel) is staged
+        // before the launch wait, while the kernel before this one drains
+        for (int i = threadIdx.x; i < img_words; i += kAdvanceThreads)
+            reinterpret_cast<uint4*>(adv_smem)[i] = __ldg(img + i);
+        __syncthreads();
+    }
     pdl_wait();
     pdl_trigger();
     const int b = blockIdx.x * kAdvanceThreads + threadIdx.x;
     if (b >= batch) return;
-    advance_row<STACK, MODE>(v, states, stacks, b, tokens[b], states_out, stacks_out);
+    if constexpr (MODE == kDenseGlobal) {
+        advance_row<STACK, kDenseGlobal>(v, states, stacks, b, tokens[b], states_out, stacks_out);
+    } else {
+        Tab<E, MODE> tab;
+        tab.dense = reinterpret_cast<const E*>(adv_smem);
+        tab.sp = reinterpret_cast<const uint32_t*>(adv_smem);
+        tab.tgt = reinterpret_cast<const E*>(adv_smem + tgt_off);
+        tab.K = (uint32_t)v.K;
+        advance_row_with<STACK>(v, tab, reinterpret_cast<const uint16_t*>(adv_smem + ret_off), states, stacks, b,
+                                tokens[b], states_out, stacks_out);
+    }
 }
 
 // Opportunistic masking, the check: is row b's proposal (its unmasked argmax)
@@ -1842,25 +1862,58 @@ cudaError_t launch_mask_sample(const LaunchEnv& env, const void* logits, int dty
                               counters, nullptr, st, nullptr, 0, nullptr, &sa);
 }
 
+// The table image of `mode` staged in shared memory (the step kernel's image:
+// dense [Q][K] then pop targets, or the sparse rows, entries, pop targets);
+// kDenseGlobal reads the dense image from global memory.
+template <bool STACK, int MODE>
+cudaError_t launch_advance_m(const StepView& v, const int32_t* states, const uint64_t* stacks, const int32_t* tokens,
+                             int32_t batch, int32_t* states_out, uint64_t* stacks_out, cudaStream_t st) {
+    const unsigned grid = (unsigned)((batch + kAdvanceThreads - 1) / kAdvanceThreads);
+    const uint4* img = nullptr;
+    int bytes = 0, tgt_off = 0, ret_off = 0;
+    if constexpr (MODE != kDenseGlobal) {
+        const size_t esz = STACK ? 4 : 2;
+        bytes = (int)table_smem_bytes(v, STACK, MODE);
+        if (MODE == kDenseSmem) {
+            img = reinterpret_cast<const uint4*>(STACK ? (const void*)v.t32 : (const void*)v.t16);
+            ret_off = align16((int)((size_t)v.Q * v.K * esz));
+        } else {
+            img = reinterpret_cast<const uint4*>(v.sp_info);
+            tgt_off = align16(v.Q * (MODE == kSparse32Smem ? 8 : 16));
+            ret_off = tgt_off + align16((int)((size_t)v.sp_nnz * esz));
+        }
+        static int configured[kMaxDevices] = {0};
+        static std::mutex mu;
+        int dev = 0;
+        cudaGetDevice(&dev);
+        if (bytes > 48 * 1024 && dev < kMaxDevices) {
+            std::lock_guard<std::mutex> lk(mu);
+            if (configured[dev] < bytes) {
+                cudaError_t e =
+                    cudaFuncSetAttribute(advance_kernel<STACK, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+                if (e != cudaSuccess) return e;
+                configured[dev] = bytes;
+            }
+        }
+    }
+    return launch_pdl(advance_kernel<STACK, MODE>, dim3(grid), dim3(kAdvanceThreads), (size_t)bytes, st, v, img,
+                      bytes / 16, tgt_off, ret_off, states, stacks, tokens, batch, states_out, stacks_out);
+}
+
 template <bool STACK>
 cudaError_t launch_advance_s(const StepView& v, int mode, const int32_t* states, const uint64_t* stacks,
                              const int32_t* tokens, int32_t batch, int32_t* states_out, uint64_t* stacks_out,
                              cudaStream_t st) {
-    const unsigned grid = (unsigned)((batch + kAdvanceThreads - 1) / kAdvanceThreads);
     switch (mode) {
+        case kDenseSmem:
+            return launch_advance_m<STACK, kDenseSmem>(v, states, stacks, tokens, batch, states_out, stacks_out, st);
         case kSparse32Smem:
-            return launch_pdl(advance_kernel<STACK, kSparse32Smem>, dim3(grid), dim3(kAdvanceThreads), 0, st, v, states,
-                              stacks, tokens, batch, states_out, stacks_out);
-            break;
+            return launch_advance_m<STACK, kSparse32Smem>(v, states, stacks, tokens, batch, states_out, stacks_out, st);
         case kSparse64Smem:
-            return launch_pdl(advance_kernel<STACK, kSparse64Smem>, dim3(grid), dim3(kAdvanceThreads), 0, st, v, states,
-                              stacks, tokens, batch, states_out, stacks_out);
-            break;
+            return launch_advance_m<STACK, kSparse64Smem>(v, states, stacks, tokens, batch, states_out, stacks_out, st);
         default:
-            return launch_pdl(advance_kernel<STACK, kDenseGlobal>, dim3(grid), dim3(kAdvanceThreads), 0, st, v, states,
-                              stacks, tokens, batch, states_out, stacks_out);
+            return launch_advance_m<STACK, kDenseGlobal>(v, states, stacks, tokens, batch, states_out, stacks_out, st);
     }
-    return cudaGetLastError();
 }
 
 cudaError_t launch_advance(const StepView& v, bool stack, int mode, const int32_t* states, const uint64_t* stacks,

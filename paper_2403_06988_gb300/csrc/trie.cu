@@ -49,7 +49,8 @@ namespace {
 
 constexpr int kTileThreads = 1024;
 constexpr int kTileWarps = kTileThreads / 32;
-constexpr int kClearThreads = 256;          // 8 rows per CTA, one warp each
+constexpr int kClearThreads = 256;          // 8 warps per CTA
+constexpr int kClearSplit = 4;              // warps per row
 constexpr int kTrieCfg = 4096;              // (slot, row) configurations per row block
 constexpr int kTrieRowBlock = 512;          // most rows per block
 constexpr int kTrieEmitWarp = 32;           // longer token ranges are spread over the warp's lanes
@@ -108,33 +109,48 @@ __device__ __forceinline__ void set_bit(uint32_t* word, uint32_t bit) {
 // ---------------------------------------------------------------------------
 // tree_clear_kernel
 // ---------------------------------------------------------------------------
+// kClearSplit warps per row, each on a slice of its mask (and next states);
+// the warp whose slice holds EOS sets it after clearing.
 template <bool NEXT>
 __global__ void __launch_bounds__(kClearThreads)
     tree_clear_kernel(const __grid_constant__ StepView v, const __grid_constant__ TreeArgs a, const RowList list) {
     pdl_wait();
     pdl_trigger();
     const int lane = threadIdx.x & 31;
-    const int i = blockIdx.x * (kClearThreads / 32) + (threadIdx.x >> 5);
+    const int gw = blockIdx.x * (kClearThreads / 32) + (threadIdx.x >> 5);
+    const int i = gw / kClearSplit, part = gw - i * kClearSplit;
     if (i >= list.rows(a.batch)) return;
-    const int W = v.W, V = v.V;
+    const int W = v.W, V = v.V, eos = v.eos_id;
     uint32_t* mrow = a.mask ? a.mask + (size_t)i * W : nullptr;
     int32_t* nrow = NEXT && a.next ? a.next + (size_t)i * V : nullptr;
+    bool eos_m = false, eos_n = false;   // this warp's slices hold EOS
     if (mrow) {
-        if ((W & 3) == 0 && (reinterpret_cast<uintptr_t>(mrow) & 15) == 0) {
-            for (int j = lane; j < W / 4; j += 32) reinterpret_cast<uint4*>(mrow)[j] = make_uint4(0u, 0u, 0u, 0u);
+        const bool vec = (W & 3) == 0 && (reinterpret_cast<uintptr_t>(mrow) & 15) == 0;
+        const int n = vec ? W / 4 : W, c = (n + kClearSplit - 1) / kClearSplit;
+        const int j0 = part * c, j1 = min(n, j0 + c);
+        if (vec) {
+            for (int j = j0 + lane; j < j1; j += 32) reinterpret_cast<uint4*>(mrow)[j] = make_uint4(0u, 0u, 0u, 0u);
         } else {
-            for (int j = lane; j < W; j += 32) mrow[j] = 0u;
+            for (int j = j0 + lane; j < j1; j += 32) mrow[j] = 0u;
         }
+        const int e = vec ? (eos >> 5) >> 2 : eos >> 5;
+        eos_m = eos >= 0 && e >= j0 && e < j1;
     }
     if (nrow) {
-        if ((V & 3) == 0 && (reinterpret_cast<uintptr_t>(nrow) & 15) == 0) {
-            for (int j = lane; j < V / 4; j += 32) __stcs(reinterpret_cast<int4*>(nrow) + j, make_int4(0, 0, 0, 0));
+        const bool vec = (V & 3) == 0 && (reinterpret_cast<uintptr_t>(nrow) & 15) == 0;
+        const int n = vec ? V / 4 : V, c = (n + kClearSplit - 1) / kClearSplit;
+        const int j0 = part * c, j1 = min(n, j0 + c);
+        if (vec) {
+            for (int j = j0 + lane; j < j1; j += 32) __stcs(reinterpret_cast<int4*>(nrow) + j, make_int4(0, 0, 0, 0));
         } else {
-            for (int j = lane; j < V; j += 32) nrow[j] = 0;
+            for (int j = j0 + lane; j < j1; j += 32) nrow[j] = 0;
         }
+        const int e = vec ? eos >> 2 : eos;
+        eos_n = eos >= 0 && e >= j0 && e < j1;
     }
-    __syncwarp();   // the row is clear before its EOS bit is set
-    if (lane == 0) {   // the row's configuration: invalid ones set the error word; EOS
+    __syncwarp();   // the slice is clear before its EOS bit is set
+    if (lane == 0 && (part == 0 || eos_m || eos_n)) {
+        // the row's configuration (invalid ones set the error word, once per row)
         const int b = list.row(i);
         uint4 rc;
         if (a.row_is_state) {
@@ -144,12 +160,12 @@ __global__ void __launch_bounds__(kClearThreads)
             const int32_t sv = __ldg(a.states + b);
             const unsigned long long w =
                 a.stacks ? __ldg(reinterpret_cast<const unsigned long long*>(a.stacks) + b) : 0ull;
-            rc = decode_row(v, sv, w, a.stacks != nullptr, v.accept_bits, true);
+            rc = decode_row(v, sv, w, a.stacks != nullptr, v.accept_bits, part == 0);
         }
         // EOS: allowed iff the state accepts and the stack is empty; the state stays
-        if ((rc.w & 2u) && v.eos_id >= 0) {
-            if (mrow) set_bit(mrow + (v.eos_id >> 5), 1u << (v.eos_id & 31));
-            if (nrow) nrow[v.eos_id] = (int32_t)rc.x;
+        if (rc.w & 2u) {
+            if (eos_m) set_bit(mrow + (eos >> 5), 1u << (eos & 31));
+            if (eos_n) nrow[eos] = (int32_t)rc.x;
         }
     }
 }
@@ -271,11 +287,9 @@ struct TileCtx {
     }
 };
 
-// At most 56 registers: a 1024-thread CTA then leaves room on its SM for the
-// next step's tree_clear_kernel CTAs, which start (and wait on this kernel)
-// while it drains instead of after it.
+// 1024 threads a CTA: at most 64 registers a thread.
 template <bool STACK, int MODE, bool NEXT>
-__global__ void __maxnreg__(56)
+__global__ void __maxnreg__(64)
     tree_tile_kernel(const __grid_constant__ StepView v, const __grid_constant__ TrieView tv,
                      const uint4* __restrict__ img, const __grid_constant__ TreeArgs a, const RowList list) {
     using E = typename std::conditional<STACK, uint32_t, uint16_t>::type;
@@ -499,7 +513,7 @@ cudaError_t launch_tree_t(const StepView& v, const TrieView& tv, const LaunchEnv
             configured[dev] = L.total;
         }
     }
-    const int clear_grid = (a.batch + kClearThreads / 32 - 1) / (kClearThreads / 32);
+    const int clear_grid = (int)(((int64_t)a.batch * kClearSplit + kClearThreads / 32 - 1) / (kClearThreads / 32));
     cudaError_t e = launch_pdl(tree_clear_kernel<NEXT>, dim3(clear_grid), dim3(kClearThreads), 0, st, v, a, list);
     if (e != cudaSuccess) return e;
     return launch_pdl(tile, dim3(tv.grid), dim3(kTileThreads), (size_t)L.total, st, v, tv, img, a, list);

@@ -264,10 +264,10 @@ __device__ __forceinline__ uint4 read_row_rw(const StepView& v, const int32_t* s
 // C.update() for one row: row b's configuration walks token t (t < 0 or EOS:
 // the start state; a rejected token: state 0; t >= V: state 0 and the error
 // word).  Reads the configuration before writing, so the outputs may alias it.
-template <bool STACK, int MODE>
-__device__ __forceinline__ void advance_row(const StepView& v, const int32_t* states, const uint64_t* stacks, int b,
-                                            int32_t t, int32_t* states_out, uint64_t* stacks_out) {
-    using E = typename std::conditional<STACK, uint32_t, uint16_t>::type;
+template <bool STACK, typename TabT>
+__device__ __forceinline__ void advance_row_with(const StepView& v, const TabT& tab, const uint16_t* ret,
+                                                 const int32_t* states, const uint64_t* stacks, int b, int32_t t,
+                                                 int32_t* states_out, uint64_t* stacks_out) {
     uint32_t s = 0, bits = 0, depth = 0;
     if (t < 0 || t == v.eos_id) {
         s = (uint32_t)v.start;   // the sequence ended; the next one starts from init
@@ -276,12 +276,6 @@ __device__ __forceinline__ void advance_row(const StepView& v, const int32_t* st
     } else {
         const uint4 rc = read_row_rw(v, states, stacks, b, true);
         if (rc.w & 1u) {
-            // the table image the step kernel staged (L2-resident) read from global memory
-            Tab<E, MODE == kDenseSmem ? kDenseGlobal : MODE> tab;
-            tab.dense = reinterpret_cast<const E*>(STACK ? (const void*)v.t32 : (const void*)v.t16);
-            tab.sp = v.sp_info;
-            tab.tgt = reinterpret_cast<const E*>(v.sp_tgt);
-            tab.K = (uint32_t)v.K;
             const int p = __ldg(v.pos_of + t);
             const int len = (int)(__ldg(v.info + p) >> 16);
             const uint8_t* hp = reinterpret_cast<const uint8_t*>(v.head + 2 * (size_t)p);
@@ -289,13 +283,27 @@ __device__ __forceinline__ void advance_row(const StepView& v, const int32_t* st
             if (len > 0) {
                 bits = rc.y;
                 depth = rc.z;
-                s = walk<STACK, 0>(tab, v.ret, (uint32_t)v.max_depth, rc.x, bits, depth, hp, len, tail);
+                s = walk<STACK, 0>(tab, ret, (uint32_t)v.max_depth, rc.x, bits, depth, hp, len, tail);
                 if (s == 0) bits = depth = 0;
             }
         }
     }
     states_out[b] = (int32_t)s;
     if (stacks_out) stacks_out[b] = ((uint64_t)depth << 32) | bits;
+}
+
+// advance_row_with over the table image the step kernel stages, read from
+// global memory (L2-resident)
+template <bool STACK, int MODE>
+__device__ __forceinline__ void advance_row(const StepView& v, const int32_t* states, const uint64_t* stacks, int b,
+                                            int32_t t, int32_t* states_out, uint64_t* stacks_out) {
+    using E = typename std::conditional<STACK, uint32_t, uint16_t>::type;
+    Tab<E, MODE == kDenseSmem ? kDenseGlobal : MODE> tab;
+    tab.dense = reinterpret_cast<const E*>(STACK ? (const void*)v.t32 : (const void*)v.t16);
+    tab.sp = v.sp_info;
+    tab.tgt = reinterpret_cast<const E*>(v.sp_tgt);
+    tab.K = (uint32_t)v.K;
+    advance_row_with<STACK>(v, tab, v.ret, states, stacks, b, t, states_out, stacks_out);
 }
 }  // namespace
 }  // namespace domino
