@@ -95,6 +95,7 @@ struct StepView {
 // node are set by the one batch that lists that node as an emitting slot.
 constexpr int kTrieTile = 64;
 constexpr int kTrieBranch = 8;
+constexpr int kTrieInterleave = 2;      // places of the tree a CTA's units are drawn from
 constexpr int kTrieMaxSlots = 48;             // slots per batch
 constexpr int32_t kTrieMaxNodes = (1 << 24) - 1;
 
@@ -103,10 +104,11 @@ struct TrieView {
     const int32_t* dtok;      // original ids in preorder
     const uint4* upper;       // [n_upper]: {node, path offset, path length, 0}
     const uint8_t* upath;     // classes of the upper nodes' paths from the root
-    const uint4* batch;       // [n_batches][2]: {first unit, end unit, first node, end node},
-                              //                 {first token, end token, first slot, end slot}
+    const uint4* batch;       // [n_batches][2]: {first unit, end unit, first range, end range},
+                              //                 {first slot, end slot, staged nodes, staged tokens}
+    const uint4* range;       // {first node, end node, first token, end token}: staged one after the other
     const uint4* slot;        // {upper index, first token ending at its node, tokens it sets (0: none), 0}
-    const uint2* unit;        // {root node, slot index within the batch}
+    const uint2* unit;        // {root's staged index, slot index within the batch}
     const int32_t* cta_batch; // [grid + 1]: CTA c takes batches [cta_batch[c], cta_batch[c + 1])
     int32_t n_nodes, n_upper, grid;
     int32_t max_nodes, max_toks, max_units, max_slots, max_path;   // the largest batch

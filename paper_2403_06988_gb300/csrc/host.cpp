@@ -60,7 +60,7 @@ struct domino_ctx {
     DevBuf d_err, d_partials, d_counters, d_lse_tmp, d_fpart;
     bool arena_ready = false;
     // prefix tree of the class strings and its per-CTA batches (see TrieView)
-    DevBuf d_tnode, d_tdtok, d_tupper, d_tupath, d_tbatch, d_tslot, d_tunit, d_tcta;
+    DevBuf d_tnode, d_tdtok, d_tupper, d_tupath, d_tbatch, d_trange, d_tslot, d_tunit, d_tcta;
     std::vector<uint4> t_node;       // host copies (domino_get_prefix_tree)
     std::vector<int32_t> t_dtok;
     std::vector<uint4> t_upper;      // {node, path offset, path length, 0}
@@ -68,6 +68,7 @@ struct domino_ctx {
     std::vector<uint2> t_unit;       // {root node, parent upper index}
     // per-CTA batches (see TrieView)
     std::vector<uint4> t_batch;      // two per batch
+    std::vector<uint4> t_range;      // {first node, end node, first token, end token}
     std::vector<uint4> t_slot;
     std::vector<uint2> t_bunit;      // {root node, slot within the batch}
     std::vector<int32_t> t_cta;      // [grid + 1] first batch of each CTA
@@ -96,8 +97,9 @@ struct domino_ctx {
     cudaEvent_t ev_cfg = nullptr;
     cudaEvent_t ev_chunk[8] = {};
     cudaEvent_t ev_t[4] = {};       // the chunked copy's start and end (2, 3)
-    // host wall time of the last settled call of each path for pinned bf16
-    // logits: [0] the chunked copy, [1] the in-place read (0: not yet seen)
+    // host wall time of each path for pinned bf16 logits, a moving average
+    // over settled calls: [0] the chunked copy, [1] the in-place read (0: not
+    // yet seen)
     double t_wall_ms[2] = {0.0, 0.0};
     // Recorded host-buffer steps: a call whose buffers, sizes and path match an
     // earlier one replays that call's CUDA graph instead of issuing each copy
@@ -375,88 +377,131 @@ bool cut_batches(domino_ctx* h) {
     int64_t total = 0;
     for (size_t u = 0; u < unit.size(); u++) total += unit_nodes[u];
     const int per_node = 8 + (self ? 8 : 0);
+    if (unit.empty()) return false;
+    // the upper nodes whose tokens a unit's batch sets: those with tokens
+    // between the previous unit's root and its own (trailing ones: the last)
+    std::vector<std::vector<uint32_t>> emit_at(unit.size());
+    {
+        size_t ui = 0;
+        for (size_t u = 0; u < upper.size(); u++) {
+            if (node[2 * (size_t)upper[u].x].z == 0) continue;
+            while (ui < unit.size() && unit[ui].x < upper[u].x) ui++;
+            emit_at[std::min(ui, unit.size() - 1)].push_back((uint32_t)u);
+        }
+    }
+    // The units in preorder are cut into grid x kTrieInterleave chunks of
+    // equal cost; CTA c takes chunks c, c + grid, ...  The rows live at a
+    // unit vary from one batch of rows to the next, and nearby units share
+    // their upper nodes, so a CTA's share drawn from several places of the
+    // tree varies less than one run of it.
+    const int nchunk = grid * kTrieInterleave;
+    std::vector<size_t> cbeg((size_t)nchunk + 1, unit.size());
+    {
+        int64_t done = 0;
+        size_t u = 0;
+        for (int j = 0; j < nchunk; j++) {
+            cbeg[(size_t)j] = u;
+            const int64_t goal = total * (j + 1) / nchunk;
+            while (u < unit.size() && (done < goal || j == nchunk - 1)) done += unit_nodes[u++];
+        }
+    }
     for (int64_t budget = (int64_t)smem - fixed - table; budget >= 4096; budget = budget * 9 / 10) {
-        std::vector<uint4> batch, slot;
+        std::vector<uint4> batch, slot, range;
         std::vector<uint2> bunit;
         std::vector<int32_t> cta((size_t)grid + 1, 0);
         int32_t mx_nodes = 0, mx_toks = 0, mx_units = 0, mx_slots = 0, mx_path = 0;
-        size_t u = 0, up = 0;   // next unit, next upper node whose tokens are unassigned
-        int64_t done = 0;
         bool ok = true;
         for (int c = 0; c < grid && ok; c++) {
             cta[(size_t)c] = (int32_t)(batch.size() / 2);
-            const int64_t goal = total * (c + 1) / grid;
-            size_t ue = u;
-            while (ue < unit.size() && (done < goal || c == grid - 1)) done += unit_nodes[ue++];
-            while (u < ue && ok) {
-                // one batch: units [u, b1) of this CTA
-                const uint32_t n0 = unit[u].x, t0 = node[2 * (size_t)n0].y;
-                const size_t slot0 = slot.size(), unit0 = bunit.size();
+            std::vector<std::pair<size_t, size_t>> runs;   // this CTA's unit runs, in preorder
+            for (int k = 0; k < kTrieInterleave; k++) {
+                const size_t j = (size_t)c + (size_t)k * grid;
+                if (cbeg[j] < cbeg[j + 1]) runs.emplace_back(cbeg[j], cbeg[j + 1]);
+            }
+            size_t ri = 0, u = runs.empty() ? 0 : runs[0].first;
+            while (ri < runs.size() && ok) {
+                // one batch: units of this CTA's runs from u on, staged as node
+                // and token ranges one after the other
+                const size_t slot0 = slot.size(), unit0 = bunit.size(), range0 = range.size();
                 std::vector<std::pair<uint32_t, uint32_t>> slots;   // (upper index, slot)
                 auto slot_of = [&](uint32_t ui, bool emit) -> int {
-                    for (auto& p : slots)
-                        if (p.first == ui) return (int)p.second;
-                    if ((int)slots.size() >= kTrieMaxSlots) return -1;
                     const uint32_t n = upper[ui].x;
+                    for (auto& p : slots)
+                        if (p.first == ui) {
+                            if (emit) slot[slot0 + p.second].z = node[2 * (size_t)n].z;
+                            return (int)p.second;
+                        }
+                    if ((int)slots.size() >= kTrieMaxSlots) return -1;
                     slot.push_back(make_uint4(ui, node[2 * (size_t)n].y, emit ? node[2 * (size_t)n].z : 0u, 0u));
                     slots.emplace_back(ui, (uint32_t)slots.size());
                     mx_path = std::max<int32_t>(mx_path, (int32_t)upper[ui].z);
                     return (int)slots.size() - 1;
                 };
-                auto bytes_now = [&](uint32_t n1, uint32_t t1) {
-                    return (int64_t)(n1 - n0) * per_node + (int64_t)(t1 - t0) * 4 +
-                           (int64_t)(bunit.size() - unit0) * 4 + (int64_t)slots.size() * (16 + 64);
+                int64_t nodes_b = 0, toks_b = 0;   // staged by the closed ranges
+                bool open = false;
+                uint32_t rn0 = 0, rn1 = 0, rt0 = 0, rt1 = 0;   // the open range
+                auto close_range = [&]() {
+                    if (!open) return;
+                    range.push_back(make_uint4(rn0, rn1, rt0, rt1));
+                    nodes_b += rn1 - rn0;
+                    toks_b += rt1 - rt0;
+                    open = false;
                 };
-                size_t b1 = u;
-                while (b1 < ue) {
-                    // the upper nodes in front of unit b1 set their tokens here
-                    const size_t keep_slots = slot.size(), keep_units = bunit.size();
-                    const size_t keep_up = up;
+                size_t added = 0;
+                while (ri < runs.size()) {
+                    if (u >= runs[ri].second) {   // the run is done: its range closes
+                        close_range();
+                        if (++ri < runs.size()) u = runs[ri].first;
+                        continue;
+                    }
+                    const size_t keep_slots = slot.size();
                     const auto keep_list = slots;
+                    std::vector<uint32_t> keep_z;
+                    for (size_t k = slot0; k < slot.size(); k++) keep_z.push_back(slot[k].z);
                     bool fit = true;
-                    while (fit && up < upper.size() && upper[up].x < unit[b1].x) {
-                        if (node[2 * (size_t)upper[up].x].z > 0) fit = slot_of((uint32_t)up, true) >= 0;
-                        up++;
-                    }
-                    int sl = fit ? slot_of(unit[b1].y, false) : -1;
+                    for (uint32_t e : emit_at[u])
+                        if (fit) fit = slot_of(e, true) >= 0;
+                    const int sl = fit ? slot_of(unit[u].y, false) : -1;
                     fit = sl >= 0;
-                    const uint32_t n1 = skip_of(unit[b1].x), t1 = node[2 * (size_t)unit[b1].x].w;
-                    if (fit) {
-                        bunit.push_back(make_uint2(unit[b1].x, (uint32_t)sl));
-                        fit = n1 - n0 <= 0xFFFFu && t1 - t0 <= 0xFFFFu && bytes_now(n1, t1) <= budget;
-                    }
-                    if (!fit) {   // undo the additions of this unit
+                    const uint32_t n0 = open ? rn0 : unit[u].x, t0 = open ? rt0 : node[2 * (size_t)unit[u].x].y;
+                    const uint32_t n1 = skip_of(unit[u].x), t1 = node[2 * (size_t)unit[u].x].w;
+                    const int64_t nodes_all = nodes_b + (n1 - n0), toks_all = toks_b + (t1 - t0);
+                    if (fit)
+                        fit = nodes_all <= 0xFFFF && toks_all <= 0xFFFF &&
+                              nodes_all * per_node + toks_all * 4 + (int64_t)(bunit.size() - unit0 + 1) * 4 +
+                                      (int64_t)slots.size() * (16 + 64) <=
+                                  budget;
+                    if (!fit) {   // undo this unit's slots; the batch ends before it
                         slot.resize(keep_slots);
-                        bunit.resize(keep_units);
-                        up = keep_up;
                         slots = keep_list;
-                        if (b1 == u) ok = false;   // a unit alone does not fit
+                        for (size_t k = slot0; k < slot.size(); k++) slot[k].z = keep_z[k - slot0];
+                        if (added == 0) ok = false;   // a unit alone does not fit
                         break;
                     }
-                    b1++;
+                    bunit.push_back(make_uint2((uint32_t)(nodes_b + (unit[u].x - n0)), (uint32_t)sl));
+                    if (!open) {
+                        rn0 = n0;
+                        rt0 = t0;
+                        open = true;
+                    }
+                    rn1 = n1;
+                    rt1 = t1;
+                    added++;
+                    u++;
                 }
                 if (!ok) break;
-                if (c == grid - 1 && b1 == ue) {   // the last CTA sets the tokens of the trailing upper nodes
-                    while (up < upper.size()) {
-                        if (node[2 * (size_t)upper[up].x].z > 0 && slot_of((uint32_t)up, true) < 0) {
-                            ok = false;
-                            break;
-                        }
-                        up++;
-                    }
-                }
-                const uint32_t n1 = skip_of(unit[b1 - 1].x), t1 = node[2 * (size_t)unit[b1 - 1].x].w;
-                batch.push_back(make_uint4((uint32_t)unit0, (uint32_t)bunit.size(), n0, n1));
-                batch.push_back(make_uint4(t0, t1, (uint32_t)slot0, (uint32_t)slot.size()));
-                mx_nodes = std::max<int32_t>(mx_nodes, (int32_t)(n1 - n0));
-                mx_toks = std::max<int32_t>(mx_toks, (int32_t)(t1 - t0));
+                close_range();
+                batch.push_back(make_uint4((uint32_t)unit0, (uint32_t)bunit.size(), (uint32_t)range0,
+                                           (uint32_t)range.size()));
+                batch.push_back(make_uint4((uint32_t)slot0, (uint32_t)slot.size(), (uint32_t)nodes_b,
+                                           (uint32_t)toks_b));
+                mx_nodes = std::max<int32_t>(mx_nodes, (int32_t)nodes_b);
+                mx_toks = std::max<int32_t>(mx_toks, (int32_t)toks_b);
                 mx_units = std::max<int32_t>(mx_units, (int32_t)(bunit.size() - unit0));
                 mx_slots = std::max<int32_t>(mx_slots, (int32_t)(slot.size() - slot0));
-                u = b1;
             }
         }
         if (!ok) continue;
-        if (unit.empty()) return false;
         cta[(size_t)grid] = (int32_t)(batch.size() / 2);
         TrieView tv{};
         tv.max_nodes = mx_nodes;
@@ -466,6 +511,7 @@ bool cut_batches(domino_ctx* h) {
         tv.max_path = mx_path;
         if (trie_tile_smem_bytes(v, tv, h->stack, (int)table) > smem) continue;   // the maxima together: cut tighter
         h->t_batch.swap(batch);
+        h->t_range.swap(range);
         h->t_slot.swap(slot);
         h->t_bunit.swap(bunit);
         h->t_cta.swap(cta);
@@ -492,6 +538,7 @@ int build_trie(domino_ctx* h) {
     if ((rc = up(h->d_tupper, h->t_upper.data(), h->t_upper.size() * sizeof(uint4)))) return rc;
     if ((rc = up(h->d_tupath, h->t_upath.data(), h->t_upath.size()))) return rc;
     if ((rc = up(h->d_tbatch, h->t_batch.data(), h->t_batch.size() * sizeof(uint4)))) return rc;
+    if ((rc = up(h->d_trange, h->t_range.data(), h->t_range.size() * sizeof(uint4)))) return rc;
     if ((rc = up(h->d_tslot, h->t_slot.data(), h->t_slot.size() * sizeof(uint4)))) return rc;
     if ((rc = up(h->d_tunit, h->t_bunit.data(), h->t_bunit.size() * sizeof(uint2)))) return rc;
     if ((rc = up(h->d_tcta, h->t_cta.data(), h->t_cta.size() * 4))) return rc;
@@ -639,6 +686,7 @@ TrieView make_trie_view(const domino_ctx* h) {
     tv.upper = (const uint4*)h->d_tupper.p;
     tv.upath = (const uint8_t*)h->d_tupath.p;
     tv.batch = (const uint4*)h->d_tbatch.p;
+    tv.range = (const uint4*)h->d_trange.p;
     tv.slot = (const uint4*)h->d_tslot.p;
     tv.unit = (const uint2*)h->d_tunit.p;
     tv.cta_batch = (const int32_t*)h->d_tcta.p;
@@ -757,7 +805,7 @@ int domino_destroy(domino_t h) {
                          &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_self, &h->d_tok_cls, &h->d_err, &h->d_fpart, &h->d_partials,
                          &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_mask, &h->s_io,
                          &h->o_prop, &h->o_rows, &h->o_count, &h->d_tnode, &h->d_tdtok, &h->d_tupper, &h->d_tupath, &h->d_tbatch, &h->d_tslot,
-                         &h->d_tunit, &h->d_tcta};
+                         &h->d_tunit, &h->d_tcta, &h->d_trange};
         for (auto* b : all) dev_free(*b);
         for (cudaEvent_t& e : h->ev_chunk)
             if (e) cudaEventDestroy(e);
@@ -1482,7 +1530,7 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
     // link, while the walk runs.  Or they are copied in chunks while the mask
     // step runs and decoded as they land.  Which is faster depends on the
     // masks' density and on the link's read granularity, so it is measured:
-    // each path's host wall time is taken on settled calls (no buffer growth,
+    // each path's host wall time is averaged over settled calls (no buffer growth,
     // no recording), the faster one is used, and every 64th call takes the
     // other to keep its time current.
     const auto t_enter = std::chrono::steady_clock::now();
@@ -1595,9 +1643,13 @@ int domino_decode_step_host(domino_t h, const void* logits_host, int32_t dtype, 
     if (lse_host) std::memcpy(lse_host, io + L.lse, (size_t)batch * 4);
     std::memcpy(states_host, io + L.st, (size_t)batch * 4);
     if (stacks) std::memcpy(stacks_host, io + L.sk, (size_t)batch * 8);
-    if (choice && !grow && !record && h->host_calls > 1)
-        h->t_wall_ms[mapped ? 1 : 0] =
-            std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t_enter).count();
+    if (choice && !grow && !record && h->host_calls > 1) {
+        // a moving average, so that one slow call (the host preempted, a
+        // shared link) does not send the next 64 calls down the slower path
+        const double t = std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t_enter).count();
+        double& avg = h->t_wall_ms[mapped ? 1 : 0];
+        avg = avg == 0.0 ? t : 0.75 * avg + 0.25 * t;
+    }
     return DOMINO_OK;
 }
 

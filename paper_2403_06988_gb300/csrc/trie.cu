@@ -341,35 +341,49 @@ __global__ void __maxnreg__(64)
     uint2* wustk = ustk + warp * kTrieBranch;
     bool waited = false;
     for (int bj = b0; bj < b1; ++bj) {
-        const uint4 bA = __ldg(tv.batch + 2 * bj);       // units [x, y), nodes [z, w)
-        const uint4 bB = __ldg(tv.batch + 2 * bj + 1);   // tokens [x, y), slots [z, w)
-        const int nk = (int)(bA.y - bA.x), nn = (int)(bA.w - bA.z), nt = (int)(bB.y - bB.x);
-        const int ns = (int)(bB.w - bB.z);
+        const uint4 bA = __ldg(tv.batch + 2 * bj);       // units [x, y), ranges [z, w)
+        const uint4 bB = __ldg(tv.batch + 2 * bj + 1);   // slots [x, y), staged nodes z, tokens w
+        const int nk = (int)(bA.y - bA.x), nn = (int)bB.z, nt = (int)bB.w;
+        const int ns = (int)(bB.y - bB.x);
         __syncthreads();   // the previous batch is done with shared memory
         if (tid == 0) ctl[kCtlBad] = 0;
         __syncthreads();
-        for (int n = tid; n < nn; n += kTileThreads) {
-            const uint4 r0 = __ldg(tv.node + 2 * ((size_t)bA.z + n));
-            // preorder (a subtree ends after its root) and the node's tokens
-            // inside the batch's: the walk relies on both.  The upper nodes
-            // between a batch's units are staged too (never walked); their
-            // subtrees end past the batch, so skips are clamped to its end.
-            const uint32_t xs = min((r0.x & 0xFFFFFFu) - bA.z, (uint32_t)nn), tl = r0.y - bB.x;
-            if (xs <= (uint32_t)n || tl > (uint32_t)nt || r0.z > (uint32_t)nt - tl) ctl[kCtlBad] = 1;
-            snode[n] = make_uint2(xs | ((r0.x >> 24) << 16), tl | (r0.z << 16));
-            if (use_self) {
-                const uint4 r1 = __ldg(tv.node + 2 * ((size_t)bA.z + n) + 1);
-                ssub[n] = ((unsigned long long)r1.y << 32) | r1.x;
+        // the batch's node and token ranges, staged one after the other; a
+        // node's subtree end and first token become staged indices
+        int sb = 0, tb = 0;
+        for (uint32_t ri = bA.z; ri < bA.w; ++ri) {
+            const uint4 R = __ldg(tv.range + ri);   // {first node, end node, first token, end token}
+            const int rn = (int)(R.y - R.x), rt = (int)(R.w - R.z);
+            if (rn < 0 || rt < 0 || sb + rn > nn || tb + rt > nt) {
+                if (tid == 0) ctl[kCtlBad] = 1;
+                break;
             }
+            for (int n = tid; n < rn; n += kTileThreads) {
+                const uint4 r0 = __ldg(tv.node + 2 * ((size_t)R.x + n));
+                // preorder (a subtree ends after its root) and the node's tokens
+                // inside the range's: the walk relies on both.  The upper nodes
+                // between a range's units are staged too (never walked); their
+                // subtrees end past the range, so skips are clamped to its end.
+                const uint32_t xs = min((r0.x & 0xFFFFFFu) - R.x, (uint32_t)rn), tl = r0.y - R.z;
+                if (xs <= (uint32_t)n || tl > (uint32_t)rt || r0.z > (uint32_t)rt - tl) ctl[kCtlBad] = 1;
+                snode[sb + n] = make_uint2((xs + sb) | ((r0.x >> 24) << 16), (tl + tb) | (r0.z << 16));
+                if (use_self) {
+                    const uint4 r1 = __ldg(tv.node + 2 * ((size_t)R.x + n) + 1);
+                    ssub[sb + n] = ((unsigned long long)r1.y << 32) | r1.x;
+                }
+            }
+            for (int j = tid; j < rt; j += kTileThreads) stok[tb + j] = __ldg(tv.dtok + R.z + j);
+            sb += rn;
+            tb += rt;
         }
-        for (int j = tid; j < nt; j += kTileThreads) stok[j] = __ldg(tv.dtok + bB.x + j);
+        if ((sb != nn || tb != nt) && tid == 0) ctl[kCtlBad] = 1;
         for (int k = tid; k < nk; k += kTileThreads) {
             const uint2 un = __ldg(tv.unit + bA.x + k);
-            if (un.x < bA.z || un.x >= bA.w || un.y >= (uint32_t)ns) ctl[kCtlBad] = 1;
-            sunit[k] = (un.x - bA.z) | (un.y << 16);
+            if (un.x >= (uint32_t)nn || un.y >= (uint32_t)ns) ctl[kCtlBad] = 1;
+            sunit[k] = un.x | (un.y << 16);
         }
         for (int k = tid; k < ns; k += kTileThreads) {
-            const uint4 sl = __ldg(tv.slot + bB.z + k);   // {upper index, first token, tokens set, 0}
+            const uint4 sl = __ldg(tv.slot + bB.x + k);   // {upper index, first token, tokens set, 0}
             const uint4 up = __ldg(tv.upper + sl.x);      // {node, path offset, path length, 0}
             if (up.z > (uint32_t)tv.max_path) ctl[kCtlBad] = 1;
             sslot[k] = make_uint4(min(up.z, (uint32_t)tv.max_path), 0u, sl.y, sl.z);
