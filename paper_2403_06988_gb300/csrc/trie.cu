@@ -470,23 +470,28 @@ __global__ void __maxnreg__(64)
                     cx.emit_one(r0 + r, __ldg(tv.dtok + sl.z + j), cfg[k * nr + r] & 0xFFFFu);
                 }
             }
-            // 3. warps claim units; a unit is walked for its slot's live rows,
-            // 32 at a time
+            // 3. warps claim (unit, chunk of 32 of its slot's live rows) items,
+            // chunk-major: every unit's first chunk, then every second chunk,
+            // so that units with many live rows do not leave one warp working
+            // while the others wait at the barrier
+            int maxc = 0;   // the most chunks any slot has
+            for (int k = lane; k < ns; k += 32) maxc = max(maxc, (lcount[k] + 31) >> 5);
+            maxc = __reduce_max_sync(0xffffffffu, maxc);
             for (;;) {
-                int k = 0;
-                if (lane == 0) k = atomicAdd(&ctl[kCtlUnit], 1);
-                k = __shfl_sync(0xffffffffu, k, 0);
-                if (k >= nk) break;
+                int i = 0;
+                if (lane == 0) i = atomicAdd(&ctl[kCtlUnit], 1);
+                i = __shfl_sync(0xffffffffu, i, 0);
+                if (i >= nk * maxc) break;
+                const int c = i / nk, k = i - c * nk;
                 const uint32_t un = sunit[k];
                 const int x0 = (int)(un & 0xFFFFu), sl = (int)(un >> 16);
-                const int n = lcount[sl];
-                for (int c = 0; c < n; c += 32) {
-                    const bool on = c + lane < n;
-                    const int r = on ? lrows[sl * rb + c + lane] : 0;
-                    const uint32_t sd = on ? cfg[sl * nr + r] : 0u;
-                    const uint32_t bits = STACK && on ? cfg[kTrieCfg + sl * nr + r] : 0u;
-                    cx.walk(lane, r0 + r, x0, sd & 0xFFFFu, bits, sd >> 16, wstk, wstkb, wustk);
-                }
+                const int n = lcount[sl] - 32 * c;
+                if (n <= 0) continue;
+                const bool on = lane < n;
+                const int r = on ? lrows[sl * rb + 32 * c + lane] : 0;
+                const uint32_t sd = on ? cfg[sl * nr + r] : 0u;
+                const uint32_t bits = STACK && on ? cfg[kTrieCfg + sl * nr + r] : 0u;
+                cx.walk(lane, r0 + r, x0, sd & 0xFFFFu, bits, sd >> 16, wstk, wstkb, wustk);
             }
             __syncthreads();
         }
