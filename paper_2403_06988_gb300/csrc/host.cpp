@@ -408,6 +408,7 @@ bool cut_batches(domino_ctx* h) {
     for (int64_t budget = (int64_t)smem - fixed - table; budget >= 4096; budget = budget * 9 / 10) {
         std::vector<uint4> batch, slot, range;
         std::vector<uint2> bunit;
+        std::vector<int64_t> bweight;   // the estimated cost of each bunit entry
         std::vector<int32_t> cta((size_t)grid + 1, 0);
         int32_t mx_nodes = 0, mx_toks = 0, mx_units = 0, mx_slots = 0, mx_path = 0;
         bool ok = true;
@@ -479,6 +480,7 @@ bool cut_batches(domino_ctx* h) {
                         break;
                     }
                     bunit.push_back(make_uint2((uint32_t)(nodes_b + (unit[u].x - n0)), (uint32_t)sl));
+                    bweight.push_back(unit_nodes[u]);
                     if (!open) {
                         rn0 = n0;
                         rt0 = t0;
@@ -491,6 +493,20 @@ bool cut_batches(domino_ctx* h) {
                 }
                 if (!ok) break;
                 close_range();
+                {   // the costliest units first: the warps' last claims are short ones
+                    std::vector<size_t> ord(bunit.size() - unit0);
+                    for (size_t k = 0; k < ord.size(); k++) ord[k] = unit0 + k;
+                    std::stable_sort(ord.begin(), ord.end(),
+                                     [&](size_t x, size_t y) { return bweight[x] > bweight[y]; });
+                    std::vector<uint2> su;
+                    std::vector<int64_t> sw;
+                    for (size_t k : ord) {
+                        su.push_back(bunit[k]);
+                        sw.push_back(bweight[k]);
+                    }
+                    std::copy(su.begin(), su.end(), bunit.begin() + (ptrdiff_t)unit0);
+                    std::copy(sw.begin(), sw.end(), bweight.begin() + (ptrdiff_t)unit0);
+                }
                 batch.push_back(make_uint4((uint32_t)unit0, (uint32_t)bunit.size(), (uint32_t)range0,
                                            (uint32_t)range.size()));
                 batch.push_back(make_uint4((uint32_t)slot0, (uint32_t)slot.size(), (uint32_t)nodes_b,
