@@ -100,18 +100,21 @@ constexpr int kTrieMaxSlots = 48;             // slots per batch
 constexpr int32_t kTrieMaxNodes = (1 << 24) - 1;
 
 struct TrieView {
-    const uint4* node;        // [n_nodes][2]
+    const uint4* node;        // the walk's records, two each: {end record, first node, nodes, first token},
+                              //   {tokens ending at the last node, classes below it (64 bits), 0}
+    const uint8_t* ncls;      // [n_nodes]: each node's class (the records' classes, in order)
     const int32_t* dtok;      // original ids in preorder
     const uint4* upper;       // [n_upper]: {node, path offset, path length, 0}
     const uint8_t* upath;     // classes of the upper nodes' paths from the root
     const uint4* batch;       // [n_batches][2]: {first unit, end unit, first range, end range},
                               //                 {first slot, end slot, staged nodes, staged tokens}
-    const uint4* range;       // {first node, end node, first token, end token}: staged one after the other
+    const uint4* range;       // two each: {first record, end record, first token, end token},
+                              //   {first node, end node, 0, 0}; staged one after the other
     const uint4* slot;        // {upper index, first token ending at its node, tokens it sets (0: none), 0}
     const uint2* unit;        // {root's staged index, slot index within the batch}
     const int32_t* cta_batch; // [grid + 1]: CTA c takes batches [cta_batch[c], cta_batch[c + 1])
     int32_t n_nodes, n_upper, grid;
-    int32_t max_nodes, max_toks, max_units, max_slots, max_path;   // the largest batch
+    int32_t max_nodes, max_cls, max_toks, max_units, max_slots, max_path;   // the largest batch (records, nodes, ...)
 };
 
 struct LaunchEnv {

@@ -60,8 +60,11 @@ struct domino_ctx {
     DevBuf d_err, d_partials, d_counters, d_lse_tmp, d_fpart;
     bool arena_ready = false;
     // prefix tree of the class strings and its per-CTA batches (see TrieView)
-    DevBuf d_tnode, d_tdtok, d_tupper, d_tupath, d_tbatch, d_trange, d_tslot, d_tunit, d_tcta;
+    DevBuf d_tnode, d_tncls, d_tdtok, d_tupper, d_tupath, d_tbatch, d_trange, d_tslot, d_tunit, d_tcta;
     std::vector<uint4> t_node;       // host copies (domino_get_prefix_tree)
+    std::vector<uint4> t_cnode;      // the walk's records (chains of nodes), two per record
+    std::vector<uint32_t> t_hc;      // [n_nodes + 1]: records before each node
+    std::vector<uint8_t> t_ncls;     // each node's class
     std::vector<int32_t> t_dtok;
     std::vector<uint4> t_upper;      // {node, path offset, path length, 0}
     std::vector<uint8_t> t_upath;
@@ -73,7 +76,7 @@ struct domino_ctx {
     std::vector<uint2> t_bunit;      // {root node, slot within the batch}
     std::vector<int32_t> t_cta;      // [grid + 1] first batch of each CTA
     int32_t t_nodes = 0, t_grid = 0;
-    int32_t t_max_nodes = 0, t_max_toks = 0, t_max_units = 0, t_max_slots = 0, t_max_path = 0;
+    int32_t t_max_nodes = 0, t_max_cls = 0, t_max_toks = 0, t_max_units = 0, t_max_slots = 0, t_max_path = 0;
     int t_mode = kDenseGlobal;       // where the tile kernel reads transitions
     bool trie_built = false;         // host arrays valid
     bool trie_ready = false;         // device copies valid
@@ -186,6 +189,9 @@ void clear_host_graphs(domino_ctx* h) {
 void build_trie_host(domino_ctx* h) {
     h->trie_built = h->trie_ready = false;
     h->t_node.clear();
+    h->t_cnode.clear();
+    h->t_hc.clear();
+    h->t_ncls.clear();
     h->t_dtok.clear();
     h->t_upper.clear();
     h->t_upath.clear();
@@ -289,6 +295,41 @@ void build_trie_host(domino_ctx* h) {
         node[2 * (size_t)n] = make_uint4(skip[n] | ((uint32_t)ncls[n] << 24), tok_lo[n], n_end[n], tok_hi[n]);
         node[2 * (size_t)n + 1] = make_uint4((uint32_t)sub[n], (uint32_t)(sub[n] >> 32), 0u, 0u);
     }
+    // Chains: inside a unit, a node with one child and no token ending at it
+    // is walked together with that child.  The walk's records are the chains'
+    // first nodes (heads); a record covers `len` nodes (at most 255), its
+    // classes are those nodes' classes, and its tokens and classes-below are
+    // those of its last node.  Upper nodes stay records of their own.
+    std::vector<uint32_t> nchild(N, 0);
+    for (uint32_t n = 1; n < N; n++) nchild[parent[n]]++;
+    std::vector<uint8_t> head(N, 1);
+    std::vector<uint32_t> clen(N, 1);   // a head's chain length
+    for (const uint2& u : unit) {
+        uint32_t cur = u.x;
+        for (uint32_t n = u.x + 1; n < skip[u.x]; n++) {
+            const uint32_t pp = parent[n];
+            if (nchild[pp] == 1 && n_end[pp] == 0 && pp + 1 == n && clen[cur] < 255 &&
+                cur + clen[cur] == n) {
+                head[n] = 0;
+                clen[cur]++;
+            } else {
+                cur = n;
+            }
+        }
+    }
+    std::vector<uint32_t> hc((size_t)N + 1, 0);   // heads before each node
+    for (uint32_t n = 0; n < N; n++) hc[n + 1] = hc[n] + head[n];
+    std::vector<uint4> cnode((size_t)hc[N] * 2);
+    for (uint32_t n = 0; n < N; n++) {
+        if (!head[n]) continue;
+        const uint32_t b = n + clen[n] - 1;   // the chain's last node
+        const size_t c = hc[n];
+        cnode[2 * c] = make_uint4(hc[skip[n]], n, clen[n], tok_lo[n]);
+        cnode[2 * c + 1] = make_uint4(n_end[b], (uint32_t)sub[b], (uint32_t)(sub[b] >> 32), 0u);
+    }
+    h->t_cnode.swap(cnode);
+    h->t_hc.swap(hc);
+    h->t_ncls.swap(ncls);
     h->t_node.swap(node);
     h->t_dtok.swap(dtok);
     h->t_upper.swap(upper);
@@ -376,7 +417,8 @@ bool cut_batches(domino_ctx* h) {
     }
     int64_t total = 0;
     for (size_t u = 0; u < unit.size(); u++) total += unit_nodes[u];
-    const int per_node = 8 + (self ? 8 : 0);
+    const int per_rec = 16 + (self ? 8 : 0);   // a staged walk record (and its classes below)
+    const std::vector<uint32_t>& hc = h->t_hc;
     if (unit.empty()) return false;
     // the upper nodes whose tokens a unit's batch sets: those with tokens
     // between the previous unit's root and its own (trailing ones: the last)
@@ -410,7 +452,7 @@ bool cut_batches(domino_ctx* h) {
         std::vector<uint2> bunit;
         std::vector<int64_t> bweight;   // the estimated cost of each bunit entry
         std::vector<int32_t> cta((size_t)grid + 1, 0);
-        int32_t mx_nodes = 0, mx_toks = 0, mx_units = 0, mx_slots = 0, mx_path = 0;
+        int32_t mx_nodes = 0, mx_cls = 0, mx_toks = 0, mx_units = 0, mx_slots = 0, mx_path = 0;
         bool ok = true;
         for (int c = 0; c < grid && ok; c++) {
             cta[(size_t)c] = (int32_t)(batch.size() / 2);
@@ -438,13 +480,15 @@ bool cut_batches(domino_ctx* h) {
                     mx_path = std::max<int32_t>(mx_path, (int32_t)upper[ui].z);
                     return (int)slots.size() - 1;
                 };
-                int64_t nodes_b = 0, toks_b = 0;   // staged by the closed ranges
+                int64_t recs_b = 0, cls_b = 0, toks_b = 0;   // staged by the closed ranges
                 bool open = false;
-                uint32_t rn0 = 0, rn1 = 0, rt0 = 0, rt1 = 0;   // the open range
+                uint32_t rn0 = 0, rn1 = 0, rt0 = 0, rt1 = 0;   // the open range (nodes, tokens)
                 auto close_range = [&]() {
                     if (!open) return;
-                    range.push_back(make_uint4(rn0, rn1, rt0, rt1));
-                    nodes_b += rn1 - rn0;
+                    range.push_back(make_uint4(hc[rn0], hc[rn1], rt0, rt1));
+                    range.push_back(make_uint4(rn0, rn1, 0u, 0u));
+                    recs_b += hc[rn1] - hc[rn0];
+                    cls_b += rn1 - rn0;
                     toks_b += rt1 - rt0;
                     open = false;
                 };
@@ -466,11 +510,12 @@ bool cut_batches(domino_ctx* h) {
                     fit = sl >= 0;
                     const uint32_t n0 = open ? rn0 : unit[u].x, t0 = open ? rt0 : node[2 * (size_t)unit[u].x].y;
                     const uint32_t n1 = skip_of(unit[u].x), t1 = node[2 * (size_t)unit[u].x].w;
-                    const int64_t nodes_all = nodes_b + (n1 - n0), toks_all = toks_b + (t1 - t0);
+                    const int64_t recs_all = recs_b + (hc[n1] - hc[n0]), cls_all = cls_b + (n1 - n0);
+                    const int64_t toks_all = toks_b + (t1 - t0);
                     if (fit)
-                        fit = nodes_all <= 0xFFFF && toks_all <= 0xFFFF &&
-                              nodes_all * per_node + toks_all * 4 + (int64_t)(bunit.size() - unit0 + 1) * 4 +
-                                      (int64_t)slots.size() * (16 + 64) <=
+                        fit = recs_all <= 0xFFFF && toks_all <= 0xFFFF &&
+                              recs_all * per_rec + ((cls_all + 15) & ~15) + toks_all * 4 +
+                                      (int64_t)(bunit.size() - unit0 + 1) * 4 + (int64_t)slots.size() * (16 + 64) <=
                                   budget;
                     if (!fit) {   // undo this unit's slots; the batch ends before it
                         slot.resize(keep_slots);
@@ -479,7 +524,7 @@ bool cut_batches(domino_ctx* h) {
                         if (added == 0) ok = false;   // a unit alone does not fit
                         break;
                     }
-                    bunit.push_back(make_uint2((uint32_t)(nodes_b + (unit[u].x - n0)), (uint32_t)sl));
+                    bunit.push_back(make_uint2((uint32_t)(recs_b + (hc[unit[u].x] - hc[n0])), (uint32_t)sl));
                     bweight.push_back(unit_nodes[u]);
                     if (!open) {
                         rn0 = n0;
@@ -507,11 +552,12 @@ bool cut_batches(domino_ctx* h) {
                     std::copy(su.begin(), su.end(), bunit.begin() + (ptrdiff_t)unit0);
                     std::copy(sw.begin(), sw.end(), bweight.begin() + (ptrdiff_t)unit0);
                 }
-                batch.push_back(make_uint4((uint32_t)unit0, (uint32_t)bunit.size(), (uint32_t)range0,
-                                           (uint32_t)range.size()));
-                batch.push_back(make_uint4((uint32_t)slot0, (uint32_t)slot.size(), (uint32_t)nodes_b,
+                batch.push_back(make_uint4((uint32_t)unit0, (uint32_t)bunit.size(), (uint32_t)(range0 / 2),
+                                           (uint32_t)(range.size() / 2)));
+                batch.push_back(make_uint4((uint32_t)slot0, (uint32_t)slot.size(), (uint32_t)recs_b,
                                            (uint32_t)toks_b));
-                mx_nodes = std::max<int32_t>(mx_nodes, (int32_t)nodes_b);
+                mx_nodes = std::max<int32_t>(mx_nodes, (int32_t)recs_b);
+                mx_cls = std::max<int32_t>(mx_cls, (int32_t)cls_b);
                 mx_toks = std::max<int32_t>(mx_toks, (int32_t)toks_b);
                 mx_units = std::max<int32_t>(mx_units, (int32_t)(bunit.size() - unit0));
                 mx_slots = std::max<int32_t>(mx_slots, (int32_t)(slot.size() - slot0));
@@ -521,6 +567,7 @@ bool cut_batches(domino_ctx* h) {
         cta[(size_t)grid] = (int32_t)(batch.size() / 2);
         TrieView tv{};
         tv.max_nodes = mx_nodes;
+        tv.max_cls = mx_cls;
         tv.max_toks = mx_toks;
         tv.max_units = mx_units;
         tv.max_slots = mx_slots;
@@ -533,6 +580,7 @@ bool cut_batches(domino_ctx* h) {
         h->t_cta.swap(cta);
         h->t_grid = grid;
         h->t_max_nodes = mx_nodes;
+        h->t_max_cls = mx_cls;
         h->t_max_toks = mx_toks;
         h->t_max_units = mx_units;
         h->t_max_slots = mx_slots;
@@ -549,7 +597,8 @@ int build_trie(domino_ctx* h) {
     if (!h->trie_built || !cut_batches(h)) return DOMINO_OK;
     int rc;
     auto up = [&](DevBuf& b, const void* p, size_t n) { return dev_upload(b, p, std::max<size_t>(16, n)); };
-    if ((rc = up(h->d_tnode, h->t_node.data(), h->t_node.size() * sizeof(uint4)))) return rc;
+    if ((rc = up(h->d_tnode, h->t_cnode.data(), h->t_cnode.size() * sizeof(uint4)))) return rc;
+    if ((rc = up(h->d_tncls, h->t_ncls.data(), h->t_ncls.size()))) return rc;
     if ((rc = up(h->d_tdtok, h->t_dtok.data(), h->t_dtok.size() * 4))) return rc;
     if ((rc = up(h->d_tupper, h->t_upper.data(), h->t_upper.size() * sizeof(uint4)))) return rc;
     if ((rc = up(h->d_tupath, h->t_upath.data(), h->t_upath.size()))) return rc;
@@ -698,6 +747,7 @@ int choose_mode(const domino_ctx* h, const StepView& v, bool next) {
 TrieView make_trie_view(const domino_ctx* h) {
     TrieView tv{};
     tv.node = (const uint4*)h->d_tnode.p;
+    tv.ncls = (const uint8_t*)h->d_tncls.p;
     tv.dtok = (const int32_t*)h->d_tdtok.p;
     tv.upper = (const uint4*)h->d_tupper.p;
     tv.upath = (const uint8_t*)h->d_tupath.p;
@@ -710,6 +760,7 @@ TrieView make_trie_view(const domino_ctx* h) {
     tv.n_upper = (int32_t)h->t_upper.size();
     tv.grid = h->t_grid;
     tv.max_nodes = h->t_max_nodes;
+    tv.max_cls = h->t_max_cls;
     tv.max_toks = h->t_max_toks;
     tv.max_units = h->t_max_units;
     tv.max_slots = h->t_max_slots;
@@ -821,7 +872,7 @@ int domino_destroy(domino_t h) {
                          &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_self, &h->d_tok_cls, &h->d_err, &h->d_fpart, &h->d_partials,
                          &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_mask, &h->s_io,
                          &h->o_prop, &h->o_rows, &h->o_count, &h->d_tnode, &h->d_tdtok, &h->d_tupper, &h->d_tupath, &h->d_tbatch, &h->d_tslot,
-                         &h->d_tunit, &h->d_tcta, &h->d_trange};
+                         &h->d_tunit, &h->d_tcta, &h->d_trange, &h->d_tncls};
         for (auto* b : all) dev_free(*b);
         for (cudaEvent_t& e : h->ev_chunk)
             if (e) cudaEventDestroy(e);

@@ -64,7 +64,8 @@ enum TileCtl : int {
 
 // Shared-memory layout of the tile kernel (byte offsets).
 struct TileLayout {
-    int accept, self, table, nodes, sub, toks, units, slots, paths, rowcfg, cfg, lrows, lcount, stk, ustk, ctl, total;
+    int accept, self, table, nodes, sub, cls, toks, units, slots, paths, rowcfg, cfg, lrows, lcount, stk, ustk, ctl,
+        total;
 };
 
 __host__ __device__ inline TileLayout tile_layout(int Q, bool self, bool stack, int table_bytes, const TrieView& tv) {
@@ -73,8 +74,9 @@ __host__ __device__ inline TileLayout tile_layout(int Q, bool self, bool stack, 
     L.accept = o;  o += align16(((Q + 31) / 32) * 4);
     L.self = o;    o += self ? align16(Q * 8) : 0;
     L.table = o;   o += align16(table_bytes);
-    L.nodes = o;   o += align16(tv.max_nodes * 8);
+    L.nodes = o;   o += align16(tv.max_nodes * 16);
     L.sub = o;     o += self ? align16(tv.max_nodes * 8) : 0;
+    L.cls = o;     o += align16(tv.max_cls);
     L.toks = o;    o += align16(tv.max_toks * 4);
     L.units = o;   o += align16(tv.max_units * 4);
     L.slots = o;   o += align16(tv.max_slots * 16);
@@ -186,7 +188,8 @@ struct TileCtx {
     const uint16_t* ret;
     uint32_t maxd;
     const unsigned long long* s_self;   // nullptr: no self-loop skip
-    const uint2* snode;                 // {skip - nb | cls << 16, tok - tb | n_end << 16}
+    const uint4* snode;                 // {end | nodes << 16, first token | tokens << 16, first class, 0}
+    const uint8_t* scls;                // the records' classes
     const unsigned long long* ssub;
     const int32_t* stok;
     int nn, nt;                         // staged nodes and tokens
@@ -231,10 +234,15 @@ struct TileCtx {
         int x = x0, end = x0 + 1, sp = 0;
         for (;;) {
             while (x < end) {
-                const uint2 rec = snode[x];   // checked when staged
-                const int xs = (int)(rec.x & 0xFFFFu);
+                const uint4 rec = snode[x];   // checked when staged
+                const int xs = (int)(rec.x & 0xFFFFu), nc = (int)(rec.x >> 16);
                 uint32_t b2 = bits, d2 = depth;
-                const uint32_t s2 = step_once<STACK>(tab, ret, maxd, s, (rec.x >> 16) & 0xFFu, b2, d2);
+                // the record's chain of classes (no token ends before its last node)
+                uint32_t s2 = step_once<STACK>(tab, ret, maxd, s, scls[rec.z], b2, d2);
+                for (int k = 1; k < nc; ++k) {
+                    if (!__any_sync(0xffffffffu, s2 != 0)) break;
+                    if (s2) s2 = step_once<STACK>(tab, ret, maxd, s2, scls[rec.z + k], b2, d2);
+                }
                 const bool on = s2 != 0;
                 if (__ballot_sync(0xffffffffu, on)) {
                     const int tl = (int)(rec.y & 0xFFFFu), ne = (int)(rec.y >> 16);
@@ -246,7 +254,7 @@ struct TileCtx {
                             // subtree is allowed with it
                             const bool keep = on && (ssub[x] & ~s_self[s2]) == 0ull;
                             if (__ballot_sync(0xffffffffu, keep)) {
-                                const int th = xs < nn ? (int)(snode[xs].y & 0xFFFFu) : nt;
+                                const int th = xs < nn ? (int)(snode[xs].y & 0xFFFFu) : nt;   // the subtree's tokens end
                                 emit(lane, keep, row, tl + ne, th, s2);
                             }
                             desc = desc && !keep;
@@ -299,7 +307,9 @@ __global__ void __maxnreg__(64)
     const TileLayout L = tile_layout(v.Q, use_self, STACK, MODE == kDenseGlobal ? 0 : a.img_bytes, tv);
     uint32_t* s_accept = reinterpret_cast<uint32_t*>(smem + L.accept);
     unsigned long long* s_self = reinterpret_cast<unsigned long long*>(smem + L.self);
-    uint2* snode = reinterpret_cast<uint2*>(smem + L.nodes);
+    // a staged walk record: {end record | nodes << 16, first token | tokens << 16, first class, 0}
+    uint4* snode = reinterpret_cast<uint4*>(smem + L.nodes);
+    uint8_t* scls = reinterpret_cast<uint8_t*>(smem + L.cls);
     unsigned long long* ssub = reinterpret_cast<unsigned long long*>(smem + L.sub);
     int32_t* stok = reinterpret_cast<int32_t*>(smem + L.toks);
     uint32_t* sunit = reinterpret_cast<uint32_t*>(smem + L.units);   // root - nb | slot << 16
@@ -348,33 +358,38 @@ __global__ void __maxnreg__(64)
         __syncthreads();   // the previous batch is done with shared memory
         if (tid == 0) ctl[kCtlBad] = 0;
         __syncthreads();
-        // the batch's node and token ranges, staged one after the other; a
-        // node's subtree end and first token become staged indices
-        int sb = 0, tb = 0;
+        // the batch's record, class and token ranges, staged one after the
+        // other; a record's subtree end, first class and first token become
+        // staged indices
+        int sb = 0, tb = 0, cb = 0;
         for (uint32_t ri = bA.z; ri < bA.w; ++ri) {
-            const uint4 R = __ldg(tv.range + ri);   // {first node, end node, first token, end token}
-            const int rn = (int)(R.y - R.x), rt = (int)(R.w - R.z);
-            if (rn < 0 || rt < 0 || sb + rn > nn || tb + rt > nt) {
+            const uint4 R = __ldg(tv.range + 2 * ri);       // {first record, end record, first token, end token}
+            const uint4 Rn = __ldg(tv.range + 2 * ri + 1);  // {first node, end node, 0, 0}
+            const int rn = (int)(R.y - R.x), rt = (int)(R.w - R.z), rc = (int)(Rn.y - Rn.x);
+            if (rn < 0 || rt < 0 || rc < 0 || sb + rn > nn || tb + rt > nt || cb + rc > tv.max_cls) {
                 if (tid == 0) ctl[kCtlBad] = 1;
                 break;
             }
             for (int n = tid; n < rn; n += kTileThreads) {
                 const uint4 r0 = __ldg(tv.node + 2 * ((size_t)R.x + n));
-                // preorder (a subtree ends after its root) and the node's tokens
-                // inside the range's: the walk relies on both.  The upper nodes
-                // between a range's units are staged too (never walked); their
-                // subtrees end past the range, so skips are clamped to its end.
-                const uint32_t xs = min((r0.x & 0xFFFFFFu) - R.x, (uint32_t)rn), tl = r0.y - R.z;
-                if (xs <= (uint32_t)n || tl > (uint32_t)rt || r0.z > (uint32_t)rt - tl) ctl[kCtlBad] = 1;
-                snode[sb + n] = make_uint2((xs + sb) | ((r0.x >> 24) << 16), (tl + tb) | (r0.z << 16));
-                if (use_self) {
-                    const uint4 r1 = __ldg(tv.node + 2 * ((size_t)R.x + n) + 1);
-                    ssub[sb + n] = ((unsigned long long)r1.y << 32) | r1.x;
-                }
+                const uint4 r1 = __ldg(tv.node + 2 * ((size_t)R.x + n) + 1);
+                // preorder (a subtree ends after its record), the record's nodes
+                // and tokens inside the range's: the walk relies on all three.
+                // The upper nodes between a range's units are staged too (never
+                // walked); their subtrees end past the range, so skips are
+                // clamped to its end.
+                const uint32_t xs = min(r0.x - R.x, (uint32_t)rn), tl = r0.w - R.z, fc = r0.y - Rn.x;
+                if (xs <= (uint32_t)n || tl > (uint32_t)rt || r1.x > (uint32_t)rt - tl || r0.z == 0u ||
+                    r0.z > 255u || fc >= (uint32_t)rc || r0.z > (uint32_t)rc - fc)
+                    ctl[kCtlBad] = 1;
+                snode[sb + n] = make_uint4((xs + sb) | (min(r0.z, 255u) << 16), (tl + tb) | (r1.x << 16), fc + cb, 0u);
+                if (use_self) ssub[sb + n] = ((unsigned long long)r1.z << 32) | r1.y;
             }
+            for (int j = tid; j < rc; j += kTileThreads) scls[cb + j] = __ldg(tv.ncls + Rn.x + j);
             for (int j = tid; j < rt; j += kTileThreads) stok[tb + j] = __ldg(tv.dtok + R.z + j);
             sb += rn;
             tb += rt;
+            cb += rc;
         }
         if ((sb != nn || tb != nt) && tid == 0) ctl[kCtlBad] = 1;
         for (int k = tid; k < nk; k += kTileThreads) {
@@ -403,7 +418,8 @@ __global__ void __maxnreg__(64)
             if (tid == 0) atomicOr(v.err, DOMINO_DEVERR_INTERNAL);
             continue;
         }
-        const TileCtx<STACK, MODE, NEXT> cx{v, a, tab, ret, maxd, use_self ? s_self : nullptr, snode, ssub, stok, nn, nt};
+        const TileCtx<STACK, MODE, NEXT> cx{v, a, tab, ret, maxd, use_self ? s_self : nullptr, snode, scls, ssub, stok,
+                                            nn, nt};
         const int nrows = list.rows(a.batch);
         const int rb = max(1, min(kTrieRowBlock, kTrieCfg / max(ns, 1)));
         for (int r0 = 0; r0 < nrows; r0 += rb) {
