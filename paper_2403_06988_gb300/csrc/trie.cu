@@ -14,27 +14,26 @@
 //                     states) and sets EOS when the state accepts with an
 //                     empty stack.
 //  tree_tile_kernel   persistent CTAs, one per SM.  For each of its batches a
-//                     CTA stages the batch's units (compact node records, the
-//                     units' tokens) in shared memory next to the transition
-//                     table; then, a block of rows at a time:
+//                     CTA stages the batch's walk records (chains of nodes
+//                     with one child and no token, walked as one record),
+//                     their classes and the units' tokens in shared memory
+//                     next to the transition table; then, a block of rows at
+//                     a time:
 //                       1. each row's configuration at every slot (the upper
 //                          nodes the units hang off), by walking the slot's
 //                          path from the row's configuration;
-//                       2. per slot, the list of rows live there; emitting
-//                          slots set the bits of the tokens ending at them;
-//                       3. warps claim units: a warp walks its unit for up to
-//                          32 of the slot's live rows at once, one row per
-//                          lane, in lockstep over the unit's nodes in
-//                          preorder; a subtree is entered while it is live for
-//                          some lane and skipped when it is dead for all; the
-//                          siblings still to visit are kept on a per-warp
-//                          stack (one level per branching node, at most
-//                          kTrieBranch).  A node's tokens set their bits with
-//                          global reductions (and store their next state): a
-//                          few at a time for all the lanes a node is live in,
-//                          or, for long token ranges -- and whole subtrees
-//                          whose classes all loop on a lane's state (the
-//                          self-loop skip) -- spread over the warp's lanes.
+//                       2. per slot, the list of rows live there;
+//                       3. the emitting slots' (row, token) items, spread over
+//                          the CTA; then every (unit, row live at the unit's
+//                          slot) pair, one thread each: the thread walks the
+//                          unit depth first from the row's configuration,
+//                          skipping a record's subtree when the record dies,
+//                          with the siblings still to visit on its own stack
+//                          (one entry per branching record, at most
+//                          kTrieBranch).  A record's tokens set their bits with
+//                          global reductions (and store their next state);
+//                          so do whole subtrees whose classes all loop on the
+//                          row's state (the self-loop skip).
 #include <cuda_runtime.h>
 
 #include <climits>
@@ -48,12 +47,10 @@ namespace domino {
 namespace {
 
 constexpr int kTileThreads = 1024;
-constexpr int kTileWarps = kTileThreads / 32;
 constexpr int kClearThreads = 256;          // 8 warps per CTA
 constexpr int kClearSplit = 4;              // warps per row
 constexpr int kTrieCfg = 4096;              // (slot, row) configurations per row block
 constexpr int kTrieRowBlock = 512;          // most rows per block
-constexpr int kTrieEmitWarp = 32;           // longer token ranges are spread over the warp's lanes
 constexpr int kTrieMaxDevices = 64;
 
 enum TileCtl : int {
@@ -64,7 +61,7 @@ enum TileCtl : int {
 
 // Shared-memory layout of the tile kernel (byte offsets).
 struct TileLayout {
-    int accept, self, table, nodes, sub, cls, toks, units, slots, paths, rowcfg, cfg, lrows, lcount, stk, ustk, ctl,
+    int accept, self, table, nodes, sub, cls, toks, units, upre, slots, paths, rowcfg, cfg, lrows, lcount, epre, ctl,
         total;
 };
 
@@ -79,14 +76,14 @@ __host__ __device__ inline TileLayout tile_layout(int Q, bool self, bool stack, 
     L.cls = o;     o += align16(tv.max_cls);
     L.toks = o;    o += align16(tv.max_toks * 4);
     L.units = o;   o += align16(tv.max_units * 4);
+    L.upre = o;    o += align16((tv.max_units + 1) * 4);
     L.slots = o;   o += align16(tv.max_slots * 16);
     L.paths = o;   o += align16(tv.max_slots * tv.max_path);
     L.rowcfg = o;  o += kTrieRowBlock * 16;
     L.cfg = o;     o += kTrieCfg * (stack ? 8 : 4);
     L.lrows = o;   o += kTrieCfg * 2;
     L.lcount = o;  o += align16(kTrieMaxSlots * 4);
-    L.stk = o;     o += kTileWarps * kTrieBranch * 32 * (stack ? 8 : 4);
-    L.ustk = o;    o += kTileWarps * kTrieBranch * 8;
+    L.epre = o;    o += align16((kTrieMaxSlots + 1) * 4);
     L.ctl = o;     o += kCtlWords * 4;
     L.total = align16(o);
     return L;
@@ -206,72 +203,45 @@ struct TileCtx {
             if (a.next) a.next[(size_t)row * v.V + t] = (int32_t)s;
         }
     }
-    // Staged tokens [lo, hi) (the same for all lanes) allowed with state s in
-    // the lanes where `on`, each in its lane's row.  Few tokens: a loop over
-    // them, every lane setting its own row's bit.  Many: for each lane that is
-    // on, the warp's lanes split the range.  Warp-uniform control flow.
-    __device__ __forceinline__ void emit(int lane, bool on, int row, int lo, int hi, uint32_t s) const {
-        if (hi - lo <= kTrieEmitWarp) {
-            for (int j = lo; j < hi; ++j) {
-                const int t = stok[j];
-                if (on) emit_one(row, t, s);
-            }
-            return;
-        }
-        for (unsigned m = __ballot_sync(0xffffffffu, on); m; m &= m - 1) {
-            const int src = __ffs(m) - 1;
-            const int r = __shfl_sync(0xffffffffu, row, src);
-            const uint32_t ss = __shfl_sync(0xffffffffu, s, src);
-            for (int j = lo + lane; j < hi; j += 32) emit_one(r, stok[j], ss);
-        }
-    }
-
-    // One warp walks unit root x0 (staged index) for its lanes' rows, in
-    // lockstep: (s, bits, depth) is the lane's configuration at the unit's
-    // parent (s = 0: no row).  stk / ustk: the warp's stack.
-    __device__ __forceinline__ void walk(int lane, int row, int x0, uint32_t s, uint32_t bits, uint32_t depth,
-                                         uint32_t* stk, uint32_t* stkb, uint2* ustk) const {
+    // One lane walks unit root x0 for its own row from the configuration
+    // (s, bits, depth) at the unit's parent: depth first over the records in
+    // preorder, the siblings still to visit on the lane's own stack (one entry
+    // per branching record, at most kTrieBranch).
+    __device__ __forceinline__ void walk_lane(int row, int x0, uint32_t s, uint32_t bits, uint32_t depth) const {
         int x = x0, end = x0 + 1, sp = 0;
+        uint32_t kx[kTrieBranch], ks[kTrieBranch], kb[STACK ? kTrieBranch : 1];
         for (;;) {
             while (x < end) {
                 const uint4 rec = snode[x];   // checked when staged
                 const int xs = (int)(rec.x & 0xFFFFu), nc = (int)(rec.x >> 16);
-                uint32_t b2 = bits, d2 = depth;
-                // the record's chain of classes (no token ends before its last node)
-                uint32_t s2 = step_once<STACK>(tab, ret, maxd, s, scls[rec.z], b2, d2);
-                for (int k = 1; k < nc; ++k) {
-                    if (!__any_sync(0xffffffffu, s2 != 0)) break;
-                    if (s2) s2 = step_once<STACK>(tab, ret, maxd, s2, scls[rec.z + k], b2, d2);
-                }
-                const bool on = s2 != 0;
-                if (__ballot_sync(0xffffffffu, on)) {
+                uint32_t b2 = bits, d2 = depth, s2 = s;
+                for (int k = 0; k < nc && s2 != 0; ++k)
+                    s2 = step_once<STACK>(tab, ret, maxd, s2, scls[rec.z + k], b2, d2);
+                if (s2 != 0) {
                     const int tl = (int)(rec.y & 0xFFFFu), ne = (int)(rec.y >> 16);
-                    if (ne) emit(lane, on, row, tl, tl + ne, s2);
+                    for (int j = tl; j < tl + ne; ++j) emit_one(row, stok[j], s2);
                     if (xs > x + 1) {   // x has children
-                        bool desc = on;
-                        if (s_self) {
+                        bool desc = true;
+                        if (s_self && (ssub[x] & ~s_self[s2]) == 0ull) {
                             // every class below keeps the state: the whole
                             // subtree is allowed with it
-                            const bool keep = on && (ssub[x] & ~s_self[s2]) == 0ull;
-                            if (__ballot_sync(0xffffffffu, keep)) {
-                                const int th = xs < nn ? (int)(snode[xs].y & 0xFFFFu) : nt;   // the subtree's tokens end
-                                emit(lane, keep, row, tl + ne, th, s2);
-                            }
-                            desc = desc && !keep;
+                            const int th = xs < nn ? (int)(snode[xs].y & 0xFFFFu) : nt;   // the subtree's tokens end
+                            for (int j = tl + ne; j < th; ++j) emit_one(row, stok[j], s2);
+                            desc = false;
                         }
-                        if (__ballot_sync(0xffffffffu, desc)) {
+                        if (desc) {
                             if (xs < end) {
                                 if (sp == kTrieBranch) {   // the tree bounds the stack by kTrieBranch
-                                    if (lane == 0) fail();
+                                    fail();
                                     return;
                                 }
-                                stk[sp * 32 + lane] = pack_sd(s, depth);
-                                if constexpr (STACK) stkb[sp * 32 + lane] = bits;
-                                if (lane == 0) ustk[sp] = make_uint2((uint32_t)xs, (uint32_t)end);
+                                kx[sp] = (uint32_t)xs | ((uint32_t)end << 16);
+                                ks[sp] = pack_sd(s, depth);
+                                if constexpr (STACK) kb[sp] = bits;
                                 ++sp;
                             }
                             end = xs;
-                            s = desc ? s2 : 0u;
+                            s = s2;
                             bits = b2;
                             depth = d2;
                             x = x + 1;
@@ -283,14 +253,11 @@ struct TileCtx {
             }
             if (sp == 0) return;
             --sp;
-            __syncwarp();
-            const uint2 u = ustk[sp];
-            x = (int)u.x;
-            end = (int)u.y;
-            const uint32_t sd = stk[sp * 32 + lane];
-            s = sd & 0xFFFFu;
-            depth = sd >> 16;
-            if constexpr (STACK) bits = stkb[sp * 32 + lane];
+            x = (int)(kx[sp] & 0xFFFFu);
+            end = (int)(kx[sp] >> 16);
+            s = ks[sp] & 0xFFFFu;
+            depth = ks[sp] >> 16;
+            if constexpr (STACK) bits = kb[sp];
         }
     }
 };
@@ -313,14 +280,14 @@ __global__ void __maxnreg__(64)
     unsigned long long* ssub = reinterpret_cast<unsigned long long*>(smem + L.sub);
     int32_t* stok = reinterpret_cast<int32_t*>(smem + L.toks);
     uint32_t* sunit = reinterpret_cast<uint32_t*>(smem + L.units);   // root - nb | slot << 16
+    int* upre = reinterpret_cast<int*>(smem + L.upre);               // the units' first (row, unit) pairs
     uint4* sslot = reinterpret_cast<uint4*>(smem + L.slots);         // {path length, 0, first token, tokens set}
     uint8_t* spath = reinterpret_cast<uint8_t*>(smem + L.paths);
     uint4* rowcfg = reinterpret_cast<uint4*>(smem + L.rowcfg);
     uint32_t* cfg = reinterpret_cast<uint32_t*>(smem + L.cfg);       // [slot][row] state | depth << 16 (+ bits)
     uint16_t* lrows = reinterpret_cast<uint16_t*>(smem + L.lrows);   // [slot][k] live rows of the block
     int* lcount = reinterpret_cast<int*>(smem + L.lcount);
-    uint32_t* stk = reinterpret_cast<uint32_t*>(smem + L.stk);
-    uint2* ustk = reinterpret_cast<uint2*>(smem + L.ustk);
+    int* epre = reinterpret_cast<int*>(smem + L.epre);   // the emitting slots' first (row, token) items
     int* ctl = reinterpret_cast<int*>(smem + L.ctl);
     const int b0 = __ldg(tv.cta_batch + blockIdx.x), b1 = __ldg(tv.cta_batch + blockIdx.x + 1);
     if (b0 >= b1) {   // no units for this CTA
@@ -346,9 +313,6 @@ __global__ void __maxnreg__(64)
         ret = reinterpret_cast<const uint16_t*>(t + a.img_ret_off);
     }
     const uint32_t maxd = (uint32_t)v.max_depth;
-    uint32_t* wstk = stk + warp * kTrieBranch * 32 * (STACK ? 2 : 1);
-    uint32_t* wstkb = wstk + kTrieBranch * 32;
-    uint2* wustk = ustk + warp * kTrieBranch;
     bool waited = false;
     for (int bj = b0; bj < b1; ++bj) {
         const uint4 bA = __ldg(tv.batch + 2 * bj);       // units [x, y), ranges [z, w)
@@ -475,39 +439,75 @@ __global__ void __maxnreg__(64)
                 }
             }
             __syncthreads();
-            // emitting slots: the tokens that end at their nodes, for every row
-            // live there, spread over the CTA (read from the preorder list)
-            for (int k = 0; k < ns; ++k) {
-                const uint4 sl = sslot[k];
-                const int nl = lcount[k], nt_k = (int)sl.w;
-                for (int f = tid; f < nl * nt_k; f += kTileThreads) {
-                    const int li = f / nt_k, j = f - li * nt_k;
-                    const int r = lrows[k * rb + li];
-                    cx.emit_one(r0 + r, __ldg(tv.dtok + sl.z + j), cfg[k * nr + r] & 0xFFFFu);
+            // 3. the (unit, live row at the unit's slot) pairs, one lane each:
+            // most rows die at the unit's first record, so lanes that walk
+            // their own pairs waste far fewer lookups than a warp walking a
+            // unit for all its rows in lockstep.  Warp 0 forms the pairs'
+            // prefix over the units (a unit's pairs are consecutive).
+            if (warp == 1) {
+                // emitting slots: (live row, token ending at the slot's node)
+                // items, prefix over the slots
+                int e0 = 0, e1 = 0;
+                if (lane < ns) e0 = lcount[lane] * (int)sslot[lane].w;
+                if (lane + 32 < ns) e1 = lcount[lane + 32] * (int)sslot[lane + 32].w;
+                int i0 = e0, i1 = e1;
+#pragma unroll
+                for (int off = 1; off < 32; off <<= 1) {
+                    const int y0 = __shfl_up_sync(0xffffffffu, i0, off), y1 = __shfl_up_sync(0xffffffffu, i1, off);
+                    if (lane >= off) i0 += y0, i1 += y1;
                 }
+                const int tot0 = __shfl_sync(0xffffffffu, i0, 31);
+                if (lane < ns) epre[lane] = i0 - e0;
+                if (lane + 32 < ns) epre[lane + 32] = tot0 + i1 - e1;
+                if (lane == 31) epre[ns] = tot0 + (ns > 32 ? i1 : 0);
             }
-            // 3. warps claim (unit, chunk of 32 of its slot's live rows) items,
-            // chunk-major: every unit's first chunk, then every second chunk,
-            // so that units with many live rows do not leave one warp working
-            // while the others wait at the barrier
-            int maxc = 0;   // the most chunks any slot has
-            for (int k = lane; k < ns; k += 32) maxc = max(maxc, (lcount[k] + 31) >> 5);
-            maxc = __reduce_max_sync(0xffffffffu, maxc);
-            for (;;) {
-                int i = 0;
-                if (lane == 0) i = atomicAdd(&ctl[kCtlUnit], 1);
-                i = __shfl_sync(0xffffffffu, i, 0);
-                if (i >= nk * maxc) break;
-                const int c = i / nk, k = i - c * nk;
-                const uint32_t un = sunit[k];
+            if (warp == 0) {
+                const int per = (nk + 31) / 32, k0 = lane * per, k1 = min(nk, k0 + per);
+                int sum = 0;
+                for (int k = k0; k < k1; ++k) sum += lcount[sunit[k] >> 16];
+                int incl = sum;
+#pragma unroll
+                for (int off = 1; off < 32; off <<= 1) {
+                    const int y = __shfl_up_sync(0xffffffffu, incl, off);
+                    if (lane >= off) incl += y;
+                }
+                int run = incl - sum;
+                for (int k = k0; k < k1; ++k) {
+                    upre[k] = run;
+                    run += lcount[sunit[k] >> 16];
+                }
+                if (lane == 31) upre[nk] = incl;
+            }
+            __syncthreads();
+            // the emitting slots' items, spread over the CTA (tokens read from
+            // the preorder list in global memory: all loads independent)
+            for (int f = tid; f < epre[ns]; f += kTileThreads) {
+                int k = 0, hi = ns;   // the slot: epre[k] <= f < epre[k + 1]
+                while (hi - k > 1) {
+                    const int mid = (k + hi) >> 1;
+                    if (epre[mid] <= f) k = mid;
+                    else hi = mid;
+                }
+                const uint4 sl = sslot[k];
+                const int g = f - epre[k], nt_k = (int)sl.w;
+                const int li = g / nt_k, j = g - li * nt_k;
+                const int r = lrows[k * rb + li];
+                cx.emit_one(r0 + r, __ldg(tv.dtok + sl.z + j), cfg[k * nr + r] & 0xFFFFu);
+            }
+            const int npairs = upre[nk];
+            for (int i = tid; i < npairs; i += kTileThreads) {
+                int lo = 0, hi = nk;   // the unit: upre[lo] <= i < upre[lo + 1]
+                while (hi - lo > 1) {
+                    const int mid = (lo + hi) >> 1;
+                    if (upre[mid] <= i) lo = mid;
+                    else hi = mid;
+                }
+                const uint32_t un = sunit[lo];
                 const int x0 = (int)(un & 0xFFFFu), sl = (int)(un >> 16);
-                const int n = lcount[sl] - 32 * c;
-                if (n <= 0) continue;
-                const bool on = lane < n;
-                const int r = on ? lrows[sl * rb + 32 * c + lane] : 0;
-                const uint32_t sd = on ? cfg[sl * nr + r] : 0u;
-                const uint32_t bits = STACK && on ? cfg[kTrieCfg + sl * nr + r] : 0u;
-                cx.walk(lane, r0 + r, x0, sd & 0xFFFFu, bits, sd >> 16, wstk, wstkb, wustk);
+                const int r = lrows[sl * rb + (i - upre[lo])];
+                const uint32_t sd = cfg[sl * nr + r];
+                const uint32_t bits = STACK ? cfg[kTrieCfg + sl * nr + r] : 0u;
+                cx.walk_lane(r0 + r, x0, sd & 0xFFFFu, bits, sd >> 16);
             }
             __syncthreads();
         }
