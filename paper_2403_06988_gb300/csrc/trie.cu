@@ -54,7 +54,7 @@ constexpr int kTrieRowBlock = 512;          // most rows per block
 constexpr int kTrieMaxDevices = 64;
 
 enum TileCtl : int {
-    kCtlUnit = 0,     // units claimed in this row block
+    kCtlUnit = 0,     // (unit, row) pairs claimed in this row block
     kCtlBad = 1,      // a staged record failed its check
     kCtlWords = 4,
 };
@@ -494,8 +494,15 @@ __global__ void __maxnreg__(64)
                 const int r = lrows[k * rb + li];
                 cx.emit_one(r0 + r, __ldg(tv.dtok + sl.z + j), cfg[k * nr + r] & 0xFFFFu);
             }
+            // warps take 32 consecutive pairs at a time (the costliest units'
+            // first), so that no warp is left with the last long walks
             const int npairs = upre[nk];
-            for (int i = tid; i < npairs; i += kTileThreads) {
+            for (;;) {
+                int i = 0;
+                if (lane == 0) i = atomicAdd(&ctl[kCtlUnit], 32);
+                i = __shfl_sync(0xffffffffu, i, 0) + lane;
+                if (i - lane >= npairs) break;
+                if (i >= npairs) continue;
                 int lo = 0, hi = nk;   // the unit: upre[lo] <= i < upre[lo + 1]
                 while (hi - lo > 1) {
                     const int mid = (lo + hi) >> 1;
