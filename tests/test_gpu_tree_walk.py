@@ -95,3 +95,32 @@ def test_tree_walk_tiny_grammars(tree_walk, name):
     assert_exact(mask, m_o, "mask")
     assert_exact(nxt, n_o, "next")
     d.close()
+
+
+def test_tree_walk_long_chains(tree_walk):
+    """Tokens of up to 700 bytes: runs of one-child nodes longer than one walk
+    record (255 nodes), long shared prefixes that branch deep down, and
+    tokens ending inside a run."""
+    import oracle
+    a = synth.int_regex_dfa()
+    rng = np.random.default_rng(31)
+    digits = np.frombuffer(b"0123456789", np.uint8)
+    base = rng.choice(digits, 700).tobytes()
+    toks = {base, base[:255], base[:256], base[:511], b"-" + base[:600], b"x" + base[:40]}
+    for k in (3, 254, 255, 256, 300, 510, 699):   # branches deep inside the run
+        toks.add(base[:k] + bytes([48 + (base[k] - 47) % 10]) + rng.choice(digits, 20).tobytes())
+    while len(toks) < 400:
+        toks.add(rng.choice(np.frombuffer(b"-0123456789x", np.uint8), int(rng.integers(1, 12))).tobytes())
+    toks = sorted(toks)
+    toks.insert(17, b"")   # EOS
+    v = synth.Vocab.from_tokens(toks, eos_id=17)
+    d = Domino.from_parts(a, v, device=0)
+    assert d.info()["walk_tree"] == 1
+    states = np.repeat(np.arange(a.n_states, dtype=np.int32), 3)
+    mask, nxt = d.step_mask(dev(states), None, want_next=True)
+    m_o, n_o, bad = oracle.Problem.from_parts(a, v).step_mask(states, want_next=True)
+    assert bad == 0
+    assert_exact(mask, m_o, "mask")
+    assert_exact(nxt, n_o, "next")
+    assert d.device_error() == 0
+    d.close()
