@@ -16,7 +16,8 @@ from typing import Optional
 import numpy as np
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_PKG, "libdomino.so")
+# DOMINO_DEBUG_LIB=1: the bounds-checked build (build.build(debug=True))
+LIB_PATH = os.path.join(_PKG, "libdomino_debug.so" if os.environ.get("DOMINO_DEBUG_LIB") == "1" else "libdomino.so")
 HEADER = os.path.join(os.path.dirname(_PKG), "include", "domino.h")
 
 DOMINO_OK = 0
@@ -85,8 +86,9 @@ def lib() -> ctypes.CDLL:
     global _lib
     if _lib is None:
         if not os.path.exists(LIB_PATH):
-            raise ImportError(f"libdomino.so is not built ({LIB_PATH}); run __graft_entry__.build() "
-                              "or python -m paper_2403_06988_gb300.build")
+            raise ImportError(f"{os.path.basename(LIB_PATH)} is not built ({LIB_PATH}); run "
+                              "__graft_entry__.build() or python -m paper_2403_06988_gb300.build "
+                              "(build.build(debug=True) for the debug library)")
         L = ctypes.CDLL(LIB_PATH)
         for name, args in _SIGS.items():
             f = getattr(L, name)

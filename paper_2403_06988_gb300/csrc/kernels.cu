@@ -321,6 +321,7 @@ __global__ void __launch_bounds__(kStepThreads, 1)
 
     Tab<E, MODE> tab;
     tab.K = (uint32_t)K;
+    debug_bounds(tab, v);
     const uint16_t* ret;
     if constexpr (MODE == kDenseGlobal) {
         tab.dense = reinterpret_cast<const E*>(STACK ? (const void*)v.t32 : (const void*)v.t16);
@@ -1282,6 +1283,7 @@ __global__ void __launch_bounds__(kAdvanceThreads)
         tab.sp = reinterpret_cast<const uint32_t*>(adv_smem);
         tab.tgt = reinterpret_cast<const E*>(adv_smem + tgt_off);
         tab.K = (uint32_t)v.K;
+        debug_bounds(tab, v);
         advance_row_with<STACK>(v, tab, reinterpret_cast<const uint16_t*>(adv_smem + ret_off), states, stacks, b,
                                 tokens[b], states_out, stacks_out);
     }
@@ -1315,6 +1317,7 @@ __global__ void __launch_bounds__(kAdvanceThreads)
                 tab.sp = v.sp_info;
                 tab.tgt = reinterpret_cast<const E*>(v.sp_tgt);
                 tab.K = (uint32_t)v.K;
+                debug_bounds(tab, v);
                 const int p = __ldg(v.pos_of + t);
                 const int len = (int)(__ldg(v.info + p) >> 16);
                 if (len > 0) {
@@ -1385,6 +1388,7 @@ __global__ void __launch_bounds__(kAdvanceThreads)
     tab.sp = v.sp_info;
     tab.tgt = reinterpret_cast<const E*>(v.sp_tgt);
     tab.K = (uint32_t)v.K;
+    debug_bounds(tab, v);
     const int32_t sv = __ldg(states + b);
     const unsigned long long wv = stacks ? __ldg(reinterpret_cast<const unsigned long long*>(stacks) + b) : 0ull;
     const uint4 rc = decode_row(v, sv, wv, stacks != nullptr, v.accept_bits, false);

@@ -299,6 +299,7 @@ __global__ void __maxnreg__(64)
         for (int i = tid; i < v.Q; i += kTileThreads) s_self[i] = __ldg(v.self_mask + i);
     Tab<E, MODE> tab;
     tab.K = (uint32_t)v.K;
+    debug_bounds(tab, v);
     const uint16_t* ret;
     if constexpr (MODE == kDenseGlobal) {
         tab.dense = reinterpret_cast<const E*>(STACK ? (const void*)v.t32 : (const void*)v.t16);

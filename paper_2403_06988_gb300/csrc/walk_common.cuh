@@ -114,7 +114,26 @@ struct Tab {
     const uint32_t* sp;
     const E* tgt;
     uint32_t K;
+#ifdef DOMINO_DEBUG
+    // the debug build's bounds (set by debug_bounds): a lookup outside the
+    // table sets DOMINO_DEVERR_INTERNAL and reads as the dead state
+    uint32_t Q = 0xFFFFFFFFu, nnz = 0xFFFFFFFFu;
+    uint32_t* err = nullptr;
+    __device__ __forceinline__ bool out_of_bounds(uint32_t s, uint32_t c) const {
+        if (s < Q && c < K) return false;
+        if (err) atomicOr(err, DOMINO_DEVERR_INTERNAL);
+        return true;
+    }
+    __device__ __forceinline__ bool bad_entry(uint32_t i) const {
+        if (i < nnz) return false;
+        if (err) atomicOr(err, DOMINO_DEVERR_INTERNAL);
+        return true;
+    }
+#endif
     __device__ __forceinline__ uint32_t get(uint32_t s, uint32_t c) const {
+#ifdef DOMINO_DEBUG
+        if (out_of_bounds(s, c)) return 0u;
+#endif
         if constexpr (MODE == kDenseSmem) {
             return dense[s * K + c];
         } else if constexpr (MODE == kDenseGlobal) {
@@ -122,15 +141,34 @@ struct Tab {
         } else if constexpr (MODE == kSparse32Smem) {
             const uint2 ri = reinterpret_cast<const uint2*>(sp)[s];
             if (!((ri.x >> c) & 1u)) return 0u;
+#ifdef DOMINO_DEBUG
+            if (bad_entry(ri.y + __popc(ri.x & ((1u << c) - 1u)))) return 0u;
+#endif
             return tgt[ri.y + __popc(ri.x & ((1u << c) - 1u))];
         } else {
             const uint4 ri = reinterpret_cast<const uint4*>(sp)[s];
             const unsigned long long m = ((unsigned long long)ri.y << 32) | ri.x;
             if (!((m >> c) & 1ull)) return 0u;
+#ifdef DOMINO_DEBUG
+            if (bad_entry(ri.z + (uint32_t)__popcll(m & ((1ull << c) - 1ull)))) return 0u;
+#endif
             return tgt[ri.z + __popcll(m & ((1ull << c) - 1ull))];
         }
     }
 };
+
+// The debug build's table bounds for tab (a no-op otherwise).
+template <typename T>
+__device__ __forceinline__ void debug_bounds(T& tab, const StepView& v) {
+#ifdef DOMINO_DEBUG
+    tab.Q = (uint32_t)v.Q;
+    tab.nnz = v.sp_nnz > 0 ? (uint32_t)v.sp_nnz : 0xFFFFFFFFu;
+    tab.err = v.err;
+#else
+    (void)tab;
+    (void)v;
+#endif
+}
 
 // One pushdown step for table entry e (bits 0..15 next, 16..17 kind, 18 sym,
 // 19..31 pop-target triple).  Returns the next state, 0 when rejected.
@@ -303,6 +341,7 @@ __device__ __forceinline__ void advance_row(const StepView& v, const int32_t* st
     tab.sp = v.sp_info;
     tab.tgt = reinterpret_cast<const E*>(v.sp_tgt);
     tab.K = (uint32_t)v.K;
+    debug_bounds(tab, v);
     advance_row_with<STACK>(v, tab, v.ret, states, stacks, b, t, states_out, stacks_out);
 }
 }  // namespace
