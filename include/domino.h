@@ -29,8 +29,11 @@
  *    (all tokens rejected, next state 0) and set a bit of the sticky device
  *    error word read by domino_get_device_error.  No kernel traps.
  *  - A handle is not thread-safe; calls on one handle must be serialised by
- *    the caller (the kernels of different calls may overlap on the GPU only
- *    if the caller puts them on different streams).
+ *    the caller, and their kernels must not overlap on the GPU either (issue
+ *    them on one stream, or order the streams with events): the handle's
+ *    scratch (the logits pass's partials and tickets, the fused decode's
+ *    partials, the host-buffer step's staging) is shared by its calls.
+ *    Different handles are independent.
  */
 #ifndef DOMINO_H
 #define DOMINO_H

@@ -86,12 +86,14 @@ struct StepView {
 // below n (K <= 64, for the self-loop skip).
 // Upper nodes: the root and every node whose subtree has more than kTrieTile
 // nodes or more than kTrieBranch branching levels (an ancestor of an upper
-// node is upper).  Units: the subtrees hanging off upper nodes.  The units are
-// cut into per-CTA batches that fit in shared memory; for a block of rows a
-// CTA computes each row's configuration at the upper nodes its units hang
-// off ("slots"), then a warp walks a unit for up to 32 rows live at its slot
-// at once, in lockstep over the unit's nodes, with a stack of at most
-// kTrieBranch levels (tree_tile_kernel).  The tokens that end at an upper
+// node is upper).  Units: the subtrees hanging off upper nodes.  Inside a
+// unit, a node with one child and no token is walked together with its child:
+// the walk's records are such runs (up to 255 nodes).  The units are cut into
+// per-CTA batches that fit in shared memory; for a block of rows a CTA
+// computes each row's configuration at the upper nodes its units hang off
+// ("slots"), then each (unit, row live at its slot) pair is walked by one
+// thread, depth first over the unit's records, with a stack of at most
+// kTrieBranch entries (tree_tile_kernel).  The tokens that end at an upper
 // node are set by the one batch that lists that node as an emitting slot.
 constexpr int kTrieTile = 64;
 constexpr int kTrieBranch = 8;

@@ -341,12 +341,15 @@ void build_trie_host(domino_ctx* h) {
 
 // Cuts the units into per-CTA batches that fit in the tile kernel's shared
 // memory next to the transition table, for a grid of one CTA per SM.  Units
-// are dealt out in preorder, about the same number of nodes per CTA; a batch
-// holds a run of one CTA's units, the upper nodes they hang off (slots), and
-// the upper nodes in front of them whose tokens it sets (emitting slots: each
-// upper node with tokens is set by exactly one batch).  Chooses the table
-// placement: in shared memory when that leaves room for batches, else through
-// L1/L2.  false: some unit alone does not fit (the per-token walk is used).
+// are weighed by their estimated walk cost, cut in preorder into kTrieInterleave
+// chunks per CTA of equal weight, and CTA c takes chunks c, c + grid, ...; a
+// batch holds some of one CTA's units (staged as node, record and token ranges
+// one after the other, costliest units first), the upper nodes they hang off
+// (slots), and the upper nodes whose tokens it sets (emitting slots: each upper
+// node with tokens is set by the batch of the first unit after it in preorder).
+// Chooses the table placement: in shared memory when that leaves room for
+// batches, else through L1/L2.  false: some unit alone does not fit (the
+// per-token walk is used).
 bool cut_batches(domino_ctx* h) {
     const int smem = h->env.max_smem_optin > 0 ? h->env.max_smem_optin : 232448;
     const int grid = h->env.num_sms > 0 ? h->env.num_sms : 1;
