@@ -71,6 +71,33 @@ def test_tree_walk_precompute_config2(tree_walk):
     d.close()
 
 
+@pytest.mark.parametrize("n_tok,eos", [(1001, 0), (1003, 1002), (2050, 977), (4096, 4095)])
+def test_tree_walk_precompute_ragged_vocab(tree_walk, n_tok, eos):
+    """The precompute over 20000 states with vocabularies whose rows start off
+    16-byte boundaries (V % 4 != 0); EOS first, last or inside a word (2000
+    accepting states); with and without the mask."""
+    import oracle
+    w = synth.workload(4)
+    a = w.automaton
+    toks = [t for t in w.vocab.tokens()[:n_tok] if t][: n_tok - 1]
+    toks.insert(eos, b"")
+    v = synth.Vocab.from_tokens(toks, eos_id=eos)
+    assert v.n_tokens == n_tok
+    d = Domino.from_parts(a, v, device=0)
+    assert d.info()["walk_tree"] == 1
+    Q = a.n_states
+    m_o, n_o, _ = oracle.Problem.from_parts(a, v).step_mask(np.arange(Q, dtype=np.int32), want_next=True,
+                                                            n_threads=NT)
+    assert m_o[:, eos >> 5].any() and (n_o[:, eos] != 0).any()
+    nxt, mask = d.precompute_table()
+    assert_exact(mask, m_o, "table mask")
+    assert_exact(nxt, n_o, "table next")
+    nxt, _ = d.precompute_table(want_mask=False)
+    assert_exact(nxt, n_o, "table next without the mask")
+    assert d.device_error() == 0
+    d.close()
+
+
 @pytest.mark.parametrize("name", ["dyck2", "int_regex", "dyck_ctx"])
 def test_tree_walk_tiny_grammars(tree_walk, name):
     import oracle
