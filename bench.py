@@ -460,7 +460,8 @@ def run_precompute(args, dist: Dist):
         "e2e": {"value": n * Q * V * Ke / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": out_bytes, "steps": Ke,
                 "api": "domino_precompute_table + copy of the table to pinned host memory"},
-        "gpu_launches": K,
+        # the tree walk: tree_clear_kernel then tree_tile_kernel; else one step_kernel
+        "gpu_launches": K * (2 if info["walk_tree"] else 1),
         "clocks": sampler.summary(),
     }
     if dist.rank == 0 and n == 1 and not args.no_cpu_baseline:

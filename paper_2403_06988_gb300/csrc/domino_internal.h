@@ -115,7 +115,7 @@ struct TrieView {
     const uint4* slot;        // {upper index, first token ending at its node, tokens it sets (0: none), 0}
     const uint2* unit;        // {root's staged index, slot index within the batch}
     const int32_t* cta_batch; // [grid + 1]: CTA c takes batches [cta_batch[c], cta_batch[c + 1])
-    int32_t n_nodes, n_upper, grid;
+    int32_t n_nodes, n_upper, grid, n_batches;
     int32_t max_nodes, max_cls, max_toks, max_units, max_slots, max_path;   // the largest batch (records, nodes, ...)
 };
 
@@ -152,10 +152,13 @@ cudaError_t launch_fused_combine(const StepView& v, bool stack, int mode, const 
 // mask / next / row_ids / row_count as launch_step_mask.  mode: where the tile
 // kernel reads transitions.
 int trie_tile_smem_bytes(const StepView& v, const TrieView& tv, bool stack, int table_bytes);
+// row_next (the precompute: row_is_state, next states written, no row list):
+// tv.n_batches device words through which the CTAs share out the batches' row
+// blocks (nullptr: each CTA walks every row of its own batches).
 cudaError_t launch_trie_step(const StepView& v, const TrieView& tv, const LaunchEnv& env, bool stack, int mode,
                              const int32_t* states, const uint64_t* stacks, int32_t batch, bool row_is_state,
                              uint32_t* mask, int32_t* next, cudaStream_t st, const int32_t* row_ids = nullptr,
-                             const int32_t* row_count = nullptr);
+                             const int32_t* row_count = nullptr, int32_t* row_next = nullptr);
 
 // Log-probabilities only (bf16 logits, rows on 16-byte boundaries), given the
 // rows' lse: logprobs[b][t] = logit - lse[b] for allowed t, -inf else.

@@ -61,6 +61,7 @@ struct domino_ctx {
     bool arena_ready = false;
     // prefix tree of the class strings and its per-CTA batches (see TrieView)
     DevBuf d_tnode, d_tncls, d_tdtok, d_tupper, d_tupath, d_tbatch, d_trange, d_tslot, d_tunit, d_tcta;
+    DevBuf d_trow;                   // the precompute's row counter per batch
     std::vector<uint4> t_node;       // host copies (domino_get_prefix_tree)
     std::vector<uint4> t_cnode;      // the walk's records (chains of nodes), two per record
     std::vector<uint32_t> t_hc;      // [n_nodes + 1]: records before each node
@@ -610,6 +611,7 @@ int build_trie(domino_ctx* h) {
     if ((rc = up(h->d_tslot, h->t_slot.data(), h->t_slot.size() * sizeof(uint4)))) return rc;
     if ((rc = up(h->d_tunit, h->t_bunit.data(), h->t_bunit.size() * sizeof(uint2)))) return rc;
     if ((rc = up(h->d_tcta, h->t_cta.data(), h->t_cta.size() * 4))) return rc;
+    if ((rc = dev_reserve(h->d_trow, std::max<size_t>(1, h->t_batch.size() / 2) * 4))) return rc;
     h->trie_ready = true;
     return DOMINO_OK;
 }
@@ -762,6 +764,7 @@ TrieView make_trie_view(const domino_ctx* h) {
     tv.n_nodes = h->t_nodes;
     tv.n_upper = (int32_t)h->t_upper.size();
     tv.grid = h->t_grid;
+    tv.n_batches = (int32_t)(h->t_batch.size() / 2);
     tv.max_nodes = h->t_max_nodes;
     tv.max_cls = h->t_max_cls;
     tv.max_toks = h->t_max_toks;
@@ -875,7 +878,7 @@ int domino_destroy(domino_t h) {
                          &h->d_eos_slot, &h->d_dense, &h->d_sparse, &h->d_accept, &h->d_self, &h->d_tok_cls, &h->d_err, &h->d_fpart, &h->d_partials,
                          &h->d_counters, &h->d_lse_tmp, &h->s_logits, &h->s_mask, &h->s_io,
                          &h->o_prop, &h->o_rows, &h->o_count, &h->d_tnode, &h->d_tdtok, &h->d_tupper, &h->d_tupath, &h->d_tbatch, &h->d_tslot,
-                         &h->d_tunit, &h->d_tcta, &h->d_trange, &h->d_tncls};
+                         &h->d_tunit, &h->d_tcta, &h->d_trange, &h->d_tncls, &h->d_trow};
         for (auto* b : all) dev_free(*b);
         for (cudaEvent_t& e : h->ev_chunk)
             if (e) cudaEventDestroy(e);
@@ -1231,7 +1234,8 @@ int domino_precompute_table(domino_t h, int32_t* next_dev, uint32_t* mask_dev, v
     StepView v = make_view(h);
     if (use_tree(h)) {
         return cuda_status(launch_trie_step(v, make_trie_view(h), h->env, false, h->t_mode, nullptr, nullptr, h->Q,
-                                            true, mask_dev, next_dev, (cudaStream_t)stream));
+                                            true, mask_dev, next_dev, (cudaStream_t)stream, nullptr, nullptr,
+                                            (int32_t*)h->d_trow.p));
     }
     const int mode = choose_mode(h, v, next_dev != nullptr);
     return cuda_status(launch_step_mask(v, h->env, false, mode, nullptr, nullptr, h->Q, true, mask_dev, next_dev,

@@ -34,6 +34,11 @@
 //                          global reductions (and store their next state);
 //                          so do whole subtrees whose classes all loop on the
 //                          row's state (the self-loop skip).
+//
+// With many rows (the precompute: every state a row) a CTA claims its batches'
+// row blocks from a global counter per batch, and a CTA done with its own
+// batches stages the batch with the most rows left and claims row blocks from
+// it too, so that the CTAs end together.
 #include <cuda_runtime.h>
 
 #include <climits>
@@ -56,6 +61,7 @@ constexpr int kTrieMaxDevices = 64;
 enum TileCtl : int {
     kCtlUnit = 0,     // (unit, row) pairs claimed in this row block
     kCtlBad = 1,      // a staged record failed its check
+    kCtlRow = 2,      // the row block claimed (shared row counters)
     kCtlWords = 4,
 };
 
@@ -97,6 +103,7 @@ struct TreeArgs {
     uint32_t* mask;
     int32_t* next;
     int32_t img_bytes, img_tgt_off, img_ret_off;
+    int32_t* row_next;      // [batches]: rows claimed of each batch (zero at launch), or nullptr
 };
 
 // Sets a mask bit without waiting for the result (a reduction, not an atomic
@@ -262,8 +269,37 @@ struct TileCtx {
     }
 };
 
-// 1024 threads a CTA: at most 64 registers a thread.
-template <bool STACK, int MODE, bool NEXT>
+// The rows per block of a batch with `ns` slots.
+__device__ __forceinline__ int rows_per_block(int ns) { return max(1, min(kTrieRowBlock, kTrieCfg / max(ns, 1))); }
+
+// The batch with the most rows left (ties: the lowest index), if at least two
+// of its row blocks are left; -1 otherwise.  Every thread of the CTA calls it;
+// red holds 33 ints of scratch.
+__device__ __forceinline__ int pick_batch(const TrieView& tv, const int32_t* row_next, int nrows, int* red, int tid) {
+    const int nb = __ldg(tv.cta_batch + tv.grid);
+    unsigned best = 0u;   // rows left << 16 | (0xFFFF - batch)
+    for (int b = tid; b < nb; b += kTileThreads) {
+        const int taken = *reinterpret_cast<const volatile int32_t*>(row_next + b);
+        const uint4 bB = __ldg(tv.batch + 2 * b + 1);
+        const int rem = nrows - min(nrows, max(taken, 0));
+        if (rem >= 2 * rows_per_block((int)(bB.y - bB.x)))
+            best = max(best, ((unsigned)rem << 16) | (0xFFFFu - (unsigned)b));
+    }
+    best = __reduce_max_sync(0xffffffffu, best);
+    __syncthreads();   // red is free
+    if ((tid & 31) == 0) red[tid >> 5] = (int)best;
+    __syncthreads();
+    if (tid < 32) {
+        const unsigned w = __reduce_max_sync(0xffffffffu, (unsigned)red[tid]);
+        if (tid == 0) red[32] = w == 0u ? -1 : (int)(0xFFFFu - (w & 0xFFFFu));
+    }
+    __syncthreads();
+    return red[32];
+}
+
+// 1024 threads a CTA: at most 64 registers a thread.  STEAL: row blocks
+// claimed from a.row_next, other CTAs' batches taken once a CTA's own are done.
+template <bool STACK, int MODE, bool NEXT, bool STEAL>
 __global__ void __maxnreg__(64)
     tree_tile_kernel(const __grid_constant__ StepView v, const __grid_constant__ TrieView tv,
                      const uint4* __restrict__ img, const __grid_constant__ TreeArgs a, const RowList list) {
@@ -290,7 +326,7 @@ __global__ void __maxnreg__(64)
     int* epre = reinterpret_cast<int*>(smem + L.epre);   // the emitting slots' first (row, token) items
     int* ctl = reinterpret_cast<int*>(smem + L.ctl);
     const int b0 = __ldg(tv.cta_batch + blockIdx.x), b1 = __ldg(tv.cta_batch + blockIdx.x + 1);
-    if (b0 >= b1) {   // no units for this CTA
+    if (b0 >= b1 && !STEAL) {   // no units for this CTA
         pdl_wait();
         return;
     }
@@ -315,7 +351,19 @@ __global__ void __maxnreg__(64)
     }
     const uint32_t maxd = (uint32_t)v.max_depth;
     bool waited = false;
-    for (int bj = b0; bj < b1; ++bj) {
+    for (int own = b0;;) {
+        int bj = own;
+        if (own < b1) {
+            ++own;
+        } else {
+            if constexpr (!STEAL) break;
+            if (!waited) {   // the row counters are zeroed before the clear kernel
+                pdl_wait();
+                waited = true;
+            }
+            bj = pick_batch(tv, a.row_next, list.rows(a.batch), lcount, tid);
+            if (bj < 0) break;
+        }
         const uint4 bA = __ldg(tv.batch + 2 * bj);       // units [x, y), ranges [z, w)
         const uint4 bB = __ldg(tv.batch + 2 * bj + 1);   // slots [x, y), staged nodes z, tokens w
         const int nk = (int)(bA.y - bA.x), nn = (int)bB.z, nt = (int)bB.w;
@@ -386,8 +434,14 @@ __global__ void __maxnreg__(64)
         const TileCtx<STACK, MODE, NEXT> cx{v, a, tab, ret, maxd, use_self ? s_self : nullptr, snode, scls, ssub, stok,
                                             nn, nt};
         const int nrows = list.rows(a.batch);
-        const int rb = max(1, min(kTrieRowBlock, kTrieCfg / max(ns, 1)));
-        for (int r0 = 0; r0 < nrows; r0 += rb) {
+        const int rb = rows_per_block(ns);
+        for (int r0 = 0;; r0 += rb) {
+            if constexpr (STEAL) {   // the previous block ended with a barrier
+                if (tid == 0) ctl[kCtlRow] = atomicAdd(a.row_next + bj, rb);
+                __syncthreads();
+                r0 = ctl[kCtlRow];
+            }
+            if (r0 >= nrows) break;
             const int nr = min(rb, nrows - r0);
             if (tid < ns) lcount[tid] = 0;
             if (tid == 0) ctl[kCtlUnit] = 0;
@@ -522,6 +576,18 @@ __global__ void __maxnreg__(64)
     }
 }
 
+template <typename K>
+cudaError_t allow_smem(K kern, int bytes, int* configured, std::mutex& mu) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (bytes <= 48 * 1024 || dev >= kTrieMaxDevices) return cudaSuccess;
+    std::lock_guard<std::mutex> lk(mu);
+    if (configured[dev] >= bytes) return cudaSuccess;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess) configured[dev] = bytes;
+    return e;
+}
+
 template <bool STACK, int MODE, bool NEXT>
 cudaError_t launch_tree_t(const StepView& v, const TrieView& tv, const LaunchEnv& env, TreeArgs a,
                           const RowList& list, cudaStream_t st) {
@@ -543,21 +609,28 @@ cudaError_t launch_tree_t(const StepView& v, const TrieView& tv, const LaunchEnv
     const TileLayout L = tile_layout(v.Q, v.self_mask != nullptr, STACK, img_bytes, tv);
     if (L.total > env.max_smem_optin || tv.max_slots > kTrieMaxSlots || tv.grid > env.num_sms)
         return cudaErrorInvalidConfiguration;
-    auto tile = tree_tile_kernel<STACK, MODE, NEXT>;
-    static int configured[kTrieMaxDevices] = {0};
     static std::mutex mu;
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (L.total > 48 * 1024 && dev < kTrieMaxDevices) {
-        std::lock_guard<std::mutex> lk(mu);
-        if (configured[dev] < L.total) {
-            cudaError_t e = cudaFuncSetAttribute(tile, cudaFuncAttributeMaxDynamicSharedMemorySize, L.total);
+    // the precompute (every state a row): shared row counters and stealing
+    const bool steal = !STACK && NEXT && a.row_next && a.row_is_state && !list.ids && tv.n_batches > 0 &&
+                       tv.n_batches <= 0xFFFF && a.batch <= 0xFFFF;
+    if (!steal) a.row_next = nullptr;
+    const int clear_grid = (int)(((int64_t)a.batch * kClearSplit + kClearThreads / 32 - 1) / (kClearThreads / 32));
+    cudaError_t e = cudaSuccess;
+    if constexpr (!STACK && NEXT) {
+        if (steal) {
+            auto tile = tree_tile_kernel<false, MODE, true, true>;
+            static int configured[kTrieMaxDevices] = {0};
+            if ((e = allow_smem(tile, L.total, configured, mu)) != cudaSuccess) return e;
+            if ((e = cudaMemsetAsync(a.row_next, 0, (size_t)tv.n_batches * 4, st)) != cudaSuccess) return e;
+            e = launch_pdl(tree_clear_kernel<NEXT>, dim3(clear_grid), dim3(kClearThreads), 0, st, v, a, list);
             if (e != cudaSuccess) return e;
-            configured[dev] = L.total;
+            return launch_pdl(tile, dim3(tv.grid), dim3(kTileThreads), (size_t)L.total, st, v, tv, img, a, list);
         }
     }
-    const int clear_grid = (int)(((int64_t)a.batch * kClearSplit + kClearThreads / 32 - 1) / (kClearThreads / 32));
-    cudaError_t e = launch_pdl(tree_clear_kernel<NEXT>, dim3(clear_grid), dim3(kClearThreads), 0, st, v, a, list);
+    auto tile = tree_tile_kernel<STACK, MODE, NEXT, false>;
+    static int configured[kTrieMaxDevices] = {0};
+    if ((e = allow_smem(tile, L.total, configured, mu)) != cudaSuccess) return e;
+    e = launch_pdl(tree_clear_kernel<NEXT>, dim3(clear_grid), dim3(kClearThreads), 0, st, v, a, list);
     if (e != cudaSuccess) return e;
     return launch_pdl(tile, dim3(tv.grid), dim3(kTileThreads), (size_t)L.total, st, v, tv, img, a, list);
 }
@@ -582,9 +655,10 @@ int trie_tile_smem_bytes(const StepView& v, const TrieView& tv, bool stack, int 
 cudaError_t launch_trie_step(const StepView& v, const TrieView& tv, const LaunchEnv& env, bool stack, int mode,
                              const int32_t* states, const uint64_t* stacks, int32_t batch, bool row_is_state,
                              uint32_t* mask, int32_t* next, cudaStream_t st, const int32_t* row_ids,
-                             const int32_t* row_count) {
+                             const int32_t* row_count, int32_t* row_next) {
     if (batch <= 0) return cudaSuccess;
     TreeArgs a{};
+    a.row_next = row_next;
     a.states = states;
     a.stacks = stacks;
     a.batch = batch;
